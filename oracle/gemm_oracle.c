@@ -1,0 +1,111 @@
+/*
+ * gemm_oracle.c -- the CPU oracle for the exact integer GEMM  C += A*B.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call, link or
+ * load this file or the library built from it; only the test-suite, the smoke
+ * check and the timed CPU baseline of the benchmark use it.  It shares no code,
+ * header, table or helper with the CUDA library.
+ *
+ * What it computes (paper, Section 4.1, the GEMM definition): A is m x k,
+ * B is k x n, C is m x n, and C is updated in place by the product A*B.  The
+ * paper's micro-kernel (Section 4.1, loop L6 of Figure 1) builds that update as
+ * a sequence of rank-1 updates, one per index p of the reduction dimension,
+ * and its AIE accumulators are wide (48-bit) precisely so that the 16-bit
+ * products are summed without overflow (Section 6.2, closing remarks).
+ *
+ * The oracle is that definition written out: for every row i, every p and
+ * every column j, C[i][j] += A[i][p] * B[p][j], each product formed exactly
+ * (a 16x16-bit product needs at most 31 bits) and summed in 64-bit unsigned
+ * arithmetic, i.e. modulo 2^64.  Because addition modulo 2^64 is associative
+ * and commutative, the final C is unique whatever order a fast implementation
+ * sums in, so the comparison against a GPU result is bit-exact.  The int8
+ * variant is the same update with int8 operands and an int32 C, taken modulo
+ * 2^32 (computed in 64 bits, then truncated, which is the same thing).
+ *
+ * Storage is row-major with leading dimensions: A[i*lda+p], B[p*ldb+j],
+ * C[i*ldc+j]; entries of C outside the m x n block are never read or written.
+ * All pointers are HOST pointers.  nthreads > 1 splits the rows i across
+ * OpenMP threads (each thread owns whole rows of C, so the sum for each entry
+ * is still the plain sequential loop over p); it exists only so that large
+ * cases finish in reasonable time on many cores.
+ *
+ * Return value: 0 on success, 1 on an invalid argument (negative size, ld too
+ * small, null pointer with a non-zero size).
+ */
+#include <stdint.h>
+#include <stddef.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+static int oracle_check(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda,
+                        const void* B, int64_t ldb, const void* C, int64_t ldc) {
+  if (m < 0 || n < 0 || k < 0) return 1;
+  if (m == 0 || n == 0) return 0;
+  if (ldc < n) return 1;
+  if (C == NULL) return 1;
+  if (k == 0) return 0;
+  if (lda < k || ldb < n) return 1;
+  if (A == NULL || B == NULL) return 1;
+  return 0;
+}
+
+/* C (int64, m x n) += A (int16, m x k) * B (int16, k x n), modulo 2^64. */
+int gemm_oracle_i16(int64_t m, int64_t n, int64_t k,
+                    const int16_t* A, int64_t lda,
+                    const int16_t* B, int64_t ldb,
+                    int64_t* C, int64_t ldc, int nthreads) {
+  if (oracle_check(m, n, k, A, lda, B, ldb, C, ldc)) return 1;
+  if (m == 0 || n == 0 || k == 0) return 0;
+#ifdef _OPENMP
+  if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads)
+#else
+  (void)nthreads;
+#endif
+  for (int64_t i = 0; i < m; ++i) {
+    uint64_t* c = (uint64_t*)(C + i * ldc);
+    for (int64_t p = 0; p < k; ++p) {
+      /* one rank-1 term: row i of C gains A[i][p] times row p of B */
+      const int64_t a = (int64_t)A[i * lda + p];
+      const int16_t* b = B + p * ldb;
+      for (int64_t j = 0; j < n; ++j)
+        c[j] += (uint64_t)(a * (int64_t)b[j]);
+    }
+  }
+  return 0;
+}
+
+/* C (int32, m x n) += A (int8, m x k) * B (int8, k x n), modulo 2^32. */
+int gemm_oracle_i8(int64_t m, int64_t n, int64_t k,
+                   const int8_t* A, int64_t lda,
+                   const int8_t* B, int64_t ldb,
+                   int32_t* C, int64_t ldc, int nthreads) {
+  if (oracle_check(m, n, k, A, lda, B, ldb, C, ldc)) return 1;
+  if (m == 0 || n == 0 || k == 0) return 0;
+#ifdef _OPENMP
+  if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads)
+#else
+  (void)nthreads;
+#endif
+  for (int64_t i = 0; i < m; ++i) {
+    int32_t* c = C + i * ldc;
+    for (int64_t j = 0; j < n; ++j) {
+      uint64_t s = (uint64_t)(int64_t)c[j];
+      for (int64_t p = 0; p < k; ++p)
+        s += (uint64_t)((int64_t)A[i * lda + p] * (int64_t)B[p * ldb + j]);
+      c[j] = (int32_t)(uint32_t)s; /* keep the low 32 bits: modulo 2^32 */
+    }
+  }
+  return 0;
+}
+
+/* Threads the library was built to use (1 without OpenMP). */
+int gemm_oracle_max_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}

@@ -1,0 +1,241 @@
+"""Checks that pin the CPU oracle to facts fixed outside itself.
+
+Each check returns a list of failure strings (empty = pass) so the same
+checks serve both the regular tests and the mutation tests, which plant a
+mistake in a copy of the oracle's C source and require some check to fail.
+
+What pins the oracle (the GEMM definition of Section 4.1, C += A*B):
+  * hand-computed cases (tests/golden/hand_cases.json), each with its working;
+  * brute force with Python's arbitrary-precision integers on tiny shapes;
+  * numpy's integer matmul on int64 arrays (an exact library routine);
+  * closed forms: all-ones gives C += k, extreme operands give k*2^30 etc.;
+  * identity and permutation matrices;
+  * the paper's blocked algorithm (Figure 1, loops L1-L3): summing the GEMM
+    over k_c-blocks of the reduction dimension and m_c/n_c-blocks of C gives
+    the unblocked result;
+  * modular wrap-around and untouched padding outside the m x n block of C.
+"""
+from __future__ import annotations
+
+import json
+import os
+
+import numpy as np
+
+import gemm_inputs as gi
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "hand_cases.json")
+TINY = (0, 1, 2, 3, 5, 8, 17)
+
+
+def golden_cases():
+    with open(GOLDEN) as f:
+        return json.load(f)["cases"]
+
+
+def _arrays(case):
+    op = np.int16 if case["kind"] == "i16" else np.int8
+    cd = np.int64 if case["kind"] == "i16" else np.int32
+    A = np.array(case["A"], dtype=op).reshape(case["m"], case["k"])
+    B = np.array(case["B"], dtype=op).reshape(case["k"], case["n"])
+    C = np.array(case["C_in"], dtype=cd).reshape(case["m"], case["n"])
+    E = np.array(case["C_out"], dtype=cd).reshape(case["m"], case["n"])
+    return A, B, C, E
+
+
+def bigint_gemm(A, B, C, bits):
+    """C + A*B with Python integers, reduced to a two's-complement `bits`-bit value."""
+    m, k = A.shape
+    n = B.shape[1]
+    out = np.empty_like(C)
+    mod = 1 << bits
+    for i in range(m):
+        for j in range(n):
+            s = int(C[i, j])
+            for p in range(k):
+                s += int(A[i, p]) * int(B[p, j])
+            s %= mod
+            if s >= mod >> 1:
+                s -= mod
+            out[i, j] = s
+    return out
+
+
+def numpy_gemm(A, B, C):
+    """C + A*B through numpy's exact int64 matmul (wraps modulo 2^64)."""
+    P = np.matmul(A.astype(np.int64), B.astype(np.int64))
+    with np.errstate(over="ignore"):
+        R = C.astype(np.int64) + P
+    return R.astype(C.dtype)  # int32 C: astype keeps the low 32 bits (mod 2^32)
+
+
+def _run(lib, A, B, C, nthreads=1):
+    X = C.copy()
+    oracle.gemm(A, B, X, nthreads=nthreads, lib=lib)
+    return X
+
+
+def check_golden(lib):
+    bad = []
+    for case in golden_cases():
+        A, B, C, E = _arrays(case)
+        got = _run(lib, A, B, C)
+        if not np.array_equal(got, E):
+            bad.append(f"golden {case['name']}: {got.tolist()} != {E.tolist()}")
+    return bad
+
+
+def check_bruteforce(lib, shapes=None, kinds=("i16", "i8")):
+    bad = []
+    shapes = shapes or [(m, n, k) for m in TINY for n in TINY for k in TINY]
+    for kind in kinds:
+        bits = 64 if kind == "i16" else 32
+        for idx, (m, n, k) in enumerate(shapes):
+            A, B, C = gi.random_problem(7000 + idx, m, n, k, kind)
+            exp = bigint_gemm(A, B, C, bits)
+            got = _run(lib, A, B, C)
+            if not np.array_equal(got, exp):
+                bad.append(f"bruteforce {kind} {m}x{n}x{k}")
+    return bad
+
+
+def check_extreme_bruteforce(lib):
+    """All-minimum / all-maximum operands, where any int32 shortcut overflows."""
+    bad = []
+    for kind, lo, hi in (("i16", -32768, 32767), ("i8", -128, 127)):
+        op = np.int16 if kind == "i16" else np.int8
+        cd = np.int64 if kind == "i16" else np.int32
+        bits = 64 if kind == "i16" else 32
+        for (m, n, k) in ((3, 5, 17), (8, 2, 33), (1, 1, 130)):
+            for a, b in ((lo, lo), (hi, lo), (hi, hi)):
+                A = np.full((m, k), a, op)
+                B = np.full((k, n), b, op)
+                C = np.zeros((m, n), cd)
+                if not np.array_equal(_run(lib, A, B, C), bigint_gemm(A, B, C, bits)):
+                    bad.append(f"extreme {kind} {m}x{n}x{k} a={a} b={b}")
+    return bad
+
+
+def check_numpy(lib, shapes=((64, 48, 80), (129, 70, 301), (256, 256, 256))):
+    bad = []
+    for idx, (m, n, k) in enumerate(shapes):
+        for kind in ("i16", "i8"):
+            A, B, C = gi.random_problem(9100 + idx, m, n, k, kind)
+            if not np.array_equal(_run(lib, A, B, C), numpy_gemm(A, B, C)):
+                bad.append(f"numpy {kind} {m}x{n}x{k}")
+    return bad
+
+
+def check_closed_forms(lib):
+    bad = []
+    for k in (1, 2, 7, 300):
+        m, n = 3, 4
+        ones = _run(lib, np.ones((m, k), np.int16), np.ones((k, n), np.int16), np.zeros((m, n), np.int64))
+        if not (ones == k).all():
+            bad.append(f"all-ones k={k}")
+        mm = _run(lib, np.full((m, k), -32768, np.int16), np.full((k, n), -32768, np.int16),
+                  np.zeros((m, n), np.int64))
+        if not (mm == k * (1 << 30)).all():
+            bad.append(f"min*min k={k}")
+        xm = _run(lib, np.full((m, k), 32767, np.int16), np.full((k, n), -32768, np.int16),
+                  np.zeros((m, n), np.int64))
+        if not (xm == -k * 1073709056).all():
+            bad.append(f"max*min k={k}")
+        i8 = _run(lib, np.full((m, k), -128, np.int8), np.full((k, n), -128, np.int8),
+                  np.zeros((m, n), np.int32))
+        if not (i8 == k * 16384).all():  # k * 2^14 < 2^31 for every k here
+            bad.append(f"i8 min*min k={k}")
+    return bad
+
+
+def check_identity_permutation(lib):
+    bad = []
+    m, n = 37, 23
+    _, B, C = gi.random_problem(31, m, n, m, "i16")
+    eye = np.eye(m, dtype=np.int16)
+    if not np.array_equal(_run(lib, eye, B, C), C + B.astype(np.int64)):
+        bad.append("identity")
+    perm = np.array(gi.uniform_int(77, (m,), 0, 1 << 30, np.int64).argsort(kind="stable"))
+    P = np.zeros((m, m), np.int16)
+    P[np.arange(m), perm] = 1
+    if not np.array_equal(_run(lib, P, B, C), C + B[perm].astype(np.int64)):
+        bad.append("permutation")
+    return bad
+
+
+def check_blocked(lib, m=70, n=45, k=133, mc=32, nc=16, kc=40):
+    """Figure 1 of the paper: loops L1 (n_c), L2 (k_c), L3 (m_c) around C += A_c B_c."""
+    A, B, C = gi.random_problem(55, m, n, k, "i16")
+    full = _run(lib, A, B, C)
+    X = C.copy()
+    for jc in range(0, n, nc):
+        for pc in range(0, k, kc):
+            for ic in range(0, m, mc):
+                sub = X[ic:ic + mc, jc:jc + nc]  # a strided view: leading dimension n
+                oracle.gemm(A[ic:ic + mc, pc:pc + kc], B[pc:pc + kc, jc:jc + nc], sub, lib=lib)
+    return [] if np.array_equal(full, X) else ["blocked"]
+
+
+def check_padding(lib):
+    """Leading dimensions larger than the rows: only the m x n block of C changes."""
+    bad = []
+    m, n, k = 9, 11, 13
+    A, B, C = gi.random_problem(66, m, n, k, "i16")
+    exp = numpy_gemm(A, B, C)
+    Ap = np.full((m, k + 5), 12345, np.int16)
+    Bp = np.full((k, n + 3), -777, np.int16)
+    Cp = np.full((m, n + 7), -424242, np.int64)
+    Ap[:, :k] = A
+    Bp[:, :n] = B
+    Cp[:, :n] = C
+    oracle.gemm(Ap[:, :k], Bp[:, :n], Cp[:, :n], lib=lib)
+    if not np.array_equal(Cp[:, :n], exp):
+        bad.append("padded result")
+    if not (Cp[:, n:] == -424242).all():
+        bad.append("padding of C touched")
+    return bad
+
+
+def check_linearity(lib):
+    bad = []
+    m, n, k = 20, 30, 40
+    A1, B, C = gi.random_problem(81, m, n, k, "i16", a_range=(-16384, 16383))
+    A2, _, _ = gi.random_problem(82, m, n, k, "i16", a_range=(-16384, 16383))
+    z = np.zeros((m, n), np.int64)
+    lhs = _run(lib, (A1 + A2).astype(np.int16), B, z)
+    rhs = _run(lib, A1, B, z) + _run(lib, A2, B, z)
+    if not np.array_equal(lhs, rhs):
+        bad.append("linear in A")
+    B1, B2 = B // 2, B - B // 2
+    if not np.array_equal(_run(lib, A1, B, z), _run(lib, A1, B1.astype(np.int16), z) + _run(lib, A1, B2.astype(np.int16), z)):
+        bad.append("linear in B")
+    if not np.array_equal(_run(lib, A1, B, C) - _run(lib, A1, B, z), C):
+        bad.append("offset by C_in")
+    return bad
+
+
+def check_transpose(lib):
+    m, n, k = 13, 29, 7
+    A, B, C = gi.random_problem(91, m, n, k, "i16")
+    X = _run(lib, A, B, C)
+    Y = _run(lib, np.ascontiguousarray(B.T), np.ascontiguousarray(A.T), np.ascontiguousarray(C.T))
+    return [] if np.array_equal(X, Y.T) else ["transpose identity (AB)^T = B^T A^T"]
+
+
+ALL_CHECKS = (check_golden, check_extreme_bruteforce, check_closed_forms, check_identity_permutation,
+              check_blocked, check_padding, check_linearity, check_transpose, check_numpy)
+
+
+def pin_failures(lib, bruteforce_shapes=None):
+    bad = []
+    for chk in ALL_CHECKS:
+        try:
+            bad += chk(lib)
+        except Exception as e:  # a crash of a mutant counts as detected
+            bad.append(f"{chk.__name__} raised {type(e).__name__}: {e}")
+    try:
+        bad += check_bruteforce(lib, shapes=bruteforce_shapes)
+    except Exception as e:
+        bad.append(f"bruteforce raised {e}")
+    return bad

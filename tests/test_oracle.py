@@ -1,0 +1,134 @@
+"""The CPU oracle against what the paper and the mathematics fix (no GPU)."""
+import os
+import re
+import subprocess
+import tempfile
+
+import numpy as np
+import pytest
+
+import gemm_inputs as gi
+import oracle
+import oracle_pins as pins
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return oracle.load()
+
+
+def test_golden_hand_cases(lib):
+    assert pins.check_golden(lib) == []
+
+
+@pytest.mark.parametrize("kind", ["i16", "i8"])
+def test_bruteforce_tiny_shapes(lib, kind):
+    assert pins.check_bruteforce(lib, kinds=(kind,)) == []
+
+
+def test_extreme_values(lib):
+    assert pins.check_extreme_bruteforce(lib) == []
+
+
+def test_numpy_integer_matmul(lib):
+    assert pins.check_numpy(lib) == []
+
+
+def test_closed_forms(lib):
+    assert pins.check_closed_forms(lib) == []
+
+
+def test_identity_and_permutation(lib):
+    assert pins.check_identity_permutation(lib) == []
+
+
+def test_blocked_algorithm_equivalence(lib):
+    assert pins.check_blocked(lib) == []
+
+
+def test_padding_untouched(lib):
+    assert pins.check_padding(lib) == []
+
+
+def test_linearity(lib):
+    assert pins.check_linearity(lib) == []
+
+
+def test_transpose_identity(lib):
+    assert pins.check_transpose(lib) == []
+
+
+def test_zero_sizes_and_k0(lib):
+    A, B, C = gi.random_problem(5, 4, 6, 0, "i16")
+    X = C.copy()
+    oracle.gemm(A, B, X, lib=lib)
+    assert np.array_equal(X, C)
+    for m, n in ((0, 5), (5, 0), (0, 0)):
+        A, B, C = gi.random_problem(6, m, n, 3, "i16")
+        oracle.gemm(A, B, C, lib=lib)
+
+
+def test_invalid_arguments_rejected(lib):
+    i64 = np.zeros((2, 2), np.int64)
+    a = np.zeros((2, 2), np.int16)
+    f = lib.gemm_oracle_i16
+    p = a.ctypes.data
+    c = i64.ctypes.data
+    assert f(-1, 2, 2, p, 2, p, 2, c, 2, 1) == 1
+    assert f(2, 2, 2, p, 1, p, 2, c, 2, 1) == 1   # lda < k
+    assert f(2, 2, 2, p, 2, p, 1, c, 2, 1) == 1   # ldb < n
+    assert f(2, 2, 2, p, 2, p, 2, c, 1, 1) == 1   # ldc < n
+    assert f(2, 2, 2, 0, 2, p, 2, c, 2, 1) == 1   # null A
+    assert f(2, 2, 2, p, 2, p, 2, c, 2, 1) == 0
+
+
+def test_threads_do_not_change_result(lib):
+    A, B, C = gi.random_problem(12, 97, 33, 65, "i16")
+    X1, X4 = C.copy(), C.copy()
+    oracle.gemm(A, B, X1, nthreads=1, lib=lib)
+    oracle.gemm(A, B, X4, nthreads=4, lib=lib)
+    assert np.array_equal(X1, X4)
+
+
+def test_workload_small_case_matches_numpy(lib):
+    """The 256^3 workload (C in [-2^20, 2^20]) against numpy's exact int64 matmul."""
+    w = gi.WORKLOADS["i16_256"]
+    A, B, C = gi.make_inputs(w)
+    X = C.copy()
+    oracle.gemm(A, B, X, nthreads=4, lib=lib)
+    assert np.array_equal(X, pins.numpy_gemm(A, B, C))
+
+
+# --- mutation tests: a mistake planted in a copy of the oracle must be caught ---
+
+MUTANTS = {
+    "drop_last_rank1_term": ("for (int64_t p = 0; p < k; ++p) {", "for (int64_t p = 0; p < k - 1; ++p) {"),
+    "wrong_sign": ("c[j] += (uint64_t)(a * (int64_t)b[j]);", "c[j] -= (uint64_t)(a * (int64_t)b[j]);"),
+    "transposed_A_index": ("const int64_t a = (int64_t)A[i * lda + p];", "const int64_t a = (int64_t)A[p * lda + i];"),
+    "int32_accumulator": ("c[j] += (uint64_t)(a * (int64_t)b[j]);",
+                          "c[j] = (uint64_t)(int64_t)(int32_t)(uint32_t)(c[j] + (uint64_t)(a * (int64_t)b[j]));"),
+    "overwrites_C": ("uint64_t* c = (uint64_t*)(C + i * ldc);",
+                     "uint64_t* c = (uint64_t*)(C + i * ldc); for (int64_t q = 0; q < n; ++q) c[q] = 0;"),
+    "ignores_ldb": ("const int16_t* b = B + p * ldb;", "const int16_t* b = B + p * n;"),
+    "off_by_one_column": ("for (int64_t j = 0; j < n; ++j)\n        c[j] +=", "for (int64_t j = 1; j < n; ++j)\n        c[j] +="),
+    "i8_truncates_to_16_bits": ("c[j] = (int32_t)(uint32_t)s;", "c[j] = (int32_t)(int16_t)s;"),
+    "i8_transposed_B": ("(int64_t)B[p * ldb + j]", "(int64_t)B[j * ldb + p]"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name):
+    src = open(os.path.join(os.path.dirname(oracle.__file__), "gemm_oracle.c")).read()
+    old, new = MUTANTS[name]
+    assert src.count(old) >= 1, f"mutation anchor not found: {old!r}"
+    mutated = src.replace(old, new, 1)
+    with tempfile.TemporaryDirectory() as d:
+        s = os.path.join(d, "mut.c")
+        so = os.path.join(d, "libmut.so")
+        open(s, "w").write(mutated)
+        subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", s, "-o", so], check=True,
+                       capture_output=True)
+        lib = oracle.load(so)
+        small = [(m, n, k) for m in (1, 2, 5) for n in (1, 3, 8) for k in (1, 2, 17)]
+        failures = pins.pin_failures(lib, bruteforce_shapes=small)
+    assert failures, f"mutant {name} passed every pin"
