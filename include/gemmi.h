@@ -1,0 +1,170 @@
+/*
+ * gemmi.h -- exact integer GEMM  C += A*B  on NVIDIA GB300 (sm_103a).
+ *
+ * The operation is the GEMM of Section 4.1 of the paper ("Toward Matrix
+ * Multiplication for Deep Learning Inference on the Xilinx Versal"): A is
+ * m x k, B is k x n, C is m x n, and C is updated in place, C += A*B.  The
+ * paper's micro-kernel takes INT16 operands (Section 6.1) and sums their
+ * products in 48-bit accumulators so that nothing overflows (Section 6.2);
+ * this library keeps that exactness and widens the result to a 64-bit C.
+ *
+ * Layout (all entry points): row-major with leading dimensions,
+ *     A[i*lda + p],  B[p*ldb + j],  C[i*ldc + j],
+ * lda >= max(1,k), ldb >= max(1,n), ldc >= max(1,n).  Entries of C outside the
+ * m x n block (the padding of each row) are never read or written.
+ *
+ * Semantics: bit-exact.  int16 operands accumulate into an int64 C modulo
+ * 2^64; int8 operands accumulate into an int32 C modulo 2^32.  Addition modulo
+ * 2^w is associative, so the result is unique and independent of the order in
+ * which the kernels sum.  m == 0, n == 0 or k == 0 is a no-op returning
+ * GEMMI_OK.
+ *
+ * Errors: every entry point returns a gemmi_status code; the text of the last
+ * error of the calling thread is available from gemmi_last_error().  Kernel
+ * launches are asynchronous: a device-side failure (a pipeline wait that ran
+ * past its time bound) is recorded in a per-device status word that
+ * gemmi_device_status() reads (and clears).  No device code traps.
+ */
+#ifndef GEMMI_H
+#define GEMMI_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum gemmi_status {
+  GEMMI_OK = 0,
+  GEMMI_EINVAL = 1,   /* negative size, ld too small, null pointer with a non-zero size, C overlapping A or B */
+  GEMMI_ENOMEM = 2,   /* the device workspace could not be allocated */
+  GEMMI_ECUDA = 3,    /* a CUDA runtime/driver call or a kernel launch failed */
+  GEMMI_ETIMEOUT = 4, /* a device-side pipeline wait exceeded its bound (reported by gemmi_device_status) */
+  GEMMI_EARCH = 5     /* the current device is not an sm_103 (GB300) GPU */
+} gemmi_status;
+
+/*
+ * gemm_i16 -- C (int64) += A (int16) * B (int16), exactly, modulo 2^64.
+ * Section 4.1 (problem statement), Section 6.1 (INT16 operands).
+ *
+ * A, B, C are DEVICE pointers owned by the caller; A and B are only read,
+ * C is read and written.  The call is asynchronous on the library's current
+ * stream (gemmi_set_stream; default: the legacy default stream).  The library
+ * owns a device workspace for the limb planes of A and B (grown on demand,
+ * freed by gemmi_release_workspace) and serialises its use across streams.
+ * Returns GEMMI_OK, GEMMI_EINVAL, GEMMI_ENOMEM, GEMMI_ECUDA or GEMMI_EARCH.
+ */
+int gemm_i16(int64_t m, int64_t n, int64_t k,
+             const int16_t* A, int64_t lda,
+             const int16_t* B, int64_t ldb,
+             int64_t* C, int64_t ldc);
+
+/* gemm_i16 on an explicit stream (a cudaStream_t passed as void*; NULL = legacy default stream). */
+int gemm_i16_ex(int64_t m, int64_t n, int64_t k,
+                const int16_t* A, int64_t lda,
+                const int16_t* B, int64_t ldb,
+                int64_t* C, int64_t ldc, void* stream);
+
+/*
+ * gemm_i8 -- C (int32) += A (int8) * B (int8), exactly, modulo 2^32.
+ * Section 4.1 (problem statement); the INT8 datatype of Section 6.1.
+ * Same pointer ownership, layout, stream and error behaviour as gemm_i16.
+ */
+int gemm_i8(int64_t m, int64_t n, int64_t k,
+            const int8_t* A, int64_t lda,
+            const int8_t* B, int64_t ldb,
+            int32_t* C, int64_t ldc);
+
+int gemm_i8_ex(int64_t m, int64_t n, int64_t k,
+               const int8_t* A, int64_t lda,
+               const int8_t* B, int64_t ldb,
+               int32_t* C, int64_t ldc, void* stream);
+
+/*
+ * gemm_i16_host / gemm_i8_host -- the same GEMMs on HOST buffers.
+ * A, B, C are host pointers (pinned memory gives the fastest copies).  The
+ * library copies A, B and C to device buffers it owns, runs the GEMM on its
+ * current stream, copies C back and waits for the stream, so C holds the
+ * result when the call returns.  Errors as above; a device-side timeout is
+ * returned directly as GEMMI_ETIMEOUT.
+ */
+int gemm_i16_host(int64_t m, int64_t n, int64_t k,
+                  const int16_t* A, int64_t lda,
+                  const int16_t* B, int64_t ldb,
+                  int64_t* C, int64_t ldc);
+
+int gemm_i8_host(int64_t m, int64_t n, int64_t k,
+                 const int8_t* A, int64_t lda,
+                 const int8_t* B, int64_t ldb,
+                 int32_t* C, int64_t ldc);
+
+/* Stream used by gemm_i16 / gemm_i8 / *_host (a cudaStream_t as void*). */
+void gemmi_set_stream(void* stream);
+
+/* Text of the calling thread's last error ("" if none).  Owned by the library. */
+const char* gemmi_last_error(void);
+
+/*
+ * Synchronises the current device and returns, then clears, its device status
+ * word: GEMMI_OK, or GEMMI_ETIMEOUT if a kernel gave up a pipeline wait.
+ * gemmi_device_status_detail() returns the raw word of the last read
+ * (low byte: status code; next byte: the wait site; upper half: block index).
+ */
+int gemmi_device_status(void);
+uint32_t gemmi_device_status_detail(void);
+
+/* Frees the library-owned device workspace of the current device (synchronises it). */
+int gemmi_release_workspace(void);
+
+/* Bytes of library-owned device workspace currently held on the current device. */
+size_t gemmi_workspace_bytes(void);
+
+/*
+ * Tuning and test options (process-wide).
+ *   GEMMI_OPT_SKINNY_MAX_M : int16 GEMMs with m <= this value take the
+ *                            skinny-M kernel (default 16, maximum 16; 0 disables it).
+ *   GEMMI_OPT_WAIT_TIMEOUT_US : bound on every device-side pipeline wait, in
+ *                            microseconds (default 4,000,000).
+ *   GEMMI_OPT_SKINNY_KSPLIT : number of CTAs sharing the reduction dimension
+ *                            of one skinny column block (0 = automatic).
+ * Returns GEMMI_OK or GEMMI_EINVAL.
+ */
+enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3 };
+int gemmi_set_option(int option, int64_t value);
+int64_t gemmi_get_option(int option);
+
+/*
+ * Failure-detection self-test: launches one tiny kernel whose single thread
+ * waits, with a bound of `timeout_us` microseconds, on a shared-memory barrier
+ * that nothing ever completes.  The wait gives up, the kernel records
+ * GEMMI_ETIMEOUT in the device status word and returns normally; the context
+ * stays usable.  Returns the status word's code read back by
+ * gemmi_device_status() (GEMMI_ETIMEOUT when detection works).
+ */
+int gemmi_selftest_wait_timeout(int64_t timeout_us);
+
+/*
+ * Per-kernel timing for benchmarks.  While enabled, the library records a CUDA
+ * event pair on the launching stream around each launch of the kernels below;
+ * gemmi_kernel_time() waits for the recorded events and returns the summed
+ * device time (milliseconds) and the number of timed launches of one kernel.
+ * gemmi_kernel_timing(0|1) switches recording and resets the sums.
+ *   GEMMI_KERNEL_SPLIT   : the limb split / conversion of A and B (one timed pair per call)
+ *   GEMMI_KERNEL_TC_I16  : the tcgen05 int16 GEMM kernel
+ *   GEMMI_KERNEL_TC_I8   : the tcgen05 int8 GEMM kernel
+ *   GEMMI_KERNEL_SKINNY  : the skinny-M int16 kernel
+ */
+enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
+       GEMMI_KERNEL_COUNT = 4 };
+int gemmi_kernel_timing(int enable);
+int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
+
+/* Library version string. */
+const char* gemmi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GEMMI_H */

@@ -1,0 +1,230 @@
+"""Exact integer GEMM (C += A*B) on NVIDIA GB300: Python binding of libgemmi.
+
+The C library (include/gemmi.h, built from csrc/ by `build()`) does all the
+work on the GPU; this module only marshals arguments through ctypes.  There is
+no CPU fallback: if the library is missing, every call raises.
+
+    gemm_i16(A, B, C)       torch CUDA tensors: int16 A (m x k), B (k x n), int64 C (m x n)
+    gemm_i8(A, B, C)        torch CUDA tensors: int8 A, B, int32 C
+    gemm_i16_host(A, B, C)  numpy arrays (host memory): the library copies in and out
+    gemm_i8_host(A, B, C)
+
+Matrices are row-major with unit column stride; a row stride larger than the
+row length (padding) is passed as the leading dimension.  C is updated in
+place: C += A @ B, bit-exactly (modulo 2^64 for int64 C, 2^32 for int32 C).
+The GEMM is the one of Section 4.1 of the paper; see include/gemmi.h.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libgemmi.so")
+
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EARCH = 0, 1, 2, 3, 4, 5
+OPT_SKINNY_MAX_M, OPT_WAIT_TIMEOUT_US, OPT_SKINNY_KSPLIT = 1, 2, 3
+EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
+            "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_detail",
+            "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
+            "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version")
+KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY = 0, 1, 2, 3
+
+_lib = None
+
+
+class GemmiError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"gemmi error {code}: {msg}")
+        self.code = code
+
+
+def build(force: bool = False) -> str:
+    from . import _build
+    return _build.build(force=force)
+
+
+def lib():
+    """The loaded C library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libgemmi.so not found at {LIB_PATH}: build it first "
+                               "(paper_2302_07594_gb300.build() or __graft_entry__.build())")
+        L = ctypes.CDLL(LIB_PATH)
+        i64, vp = ctypes.c_int64, ctypes.c_void_p
+        core = [i64, i64, i64, vp, i64, vp, i64, vp, i64]
+        for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host"):
+            getattr(L, name).argtypes = core
+            getattr(L, name).restype = ctypes.c_int
+        for name in ("gemm_i16_ex", "gemm_i8_ex"):
+            getattr(L, name).argtypes = core + [vp]
+            getattr(L, name).restype = ctypes.c_int
+        L.gemmi_set_stream.argtypes = [vp]
+        L.gemmi_set_stream.restype = None
+        L.gemmi_last_error.restype = ctypes.c_char_p
+        L.gemmi_device_status.restype = ctypes.c_int
+        L.gemmi_device_status_detail.restype = ctypes.c_uint32
+        L.gemmi_release_workspace.restype = ctypes.c_int
+        L.gemmi_workspace_bytes.restype = ctypes.c_size_t
+        L.gemmi_set_option.argtypes = [ctypes.c_int, i64]
+        L.gemmi_set_option.restype = ctypes.c_int
+        L.gemmi_get_option.argtypes = [ctypes.c_int]
+        L.gemmi_get_option.restype = i64
+        L.gemmi_selftest_wait_timeout.argtypes = [i64]
+        L.gemmi_selftest_wait_timeout.restype = ctypes.c_int
+        L.gemmi_kernel_timing.argtypes = [ctypes.c_int]
+        L.gemmi_kernel_timing.restype = ctypes.c_int
+        L.gemmi_kernel_time.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
+        L.gemmi_kernel_time.restype = ctypes.c_int
+        L.gemmi_version.restype = ctypes.c_char_p
+        _lib = L
+    return _lib
+
+
+def _check(rc: int):
+    if rc != OK:
+        raise GemmiError(rc, lib().gemmi_last_error().decode(errors="replace"))
+
+
+def last_error() -> str:
+    return lib().gemmi_last_error().decode(errors="replace")
+
+
+# ------------------------------------------------------------------ torch (device) entry points
+def _dev_ld(t, name):
+    if t.dim() != 2:
+        raise ValueError(f"{name} must be 2-D")
+    rows, cols = t.shape
+    if t.numel() == 0 or rows == 1:
+        return max(cols, 1)
+    if (cols > 1 and t.stride(1) != 1) or t.stride(0) < cols:
+        raise ValueError(f"{name} must be row-major with unit column stride")
+    return t.stride(0)
+
+
+def _torch_call(fn_name, A, B, C, op_dtype, c_dtype, stream):
+    import torch
+    for t, nm, dt in ((A, "A", op_dtype), (B, "B", op_dtype), (C, "C", c_dtype)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda:
+            raise TypeError(f"{nm} must be a CUDA tensor")
+        if t.dtype != dt:
+            raise TypeError(f"{nm} must be {dt}, got {t.dtype}")
+    if not (A.device == B.device == C.device):
+        raise ValueError("A, B and C must be on the same device")
+    m, k = A.shape
+    k2, n = B.shape
+    if k2 != k or tuple(C.shape) != (m, n):
+        raise ValueError(f"shape mismatch: A {tuple(A.shape)}, B {tuple(B.shape)}, C {tuple(C.shape)}")
+    if stream is None:
+        stream = torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = getattr(lib(), fn_name)(m, n, k, A.data_ptr(), _dev_ld(A, "A"), B.data_ptr(), _dev_ld(B, "B"),
+                                     C.data_ptr(), _dev_ld(C, "C"), stream.cuda_stream)
+    _check(rc)
+    return C
+
+
+def gemm_i16(A, B, C, stream=None):
+    """C += A @ B on the GPU: int16 A (m x k), int16 B (k x n), int64 C (m x n); exact modulo 2^64."""
+    import torch
+    return _torch_call("gemm_i16_ex", A, B, C, torch.int16, torch.int64, stream)
+
+
+def gemm_i8(A, B, C, stream=None):
+    """C += A @ B on the GPU: int8 A, int8 B, int32 C; exact modulo 2^32."""
+    import torch
+    return _torch_call("gemm_i8_ex", A, B, C, torch.int8, torch.int32, stream)
+
+
+# ------------------------------------------------------------------ host-buffer entry points
+def _host_ld(x, name):
+    import numpy as np
+    if not isinstance(x, np.ndarray) or x.ndim != 2:
+        raise TypeError(f"{name} must be a 2-D numpy array")
+    rows, cols = x.shape
+    if x.size == 0 or rows == 1:
+        return max(cols, 1)
+    if (cols > 1 and x.strides[1] != x.itemsize) or x.strides[0] % x.itemsize or x.strides[0] < cols * x.itemsize:
+        raise ValueError(f"{name} must be row-major with unit column stride")
+    return x.strides[0] // x.itemsize
+
+
+def _host_call(fn_name, A, B, C, op_dtype, c_dtype):
+    import numpy as np
+    for x, nm, dt in ((A, "A", op_dtype), (B, "B", op_dtype), (C, "C", c_dtype)):
+        if not isinstance(x, np.ndarray) or x.dtype != dt:
+            raise TypeError(f"{nm} must be a numpy {np.dtype(dt).name} array")
+    if not C.flags.writeable:
+        raise ValueError("C must be writeable")
+    m, k = A.shape
+    k2, n = B.shape
+    if k2 != k or C.shape != (m, n):
+        raise ValueError(f"shape mismatch: A {A.shape}, B {B.shape}, C {C.shape}")
+    rc = getattr(lib(), fn_name)(m, n, k, A.ctypes.data, _host_ld(A, "A"), B.ctypes.data, _host_ld(B, "B"),
+                                 C.ctypes.data, _host_ld(C, "C"))
+    _check(rc)
+    return C
+
+
+def gemm_i16_host(A, B, C):
+    """C += A @ B for numpy (host) arrays; the library stages the copies and waits for the result."""
+    import numpy as np
+    return _host_call("gemm_i16_host", A, B, C, np.int16, np.int64)
+
+
+def gemm_i8_host(A, B, C):
+    import numpy as np
+    return _host_call("gemm_i8_host", A, B, C, np.int8, np.int32)
+
+
+# ------------------------------------------------------------------ control
+def set_stream(stream) -> None:
+    """Stream used by the host-buffer entry points (a torch.cuda.Stream, a raw handle, or None)."""
+    handle = getattr(stream, "cuda_stream", stream) or 0
+    lib().gemmi_set_stream(ctypes.c_void_p(handle))
+
+
+def device_status() -> int:
+    """Synchronises the device; returns and clears its status word (OK or ETIMEOUT)."""
+    return int(lib().gemmi_device_status())
+
+
+def device_status_detail() -> int:
+    return int(lib().gemmi_device_status_detail())
+
+
+def set_option(option: int, value: int) -> None:
+    _check(lib().gemmi_set_option(option, value))
+
+
+def get_option(option: int) -> int:
+    return int(lib().gemmi_get_option(option))
+
+
+def release_workspace() -> None:
+    _check(lib().gemmi_release_workspace())
+
+
+def workspace_bytes() -> int:
+    return int(lib().gemmi_workspace_bytes())
+
+
+def selftest_wait_timeout(timeout_us: int = 1000) -> int:
+    return int(lib().gemmi_selftest_wait_timeout(timeout_us))
+
+
+def kernel_timing(enable: bool) -> None:
+    """Switch per-kernel CUDA-event timing on/off (resets the sums)."""
+    _check(lib().gemmi_kernel_timing(1 if enable else 0))
+
+
+def kernel_time(kernel: int):
+    """(total milliseconds, launches) of one kernel since timing was switched on."""
+    ms, n = ctypes.c_double(0.0), ctypes.c_int64(0)
+    _check(lib().gemmi_kernel_time(kernel, ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
+
+
+def version() -> str:
+    return lib().gemmi_version().decode()

@@ -1,0 +1,547 @@
+// api.cu -- the C ABI of include/gemmi.h: argument checks, workspace, dispatch.
+//
+// Dispatch (all paths bit-exact, see the kernels' headers):
+//   int16, m <= skinny limit (16) : skinny.cu   (B streamed once, tensor-core limb products)
+//   int16, otherwise              : split.cu (A and B -> fp16 limb planes) + gemm_tc.cu (tcgen05)
+//   int8                          : split.cu (A and B -> fp16 planes) + gemm_tc.cu (tcgen05)
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "gemmi.h"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace {
+
+using gemmi::LimbPlanes;
+
+thread_local std::string t_error;
+
+int set_error(int code, const std::string& msg) {
+  t_error = msg;
+  return code;
+}
+
+int cuda_error(cudaError_t e, const char* where) {
+  return set_error(GEMMI_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+constexpr int kMaxDevices = 64;
+constexpr size_t kAlign = 256;
+
+struct DeviceState {
+  bool ready = false;
+  bool arch_ok = false;
+  int sm_count = 0;
+  uint32_t* status = nullptr;   // device status word
+  void* ws = nullptr;           // limb planes / aligned copies
+  size_t ws_bytes = 0;
+  void* host_buf = nullptr;     // device staging for the *_host entry points
+  size_t host_buf_bytes = 0;
+  cudaEvent_t last_use = nullptr;
+  cudaStream_t last_stream = nullptr;
+  bool used = false;
+  uint32_t last_detail = 0;
+};
+
+std::mutex g_mutex;
+DeviceState g_dev[kMaxDevices];
+
+// Optional per-kernel timing with CUDA events recorded on the launching stream.
+struct KernelTimer {
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending;
+  std::vector<cudaEvent_t> pool;
+  double total_ms = 0.0;
+  int64_t launches = 0;
+};
+bool g_timing = false;
+KernelTimer g_timers[GEMMI_KERNEL_COUNT];
+
+cudaEvent_t timer_event(KernelTimer& t) {
+  if (!t.pool.empty()) {
+    cudaEvent_t e = t.pool.back();
+    t.pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Records the start event of a timed launch (returns null when timing is off).
+cudaEvent_t timer_begin(int kind, cudaStream_t s) {
+  if (!g_timing) return nullptr;
+  cudaEvent_t e = timer_event(g_timers[kind]);
+  cudaEventRecord(e, s);
+  return e;
+}
+
+void timer_end(int kind, cudaEvent_t start, cudaStream_t s) {
+  if (start == nullptr) return;
+  cudaEvent_t e = timer_event(g_timers[kind]);
+  cudaEventRecord(e, s);
+  g_timers[kind].pending.emplace_back(start, e);
+}
+
+void timer_collect(KernelTimer& t) {
+  for (auto& pr : t.pending) {
+    cudaEventSynchronize(pr.second);
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, pr.first, pr.second) == cudaSuccess) {
+      t.total_ms += ms;
+      t.launches += 1;
+    }
+    t.pool.push_back(pr.first);
+    t.pool.push_back(pr.second);
+  }
+  t.pending.clear();
+}
+cudaStream_t g_stream = nullptr;
+int64_t g_skinny_max_m = 16;
+int64_t g_timeout_us = 4000000;
+int64_t g_skinny_ksplit = 0;
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Current device's state, initialised on first use (caller holds g_mutex).
+int device_state(DeviceState** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return set_error(GEMMI_EINVAL, "device ordinal out of range");
+  DeviceState& d = g_dev[dev];
+  if (!d.ready) {
+    cudaDeviceProp prop;
+    e = cudaGetDeviceProperties(&prop, dev);
+    if (e != cudaSuccess) return cuda_error(e, "cudaGetDeviceProperties");
+    d.arch_ok = prop.major == 10 && prop.minor == 3;
+    d.sm_count = prop.multiProcessorCount;
+    if (d.arch_ok) {
+      e = cudaMalloc(&d.status, 256);
+      if (e != cudaSuccess) return set_error(GEMMI_ENOMEM, "cannot allocate the device status word");
+      e = cudaMemset(d.status, 0, 256);
+      if (e != cudaSuccess) return cuda_error(e, "cudaMemset(status)");
+      e = cudaEventCreateWithFlags(&d.last_use, cudaEventDisableTiming);
+      if (e != cudaSuccess) return cuda_error(e, "cudaEventCreate");
+    }
+    d.ready = true;
+  }
+  if (!d.arch_ok)
+    return set_error(GEMMI_EARCH, "the current device is not an sm_103 (GB300) GPU; this library has no other path");
+  *out = &d;
+  return GEMMI_OK;
+}
+
+// Grows a device buffer to at least `bytes` (synchronising the device before freeing the old one).
+int ensure_buffer(void** buf, size_t* have, size_t bytes) {
+  if (*have >= bytes) return GEMMI_OK;
+  if (*buf != nullptr) {
+    cudaDeviceSynchronize();
+    cudaFree(*buf);
+    *buf = nullptr;
+    *have = 0;
+  }
+  const size_t want = round_up(bytes, size_t(2) << 20);
+  if (cudaMalloc(buf, want) != cudaSuccess) {
+    cudaGetLastError();
+    *buf = nullptr;
+    return set_error(GEMMI_ENOMEM, "cannot allocate " + std::to_string(want) + " bytes of device workspace");
+  }
+  *have = want;
+  return GEMMI_OK;
+}
+
+// Orders this call's use of the workspace after the previous call's (which may be on another stream).
+int begin_workspace_use(DeviceState& d, cudaStream_t s) {
+  if (d.used && d.last_stream != s) {
+    cudaError_t e = cudaStreamWaitEvent(s, d.last_use, 0);
+    if (e != cudaSuccess) return cuda_error(e, "cudaStreamWaitEvent");
+  }
+  return GEMMI_OK;
+}
+
+int end_workspace_use(DeviceState& d, cudaStream_t s) {
+  cudaError_t e = cudaEventRecord(d.last_use, s);
+  if (e != cudaSuccess) return cuda_error(e, "cudaEventRecord");
+  d.last_stream = s;
+  d.used = true;
+  return GEMMI_OK;
+}
+
+bool overlaps(const void* a, size_t abytes, const void* b, size_t bbytes) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+  return a0 < b0 + bbytes && b0 < a0 + abytes;
+}
+
+// Checks shared by every entry point.  Returns -1 to proceed, or a status to return.
+int check_args(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B, int64_t ldb,
+               const void* C, int64_t ldc, size_t op_size, size_t c_size) {
+  if (m < 0 || n < 0 || k < 0) return set_error(GEMMI_EINVAL, "negative matrix dimension");
+  if (ldc < std::max<int64_t>(1, n)) return set_error(GEMMI_EINVAL, "ldc < max(1, n)");
+  if (lda < std::max<int64_t>(1, k)) return set_error(GEMMI_EINVAL, "lda < max(1, k)");
+  if (ldb < std::max<int64_t>(1, n)) return set_error(GEMMI_EINVAL, "ldb < max(1, n)");
+  if (m == 0 || n == 0) return GEMMI_OK;
+  if (C == nullptr) return set_error(GEMMI_EINVAL, "C is null");
+  if (k == 0) return GEMMI_OK;
+  if (A == nullptr || B == nullptr) return set_error(GEMMI_EINVAL, "A or B is null");
+  if (m > (int64_t(1) << 40) || n > (int64_t(1) << 31) || k > (int64_t(1) << 31))
+    return set_error(GEMMI_EINVAL, "matrix dimension too large");
+  const size_t a_bytes = static_cast<size_t>((m - 1) * lda + k) * op_size;
+  const size_t b_bytes = static_cast<size_t>((k - 1) * ldb + n) * op_size;
+  const size_t c_bytes = static_cast<size_t>((m - 1) * ldc + n) * c_size;
+  if (overlaps(C, c_bytes, A, a_bytes) || overlaps(C, c_bytes, B, b_bytes))
+    return set_error(GEMMI_EINVAL, "C overlaps A or B");
+  return -1;
+}
+
+uint64_t timeout_ns() { return static_cast<uint64_t>(g_timeout_us) * 1000u; }
+
+struct Layout {
+  size_t a0, a1, b0, b1, total;
+};
+
+Layout plane_layout(int64_t m, int64_t n, int64_t pitch, int nl) {
+  Layout L{};
+  const size_t a_plane = round_up(static_cast<size_t>(m) * pitch * 2, kAlign);
+  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
+  L.a0 = 0;
+  L.a1 = nl == 2 ? a_plane : 0;
+  L.b0 = a_plane * nl;
+  L.b1 = nl == 2 ? L.b0 + b_plane : L.b0;
+  L.total = a_plane * nl + b_plane * nl;
+  return L;
+}
+
+int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B,
+           int64_t ldb, void* C, int64_t ldc, cudaStream_t s) {
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const Layout L = plane_layout(m, n, pitch, nl);
+  int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
+  if (rc != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+  char* ws = static_cast<char*>(d.ws);
+  LimbPlanes pa{{ws + L.a0, ws + L.a1}, m, pitch};
+  LimbPlanes pb{{ws + L.b0, ws + L.b1}, n, pitch};
+  cudaError_t e;
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+  if (nl == 2) {
+    e = gemmi::split_rows_i16(static_cast<const int16_t*>(A), lda, m, k, pa, s);
+    if (e == cudaSuccess) e = gemmi::split_cols_i16(static_cast<const int16_t*>(B), ldb, k, n, pb, s);
+  } else {
+    e = gemmi::convert_rows_i8(static_cast<const int8_t*>(A), lda, m, k, pa, s);
+    if (e == cudaSuccess) e = gemmi::convert_cols_i8(static_cast<const int8_t*>(B), ldb, k, n, pb, s);
+  }
+  timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, "limb split launch");
+  gemmi::TcGemmArgs ta;
+  ta.m = m;
+  ta.n = n;
+  ta.k = k;
+  ta.a = pa;
+  ta.b = pb;
+  ta.C = C;
+  ta.ldc = ldc;
+  ta.status = d.status;
+  ta.timeout_ns = timeout_ns();
+  ta.num_sms = d.sm_count;
+  const char* why = "tcgen05 GEMM launch";
+  const int kind = nl == 2 ? GEMMI_KERNEL_TC_I16 : GEMMI_KERNEL_TC_I8;
+  cudaEvent_t t1 = timer_begin(kind, s);
+  e = nl == 2 ? gemmi::tc_gemm_i16(ta, s, &why) : gemmi::tc_gemm_i8(ta, s, &why);
+  timer_end(kind, t1, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return end_workspace_use(d, s);
+}
+
+int run_skinny(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
+               int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s) {
+  const bool tma_ok = reinterpret_cast<uintptr_t>(B) % 16 == 0 && (ldb * 2) % 16 == 0;
+  const int16_t* Bs = B;
+  int64_t ldbs = ldb;
+  bool used_ws = false;
+  int rc;
+  if (!tma_ok) {
+    // re-pitch B into the workspace so that every row starts on a 16-byte boundary
+    ldbs = static_cast<int64_t>(round_up(static_cast<size_t>(n), 8));
+    if ((rc = ensure_buffer(&d.ws, &d.ws_bytes, static_cast<size_t>(k) * ldbs * 2)) != GEMMI_OK) return rc;
+    if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+    cudaError_t e = cudaMemcpy2DAsync(d.ws, ldbs * 2, B, ldb * 2, n * 2, k, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy2DAsync(B)");
+    Bs = static_cast<const int16_t*>(d.ws);
+    used_ws = true;
+  }
+  gemmi::SkinnyArgs sa;
+  sa.m = m;
+  sa.n = n;
+  sa.k = k;
+  sa.A = A;
+  sa.lda = lda;
+  sa.B = Bs;
+  sa.ldb = ldbs;
+  sa.C = C;
+  sa.ldc = ldc;
+  sa.status = d.status;
+  sa.timeout_ns = timeout_ns();
+  sa.num_sms = d.sm_count;
+  sa.ksplit = static_cast<int>(g_skinny_ksplit);
+  const char* why = "skinny GEMM launch";
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SKINNY, s);
+  cudaError_t e = gemmi::skinny_gemm_i16(sa, s, &why);
+  timer_end(GEMMI_KERNEL_SKINNY, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return used_ws ? end_workspace_use(d, s) : GEMMI_OK;
+}
+
+int gemm_i16_locked(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,
+                    int64_t* C, int64_t ldc, cudaStream_t s) {
+  const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, 2, 8);
+  if (pre >= 0) return pre;
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  if (m <= g_skinny_max_m) return run_skinny(*d, m, n, k, A, lda, B, ldb, C, ldc, s);
+  return run_tc(*d, 2, m, n, k, A, lda, B, ldb, C, ldc, s);
+}
+
+int gemm_i8_locked(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
+                   int32_t* C, int64_t ldc, cudaStream_t s) {
+  const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, 1, 4);
+  if (pre >= 0) return pre;
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  return run_tc(*d, 1, m, n, k, A, lda, B, ldb, C, ldc, s);
+}
+
+int read_status_locked(DeviceState& d, bool clear) {
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, d.status, sizeof(word), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
+  d.last_detail = word;
+  if (clear && word != 0) {
+    e = cudaMemset(d.status, 0, sizeof(word));
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemset(status)");
+  }
+  if (word == 0) return GEMMI_OK;
+  const int code = static_cast<int>(word & 0xFFu);
+  char buf[160];
+  std::snprintf(buf, sizeof(buf), "device status 0x%08x: a pipeline wait (site %u, block %u) ran out of time",
+                word, (word >> 8) & 0xFFu, word >> 16);
+  return set_error(code, buf);
+}
+
+template <typename OP, typename CT, typename F>
+int host_gemm(int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda, const OP* B, int64_t ldb, CT* C,
+              int64_t ldc, F device_call) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, sizeof(OP), sizeof(CT));
+  if (pre >= 0) return pre;
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const size_t a_bytes = round_up(static_cast<size_t>(m) * k * sizeof(OP), kAlign);
+  const size_t b_bytes = round_up(static_cast<size_t>(k) * n * sizeof(OP), kAlign);
+  const size_t c_bytes = round_up(static_cast<size_t>(m) * n * sizeof(CT), kAlign);
+  if ((rc = ensure_buffer(&d->host_buf, &d->host_buf_bytes, a_bytes + b_bytes + c_bytes)) != GEMMI_OK) return rc;
+  char* base = static_cast<char*>(d->host_buf);
+  OP* dA = reinterpret_cast<OP*>(base);
+  OP* dB = reinterpret_cast<OP*>(base + a_bytes);
+  CT* dC = reinterpret_cast<CT*>(base + a_bytes + b_bytes);
+  cudaStream_t s = g_stream;
+  cudaError_t e = cudaMemcpy2DAsync(dA, k * sizeof(OP), A, lda * sizeof(OP), k * sizeof(OP), m, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2DAsync(dB, n * sizeof(OP), B, ldb * sizeof(OP), n * sizeof(OP), k, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2DAsync(dC, n * sizeof(CT), C, ldc * sizeof(CT), n * sizeof(CT), m, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_error(e, "host-to-device copy");
+  rc = device_call(m, n, k, dA, k, dB, n, dC, n, s);
+  if (rc != GEMMI_OK) return rc;
+  e = cudaMemcpy2DAsync(C, ldc * sizeof(CT), dC, n * sizeof(CT), n * sizeof(CT), m, cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_error(e, "device-to-host copy");
+  e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize");
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, d->status, sizeof(word), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
+  if (word != 0) return read_status_locked(*d, true);
+  return GEMMI_OK;
+}
+
+__global__ void wait_probe_kernel(uint32_t* status, uint64_t timeout_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    gemmi::mbar_init(gemmi::smem_u32(&bar), 1);
+    gemmi::fence_mbar_init();
+  }
+  __syncthreads();
+  // nothing ever arrives on `bar`: the bounded wait must give up and report
+  if (threadIdx.x == 0 && !gemmi::bounded_wait(gemmi::smem_u32(&bar), 0, timeout_ns))
+    gemmi::report_status(status, GEMMI_ETIMEOUT, 99);
+}
+
+}  // namespace
+
+namespace gemmi {
+cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(status, timeout_ns);
+  return cudaGetLastError();
+}
+}  // namespace gemmi
+
+extern "C" {
+
+int gemm_i16_ex(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,
+                int64_t* C, int64_t ldc, void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i16_locked(m, n, k, A, lda, B, ldb, C, ldc, static_cast<cudaStream_t>(stream));
+}
+
+int gemm_i16(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,
+             int64_t* C, int64_t ldc) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i16_locked(m, n, k, A, lda, B, ldb, C, ldc, g_stream);
+}
+
+int gemm_i8_ex(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
+               int32_t* C, int64_t ldc, void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i8_locked(m, n, k, A, lda, B, ldb, C, ldc, static_cast<cudaStream_t>(stream));
+}
+
+int gemm_i8(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
+            int32_t* C, int64_t ldc) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i8_locked(m, n, k, A, lda, B, ldb, C, ldc, g_stream);
+}
+
+int gemm_i16_host(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,
+                  int64_t* C, int64_t ldc) {
+  return host_gemm(m, n, k, A, lda, B, ldb, C, ldc, gemm_i16_locked);
+}
+
+int gemm_i8_host(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
+                 int32_t* C, int64_t ldc) {
+  return host_gemm(m, n, k, A, lda, B, ldb, C, ldc, gemm_i8_locked);
+}
+
+void gemmi_set_stream(void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  g_stream = static_cast<cudaStream_t>(stream);
+}
+
+const char* gemmi_last_error(void) { return t_error.c_str(); }
+
+int gemmi_device_status(void) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  return read_status_locked(*d, true);
+}
+
+uint32_t gemmi_device_status_detail(void) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+  return g_dev[dev].last_detail;
+}
+
+int gemmi_release_workspace(void) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return set_error(GEMMI_EINVAL, "device ordinal out of range");
+  DeviceState& d = g_dev[dev];
+  if (d.ws == nullptr && d.host_buf == nullptr) return GEMMI_OK;
+  e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
+  if (d.ws) cudaFree(d.ws);
+  if (d.host_buf) cudaFree(d.host_buf);
+  d.ws = d.host_buf = nullptr;
+  d.ws_bytes = d.host_buf_bytes = 0;
+  d.used = false;
+  return GEMMI_OK;
+}
+
+size_t gemmi_workspace_bytes(void) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+  return g_dev[dev].ws_bytes + g_dev[dev].host_buf_bytes;
+}
+
+int gemmi_set_option(int option, int64_t value) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  switch (option) {
+    case GEMMI_OPT_SKINNY_MAX_M:
+      if (value < 0 || value > 16) return set_error(GEMMI_EINVAL, "skinny limit must be in [0, 16]");
+      g_skinny_max_m = value;
+      return GEMMI_OK;
+    case GEMMI_OPT_WAIT_TIMEOUT_US:
+      if (value < 1 || value > 60000000) return set_error(GEMMI_EINVAL, "timeout must be in [1 us, 60 s]");
+      g_timeout_us = value;
+      return GEMMI_OK;
+    case GEMMI_OPT_SKINNY_KSPLIT:
+      if (value < 0 || value > 4096) return set_error(GEMMI_EINVAL, "ksplit must be in [0, 4096]");
+      g_skinny_ksplit = value;
+      return GEMMI_OK;
+    default:
+      return set_error(GEMMI_EINVAL, "unknown option");
+  }
+}
+
+int64_t gemmi_get_option(int option) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  switch (option) {
+    case GEMMI_OPT_SKINNY_MAX_M: return g_skinny_max_m;
+    case GEMMI_OPT_WAIT_TIMEOUT_US: return g_timeout_us;
+    case GEMMI_OPT_SKINNY_KSPLIT: return g_skinny_ksplit;
+    default: return -1;
+  }
+}
+
+int gemmi_selftest_wait_timeout(int64_t timeout_us) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (timeout_us < 1 || timeout_us > 10000000) return set_error(GEMMI_EINVAL, "timeout must be in [1 us, 10 s]");
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  cudaError_t e = gemmi::launch_wait_timeout_probe(d->status, static_cast<uint64_t>(timeout_us) * 1000u, g_stream);
+  if (e != cudaSuccess) return cuda_error(e, "wait probe launch");
+  return read_status_locked(*d, true);
+}
+
+int gemmi_kernel_timing(int enable) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  g_timing = enable != 0;
+  for (auto& t : g_timers) {
+    timer_collect(t);
+    t.total_ms = 0.0;
+    t.launches = 0;
+  }
+  return GEMMI_OK;
+}
+
+int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (kernel < 0 || kernel >= GEMMI_KERNEL_COUNT || total_ms == nullptr || launches == nullptr)
+    return set_error(GEMMI_EINVAL, "bad kernel id or null output");
+  timer_collect(g_timers[kernel]);
+  *total_ms = g_timers[kernel].total_ms;
+  *launches = g_timers[kernel].launches;
+  return GEMMI_OK;
+}
+
+const char* gemmi_version(void) { return "gemmi 0.1 (sm_103a)"; }
+
+}  // extern "C"

@@ -1,0 +1,492 @@
+// gemm_tc.cu -- exact integer GEMM on the 5th-generation tensor cores (tcgen05, sm_103a).
+//
+// What it computes: C += A*B (Section 4.1 of the paper) for int16 operands and
+// an int64 C, or int8 operands and an int32 C, bit-exactly.
+//
+// How.  The operands arrive as fp16 limb planes (split.cu): a = 256*h + l with
+// |h|, |l| <= 128, so for one reduction index
+//     a*b = 2^16 * (h_a h_b) + 2^8 * (h_a l_b + l_a h_b) + (l_a l_b),
+// and the GEMM is four limb GEMMs summed into three accumulators
+//     HH = Ah*Bh,   X = Ah*Bl + Al*Bh,   LL = Al*Bl.
+// Each limb product is an integer of magnitude <= 2^14 that fp16 x fp16 forms
+// exactly, and an fp32 accumulator sums integers exactly while every partial
+// sum stays below 2^24.  So each accumulator is only allowed a bounded run of
+// the reduction dimension (a "chunk": 512 indices for HH and LL, 256 for X,
+// keeping every partial sum within 2^23), after which it is drained:
+// converted to an integer and added, shifted by its weight (16, 8, 0 bits),
+// into a 64-bit running sum held in registers.  This plays the role of the
+// AIE's 48-bit accumulators (Section 6.2): wide accumulation so nothing
+// overflows, here built from exact fp32 chunks and int64 registers.  The int8
+// path is the same with one plane, one product and one accumulator (int32 sum).
+//
+// Structure (one persistent CTA per SM, 320 threads, 128x128 output tiles):
+//   warp 8      TMA producer: 2-D tiled bulk-tensor loads of 64-wide K blocks of
+//               the limb planes (128-byte swizzle) into a ring of smem stages;
+//   warp 9      MMA issuer: tcgen05.mma kind::f16 (M=128, N=128, K=16) from smem
+//               descriptors into fp32 accumulators in tensor memory (TMEM);
+//   warps 0-7   epilogue: drain accumulators (tcgen05.ld) into int64 registers,
+//               and read-modify-write C once per tile.
+// TMEM holds four 128-column accumulator slots: three live accumulators plus
+// one spare.  Chunk ends of the three accumulators are staggered, so at every
+// chunk end the MMA warp moves that accumulator into the spare slot and keeps
+// issuing while the epilogue drains the old one.  This takes the place of the
+// paper's loop L6 / micro-kernel (Figure 1, Section 5.2); the smem stage ring
+// takes the place of the B_r copies into local memory (Section 5.1).
+//
+// Every mbarrier wait is bounded (ptx.cuh); a wait that runs out records
+// GEMMI_ETIMEOUT in the device status word and the CTA winds down cleanly.
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace gemmi {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BN = 128;
+constexpr int BK = 64;                       // 64 fp16 = 128 bytes = one swizzle row
+constexpr int UMMA_K = 16;                   // K of one tcgen05.mma kind::f16
+constexpr int TILE_BYTES = BM * BK * 2;      // 16 KB per limb tile (BM == BN)
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int PRODUCER_WARP = 8;
+constexpr int MMA_WARP = 9;
+constexpr int NUM_THREADS = 320;
+constexpr int NSLOT = 4;
+constexpr int SLOT_COLS = 128;
+constexpr int TMEM_COLS = NSLOT * SLOT_COLS;  // 512
+constexpr int GROUP_M = 16;                   // tile raster: bands of 16 row tiles
+constexpr uint32_t STATUS_TIMEOUT = 4;
+
+template <int NL>
+struct Scheme;
+
+// int16: two limbs per operand, four products, three accumulators.
+template <>
+struct Scheme<2> {
+  static constexpr int STAGES = 3;
+  static constexpr int NACC = 3;
+  static constexpr int NPROD = 4;
+  // product p: (A limb, B limb, accumulator); limb 0 = high, 1 = low
+  __device__ static constexpr int a_limb(int p) { return p == 0 ? 0 : p == 1 ? 0 : p == 2 ? 1 : 1; }
+  __device__ static constexpr int b_limb(int p) { return p == 0 ? 0 : p == 1 ? 1 : p == 2 ? 0 : 1; }
+  __device__ static constexpr int acc(int p) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
+  // chunk schedule in K blocks of 64: accumulator a ends a chunk after block kb when
+  // (kb + 1 + PHASE[a]) % PERIOD[a] == 0, or at the last block of the tile.
+  // HH, LL: 8 blocks = 512 indices, |sum| <= 512 * 2^14 = 2^23;  X: 4 blocks = 256, |sum| <= 256 * 2^15 = 2^23.
+  __device__ static constexpr int period(int a) { return a == 1 ? 4 : 8; }
+  __device__ static constexpr int phase(int a) { return a == 0 ? 6 : a == 1 ? 0 : 2; }
+  __device__ static constexpr int shift(int a) { return a == 0 ? 16 : a == 1 ? 8 : 0; }
+};
+
+// int8: the value itself in one fp16 plane, one product, one accumulator.
+// 8 blocks = 512 indices, |sum| <= 512 * 2^14 = 2^23.
+template <>
+struct Scheme<1> {
+  static constexpr int STAGES = 6;
+  static constexpr int NACC = 1;
+  static constexpr int NPROD = 1;
+  __device__ static constexpr int a_limb(int) { return 0; }
+  __device__ static constexpr int b_limb(int) { return 0; }
+  __device__ static constexpr int acc(int) { return 0; }
+  __device__ static constexpr int period(int) { return 8; }
+  __device__ static constexpr int phase(int) { return 0; }
+  __device__ static constexpr int shift(int) { return 0; }
+};
+
+template <int NL>
+constexpr int stage_bytes() { return 2 * NL * TILE_BYTES; }
+
+template <int NL>
+constexpr size_t smem_bytes() {
+  // stages + barriers (full/empty per stage, full/empty per slot, one final) + TMEM holder + abort flag
+  return 1024 + static_cast<size_t>(Scheme<NL>::STAGES) * stage_bytes<NL>() + 8 * (2 * Scheme<NL>::STAGES + 2 * NSLOT + 1) + 16;
+}
+
+struct TcParams {
+  int64_t m, n, k;
+  void* C;
+  int64_t ldc;
+  int num_m_tiles, num_n_tiles, num_k_blocks;
+  int c_vec;
+  uint64_t timeout_ns;
+  uint32_t* status;
+};
+
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& mt, int& nt) {
+  const int per_group = GROUP_M * num_n;
+  const int group = t / per_group;
+  const int first_m = group * GROUP_M;
+  const int rows_here = min(GROUP_M, num_m - first_m);
+  const int in_group = t - group * per_group;
+  mt = first_m + in_group % rows_here;
+  nt = in_group / rows_here;
+}
+
+template <int NL>
+__device__ __forceinline__ bool chunk_ends(int a, int kb, int nkb) {
+  using S = Scheme<NL>;
+  return kb == nkb - 1 || ((kb + 1 + S::phase(a)) % S::period(a)) == 0;
+}
+
+__device__ __forceinline__ int32_t f32_to_i32(uint32_t bits) {
+  int32_t v;
+  asm("cvt.rni.s32.f32 %0, %1;" : "=r"(v) : "f"(__uint_as_float(bits)));
+  return v;
+}
+
+template <int NL>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
+               const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1, TcParams P) {
+  using S = Scheme<NL>;
+  constexpr int STAGES = S::STAGES;
+  constexpr int SB = stage_bytes<NL>();
+  // C element type and the unsigned type of the running sum (wrap-around is modular, never UB)
+  using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
+  using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * SB);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t sfull0 = empty0 + 8 * STAGES;
+  const uint32_t sempty0 = sfull0 + 8 * NSLOT;
+  const uint32_t final_bar = sempty0 + 8 * NSLOT;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2 * NSLOT + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int s = 0; s < NSLOT; ++s) {
+      mbar_init(sfull0 + 8 * s, 1);
+      mbar_init(sempty0 + 8 * s, NUM_EPI_WARPS);
+    }
+    mbar_init(final_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == MMA_WARP) {
+    tmem_alloc(smem_u32(tmem_holder), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
+  const int nkb = P.num_k_blocks;
+
+  if (warp == PRODUCER_WARP) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&mapA0);
+      tma_prefetch_desc(&mapB0);
+      if (NL == 2) {
+        tma_prefetch_desc(&mapA1);
+        tma_prefetch_desc(&mapB1);
+      }
+      int stage = 0;
+      uint32_t phase = 0;
+      int64_t issued = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
+        int mt, nt;
+        tile_coords(t, P.num_m_tiles, P.num_n_tiles, mt, nt);
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!bounded_wait(empty0 + 8 * stage, phase ^ 1u, P.timeout_ns)) {
+            report_status(P.status, STATUS_TIMEOUT, 1);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          if (*abort_flag) { ok = false; break; }
+          const uint32_t fb = full0 + 8 * stage;
+          mbar_arrive_expect_tx(fb, SB);
+          const uint32_t base = smem_u32(smem + stage * SB);
+          tma_load_2d(base, &mapA0, fb, kb * BK, mt * BM);
+          if (NL == 2) tma_load_2d(base + TILE_BYTES, &mapA1, fb, kb * BK, mt * BM);
+          tma_load_2d(base + NL * TILE_BYTES, &mapB0, fb, kb * BK, nt * BN);
+          if (NL == 2) tma_load_2d(base + (NL + 1) * TILE_BYTES, &mapB1, fb, kb * BK, nt * BN);
+          ++issued;
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // Make sure no bulk copy is still landing in shared memory when the CTA exits.
+      const int64_t first = issued > STAGES ? issued - STAGES : 0;
+      for (int64_t i = first; i < issued; ++i) {
+        const int s = static_cast<int>(i % STAGES);
+        const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
+        bounded_wait(full0 + 8 * s, par, P.timeout_ns);
+      }
+    }
+  } else if (warp == MMA_WARP) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int slot_of[3] = {0, 1, 2};
+      int spare = S::NACC;  // first slot not owned by a live accumulator
+      uint32_t use_parity = 0;  // bit s: parity of the number of times slot s has been acquired
+      bool need_acquire[3] = {true, true, true};
+      bool fresh[3] = {true, true, true};
+      bool ok = true;
+      for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
+        for (int kb = 0; kb < nkb && ok; ++kb) {
+          if (!bounded_wait(full0 + 8 * stage, phase, P.timeout_ns)) {
+            report_status(P.status, STATUS_TIMEOUT, 2);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = smem_u32(smem + stage * SB);
+#pragma unroll
+          for (int p = 0; p < S::NPROD; ++p) {
+            const int a = S::acc(p);
+            if (need_acquire[a]) {
+              const int s = slot_of[a];
+              if (!bounded_wait(sempty0 + 8 * s, ((use_parity >> s) & 1u) ^ 1u, P.timeout_ns)) {
+                report_status(P.status, STATUS_TIMEOUT, 3);
+                *abort_flag = 1;
+                ok = false;
+                break;
+              }
+              use_parity ^= 1u << s;
+              need_acquire[a] = false;
+              tc_fence_after();
+            }
+            const uint32_t d = tmem_base + static_cast<uint32_t>(slot_of[a] * SLOT_COLS);
+            const uint64_t adesc = smem_desc_kmajor_sw128(base + S::a_limb(p) * TILE_BYTES);
+            const uint64_t bdesc = smem_desc_kmajor_sw128(base + (NL + S::b_limb(p)) * TILE_BYTES);
+#pragma unroll
+            for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+              // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
+              const uint32_t acc_flag = (fresh[a] && kk == 0) ? 0u : 1u;
+              tc_mma_f16(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, acc_flag);
+            }
+            fresh[a] = false;
+          }
+          if (!ok) break;
+          tc_commit(empty0 + 8 * stage);  // stage is free once these MMAs have read it
+#pragma unroll
+          for (int a = 0; a < S::NACC; ++a) {
+            if (chunk_ends<NL>(a, kb, nkb)) {
+              tc_commit(sfull0 + 8 * slot_of[a]);  // this accumulator's chunk is ready to drain
+              const int next = spare;
+              spare = slot_of[a];
+              slot_of[a] = next;
+              need_acquire[a] = true;
+              fresh[a] = true;
+            }
+          }
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // all MMAs issued by this thread must be complete before TMEM is released
+      tc_commit(final_bar);
+      bounded_wait(final_bar, 0, P.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 0..7)
+    const int quad = warp & 3;       // TMEM lanes 32*quad .. 32*quad+31 (hardware lane quadrant)
+    const int half = warp >> 2;      // column half of the tile: 0..63 or 64..127
+    int slot_of[3] = {0, 1, 2};
+    int spare = S::NACC;
+    uint32_t drain_parity = 0;  // bit s: parity of the number of drains of slot s
+    bool ok = true;
+    UT acc[64];
+    for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
+      int mt, nt;
+      tile_coords(t, P.num_m_tiles, P.num_n_tiles, mt, nt);
+      const int64_t row = static_cast<int64_t>(mt) * BM + quad * 32 + lane;
+      const int64_t col0 = static_cast<int64_t>(nt) * BN + half * 64;
+      CT* crow = static_cast<CT*>(P.C) + row * P.ldc + col0;
+      const bool row_ok = row < P.m;
+      const bool full_cols = col0 + 64 <= P.n;
+      // running sum starts from C itself, so the tile ends with a plain store
+      if (row_ok && full_cols && P.c_vec) {
+        if constexpr (NL == 2) {
+#pragma unroll
+          for (int c = 0; c < 64; c += 2) {
+            const longlong2 v = *reinterpret_cast<const longlong2*>(crow + c);
+            acc[c] = static_cast<UT>(v.x);
+            acc[c + 1] = static_cast<UT>(v.y);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < 64; c += 4) {
+            const int4 v = *reinterpret_cast<const int4*>(crow + c);
+            acc[c] = static_cast<UT>(v.x);
+            acc[c + 1] = static_cast<UT>(v.y);
+            acc[c + 2] = static_cast<UT>(v.z);
+            acc[c + 3] = static_cast<UT>(v.w);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 64; ++c) acc[c] = (row_ok && col0 + c < P.n) ? static_cast<UT>(crow[c]) : UT(0);
+      }
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+#pragma unroll
+        for (int a = 0; a < S::NACC; ++a) {
+          if (!chunk_ends<NL>(a, kb, nkb)) continue;
+          const int s = slot_of[a];
+          // every lane waits; the warp then decides together (tcgen05.ld needs a converged warp)
+          const bool got = bounded_wait(sfull0 + 8 * s, (drain_parity >> s) & 1u, P.timeout_ns);
+          if (!__all_sync(0xFFFFFFFFu, got)) {
+            if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 4);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          drain_parity ^= 1u << s;
+          tc_fence_after();
+          const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                                 static_cast<uint32_t>(s * SLOT_COLS + half * 64);
+#pragma unroll
+          for (int c = 0; c < 64; c += 32) {
+            uint32_t r0[16], r1[16];
+            tc_ld_32x32b_x16(taddr + c, r0);
+            tc_ld_32x32b_x16(taddr + c + 16, r1);
+            tc_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              // sign-extend to the unsigned running-sum type, then weight by 2^shift (modular)
+              acc[c + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r0[i]))) << S::shift(a);
+              acc[c + 16 + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r1[i]))) << S::shift(a);
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sempty0 + 8 * s);
+          const int next = spare;
+          spare = slot_of[a];
+          slot_of[a] = next;
+        }
+      }
+      if (!ok) break;
+      if (row_ok && full_cols && P.c_vec) {
+        if constexpr (NL == 2) {
+#pragma unroll
+          for (int c = 0; c < 64; c += 2)
+            *reinterpret_cast<longlong2*>(crow + c) =
+                make_longlong2(static_cast<long long>(acc[c]), static_cast<long long>(acc[c + 1]));
+        } else {
+#pragma unroll
+          for (int c = 0; c < 64; c += 4)
+            *reinterpret_cast<int4*>(crow + c) =
+                make_int4(static_cast<int>(acc[c]), static_cast<int>(acc[c + 1]), static_cast<int>(acc[c + 2]),
+                          static_cast<int>(acc[c + 3]));
+        }
+      } else if (row_ok) {
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (col0 + c < P.n) crow[c] = static_cast<CT>(acc[c]);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == MMA_WARP) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+template <int NL>
+cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
+  CUtensorMap maps[4];
+  const LimbPlanes* ops[2] = {&a.a, &a.b};
+  for (int o = 0; o < 2; ++o) {
+    for (int l = 0; l < 2; ++l) {
+      const void* base = ops[o]->plane[l < NL ? l : 0];
+      if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
+                                static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
+                                o == 0 ? BM : BN, 128, why))
+        return cudaErrorInvalidValue;
+    }
+  }
+  TcParams P;
+  P.m = a.m;
+  P.n = a.n;
+  P.k = a.k;
+  P.C = a.C;
+  P.ldc = a.ldc;
+  P.num_m_tiles = static_cast<int>((a.m + BM - 1) / BM);
+  P.num_n_tiles = static_cast<int>((a.n + BN - 1) / BN);
+  P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
+  const size_t esz = NL == 2 ? 8 : 4;
+  P.c_vec = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && ((a.ldc * esz) % 16 == 0);
+  P.timeout_ns = a.timeout_ns;
+  P.status = a.status;
+  const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
+  const int grid = static_cast<int>(tiles < a.num_sms ? tiles : a.num_sms);
+  constexpr size_t smem = smem_bytes<NL>();
+  cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  tc_gemm_kernel<NL><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], P);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes,
+                          const char** why) {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (g_encode == nullptr) {
+    *why = "cuTensorMapEncodeTiled is not available from the driver";
+    return false;
+  }
+  const CUtensorMapDataType dt =
+      dtype_fp16_or_i16 == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUtensorMapSwizzle sw = swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                : swizzle_bytes == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                                      : CU_TENSOR_MAP_SWIZZLE_NONE;
+  const CUresult r = g_encode(static_cast<CUtensorMap*>(map), dt, 2, const_cast<void*>(base), dims, strides, box,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *why = "cuTensorMapEncodeTiled rejected the operand layout";
+    return false;
+  }
+  return true;
+}
+
+cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why) { return launch<2>(args, s, why); }
+cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) { return launch<1>(args, s, why); }
+
+}  // namespace gemmi

@@ -1,0 +1,64 @@
+// internal.h -- host-side interfaces between the C ABI (api.cu) and the kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace gemmi {
+
+// Limb planes of one operand: NL fp16 planes of `rows` x `pitch` elements (K-major:
+// element (r, p) of plane l at planes[l][r * pitch + p]).  pitch is a multiple of 8.
+struct LimbPlanes {
+  void* plane[2];
+  int64_t rows;
+  int64_t pitch;
+};
+
+// ---- split.cu: operands -> fp16 limb planes (K-major).
+// int16: two centred 8-bit limbs, a = 256*h + l, h in [-128,128], l in [-128,127].
+// int8: one plane holding the value itself.
+cudaError_t split_rows_i16(const int16_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s);
+cudaError_t split_cols_i16(const int16_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s);
+cudaError_t convert_rows_i8(const int8_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s);
+cudaError_t convert_cols_i8(const int8_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s);
+
+// ---- gemm_tc.cu: tcgen05 GEMM on limb planes, C (int64 for NL=2, int32 for NL=1) += combine(limb products).
+struct TcGemmArgs {
+  int64_t m, n, k;
+  LimbPlanes a;  // rows = m
+  LimbPlanes b;  // rows = n (B transposed to K-major)
+  void* C;
+  int64_t ldc;
+  uint32_t* status;
+  uint64_t timeout_ns;
+  int num_sms;
+};
+cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
+cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
+
+// ---- skinny.cu: m <= 16 int16 GEMM streaming B once.
+struct SkinnyArgs {
+  int64_t m, n, k;
+  const int16_t* A;
+  int64_t lda;
+  const int16_t* B;  // k x n, row-major, 16-byte aligned base, ldb % 8 == 0
+  int64_t ldb;
+  int64_t* C;
+  int64_t ldc;
+  uint32_t* status;
+  uint64_t timeout_ns;
+  int num_sms;
+  int ksplit;  // 0 = automatic
+};
+cudaError_t skinny_gemm_i16(const SkinnyArgs& args, cudaStream_t s, const char** why);
+
+// ---- selftest of the bounded wait.
+cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
+
+// Tensor-map encoder from the driver (resolved once through the runtime).
+bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes,
+                          const char** why);
+
+}  // namespace gemmi

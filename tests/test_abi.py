@@ -1,0 +1,99 @@
+"""The C-ABI library builds, loads and exports what include/gemmi.h declares (no GPU needed).
+
+Only host-side logic runs here: argument validation happens before any device
+access, so invalid calls return GEMMI_EINVAL and empty problems return OK
+without touching a GPU.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2302_07594_gb300 as gm
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "gemmi.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    gm.build()
+    return gm.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*([a-z_0-9]+)\s*\(", text, flags=re.M)
+    return sorted(set(n for n in names if n not in ("if", "while")))
+
+
+def test_header_declares_the_core_calls():
+    names = declared_functions()
+    for core in ("gemm_i16", "gemm_i8", "gemm_i16_ex", "gemm_i8_ex", "gemmi_last_error"):
+        assert core in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    missing = [n for n in declared_functions() if not hasattr(L, n)]
+    assert missing == []
+    assert sorted(declared_functions()) == sorted(gm.EXPORTED)
+
+
+def test_no_oracle_or_cpu_fallback_symbols(L):
+    # the product library must not contain the oracle
+    blob = open(gm.LIB_PATH, "rb").read()
+    assert b"gemm_oracle" not in blob
+
+
+def test_version(L):
+    assert "sm_103a" in gm.version()
+
+
+@pytest.mark.parametrize("args", [
+    (-1, 4, 4, 4, 4, 4),    # negative m
+    (4, 4, 4, 3, 4, 4),     # lda < k
+    (4, 4, 4, 4, 3, 4),     # ldb < n
+    (4, 4, 4, 4, 4, 3),     # ldc < n
+])
+def test_invalid_arguments(L, args):
+    m, n, k, lda, ldb, ldc = args
+    dummy = ctypes.c_void_p(0x1000)
+    rc = L.gemm_i16(m, n, k, dummy, lda, ctypes.c_void_p(0x2000), ldb, ctypes.c_void_p(0x3000), ldc)
+    assert rc == gm.EINVAL
+    assert gm.last_error() != ""
+
+
+def test_null_and_overlap_rejected(L):
+    assert L.gemm_i16(4, 4, 4, None, 4, ctypes.c_void_p(0x2000), 4, ctypes.c_void_p(0x3000), 4) == gm.EINVAL
+    assert L.gemm_i16(4, 4, 4, ctypes.c_void_p(0x1000), 4, ctypes.c_void_p(0x2000), 4, None, 4) == gm.EINVAL
+    # C overlapping A
+    assert L.gemm_i16(4, 4, 4, ctypes.c_void_p(0x1000), 4, ctypes.c_void_p(0x90000), 4,
+                      ctypes.c_void_p(0x1008), 4) == gm.EINVAL
+    assert "overlap" in gm.last_error()
+
+
+def test_empty_problems_are_noops(L):
+    assert L.gemm_i16(0, 4, 4, None, 4, None, 4, None, 4) == gm.OK
+    assert L.gemm_i8(4, 0, 4, None, 4, None, 1, None, 1) == gm.OK
+    # k == 0: C untouched, A and B may be null
+    assert L.gemm_i16(3, 3, 0, None, 1, None, 3, ctypes.c_void_p(0x3000), 3) == gm.OK
+
+
+def test_options(L):
+    old = gm.get_option(gm.OPT_SKINNY_MAX_M)
+    gm.set_option(gm.OPT_SKINNY_MAX_M, 4)
+    assert gm.get_option(gm.OPT_SKINNY_MAX_M) == 4
+    gm.set_option(gm.OPT_SKINNY_MAX_M, old)
+    with pytest.raises(gm.GemmiError):
+        gm.set_option(gm.OPT_SKINNY_MAX_M, 17)
+    with pytest.raises(gm.GemmiError):
+        gm.set_option(99, 1)
+
+
+def test_missing_library_fails_loudly(tmp_path, monkeypatch):
+    monkeypatch.setattr(gm, "LIB_PATH", str(tmp_path / "absent.so"))
+    monkeypatch.setattr(gm, "_lib", None)
+    with pytest.raises(RuntimeError, match="not found"):
+        gm.lib()

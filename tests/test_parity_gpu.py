@@ -1,0 +1,311 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle, bit for bit.
+
+Expected values always come from the oracle (oracle/) run on the same seeded
+inputs (gemm_inputs.py); nothing here is produced by the CUDA path itself.
+The full-size workloads are checked on sampled rows (which the oracle
+computes one row block at a time) plus a row-sum/column-sum identity that
+covers every output:  sum_j C[i,j] = A[i,:] . (B 1),  sum_i C[i,j] = (1^T A) . B[:,j].
+"""
+import numpy as np
+import pytest
+
+import gemm_inputs as gi
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def gm():
+    import paper_2302_07594_gb300 as gm
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    gm.lib()  # raises if the library was not built
+    gm.set_option(gm.OPT_SKINNY_MAX_M, 16)
+    gm.set_option(gm.OPT_SKINNY_KSPLIT, 0)
+    yield gm
+    gm.set_option(gm.OPT_SKINNY_MAX_M, 16)
+    gm.set_option(gm.OPT_SKINNY_KSPLIT, 0)
+
+
+def expected(A, B, C, threads=8):
+    X = C.copy()
+    oracle.gemm(A, B, X, nthreads=threads)
+    return X
+
+
+def run_gpu(gm, A, B, C, kind=None):
+    kind = kind or ("i16" if A.dtype == np.int16 else "i8")
+    dA, dB, dC = (torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (A, B, C))
+    (gm.gemm_i16 if kind == "i16" else gm.gemm_i8)(dA, dB, dC)
+    torch.cuda.synchronize()
+    assert gm.device_status() == gm.OK
+    return dC.cpu().numpy()
+
+
+def assert_same(got, exp, what=""):
+    if not np.array_equal(got, exp):
+        bad = np.argwhere(got != exp)
+        i, j = bad[0]
+        raise AssertionError(f"{what}: {len(bad)} mismatches, first at ({i},{j}): got {got[i, j]} want {exp[i, j]}")
+
+
+# ------------------------------------------------------------------ small and ragged shapes, full comparison
+SHAPES_I16 = [
+    (1, 1, 1), (2, 3, 5), (17, 33, 1), (128, 128, 64), (129, 127, 65), (300, 200, 290),
+    (256, 384, 513), (200, 130, 1000), (130, 260, 2049), (512, 384, 290), (64, 513, 700),
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES_I16)
+def test_i16_shapes(gm, shape):
+    m, n, k = shape
+    A, B, C = gi.random_problem(100 + sum(shape), m, n, k, "i16")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"i16 {shape}")
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1), (20, 40, 60), (129, 130, 131), (256, 256, 1025), (300, 77, 2100)])
+def test_i8_shapes(gm, shape):
+    m, n, k = shape
+    A, B, C = gi.random_problem(200 + sum(shape), m, n, k, "i8")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"i8 {shape}")
+
+
+@pytest.mark.parametrize("k", [511, 512, 513, 1023, 1024, 1025, 4096])
+def test_i16_chunk_boundaries(gm, k):
+    A, B, C = gi.random_problem(300 + k, 160, 136, k, "i16")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"k={k}")
+
+
+# ------------------------------------------------------------------ extreme and adversarial values
+EXTREMES = [(-32768, -32768), (32767, -32768), (32767, 32767), (32640, 32640), (-1, -1), (32640, -32768), (-129, 32767)]
+
+
+@pytest.mark.parametrize("ab", EXTREMES)
+@pytest.mark.parametrize("m", [8, 200])
+def test_i16_constant_extremes(gm, ab, m):
+    a, b = ab
+    n, k = 136, 1100
+    A = np.full((m, k), a, np.int16)
+    B = np.full((k, n), b, np.int16)
+    C = gi.uniform_int(9, (m, n), -(1 << 40), 1 << 40, np.int64)
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"constant {ab}")
+
+
+@pytest.mark.parametrize("m", [8, 160])
+def test_i16_near_fp32_exactness_limit(gm, m):
+    """Limb sums pushed toward the largest magnitudes a chunk allows, with odd low bits.
+
+    32640 = 256*128 - 128 has limbs (h, l) = (128, -128): every limb product is
+    +-2^14, the most a product can be.  Mixing in values with low bits set makes
+    the partial sums large and odd, where a lossy accumulation would show.
+    """
+    n, k = 136, 2048
+    base = np.where((np.arange(k) % 7) == 3, -32767, 32640).astype(np.int16)
+    A = np.tile(base, (m, 1))
+    A[:, ::13] = 32767
+    B = np.tile(base[:, None], (1, n)).astype(np.int16)
+    B[::11, :] = -32768
+    B[5::17, ::3] = 255
+    C = np.zeros((m, n), np.int64)
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), "adversarial")
+
+
+def test_i8_extremes(gm):
+    for a, b in ((-128, -128), (127, -128), (127, 127)):
+        A = np.full((140, 3000), a, np.int8)
+        B = np.full((3000, 136), b, np.int8)
+        C = gi.uniform_int(3, (140, 136), -(1 << 30), 1 << 30, np.int32)
+        assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"i8 constant {(a, b)}")
+
+
+def test_wraparound_mod_2_64(gm):
+    A = np.full((130, 4), 32767, np.int16)
+    B = np.full((4, 130), 32767, np.int16)
+    C = np.full((130, 130), np.iinfo(np.int64).max - 5, np.int64)
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), "wrap")
+
+
+# ------------------------------------------------------------------ layouts: padding, odd leading dimensions
+@pytest.mark.parametrize("pads", [(0, 0, 0), (3, 5, 7), (8, 8, 2), (1, 0, 1)])
+@pytest.mark.parametrize("m", [5, 150])
+def test_i16_leading_dimensions(gm, pads, m):
+    pa, pb, pc = pads
+    n, k = 140, 333
+    A, B, C = gi.random_problem(400 + m + sum(pads), m, n, k, "i16")
+    exp = expected(A, B, C)
+    Ap = torch.full((m, k + pa), 12345, dtype=torch.int16)
+    Bp = torch.full((k, n + pb), -777, dtype=torch.int16)
+    Cp = torch.full((m, n + pc), -424242, dtype=torch.int64)
+    Ap[:, :k] = torch.from_numpy(A)
+    Bp[:, :n] = torch.from_numpy(B)
+    Cp[:, :n] = torch.from_numpy(C)
+    dA, dB, dC = Ap.cuda(), Bp.cuda(), Cp.cuda()
+    gm.gemm_i16(dA[:, :k], dB[:, :n], dC[:, :n])
+    torch.cuda.synchronize()
+    out = dC.cpu().numpy()
+    assert_same(out[:, :n], exp, f"padded {pads}")
+    assert (out[:, n:] == -424242).all(), "padding of C was written"
+
+
+def test_i8_leading_dimensions(gm):
+    m, n, k = 150, 131, 517
+    A, B, C = gi.random_problem(77, m, n, k, "i8")
+    exp = expected(A, B, C)
+    Ap = torch.zeros((m, k + 3), dtype=torch.int8)
+    Bp = torch.zeros((k, n + 5), dtype=torch.int8)
+    Cp = torch.full((m, n + 1), 99, dtype=torch.int32)
+    Ap[:, :k], Bp[:, :n], Cp[:, :n] = torch.from_numpy(A), torch.from_numpy(B), torch.from_numpy(C)
+    dA, dB, dC = Ap.cuda(), Bp.cuda(), Cp.cuda()
+    gm.gemm_i8(dA[:, :k], dB[:, :n], dC[:, :n])
+    torch.cuda.synchronize()
+    out = dC.cpu().numpy()
+    assert_same(out[:, :n], exp, "i8 padded")
+    assert (out[:, n:] == 99).all()
+
+
+# ------------------------------------------------------------------ skinny-M path
+@pytest.mark.parametrize("m", [1, 3, 8, 9, 16])
+@pytest.mark.parametrize("nk", [(100, 300), (4096, 1000), (33, 4097)])
+def test_skinny_shapes(gm, m, nk):
+    n, k = nk
+    A, B, C = gi.random_problem(500 + m + n + k, m, n, k, "i16")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"skinny m={m} n={n} k={k}")
+
+
+@pytest.mark.parametrize("ksplit", [1, 2, 5, 64])
+def test_skinny_ksplit(gm, ksplit):
+    gm.set_option(gm.OPT_SKINNY_KSPLIT, ksplit)
+    try:
+        A, B, C = gi.random_problem(600 + ksplit, 8, 1000, 3000, "i16")
+        assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"ksplit={ksplit}")
+    finally:
+        gm.set_option(gm.OPT_SKINNY_KSPLIT, 0)
+
+
+def test_main_kernel_on_small_m(gm):
+    """The tcgen05 path on m <= 16 (skinny path switched off)."""
+    gm.set_option(gm.OPT_SKINNY_MAX_M, 0)
+    try:
+        for m in (1, 8, 16):
+            A, B, C = gi.random_problem(700 + m, m, 260, 700, "i16")
+            assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"tc m={m}")
+    finally:
+        gm.set_option(gm.OPT_SKINNY_MAX_M, 16)
+
+
+def test_skinny_unaligned_B(gm):
+    m, n, k = 8, 203, 900
+    A, B, C = gi.random_problem(801, m, n, k, "i16")
+    exp = expected(A, B, C)
+    Bp = torch.zeros((k, n + 1), dtype=torch.int16)  # row pitch 204 elements = 408 bytes: not 16-aligned
+    Bp[:, :n] = torch.from_numpy(B)
+    dA, dB, dC = torch.from_numpy(A).cuda(), Bp.cuda(), torch.from_numpy(C).cuda()
+    gm.gemm_i16(dA, dB[:, :n], dC)
+    torch.cuda.synchronize()
+    assert_same(dC.cpu().numpy(), exp, "skinny unaligned B")
+
+
+def test_skinny_extremes(gm):
+    for a, b in ((-32768, -32768), (-1, -1), (32767, -32768), (255, 255)):
+        A = np.full((8, 2000), a, np.int16)
+        B = np.full((2000, 300), b, np.int16)
+        C = np.zeros((8, 300), np.int64)
+        assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"skinny constant {(a, b)}")
+
+
+# ------------------------------------------------------------------ the five workloads
+def _sample_rows(m, count=24):
+    rows = {0, 1, m - 1, m // 2, 127, 128, m - 129}
+    rng = gi.uniform_int(4242 + m, (count,), 0, m - 1, np.int64)
+    rows.update(int(r) for r in rng)
+    return sorted(r for r in rows if 0 <= r < m)
+
+
+@pytest.mark.parametrize("name", list(gi.WORKLOADS))
+def test_workload(gm, name):
+    w = gi.WORKLOADS[name]
+    A, B, C = gi.make_inputs(w)
+    got = run_gpu(gm, A, B, C, w.kind)
+    if w.m * w.n * w.k <= 1 << 28:
+        assert_same(got, expected(A, B, C), name)
+        return
+    rows = _sample_rows(w.m)
+    assert_same(got[rows], expected(A[rows], B, C[rows]), f"{name} sampled rows {rows[:4]}...")
+    # every output through row and column sums (exact int64 arithmetic modulo 2^64)
+    with np.errstate(over="ignore"):
+        Bsum = B.astype(np.int64).sum(axis=1)
+        row_exp = A.astype(np.int64) @ Bsum + C.astype(np.int64).sum(axis=1)
+        Asum = A.astype(np.int64).sum(axis=0)
+        col_exp = Asum @ B.astype(np.int64) + C.astype(np.int64).sum(axis=0)
+        row_got = got.astype(np.int64).sum(axis=1)
+        col_got = got.astype(np.int64).sum(axis=0)
+    if w.kind == "i8":  # int32 C: the sums compare modulo 2^32
+        row_exp, row_got, col_exp, col_got = (x & 0xFFFFFFFF for x in (row_exp, row_got, col_exp, col_got))
+    assert np.array_equal(row_got, row_exp), f"{name}: row sums differ"
+    assert np.array_equal(col_got, col_exp), f"{name}: column sums differ"
+
+
+# ------------------------------------------------------------------ host-buffer API, streams, failure detection
+def test_host_api_i16_and_i8(gm):
+    A, B, C = gi.random_problem(900, 150, 170, 400, "i16")
+    X = C.copy()
+    gm.gemm_i16_host(A, B, X)
+    assert_same(X, expected(A, B, C), "host i16")
+    A, B, C = gi.random_problem(901, 150, 170, 400, "i8")
+    X = C.copy()
+    gm.gemm_i8_host(A, B, X)
+    assert_same(X, expected(A, B, C), "host i8")
+
+
+def test_host_api_padded(gm):
+    m, n, k = 9, 50, 70
+    A, B, C = gi.random_problem(902, m, n, k, "i16")
+    big = np.full((m, n + 3), 7, np.int64)
+    big[:, :n] = C
+    gm.gemm_i16_host(A, B, big[:, :n])
+    assert_same(big[:, :n], expected(A, B, C), "host padded")
+    assert (big[:, n:] == 7).all()
+
+
+def test_non_default_stream(gm):
+    A, B, C = gi.random_problem(903, 300, 260, 500, "i16")
+    s = torch.cuda.Stream()
+    dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s):
+        gm.gemm_i16(dA, dB, dC)
+    s.synchronize()
+    assert_same(dC.cpu().numpy(), expected(A, B, C), "side stream")
+
+
+def test_repeated_calls_accumulate(gm):
+    A, B, C = gi.random_problem(904, 200, 140, 300, "i16")
+    dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+    for _ in range(3):
+        gm.gemm_i16(dA, dB, dC)
+    torch.cuda.synchronize()
+    exp = C.copy()
+    for _ in range(3):
+        oracle.gemm(A, B, exp)
+    assert_same(dC.cpu().numpy(), exp, "3x accumulate")
+
+
+def test_bounded_wait_reports_timeout(gm):
+    """A pipeline wait that can never complete gives up, reports, and leaves the context usable."""
+    assert gm.selftest_wait_timeout(2000) == gm.ETIMEOUT
+    assert (gm.device_status_detail() & 0xFF) == gm.ETIMEOUT
+    assert gm.device_status() == gm.OK  # cleared
+    A, B, C = gi.random_problem(905, 130, 130, 130, "i16")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), "after timeout self-test")
+
+
+def test_dtype_and_shape_errors(gm):
+    a = torch.zeros((4, 4), dtype=torch.int32, device="cuda")
+    with pytest.raises(TypeError):
+        gm.gemm_i16(a, a, torch.zeros((4, 4), dtype=torch.int64, device="cuda"))
+    with pytest.raises(ValueError):
+        gm.gemm_i16(torch.zeros((4, 5), dtype=torch.int16, device="cuda"),
+                    torch.zeros((4, 4), dtype=torch.int16, device="cuda"),
+                    torch.zeros((4, 4), dtype=torch.int64, device="cuda"))
