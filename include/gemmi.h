@@ -128,9 +128,16 @@ size_t gemmi_workspace_bytes(void);
  *                            microseconds (default 4,000,000).
  *   GEMMI_OPT_SKINNY_KSPLIT : number of CTAs sharing the reduction dimension
  *                            of one skinny column block (0 = automatic).
- * Returns GEMMI_OK or GEMMI_EINVAL.
+ *   GEMMI_OPT_TC_CHUNK_SCALE : length of the exact fp32 accumulation runs of the tensor-core
+ *                            GEMM: 2 (default) keeps every partial limb sum within 2^24, the limit
+ *                            of exact fp32 integer sums; 1 keeps it within 2^23 (twice the drains).
+ *   GEMMI_OPT_TC_GROUP_M   : tile raster band height in 128-row tiles (default 16).
+ *   GEMMI_OPT_TC_L2_HINTS  : L2 eviction policy of the operand tile loads, bits 0-1 for A,
+ *                            bits 2-3 for B: 0 normal, 1 evict_last, 2 evict_first (default 0).
+ * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
-enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3 };
+enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
+       GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 

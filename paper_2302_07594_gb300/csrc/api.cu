@@ -107,6 +107,9 @@ cudaStream_t g_stream = nullptr;
 int64_t g_skinny_max_m = 16;
 int64_t g_timeout_us = 4000000;
 int64_t g_skinny_ksplit = 0;
+int64_t g_tc_chunk_scale = 2;
+int64_t g_tc_group_m = 16;
+int64_t g_tc_l2_hints = 0;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -251,6 +254,10 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   ta.status = d.status;
   ta.timeout_ns = timeout_ns();
   ta.num_sms = d.sm_count;
+  ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
+  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
+  ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
   const char* why = "tcgen05 GEMM launch";
   const int kind = nl == 2 ? GEMMI_KERNEL_TC_I16 : GEMMI_KERNEL_TC_I8;
   cudaEvent_t t1 = timer_begin(kind, s);
@@ -262,27 +269,41 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
 
 int run_skinny(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
                int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s) {
-  const bool tma_ok = reinterpret_cast<uintptr_t>(B) % 16 == 0 && (ldb * 2) % 16 == 0;
+  // TMA needs 16-byte aligned row starts; operands that do not have them are re-pitched into the workspace
+  const bool b_ok = reinterpret_cast<uintptr_t>(B) % 16 == 0 && (ldb * 2) % 16 == 0;
+  const bool a_ok = reinterpret_cast<uintptr_t>(A) % 16 == 0 && (lda * 2) % 16 == 0;
   const int16_t* Bs = B;
-  int64_t ldbs = ldb;
-  bool used_ws = false;
+  const int16_t* As = A;
+  int64_t ldbs = ldb, ldas = lda;
+  const bool used_ws = !a_ok || !b_ok;
   int rc;
-  if (!tma_ok) {
-    // re-pitch B into the workspace so that every row starts on a 16-byte boundary
-    ldbs = static_cast<int64_t>(round_up(static_cast<size_t>(n), 8));
-    if ((rc = ensure_buffer(&d.ws, &d.ws_bytes, static_cast<size_t>(k) * ldbs * 2)) != GEMMI_OK) return rc;
+  if (used_ws) {
+    const int64_t ldb_new = static_cast<int64_t>(round_up(static_cast<size_t>(n), 8));
+    const int64_t lda_new = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+    const size_t b_bytes = b_ok ? 0 : round_up(static_cast<size_t>(k) * ldb_new * 2, kAlign);
+    const size_t a_bytes = a_ok ? 0 : round_up(static_cast<size_t>(m) * lda_new * 2, kAlign);
+    if ((rc = ensure_buffer(&d.ws, &d.ws_bytes, a_bytes + b_bytes)) != GEMMI_OK) return rc;
     if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
-    cudaError_t e = cudaMemcpy2DAsync(d.ws, ldbs * 2, B, ldb * 2, n * 2, k, cudaMemcpyDeviceToDevice, s);
-    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy2DAsync(B)");
-    Bs = static_cast<const int16_t*>(d.ws);
-    used_ws = true;
+    char* ws = static_cast<char*>(d.ws);
+    if (!b_ok) {
+      cudaError_t e = cudaMemcpy2DAsync(ws, ldb_new * 2, B, ldb * 2, n * 2, k, cudaMemcpyDeviceToDevice, s);
+      if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy2DAsync(B)");
+      Bs = reinterpret_cast<const int16_t*>(ws);
+      ldbs = ldb_new;
+    }
+    if (!a_ok) {
+      cudaError_t e = cudaMemcpy2DAsync(ws + b_bytes, lda_new * 2, A, lda * 2, k * 2, m, cudaMemcpyDeviceToDevice, s);
+      if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy2DAsync(A)");
+      As = reinterpret_cast<const int16_t*>(ws + b_bytes);
+      ldas = lda_new;
+    }
   }
   gemmi::SkinnyArgs sa;
   sa.m = m;
   sa.n = n;
   sa.k = k;
-  sa.A = A;
-  sa.lda = lda;
+  sa.A = As;
+  sa.lda = ldas;
   sa.B = Bs;
   sa.ldb = ldbs;
   sa.C = C;
@@ -495,6 +516,19 @@ int gemmi_set_option(int option, int64_t value) {
       if (value < 0 || value > 4096) return set_error(GEMMI_EINVAL, "ksplit must be in [0, 4096]");
       g_skinny_ksplit = value;
       return GEMMI_OK;
+    case GEMMI_OPT_TC_CHUNK_SCALE:
+      if (value != 1 && value != 2) return set_error(GEMMI_EINVAL, "chunk scale must be 1 or 2");
+      g_tc_chunk_scale = value;
+      return GEMMI_OK;
+    case GEMMI_OPT_TC_GROUP_M:
+      if (value < 1 || value > 1024) return set_error(GEMMI_EINVAL, "raster band must be in [1, 1024]");
+      g_tc_group_m = value;
+      return GEMMI_OK;
+    case GEMMI_OPT_TC_L2_HINTS:
+      if (value < 0 || value > 15 || (value & 3) == 3 || ((value >> 2) & 3) == 3)
+        return set_error(GEMMI_EINVAL, "L2 hints: 2 bits each for A and B, values 0..2");
+      g_tc_l2_hints = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -506,6 +540,9 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_SKINNY_MAX_M: return g_skinny_max_m;
     case GEMMI_OPT_WAIT_TIMEOUT_US: return g_timeout_us;
     case GEMMI_OPT_SKINNY_KSPLIT: return g_skinny_ksplit;
+    case GEMMI_OPT_TC_CHUNK_SCALE: return g_tc_chunk_scale;
+    case GEMMI_OPT_TC_GROUP_M: return g_tc_group_m;
+    case GEMMI_OPT_TC_L2_HINTS: return g_tc_l2_hints;
     default: return -1;
   }
 }

@@ -19,17 +19,24 @@
 // overflows, here built from exact fp32 chunks and int64 registers.  The int8
 // path is the same with one plane, one product and one accumulator (int32 sum).
 //
-// Structure (one persistent CTA per SM, 320 threads, 128x128 output tiles):
+// Structure (one persistent CTA per SM, 352 threads, 128x128 output tiles):
 //   warp 8      TMA producer: 2-D tiled bulk-tensor loads of 64-wide K blocks of
 //               the limb planes (128-byte swizzle) into a ring of smem stages;
-//   warp 9      MMA issuer: tcgen05.mma kind::f16 (M=128, N=128, K=16) from smem
-//               descriptors into fp32 accumulators in tensor memory (TMEM);
+//   warps 9-10  MMA issuers: tcgen05.mma kind::f16 (M=128, N=128, K=16) from smem
+//               descriptors into fp32 accumulators in tensor memory (TMEM).  A
+//               single issuing thread leaves the tensor pipe idle for every cycle
+//               it spends waiting or book-keeping (the pipe buffers almost no
+//               instructions), so two warps issue concurrently, each owning its
+//               own accumulators: HH+LL and X for int16; even and odd K blocks
+//               for int8;
 //   warps 0-7   epilogue: drain accumulators (tcgen05.ld) into int64 registers,
 //               and read-modify-write C once per tile.
-// TMEM holds four 128-column accumulator slots: three live accumulators plus
-// one spare.  Chunk ends of the three accumulators are staggered, so at every
-// chunk end the MMA warp moves that accumulator into the spare slot and keeps
-// issuing while the epilogue drains the old one.  This takes the place of the
+// TMEM holds four 128-column accumulator slots: the live accumulators plus
+// spares.  Chunk ends are staggered, so at every chunk end the owning issuer
+// moves that accumulator into the oldest spare slot and keeps issuing while the
+// epilogue drains the old one.  Every role replays the same deterministic
+// chunk schedule, so slot assignments need no communication beyond the
+// full/empty barriers of each slot.  This takes the place of the
 // paper's loop L6 / micro-kernel (Figure 1, Section 5.2); the smem stage ring
 // takes the place of the B_r copies into local memory (Section 5.1).
 //
@@ -49,63 +56,115 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BN = 128;
-constexpr int BK = 64;                       // 64 fp16 = 128 bytes = one swizzle row
 constexpr int UMMA_K = 16;                   // K of one tcgen05.mma kind::f16
-constexpr int TILE_BYTES = BM * BK * 2;      // 16 KB per limb tile (BM == BN)
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int PRODUCER_WARP = 8;
-constexpr int MMA_WARP = 9;
-constexpr int NUM_THREADS = 320;
+constexpr int MMA_WARP0 = 9;                  // issuer warps 9 and 10; warp 9 also owns the TMEM allocation
+constexpr int NISSUE = 2;
+constexpr int NUM_THREADS = (NUM_EPI_WARPS + 1 + NISSUE) * 32;
 constexpr int NSLOT = 4;
 constexpr int SLOT_COLS = 128;
 constexpr int TMEM_COLS = NSLOT * SLOT_COLS;  // 512
-constexpr int GROUP_M = 16;                   // tile raster: bands of 16 row tiles
 constexpr uint32_t STATUS_TIMEOUT = 4;
 
 template <int NL>
 struct Scheme;
 
 // int16: two limbs per operand, four products, three accumulators.
+//   product p: (A limb, B limb) = (h,h), (h,l), (l,h), (l,l); limb 0 = high, 1 = low
+//   accumulators: 0 = HH (weight 2^16), 1 = X (2^8), 2 = LL (1)
+//   issuer 0 owns HH and LL (products 0, 3), issuer 1 owns X (products 1, 2): 8 MMAs each per K block.
 template <>
 struct Scheme<2> {
-  static constexpr int STAGES = 3;
   static constexpr int NACC = 3;
   static constexpr int NPROD = 4;
-  // product p: (A limb, B limb, accumulator); limb 0 = high, 1 = low
-  __device__ static constexpr int a_limb(int p) { return p == 0 ? 0 : p == 1 ? 0 : p == 2 ? 1 : 1; }
-  __device__ static constexpr int b_limb(int p) { return p == 0 ? 0 : p == 1 ? 1 : p == 2 ? 0 : 1; }
-  __device__ static constexpr int acc(int p) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
-  // chunk schedule in K blocks of 64: accumulator a ends a chunk after block kb when
-  // (kb + 1 + PHASE[a]) % PERIOD[a] == 0, or at the last block of the tile.
-  // HH, LL: 8 blocks = 512 indices, |sum| <= 512 * 2^14 = 2^23;  X: 4 blocks = 256, |sum| <= 256 * 2^15 = 2^23.
-  __device__ static constexpr int period(int a) { return a == 1 ? 4 : 8; }
-  __device__ static constexpr int phase(int a) { return a == 0 ? 6 : a == 1 ? 0 : 2; }
+  static constexpr int EMPTY_COUNT = 2;  // both issuers read every stage
+  __device__ static constexpr int a_limb(int p) { return p >> 1; }
+  __device__ static constexpr int b_limb(int p) { return p & 1; }
+  __device__ static constexpr int acc(int p, int) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
+  __device__ static constexpr int issuer(int p, int) { return (p == 0 || p == 3) ? 0 : 1; }
+  __device__ static constexpr int owner(int a) { return a == 1 ? 1 : 0; }
   __device__ static constexpr int shift(int a) { return a == 0 ? 16 : a == 1 ? 8 : 0; }
+  // Chunk schedule, in reduction indices, for chunk scale CS (1 or 2): accumulator a ends a
+  // chunk after the K block that ends at index e when (e + PHASE[a]) % PERIOD[a] == 0, or at
+  // the last block of the tile.  HH, LL: 512*CS indices, |sum| <= 512*CS * 2^14;  X: 256*CS
+  // indices, |sum| <= 256*CS * 2^15.  CS = 1 keeps every partial sum within 2^23 (one bit below
+  // the 2^24 limit of exact fp32 integer sums), CS = 2 within 2^24.  The phases stagger the
+  // three chunk ends 128*CS indices apart (HH at 128*CS, X at 256*CS, LL at 384*CS, X at 512*CS, ...).
+  template <int CS>
+  __device__ static bool chunk_ends(int a, int kb, int nkb) {
+    const int period = (a == 1 ? 256 : 512) * CS;
+    const int phase = (a == 0 ? 384 : a == 1 ? 0 : 128) * CS;
+    return kb == nkb - 1 || (((kb + 1) * 64 + phase) % period) == 0;
+  }
 };
 
-// int8: the value itself in one fp16 plane, one product, one accumulator.
-// 8 blocks = 512 indices, |sum| <= 512 * 2^14 = 2^23.
+// int8: the value itself in one fp16 plane, one product per K block.  Two accumulators take the
+// even and the odd K blocks (issuer 0 and 1), each with chunks of 512*CS of its own reduction
+// indices, |sum| <= 512*CS * 2^14; their chunk ends are staggered by half a chunk.
 template <>
 struct Scheme<1> {
-  static constexpr int STAGES = 6;
-  static constexpr int NACC = 1;
+  static constexpr int NACC = 2;
   static constexpr int NPROD = 1;
+  static constexpr int EMPTY_COUNT = 1;  // each stage is read by one issuer
   __device__ static constexpr int a_limb(int) { return 0; }
   __device__ static constexpr int b_limb(int) { return 0; }
-  __device__ static constexpr int acc(int) { return 0; }
-  __device__ static constexpr int period(int) { return 8; }
-  __device__ static constexpr int phase(int) { return 0; }
+  __device__ static constexpr int acc(int, int kb) { return kb & 1; }
+  __device__ static constexpr int issuer(int, int kb) { return kb & 1; }
+  __device__ static constexpr int owner(int a) { return a; }
   __device__ static constexpr int shift(int) { return 0; }
+  template <int CS>
+  __device__ static bool chunk_ends(int a, int kb, int nkb) {
+    if ((kb & 1) != a) return false;
+    const int own = (kb >> 1) + 1;  // K blocks this accumulator has taken, including kb
+    return kb + 2 >= nkb || ((own * 64 + a * 256 * CS) % (512 * CS)) == 0;
+  }
 };
 
-template <int NL>
-constexpr int stage_bytes() { return 2 * NL * TILE_BYTES; }
+// Assignment of accumulators to the four TMEM slots, replayed identically by every role.
+// Spare slots form a FIFO: a chunk end moves the accumulator into the oldest spare and queues
+// its old slot.  rotate() returns the parity to wait on (the slot's empty barrier) before the
+// new slot may be written: the n-th assignment of a slot waits for its (n-1)-th drain.
+template <int NACC>
+struct SlotRing {
+  int slot_of[NACC];
+  int spares[NSLOT - NACC];
+  uint32_t assign_parity;  // bit s: parity of the number of assignments of slot s so far
 
+  __device__ __forceinline__ void init() {
+    assign_parity = 0;
+#pragma unroll
+    for (int a = 0; a < NACC; ++a) {
+      slot_of[a] = a;
+      assign_parity ^= 1u << a;
+    }
+#pragma unroll
+    for (int i = 0; i < NSLOT - NACC; ++i) spares[i] = NACC + i;
+  }
+  __device__ __forceinline__ uint32_t rotate(int a) {
+    const int old = slot_of[a];
+    const int fresh = spares[0];
+#pragma unroll
+    for (int i = 0; i + 1 < NSLOT - NACC; ++i) spares[i] = spares[i + 1];
+    spares[NSLOT - NACC - 1] = old;
+    slot_of[a] = fresh;
+    const uint32_t par = ((assign_parity >> fresh) & 1u) ^ 1u;
+    assign_parity ^= 1u << fresh;
+    return par;
+  }
+};
+
+// Tile geometry: K blocks of 64 fp16 (128-byte rows, the 128-byte swizzle span).
+constexpr int BK = 64;
 template <int NL>
-constexpr size_t smem_bytes() {
-  // stages + barriers (full/empty per stage, full/empty per slot, one final) + TMEM holder + abort flag
-  return 1024 + static_cast<size_t>(Scheme<NL>::STAGES) * stage_bytes<NL>() + 8 * (2 * Scheme<NL>::STAGES + 2 * NSLOT + 1) + 16;
-}
+struct Geom {
+  static constexpr int TILE_BYTES = BM * BK * 2;          // one limb tile (BM == BN)
+  static constexpr int SB = 2 * NL * TILE_BYTES;          // one stage: NL tiles of A and of B
+  static constexpr int STAGES = (192 * 1024) / SB;        // 192 KB of stages
+  static constexpr int SWIZZLE = BK * 2;                  // bytes per swizzled row
+  static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + 8 * (2 * STAGES + 2 * NSLOT + 1) + 16;
+  static_assert(SMEM <= 227 * 1024, "shared memory budget");
+};
 
 struct TcParams {
   int64_t m, n, k;
@@ -113,24 +172,41 @@ struct TcParams {
   int64_t ldc;
   int num_m_tiles, num_n_tiles, num_k_blocks;
   int c_vec;
+  int group_m;        // tile raster: bands of group_m row tiles, column-major inside a band
+  int hint_a;         // L2 policy of A loads: 0 normal, 1 evict_last, 2 evict_first
+  int hint_b;         // same for B
   uint64_t timeout_ns;
   uint32_t* status;
 };
 
-__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& mt, int& nt) {
-  const int per_group = GROUP_M * num_n;
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
+  const int per_group = group_m * num_n;
   const int group = t / per_group;
-  const int first_m = group * GROUP_M;
-  const int rows_here = min(GROUP_M, num_m - first_m);
+  const int first_m = group * group_m;
+  const int rows_here = min(group_m, num_m - first_m);
   const int in_group = t - group * per_group;
   mt = first_m + in_group % rows_here;
   nt = in_group / rows_here;
 }
 
-template <int NL>
-__device__ __forceinline__ bool chunk_ends(int a, int kb, int nkb) {
-  using S = Scheme<NL>;
-  return kb == nkb - 1 || ((kb + 1 + S::phase(a)) % S::period(a)) == 0;
+__device__ __forceinline__ uint64_t l2_policy(int hint) {
+  uint64_t p = 0;
+  if (hint == 1) asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  else if (hint == 2) asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const void* map, uint32_t bar, int32_t x, int32_t y,
+                                                 int hint, uint64_t policy) {
+  if (hint == 0) {
+    tma_load_2d(dst, map, bar, x, y);
+  } else {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%3, %4}], [%2], %5;"
+        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "l"(policy)
+        : "memory");
+  }
 }
 
 __device__ __forceinline__ int32_t f32_to_i32(uint32_t bits) {
@@ -139,13 +215,15 @@ __device__ __forceinline__ int32_t f32_to_i32(uint32_t bits) {
   return v;
 }
 
-template <int NL>
+template <int NL, int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
                const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1, TcParams P) {
   using S = Scheme<NL>;
-  constexpr int STAGES = S::STAGES;
-  constexpr int SB = stage_bytes<NL>();
+  using G = Geom<NL>;
+  constexpr int STAGES = G::STAGES;
+  constexpr int SB = G::SB;
+  constexpr int TILE_BYTES = G::TILE_BYTES;
   // C element type and the unsigned type of the running sum (wrap-around is modular, never UB)
   using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
   using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
@@ -167,17 +245,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
-      mbar_init(empty0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, S::EMPTY_COUNT);
     }
     for (int s = 0; s < NSLOT; ++s) {
       mbar_init(sfull0 + 8 * s, 1);
       mbar_init(sempty0 + 8 * s, NUM_EPI_WARPS);
     }
-    mbar_init(final_bar, 1);
+    mbar_init(final_bar, NISSUE);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == MMA_WARP) {
+  if (warp == MMA_WARP0) {
     tmem_alloc(smem_u32(tmem_holder), TMEM_COLS);
     tmem_relinquish();
   }
@@ -198,13 +276,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         tma_prefetch_desc(&mapA1);
         tma_prefetch_desc(&mapB1);
       }
+      const uint64_t pol_a = l2_policy(P.hint_a);
+      const uint64_t pol_b = l2_policy(P.hint_b);
       int stage = 0;
       uint32_t phase = 0;
       int64_t issued = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
         int mt, nt;
-        tile_coords(t, P.num_m_tiles, P.num_n_tiles, mt, nt);
+        tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
         for (int kb = 0; kb < nkb; ++kb) {
           if (!bounded_wait(empty0 + 8 * stage, phase ^ 1u, P.timeout_ns)) {
             report_status(P.status, STATUS_TIMEOUT, 1);
@@ -216,10 +296,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           const uint32_t fb = full0 + 8 * stage;
           mbar_arrive_expect_tx(fb, SB);
           const uint32_t base = smem_u32(smem + stage * SB);
-          tma_load_2d(base, &mapA0, fb, kb * BK, mt * BM);
-          if (NL == 2) tma_load_2d(base + TILE_BYTES, &mapA1, fb, kb * BK, mt * BM);
-          tma_load_2d(base + NL * TILE_BYTES, &mapB0, fb, kb * BK, nt * BN);
-          if (NL == 2) tma_load_2d(base + (NL + 1) * TILE_BYTES, &mapB1, fb, kb * BK, nt * BN);
+          tma_load_2d_hint(base, &mapA0, fb, kb * BK, mt * BM, P.hint_a, pol_a);
+          if (NL == 2) tma_load_2d_hint(base + TILE_BYTES, &mapA1, fb, kb * BK, mt * BM, P.hint_a, pol_a);
+          tma_load_2d_hint(base + NL * TILE_BYTES, &mapB0, fb, kb * BK, nt * BN, P.hint_b, pol_b);
+          if (NL == 2) tma_load_2d_hint(base + (NL + 1) * TILE_BYTES, &mapB1, fb, kb * BK, nt * BN, P.hint_b, pol_b);
           ++issued;
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -232,63 +312,75 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         bounded_wait(full0 + 8 * s, par, P.timeout_ns);
       }
     }
-  } else if (warp == MMA_WARP) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp >= MMA_WARP0) {
+    // ------------------------------------------------------------ MMA issuers (one thread each)
+    const int me = warp - MMA_WARP0;
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
       int stage = 0;
       uint32_t phase = 0;
-      int slot_of[3] = {0, 1, 2};
-      int spare = S::NACC;  // first slot not owned by a live accumulator
-      uint32_t use_parity = 0;  // bit s: parity of the number of times slot s has been acquired
-      bool need_acquire[3] = {true, true, true};
-      bool fresh[3] = {true, true, true};
+      SlotRing<S::NACC> ring;
+      ring.init();
+      uint32_t wait_par[S::NACC];
+      bool need_acquire[S::NACC], fresh[S::NACC];
+#pragma unroll
+      for (int a = 0; a < S::NACC; ++a) {
+        wait_par[a] = 1u;  // first use of the initial slots: nothing to wait for
+        need_acquire[a] = true;
+        fresh[a] = true;
+      }
       bool ok = true;
       for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
         for (int kb = 0; kb < nkb && ok; ++kb) {
-          if (!bounded_wait(full0 + 8 * stage, phase, P.timeout_ns)) {
-            report_status(P.status, STATUS_TIMEOUT, 2);
-            *abort_flag = 1;
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t base = smem_u32(smem + stage * SB);
+          bool mine = false;
 #pragma unroll
-          for (int p = 0; p < S::NPROD; ++p) {
-            const int a = S::acc(p);
-            if (need_acquire[a]) {
-              const int s = slot_of[a];
-              if (!bounded_wait(sempty0 + 8 * s, ((use_parity >> s) & 1u) ^ 1u, P.timeout_ns)) {
-                report_status(P.status, STATUS_TIMEOUT, 3);
-                *abort_flag = 1;
-                ok = false;
-                break;
+          for (int p = 0; p < S::NPROD; ++p) mine |= S::issuer(p, kb) == me;
+          if (mine) {
+            if (!bounded_wait(full0 + 8 * stage, phase, P.timeout_ns)) {
+              report_status(P.status, STATUS_TIMEOUT, 2);
+              *abort_flag = 1;
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t base = smem_u32(smem + stage * SB);
+#pragma unroll
+            for (int p = 0; p < S::NPROD; ++p) {
+              if (S::issuer(p, kb) != me) continue;
+              const int a = S::acc(p, kb);
+              if (need_acquire[a]) {
+                // the slot's previous chunk (any accumulator's) must have been drained
+                if (!bounded_wait(sempty0 + 8 * ring.slot_of[a], wait_par[a], P.timeout_ns)) {
+                  report_status(P.status, STATUS_TIMEOUT, 3);
+                  *abort_flag = 1;
+                  ok = false;
+                  break;
+                }
+                need_acquire[a] = false;
+                tc_fence_after();
               }
-              use_parity ^= 1u << s;
-              need_acquire[a] = false;
-              tc_fence_after();
-            }
-            const uint32_t d = tmem_base + static_cast<uint32_t>(slot_of[a] * SLOT_COLS);
-            const uint64_t adesc = smem_desc_kmajor_sw128(base + S::a_limb(p) * TILE_BYTES);
-            const uint64_t bdesc = smem_desc_kmajor_sw128(base + (NL + S::b_limb(p)) * TILE_BYTES);
+              const uint32_t d = tmem_base + static_cast<uint32_t>(ring.slot_of[a] * SLOT_COLS);
+              const uint64_t adesc = smem_desc_kmajor<G::SWIZZLE>(base + S::a_limb(p) * TILE_BYTES);
+              const uint64_t bdesc = smem_desc_kmajor<G::SWIZZLE>(base + (NL + S::b_limb(p)) * TILE_BYTES);
 #pragma unroll
-            for (int kk = 0; kk < BK / UMMA_K; ++kk) {
-              // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
-              const uint32_t acc_flag = (fresh[a] && kk == 0) ? 0u : 1u;
-              tc_mma_f16(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, acc_flag);
+              for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+                // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
+                const uint32_t acc_flag = (fresh[a] && kk == 0) ? 0u : 1u;
+                tc_mma_f16(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, acc_flag);
+              }
+              fresh[a] = false;
             }
-            fresh[a] = false;
+            if (!ok) break;
+            tc_commit(empty0 + 8 * stage);  // this issuer has finished reading the stage once its MMAs complete
           }
-          if (!ok) break;
-          tc_commit(empty0 + 8 * stage);  // stage is free once these MMAs have read it
+          // replay every chunk end (own and the other issuer's) to keep the slot ring in step
 #pragma unroll
           for (int a = 0; a < S::NACC; ++a) {
-            if (chunk_ends<NL>(a, kb, nkb)) {
-              tc_commit(sfull0 + 8 * slot_of[a]);  // this accumulator's chunk is ready to drain
-              const int next = spare;
-              spare = slot_of[a];
-              slot_of[a] = next;
+            if (!S::template chunk_ends<CS>(a, kb, nkb)) continue;
+            if (S::owner(a) == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);  // chunk ready to drain
+            const uint32_t par = ring.rotate(a);
+            if (S::owner(a) == me) {
+              wait_par[a] = par;
               need_acquire[a] = true;
               fresh[a] = true;
             }
@@ -296,7 +388,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
       }
-      // all MMAs issued by this thread must be complete before TMEM is released
+      // all MMAs issued by both threads must be complete before TMEM is released
       tc_commit(final_bar);
       bounded_wait(final_bar, 0, P.timeout_ns);
     }
@@ -304,14 +396,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const int quad = warp & 3;       // TMEM lanes 32*quad .. 32*quad+31 (hardware lane quadrant)
     const int half = warp >> 2;      // column half of the tile: 0..63 or 64..127
-    int slot_of[3] = {0, 1, 2};
-    int spare = S::NACC;
+    SlotRing<S::NACC> ring;
+    ring.init();
     uint32_t drain_parity = 0;  // bit s: parity of the number of drains of slot s
     bool ok = true;
     UT acc[64];
     for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
       int mt, nt;
-      tile_coords(t, P.num_m_tiles, P.num_n_tiles, mt, nt);
+      tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
       const int64_t row = static_cast<int64_t>(mt) * BM + quad * 32 + lane;
       const int64_t col0 = static_cast<int64_t>(nt) * BN + half * 64;
       CT* crow = static_cast<CT*>(P.C) + row * P.ldc + col0;
@@ -340,11 +432,27 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 #pragma unroll
         for (int c = 0; c < 64; ++c) acc[c] = (row_ok && col0 + c < P.n) ? static_cast<UT>(crow[c]) : UT(0);
       }
+      {
+        // warm L2 with this thread's C row segment of the next tile it will process
+        const int tn = t + gridDim.x;
+        if (tn < total_tiles) {
+          int mn, nn;
+          tile_coords(tn, P.num_m_tiles, P.num_n_tiles, P.group_m, mn, nn);
+          const int64_t prow = static_cast<int64_t>(mn) * BM + quad * 32 + lane;
+          const int64_t pcol = static_cast<int64_t>(nn) * BN + half * 64;
+          if (prow < P.m && pcol < P.n) {
+            const CT* pc = static_cast<const CT*>(P.C) + prow * P.ldc + pcol;
+            const int64_t cols = min(static_cast<int64_t>(64), P.n - pcol);
+            for (int64_t c = 0; c < cols; c += 128 / static_cast<int64_t>(sizeof(CT)))
+              asm volatile("prefetch.global.L2 [%0];" ::"l"(pc + c));
+          }
+        }
+      }
       for (int kb = 0; kb < nkb && ok; ++kb) {
 #pragma unroll
         for (int a = 0; a < S::NACC; ++a) {
-          if (!chunk_ends<NL>(a, kb, nkb)) continue;
-          const int s = slot_of[a];
+          if (!S::template chunk_ends<CS>(a, kb, nkb)) continue;
+          const int s = ring.slot_of[a];
           // every lane waits; the warp then decides together (tcgen05.ld needs a converged warp)
           const bool got = bounded_wait(sfull0 + 8 * s, (drain_parity >> s) & 1u, P.timeout_ns);
           if (!__all_sync(0xFFFFFFFFu, got)) {
@@ -373,9 +481,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(sempty0 + 8 * s);
-          const int next = spare;
-          spare = slot_of[a];
-          slot_of[a] = next;
+          ring.rotate(a);
         }
       }
       if (!ok) break;
@@ -402,7 +508,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 
   tc_fence_before();
   __syncthreads();
-  if (warp == MMA_WARP) {
+  if (warp == MMA_WARP0) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem_base, TMEM_COLS);
@@ -413,8 +519,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 
-template <int NL>
+template <int NL, int CS>
 cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
+  using G = Geom<NL>;
   CUtensorMap maps[4];
   const LimbPlanes* ops[2] = {&a.a, &a.b};
   for (int o = 0; o < 2; ++o) {
@@ -422,7 +529,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
       const void* base = ops[o]->plane[l < NL ? l : 0];
       if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
                                 static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
-                                o == 0 ? BM : BN, 128, why))
+                                o == 0 ? BM : BN, G::SWIZZLE, why))
         return cudaErrorInvalidValue;
     }
   }
@@ -437,15 +544,18 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
   const size_t esz = NL == 2 ? 8 : 4;
   P.c_vec = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && ((a.ldc * esz) % 16 == 0);
+  P.group_m = a.group_m > 0 ? a.group_m : 16;
+  P.hint_a = a.hint_a;
+  P.hint_b = a.hint_b;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
   const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
   const int grid = static_cast<int>(tiles < a.num_sms ? tiles : a.num_sms);
-  constexpr size_t smem = smem_bytes<NL>();
-  cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  constexpr size_t smem = G::SMEM;
+  cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NL, CS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  tc_gemm_kernel<NL><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], P);
+  tc_gemm_kernel<NL, CS><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], P);
   return cudaGetLastError();
 }
 
@@ -486,7 +596,11 @@ bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, ui
   return true;
 }
 
-cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why) { return launch<2>(args, s, why); }
-cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) { return launch<1>(args, s, why); }
+cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch<2, 2>(args, s, why) : launch<2, 1>(args, s, why);
+}
+cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch<1, 2>(args, s, why) : launch<1, 1>(args, s, why);
+}
 
 }  // namespace gemmi

@@ -33,6 +33,10 @@ struct TcGemmArgs {
   uint32_t* status;
   uint64_t timeout_ns;
   int num_sms;
+  int chunk_scale;  // 1: exact-sum chunks keep partial sums within 2^23; 2: within 2^24 (half the drains)
+  int group_m;   // tile raster band height (row tiles), 0 = default
+  int hint_a;    // L2 policy for A / B tile loads: 0 normal, 1 evict_last, 2 evict_first
+  int hint_b;
 };
 cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
@@ -40,7 +44,7 @@ cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why)
 // ---- skinny.cu: m <= 16 int16 GEMM streaming B once.
 struct SkinnyArgs {
   int64_t m, n, k;
-  const int16_t* A;
+  const int16_t* A;  // m x k, row-major, 16-byte aligned base, lda % 8 == 0
   int64_t lda;
   const int16_t* B;  // k x n, row-major, 16-byte aligned base, ldb % 8 == 0
   int64_t ldb;

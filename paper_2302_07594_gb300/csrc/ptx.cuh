@@ -59,15 +59,27 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait with a suspend-time hint: the thread sleeps in hardware until the phase completes or
+// about `hint_ns` nanoseconds pass, so waiting warps do not take issue slots from working ones.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits until the phase with parity `parity` of barrier `bar` has completed.
 // Returns false if that did not happen within `timeout_ns` nanoseconds.
 __device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 32; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
     if (global_timer_ns() - t0 > timeout_ns) return false;
   }
 }
@@ -145,15 +157,19 @@ __device__ __forceinline__ void tc_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[1
       : "r"(taddr));
 }
 
-// Shared-memory matrix descriptor for a K-major operand tile stored with the 128-byte
-// swizzle: rows of 128 bytes, 8-row core groups 1024 bytes apart (SBO = 1024).
-__device__ __forceinline__ uint64_t smem_desc_kmajor_sw128(uint32_t saddr) {
+// Shared-memory matrix descriptor for a K-major operand tile whose rows are SW bytes wide
+// (one swizzle span: 128 or 64) and stored with that swizzle by TMA; 8-row core groups are
+// 8 * SW bytes apart (stride byte offset).
+template <int SW>
+__device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t saddr) {
+  static_assert(SW == 128 || SW == 64, "swizzle span");
+  constexpr uint64_t layout = SW == 128 ? 2u : 4u;           // SWIZZLE_128B = 2, SWIZZLE_64B = 4
   uint64_t d = 0;
   d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);        // start address
-  d |= static_cast<uint64_t>(1u) << 16;                       // leading byte offset (unused for this layout)
-  d |= static_cast<uint64_t>((1024u >> 4) & 0x3FFFu) << 32;  // stride byte offset
+  d |= static_cast<uint64_t>(1u) << 16;                       // leading byte offset (unused for swizzled K-major)
+  d |= static_cast<uint64_t>(((8u * SW) >> 4) & 0x3FFFu) << 32;  // stride byte offset
   d |= static_cast<uint64_t>(1u) << 46;                       // descriptor version for tcgen05
-  d |= static_cast<uint64_t>(2u) << 61;                       // swizzle mode: 128 B
+  d |= layout << 61;                                          // swizzle mode
   return d;
 }
 

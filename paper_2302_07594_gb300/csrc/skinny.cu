@@ -6,24 +6,24 @@
 // large and two small dimensions (Section 2, IM2COL lowering).  This kernel is
 // built around the stream of B:
 //
-//   * B is cut into column blocks of 32 (64 bytes of int16 per row); each CTA
-//     owns one column block and a range of the reduction dimension, and a
-//     producer warp streams 128-row x 32-column tiles of it into a ring of
-//     shared-memory stages with 2-D TMA loads (64-byte swizzle);
-//   * eight consumer warps each take a 16-row slab of every stage, read it
-//     transposed with ldmatrix (so that it is the "A" operand of
-//     C^T = B^T A^T), split each int16 into 8-bit limbs
+//   * B is cut into column blocks of 256 (512 contiguous bytes of every row)
+//     and the reduction dimension into ranges, one (column block, range) per
+//     CTA, about one CTA per SM; a producer warp streams 32-row x 256-column
+//     stages of B (four 2-D TMA boxes, 128-byte swizzle) plus the matching
+//     32-column slice of A into a ring of shared-memory stages;
+//   * eight consumer warps each own 32 columns of the block.  Per 16-row step a
+//     warp reads its B slab transposed with ldmatrix (the "A" operand of
+//     C^T = B^T A^T), splits every int16 into 8-bit limbs
 //         b = 256*hi + lo,  hi = b >> 8 in [-128,127],  lo = b & 255 in [0,255],
-//     exactly representable in fp16, and multiply on the tensor cores with
+//     exactly representable in fp16, and multiplies on the tensor cores with
 //     mma.sync m16n8k16 (fp16 in, fp32 accumulate) against the limbs of A;
 //   * three fp32 accumulator sets HH, X, LL hold exact integer sums while every
-//     partial sum stays below 2^23 (a warp's run of 128 reduction indices:
-//     128 * 255 * 255 < 2^23), then are drained into int64 registers as
-//     HH*2^16 + X*2^8 + LL;
-//   * the eight warps' int64 partials are summed in shared memory and added
-//     into C (plain read-modify-write when one CTA owns the whole reduction,
-//     64-bit atomic adds -- exact and order-independent modulo 2^64 -- when the
-//     reduction dimension is split across CTAs).
+//     partial sum stays below 2^23 (a run of 128 reduction indices:
+//     128 * 255 * 255 < 2^23 and 128 * 2 * 128 * 255 < 2^23), then are drained
+//     into int64 registers as HH*2^16 + X*2^8 + LL;
+//   * each warp adds its partial sums into C: a plain read-modify-write when
+//     one CTA owns the whole reduction range of its columns, 64-bit atomic adds
+//     (exact and order-independent modulo 2^64) when the range is split.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -33,39 +33,38 @@
 namespace gemmi {
 namespace {
 
-constexpr int JB = 32;          // columns of B per CTA
-constexpr int KS = 128;         // rows of B per stage
+constexpr int JB = 256;                 // columns of B per CTA
+constexpr int BOX_J = 64;               // columns per TMA box (128 bytes, the swizzle span)
+constexpr int NBOX = JB / BOX_J;        // 4 boxes per stage
+constexpr int KS = 32;                  // rows of B per stage (two 16-row mma steps)
 constexpr int STAGES = 8;
-constexpr int STAGE_BYTES = KS * JB * 2;  // 8 KB
-constexpr int NCONS = 8;        // consumer warps, one 16-row slab of a stage each
+constexpr int B_STAGE_BYTES = KS * JB * 2;       // 16 KB
+constexpr int A_ROWS = 16;
+constexpr int A_STAGE_BYTES = A_ROWS * KS * 2;   // 1 KB: 16 rows x 32 reduction indices of A
+constexpr int STAGE_BYTES = B_STAGE_BYTES + A_STAGE_BYTES;
+constexpr int NCONS = 8;                // consumer warps, 32 columns each
 constexpr int THREADS = (NCONS + 1) * 32;
-constexpr int DRAIN_EVERY = 8;  // stages per drain: 8 k-steps of 16 = 128 reduction indices per warp
+constexpr int DRAIN_EVERY = 4;          // stages per drain: 4 x 32 = 128 reduction indices
 constexpr uint32_t STATUS_TIMEOUT = 4;
 
 struct SkParams {
   int64_t m, n, k;
-  const int16_t* A;
-  int64_t lda;
   int64_t* C;
   int64_t ldc;
-  int64_t stages_per_cta;   // K range of one CTA, in stages
+  int64_t stages_per_cta;   // reduction range of one CTA, in stages
   int64_t total_stages;
   int atomic_out;
-  int a_vec;                // A rows 4-byte aligned: 32-bit fragment loads
   uint64_t timeout_ns;
   uint32_t* status;
 };
 
-template <int NT>
-constexpr size_t sk_smem() {
-  return 1024 + STAGES * STAGE_BYTES + static_cast<size_t>(NCONS) * (2 * NT * 4 * 32) * 8 + 8 * (2 * STAGES) + 16;
-}
+constexpr size_t sk_smem() { return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 8 * (2 * STAGES) + 16; }
 
 // int16 pair -> fp16 pairs of its high (signed) and low (unsigned) bytes, exactly.
-// 0x64xx as fp16 is 1024 + xx, so the byte is recovered by one subtraction.
+// 0x64xx as fp16 is 1024 + xx, so each byte is recovered by one subtraction.
 __device__ __forceinline__ void split_pair(uint32_t x, uint32_t& hi, uint32_t& lo) {
-  const uint32_t lo_bits = (x & 0x00FF00FFu) | 0x64006400u;                // 1024 + lo
-  const uint32_t hi_bits = ((x >> 8) & 0x00FF00FFu) ^ 0x64806480u;         // 1024 + (hi + 128)
+  const uint32_t lo_bits = (x & 0x00FF00FFu) | 0x64006400u;         // 1024 + lo
+  const uint32_t hi_bits = ((x >> 8) & 0x00FF00FFu) ^ 0x64806480u;  // 1024 + (hi + 128)
   const __half2 l = __hsub2(*reinterpret_cast<const __half2*>(&lo_bits), __half2half2(__ushort_as_half(0x6400)));
   const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&hi_bits), __half2half2(__ushort_as_half(0x6480)));
   lo = *reinterpret_cast<const uint32_t*>(&l);
@@ -85,14 +84,10 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
                : "r"(addr));
 }
 
-// Two consecutive reduction indices p, p+1 of row i of A as a packed int16 pair (zero outside).
-__device__ __forceinline__ uint32_t load_a_pair(const SkParams& P, int64_t i, int64_t p) {
-  if (i >= P.m || p >= P.k) return 0u;
-  const int16_t* row = P.A + i * P.lda;
-  if (P.a_vec && p + 1 < P.k) return __ldg(reinterpret_cast<const uint32_t*>(row + p));
-  const uint32_t v0 = static_cast<uint16_t>(__ldg(row + p));
-  const uint32_t v1 = (p + 1 < P.k) ? static_cast<uint16_t>(__ldg(row + p + 1)) : 0u;
-  return v0 | (v1 << 16);
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
 }
 
 __device__ __forceinline__ int32_t f2i(float f) {
@@ -103,12 +98,10 @@ __device__ __forceinline__ int32_t f2i(float f) {
 
 template <int NT>
 __global__ void __launch_bounds__(THREADS, 1)
-skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
+skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ CUtensorMap mapA, SkParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* red = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-  constexpr int RED_PER_WARP = 2 * NT * 4 * 32;
-  uint64_t* bars = red + NCONS * RED_PER_WARP;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * STAGES;
 
@@ -133,6 +126,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&mapB);
+      tma_prefetch_desc(&mapA);
       int64_t issued = 0;
       for (int64_t i = 0; i < nst; ++i) {
         const int s = static_cast<int>(i % STAGES);
@@ -141,59 +135,70 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
           report_status(P.status, STATUS_TIMEOUT, 11);
           break;
         }
-        mbar_arrive_expect_tx(full0 + 8 * s, STAGE_BYTES);
-        tma_load_2d(smem_u32(smem + s * STAGE_BYTES), &mapB, full0 + 8 * s, static_cast<int32_t>(j_base),
-                    static_cast<int32_t>((st_begin + i) * KS));
+        const uint32_t fb = full0 + 8 * s;
+        const uint32_t dst = smem_u32(smem + s * STAGE_BYTES);
+        const int32_t krow = static_cast<int32_t>((st_begin + i) * KS);
+        mbar_arrive_expect_tx(fb, STAGE_BYTES);
+#pragma unroll
+        for (int b = 0; b < NBOX; ++b)
+          tma_load_2d(dst + b * (KS * BOX_J * 2), &mapB, fb, static_cast<int32_t>(j_base + b * BOX_J), krow);
+        tma_load_2d(dst + B_STAGE_BYTES, &mapA, fb, krow, 0);
         ++issued;
       }
       const int64_t first = issued > STAGES ? issued - STAGES : 0;
       for (int64_t i = first; i < issued; ++i)
         bounded_wait(full0 + 8 * static_cast<int>(i % STAGES), static_cast<uint32_t>((i / STAGES) & 1), P.timeout_ns);
     }
-  } else {
-    // ------------------------------------------------------------ consumers
-    const int g = lane >> 2;
-    const int t = lane & 3;
-    float hh[2][NT][4], xx[2][NT][4], ll[2][NT][4];
-    uint64_t acc[2][NT][4];
+    return;
+  }
+
+  // ------------------------------------------------------------ consumers
+  const int g = lane >> 2;
+  const int t = lane & 3;
+  float hh[2][NT][4], xx[2][NT][4], ll[2][NT][4];
+  uint64_t acc[2][NT][4];
 #pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
+  for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
+    for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
-          acc[mt][nt][c] = 0;
-        }
-    // ldmatrix row address pieces: lanes 0-7 matrix 0 (k 0-7, j 0-7), 8-15 matrix 1 (k 0-7, j 8-15),
-    // 16-23 matrix 2 (k 8-15, j 0-7), 24-31 matrix 3 (k 8-15, j 8-15)
-    const int mrow = warp * 16 + (lane & 7) + ((lane >> 4) << 3);  // row of the stage tile (k)
-    const int mchunk = (lane >> 3) & 1;                             // +8 columns (j)
-    bool ok = true;
-    for (int64_t i = 0; i < nst; ++i) {
-      const int s = static_cast<int>(i % STAGES);
-      const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
-      const bool got = bounded_wait(full0 + 8 * s, par, P.timeout_ns);
-      if (!__all_sync(0xFFFFFFFFu, got)) {
-        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 12);
-        ok = false;
-        break;
+      for (int c = 0; c < 4; ++c) {
+        hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
+        acc[mt][nt][c] = 0;
       }
-      const uint32_t tile = smem_u32(smem + s * STAGE_BYTES);
-      const int64_t k0 = (st_begin + i) * KS + warp * 16;  // first reduction index of this warp's slab
+  // this warp's 32 columns live in box warp/2, 16-byte chunks (warp%2)*4 .. +3 of each 128-byte row
+  const int box = warp >> 1;
+  const int chunk_base = (warp & 1) * 4;
+  // ldmatrix lanes: 0-7 rows 0-7 / cols 0-7, 8-15 rows 0-7 / cols 8-15, 16-23 rows 8-15 / cols 0-7,
+  // 24-31 rows 8-15 / cols 8-15 of a 16x16 (reduction x column) slab
+  const int lrow = (lane & 7) + ((lane >> 4) << 3);
+  const int lchunk = (lane >> 3) & 1;
+  for (int64_t i = 0; i < nst; ++i) {
+    const int s = static_cast<int>(i % STAGES);
+    const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
+    const bool got = bounded_wait(full0 + 8 * s, par, P.timeout_ns);
+    if (!__all_sync(0xFFFFFFFFu, got)) {
+      if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 12);
+      return;
+    }
+    const uint32_t bbox = smem_u32(smem + s * STAGE_BYTES) + box * (KS * BOX_J * 2);
+    const uint32_t abase = smem_u32(smem + s * STAGE_BYTES + B_STAGE_BYTES);  // [16 rows][32 indices] int16
+#pragma unroll
+    for (int ks = 0; ks < KS / 16; ++ks) {
       // A fragments (the mma's B operand: 16 reduction indices x 8 rows of A)
       uint32_t ahi[NT][2], alo[NT][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const int64_t row = nt * 8 + g;
-        split_pair(load_a_pair(P, row, k0 + 2 * t), ahi[nt][0], alo[nt][0]);
-        split_pair(load_a_pair(P, row, k0 + 2 * t + 8), ahi[nt][1], alo[nt][1]);
+        const uint32_t arow = abase + (nt * 8 + g) * (KS * 2) + (ks * 16 + 2 * t) * 2;
+        split_pair(lds32(arow), ahi[nt][0], alo[nt][0]);
+        split_pair(lds32(arow + 16), ahi[nt][1], alo[nt][1]);
       }
+      const int row = ks * 16 + lrow;
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt) {
-        // 64-byte swizzle: 16-byte chunk c of row r sits at chunk c ^ ((r >> 1) & 3)
-        const int chunk = mt * 2 + mchunk;
-        const uint32_t addr = tile + mrow * 64 + ((chunk ^ ((mrow >> 1) & 3)) << 4);
+        // 128-byte swizzle: 16-byte chunk c of row r is stored at chunk c ^ (r & 7)
+        const int chunk = chunk_base + mt * 2 + lchunk;
+        const uint32_t addr = bbox + row * 128 + ((chunk ^ (row & 7)) << 4);
         uint32_t b[4], bhi[4], blo[4];
         ldsm_x4_trans(addr, b);
 #pragma unroll
@@ -206,66 +211,62 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
           mma16816(ll[mt][nt], blo, alo[nt][0], alo[nt][1]);
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * s);
-      if ((i + 1) % DRAIN_EVERY == 0 || i + 1 == nst) {
-#pragma unroll
-        for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-              acc[mt][nt][c] += (static_cast<uint64_t>(static_cast<int64_t>(f2i(hh[mt][nt][c]))) << 16) +
-                                (static_cast<uint64_t>(static_cast<int64_t>(f2i(xx[mt][nt][c]))) << 8) +
-                                static_cast<uint64_t>(static_cast<int64_t>(f2i(ll[mt][nt][c])));
-              hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
-            }
-      }
     }
-    if (!__all_sync(0xFFFFFFFFu, ok)) ok = false;
-    // partials to shared memory: red[warp][((mt*NT + nt)*4 + c)*32 + lane]
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty0 + 8 * s);
+    if ((i + 1) % DRAIN_EVERY == 0 || i + 1 == nst) {
 #pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
+      for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
+        for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) red[warp * RED_PER_WARP + ((mt * NT + nt) * 4 + c) * 32 + lane] = acc[mt][nt][c];
-  }
-  __syncthreads();
-  // ------------------------------------------------------------ reduce the warps and update C
-  if (warp < NCONS) {
-    for (int idx = threadIdx.x; idx < RED_PER_WARP; idx += NCONS * 32) {
-      uint64_t sum = 0;
-#pragma unroll
-      for (int w = 0; w < NCONS; ++w) sum += red[w * RED_PER_WARP + idx];
-      const int ln = idx & 31;
-      const int c = (idx >> 5) & 3;
-      const int mn = idx >> 7;  // mt * NT + nt
-      const int mt = mn / NT, nt = mn % NT;
-      const int gg = ln >> 2, tt = ln & 3;
-      const int64_t i = nt * 8 + 2 * tt + (c & 1);             // row of C (n side of the mma)
-      const int64_t j = j_base + mt * 16 + gg + 8 * (c >> 1);  // column of C (m side of the mma)
-      if (i < P.m && j < P.n && nst > 0) {
-        unsigned long long* dst = reinterpret_cast<unsigned long long*>(P.C + i * P.ldc + j);
-        if (P.atomic_out) atomicAdd(dst, static_cast<unsigned long long>(sum));
-        else *dst = *dst + static_cast<unsigned long long>(sum);
-      }
+          for (int c = 0; c < 4; ++c) {
+            acc[mt][nt][c] += (static_cast<uint64_t>(static_cast<int64_t>(f2i(hh[mt][nt][c]))) << 16) +
+                              (static_cast<uint64_t>(static_cast<int64_t>(f2i(xx[mt][nt][c]))) << 8) +
+                              static_cast<uint64_t>(static_cast<int64_t>(f2i(ll[mt][nt][c])));
+            hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
+          }
     }
   }
+  if (nst == 0) return;
+  // C fragment (m16n8): c0 (row g, col 2t), c1 (g, 2t+1), c2 (g+8, 2t), c3 (g+8, 2t+1);
+  // the mma's rows are columns j of C, its columns are rows i of C.
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int64_t i = nt * 8 + 2 * t + (c & 1);
+        const int64_t j = j_base + warp * 32 + mt * 16 + g + 8 * (c >> 1);
+        if (i < P.m && j < P.n) {
+          unsigned long long* dst = reinterpret_cast<unsigned long long*>(P.C + i * P.ldc + j);
+          const unsigned long long v = static_cast<unsigned long long>(acc[mt][nt][c]);
+          if (P.atomic_out) atomicAdd(dst, v);
+          else *dst = *dst + v;
+        }
+      }
 }
 
 template <int NT>
 cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
-  CUtensorMap map;
-  if (!encode_tensor_map_2d(&map, 0, a.B, static_cast<uint64_t>(a.n), static_cast<uint64_t>(a.k),
-                            static_cast<uint64_t>(a.ldb) * 2, JB, KS, 64, why))
+  CUtensorMap mapB, mapA;
+  if (!encode_tensor_map_2d(&mapB, 0, a.B, static_cast<uint64_t>(a.n), static_cast<uint64_t>(a.k),
+                            static_cast<uint64_t>(a.ldb) * 2, BOX_J, KS, 128, why))
+    return cudaErrorInvalidValue;
+  if (!encode_tensor_map_2d(&mapA, 0, a.A, static_cast<uint64_t>(a.k), static_cast<uint64_t>(a.m),
+                            static_cast<uint64_t>(a.lda) * 2, KS, A_ROWS, 0, why))
     return cudaErrorInvalidValue;
   const int64_t nj = (a.n + JB - 1) / JB;
   const int64_t total_stages = (a.k + KS - 1) / KS;
   int64_t ksplit = a.ksplit;
   if (ksplit <= 0) {
-    // one CTA per column block when that already fills most SMs; else split the reduction
-    ksplit = nj * 4 >= static_cast<int64_t>(a.num_sms) * 3 ? 1 : (a.num_sms + nj - 1) / nj;
+    // about one CTA per SM: the reduction range is split across the CTAs of a column block
+    ksplit = a.num_sms / nj;
+    if (ksplit < 1) ksplit = 1;
+    // keep at least 4 stages (128 reduction indices) per CTA
+    const int64_t cap = total_stages / 4 > 0 ? total_stages / 4 : 1;
+    if (ksplit > cap) ksplit = cap;
   }
   if (ksplit > total_stages) ksplit = total_stages;
   if (ksplit < 1) ksplit = 1;
@@ -279,22 +280,19 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   P.m = a.m;
   P.n = a.n;
   P.k = a.k;
-  P.A = a.A;
-  P.lda = a.lda;
   P.C = a.C;
   P.ldc = a.ldc;
   P.stages_per_cta = per;
   P.total_stages = total_stages;
   P.atomic_out = ksplit > 1 ? 1 : 0;
-  P.a_vec = (reinterpret_cast<uintptr_t>(a.A) % 4 == 0) && (a.lda % 2 == 0);
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
-  constexpr size_t smem = sk_smem<NT>();
+  constexpr size_t smem = sk_smem();
   cudaError_t e = cudaFuncSetAttribute(skinny_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit));
-  skinny_kernel<NT><<<grid, THREADS, smem, s>>>(map, P);
+  skinny_kernel<NT><<<grid, THREADS, smem, s>>>(mapB, mapA, P);
   return cudaGetLastError();
 }
 

@@ -79,22 +79,35 @@ def test_i16_chunk_boundaries(gm, k):
 
 
 # ------------------------------------------------------------------ extreme and adversarial values
-EXTREMES = [(-32768, -32768), (32767, -32768), (32767, 32767), (32640, 32640), (-1, -1), (32640, -32768), (-129, 32767)]
+# 32640 has limbs (h, l) = (128, -128): every limb product is +-2^14, the largest possible.
+# +-32641 have limbs (128, -127) / (-128, 127): limb products 16384, -16256, 16129 -- odd and
+# within 2% of the largest, so a chunk's partial sums run up to just below its bound with the
+# low bit changing at every step, where any loss of precision in the accumulation would show.
+EXTREMES = [(-32768, -32768), (32767, -32768), (32767, 32767), (32640, 32640), (-1, -1), (32640, -32768),
+            (-129, 32767), (32641, 32641), (-32641, 32641), (-32641, -32641)]
+
+
+@pytest.fixture(params=[1, 2], ids=["chunks_2^23", "chunks_2^24"])
+def chunk_scale(request, gm):
+    old = gm.get_option(gm.OPT_TC_CHUNK_SCALE)
+    gm.set_option(gm.OPT_TC_CHUNK_SCALE, request.param)
+    yield request.param
+    gm.set_option(gm.OPT_TC_CHUNK_SCALE, old)
 
 
 @pytest.mark.parametrize("ab", EXTREMES)
 @pytest.mark.parametrize("m", [8, 200])
-def test_i16_constant_extremes(gm, ab, m):
+def test_i16_constant_extremes(gm, ab, m, chunk_scale):
     a, b = ab
-    n, k = 136, 1100
+    n, k = 136, 2600
     A = np.full((m, k), a, np.int16)
     B = np.full((k, n), b, np.int16)
     C = gi.uniform_int(9, (m, n), -(1 << 40), 1 << 40, np.int64)
-    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"constant {ab}")
+    assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"constant {ab} chunk scale {chunk_scale}")
 
 
 @pytest.mark.parametrize("m", [8, 160])
-def test_i16_near_fp32_exactness_limit(gm, m):
+def test_i16_near_fp32_exactness_limit(gm, m, chunk_scale):
     """Limb sums pushed toward the largest magnitudes a chunk allows, with odd low bits.
 
     32640 = 256*128 - 128 has limbs (h, l) = (128, -128): every limb product is
@@ -112,8 +125,8 @@ def test_i16_near_fp32_exactness_limit(gm, m):
     assert_same(run_gpu(gm, A, B, C), expected(A, B, C), "adversarial")
 
 
-def test_i8_extremes(gm):
-    for a, b in ((-128, -128), (127, -128), (127, 127)):
+def test_i8_extremes(gm, chunk_scale):
+    for a, b in ((-128, -128), (127, -128), (127, 127), (-127, -127)):
         A = np.full((140, 3000), a, np.int8)
         B = np.full((3000, 136), b, np.int8)
         C = gi.uniform_int(3, (140, 136), -(1 << 30), 1 << 30, np.int32)
@@ -309,3 +322,21 @@ def test_dtype_and_shape_errors(gm):
         gm.gemm_i16(torch.zeros((4, 5), dtype=torch.int16, device="cuda"),
                     torch.zeros((4, 4), dtype=torch.int16, device="cuda"),
                     torch.zeros((4, 4), dtype=torch.int64, device="cuda"))
+
+
+# ------------------------------------------------------------------ tuning options never change results
+@pytest.mark.parametrize("opts", [
+    {"OPT_TC_CHUNK_SCALE": 2}, {"OPT_TC_GROUP_M": 1}, {"OPT_TC_GROUP_M": 3, "OPT_TC_L2_HINTS": 1 | (2 << 2)},
+    {"OPT_TC_CHUNK_SCALE": 2, "OPT_TC_L2_HINTS": 2 | (1 << 2)},
+])
+def test_tc_options_keep_results(gm, opts):
+    saved = {k: gm.get_option(getattr(gm, k)) for k in opts}
+    try:
+        for k, v in opts.items():
+            gm.set_option(getattr(gm, k), v)
+        for kind, shape in (("i16", (300, 520, 1100)), ("i16", (129, 130, 4097)), ("i8", (260, 200, 2300))):
+            A, B, C = gi.random_problem(1000 + sum(shape), *shape, kind)
+            assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"{opts} {kind} {shape}")
+    finally:
+        for k, v in saved.items():
+            gm.set_option(getattr(gm, k), v)
