@@ -167,6 +167,35 @@ enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, 
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 
+/*
+ * gemm_i16_noalloc -- gemm_i16 for callers that must not allocate device memory.
+ * The paper has no counterpart; this entry point exists for deployment.  Some
+ * callers cannot allocate at call time: an inference server that has given all
+ * free device memory to its own pool at start-up (a cudaMalloc would fail), or a
+ * latency-critical loop that cannot absorb the device-wide synchronisation of
+ * growing or freeing a buffer.  This call allocates nothing: no cudaMalloc,
+ * cudaFree or allocating library routine.  Its scratch (the fp16 limb planes of
+ * A and B and a status word) is one fixed, file-scope device array of
+ * GEMMI_NOALLOC_SCRATCH_BYTES that every GPU loading the library holds until the
+ * process exits.
+ *
+ * Same operation, layout, pointer ownership (DEVICE pointers owned by the
+ * caller) and bit-exact result as gemm_i16, always on the tensor-core path,
+ * asynchronous on `stream` (a cudaStream_t as void*; NULL = legacy default stream).
+ * Limit: 4*(m+n)*roundup(k,8) + 256 <= GEMMI_NOALLOC_SCRATCH_BYTES (for m = n = k,
+ * up to about 2000); larger problems return GEMMI_EINVAL with a message saying so.
+ * The first call on a device looks up the array's device address (with that
+ * device current) and caches it; make that first call before any stream capture.
+ * Every call shares the one array: calls that overlap on the GPU (on different
+ * streams, or from several threads) race on it and must be serialised by the caller.
+ * Returns GEMMI_OK, GEMMI_EINVAL, GEMMI_ECUDA or GEMMI_EARCH.
+ */
+#define GEMMI_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
+int gemm_i16_noalloc(int64_t m, int64_t n, int64_t k,
+                     const int16_t* A, int64_t lda,
+                     const int16_t* B, int64_t ldb,
+                     int64_t* C, int64_t ldc, void* stream);
+
 /* Library version string. */
 const char* gemmi_version(void);
 

@@ -28,7 +28,9 @@ OPT_TC_CHUNK_SCALE, OPT_TC_GROUP_M, OPT_TC_L2_HINTS = 4, 5, 6
 EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
             "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_detail",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
-            "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version")
+            "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
+            "gemm_i16_noalloc")
+NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY = 0, 1, 2, 3
 
 _lib = None
@@ -58,7 +60,7 @@ def lib():
         for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host"):
             getattr(L, name).argtypes = core
             getattr(L, name).restype = ctypes.c_int
-        for name in ("gemm_i16_ex", "gemm_i8_ex"):
+        for name in ("gemm_i16_ex", "gemm_i8_ex", "gemm_i16_noalloc"):
             getattr(L, name).argtypes = core + [vp]
             getattr(L, name).restype = ctypes.c_int
         L.gemmi_set_stream.argtypes = [vp]
@@ -130,6 +132,17 @@ def gemm_i16(A, B, C, stream=None):
     """C += A @ B on the GPU: int16 A (m x k), int16 B (k x n), int64 C (m x n); exact modulo 2^64."""
     import torch
     return _torch_call("gemm_i16_ex", A, B, C, torch.int16, torch.int64, stream)
+
+
+def gemm_i16_noalloc(A, B, C, stream=None):
+    """gemm_i16 for callers that must not allocate device memory (see include/gemmi.h).
+
+    Uses the library's fixed scratch array instead of a workspace; problems needing more
+    than NOALLOC_SCRATCH_BYTES of limb planes raise GemmiError (EINVAL).  Calls that overlap
+    on the GPU share that array and must be serialised by the caller.
+    """
+    import torch
+    return _torch_call("gemm_i16_noalloc", A, B, C, torch.int16, torch.int64, stream)
 
 
 def gemm_i8(A, B, C, stream=None):

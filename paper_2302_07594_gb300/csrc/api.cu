@@ -412,6 +412,8 @@ __global__ void wait_probe_kernel(uint32_t* status, uint64_t timeout_ns) {
 }  // namespace
 
 namespace gemmi {
+void record_error(const char* msg) { t_error = msg; }
+
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s) {
   wait_probe_kernel<<<1, 32, 0, s>>>(status, timeout_ns);
   return cudaGetLastError();

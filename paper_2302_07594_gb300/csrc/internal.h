@@ -57,6 +57,9 @@ struct SkinnyArgs {
 };
 cudaError_t skinny_gemm_i16(const SkinnyArgs& args, cudaStream_t s, const char** why);
 
+// ---- error text of the calling thread, as returned by gemmi_last_error().
+void record_error(const char* msg);
+
 // ---- selftest of the bounded wait.
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
 
