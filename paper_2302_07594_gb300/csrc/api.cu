@@ -75,9 +75,12 @@ cudaEvent_t timer_event(KernelTimer& t) {
   return e;
 }
 
-// Records the start event of a timed launch (returns null when timing is off).
+bool is_capturing(cudaStream_t s);
+
+// Records the start event of a timed launch (returns null when timing is off or the stream is
+// being captured: an event recorded into a graph cannot be timed from the host).
 cudaEvent_t timer_begin(int kind, cudaStream_t s) {
-  if (!g_timing) return nullptr;
+  if (!g_timing || is_capturing(s)) return nullptr;
   cudaEvent_t e = timer_event(g_timers[kind]);
   cudaEventRecord(e, s);
   return e;
@@ -161,9 +164,21 @@ int ensure_buffer(void** buf, size_t* have, size_t bytes) {
   return GEMMI_OK;
 }
 
-// Orders this call's use of the workspace after the previous call's (which may be on another stream).
+bool is_capturing(cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &st) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return st != cudaStreamCaptureStatusNone;
+}
+
+// Orders this call's use of the workspace after the previous call's (which may be on another
+// stream).  Inside a stream capture the library records and waits on no event of its own: the
+// captured graph orders its nodes, and ordering graph launches against other work that uses
+// the same workspace is the caller's (as for any captured work that shares memory).
 int begin_workspace_use(DeviceState& d, cudaStream_t s) {
-  if (d.used && d.last_stream != s) {
+  if (d.used && d.last_stream != s && !is_capturing(s)) {
     cudaError_t e = cudaStreamWaitEvent(s, d.last_use, 0);
     if (e != cudaSuccess) return cuda_error(e, "cudaStreamWaitEvent");
   }
@@ -171,6 +186,7 @@ int begin_workspace_use(DeviceState& d, cudaStream_t s) {
 }
 
 int end_workspace_use(DeviceState& d, cudaStream_t s) {
+  if (is_capturing(s)) return GEMMI_OK;  // the event would belong to the graph, not to the stream
   cudaError_t e = cudaEventRecord(d.last_use, s);
   if (e != cudaSuccess) return cuda_error(e, "cudaEventRecord");
   d.last_stream = s;
@@ -269,9 +285,10 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
 
 int run_skinny(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
                int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s) {
-  // TMA needs 16-byte aligned row starts; operands that do not have them are re-pitched into the workspace
+  // TMA needs 16-byte aligned row starts of B; a B without them is re-pitched into the workspace
+  // (A is read with plain loads)
   const bool b_ok = reinterpret_cast<uintptr_t>(B) % 16 == 0 && (ldb * 2) % 16 == 0;
-  const bool a_ok = reinterpret_cast<uintptr_t>(A) % 16 == 0 && (lda * 2) % 16 == 0;
+  const bool a_ok = true;
   const int16_t* Bs = B;
   const int16_t* As = A;
   int64_t ldbs = ldb, ldas = lda;

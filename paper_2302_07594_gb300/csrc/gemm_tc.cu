@@ -552,9 +552,16 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
   const int grid = static_cast<int>(tiles < a.num_sms ? tiles : a.num_sms);
   constexpr size_t smem = G::SMEM;
-  cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NL, CS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
+  // the shared-memory opt-in is set once per device for this kernel
+  static bool attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64 || !attr_done[dev]) {
+    const cudaError_t attr = cudaFuncSetAttribute(tc_gemm_kernel<NL, CS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  static_cast<int>(smem));
+    if (attr != cudaSuccess) return attr;
+    if (dev >= 0 && dev < 64) attr_done[dev] = true;
+  }
   tc_gemm_kernel<NL, CS><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], P);
   return cudaGetLastError();
 }

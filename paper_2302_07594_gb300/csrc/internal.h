@@ -44,7 +44,7 @@ cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why)
 // ---- skinny.cu: m <= 16 int16 GEMM streaming B once.
 struct SkinnyArgs {
   int64_t m, n, k;
-  const int16_t* A;  // m x k, row-major, 16-byte aligned base, lda % 8 == 0
+  const int16_t* A;  // m x k, row-major (any alignment)
   int64_t lda;
   const int16_t* B;  // k x n, row-major, 16-byte aligned base, ldb % 8 == 0
   int64_t ldb;

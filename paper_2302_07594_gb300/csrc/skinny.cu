@@ -9,9 +9,13 @@
 //   * B is cut into column blocks of 256 (512 contiguous bytes of every row)
 //     and the reduction dimension into ranges, one (column block, range) per
 //     CTA, about one CTA per SM; a producer warp streams 32-row x 256-column
-//     stages of B (four 2-D TMA boxes, 128-byte swizzle) plus the matching
-//     32-column slice of A into a ring of shared-memory stages;
-//   * eight consumer warps each own 32 columns of the block.  Per 16-row step a
+//     stages of B (four 2-D TMA boxes, 128-byte swizzle) into a ring of
+//     shared-memory stages.  The CTA's slice of A (m <= 16 rows, at most 1024
+//     reduction indices) is split into fp16 limbs once, into shared memory, when
+//     the CTA starts, so the inner loop converts only B;
+//   * sixteen consumer warps each own 16 columns of the block (four warps per
+//     scheduler, so the latencies of one warp's dependent ldmatrix / mma chains
+//     are covered by the others).  Per 16-row step a
 //     warp reads its B slab transposed with ldmatrix (the "A" operand of
 //     C^T = B^T A^T), splits every int16 into 8-bit limbs
 //         b = 256*hi + lo,  hi = b >> 8 in [-128,127],  lo = b & 255 in [0,255],
@@ -38,17 +42,21 @@ constexpr int BOX_J = 64;               // columns per TMA box (128 bytes, the s
 constexpr int NBOX = JB / BOX_J;        // 4 boxes per stage
 constexpr int KS = 32;                  // rows of B per stage (two 16-row mma steps)
 constexpr int STAGES = 8;
-constexpr int B_STAGE_BYTES = KS * JB * 2;       // 16 KB
+constexpr int STAGE_BYTES = KS * JB * 2;         // 16 KB of B per stage
 constexpr int A_ROWS = 16;
-constexpr int A_STAGE_BYTES = A_ROWS * KS * 2;   // 1 KB: 16 rows x 32 reduction indices of A
-constexpr int STAGE_BYTES = B_STAGE_BYTES + A_STAGE_BYTES;
-constexpr int NCONS = 8;                // consumer warps, 32 columns each
+constexpr int KMAX_CTA = 1024;                   // reduction indices per CTA (bounds the A limbs in smem)
+constexpr int A_PAIRS = KMAX_CTA / 2;            // packed fp16 pairs per A row
+constexpr int A_STRIDE = A_PAIRS + 4;            // words per A limb row (+4 words: conflict-free fragment reads)
+constexpr int A_LIMB_BYTES = A_ROWS * A_STRIDE * 4;  // one limb (hi or lo) of the CTA's A slice
+constexpr int NCONS = 16;               // consumer warps, 16 columns (one m16 tile) each
 constexpr int THREADS = (NCONS + 1) * 32;
 constexpr int DRAIN_EVERY = 4;          // stages per drain: 4 x 32 = 128 reduction indices
 constexpr uint32_t STATUS_TIMEOUT = 4;
 
 struct SkParams {
   int64_t m, n, k;
+  const int16_t* A;
+  int64_t lda;
   int64_t* C;
   int64_t ldc;
   int64_t stages_per_cta;   // reduction range of one CTA, in stages
@@ -58,7 +66,10 @@ struct SkParams {
   uint32_t* status;
 };
 
-constexpr size_t sk_smem() { return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 8 * (2 * STAGES) + 16; }
+constexpr size_t sk_smem() {
+  return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * A_LIMB_BYTES + 8 * (2 * STAGES) + 16;
+}
+static_assert(sk_smem() <= 227 * 1024, "shared memory budget");
 
 // int16 pair -> fp16 pairs of its high (signed) and low (unsigned) bytes, exactly.
 // 0x64xx as fp16 is 1024 + xx, so each byte is recovered by one subtraction.
@@ -98,10 +109,12 @@ __device__ __forceinline__ int32_t f2i(float f) {
 
 template <int NT>
 __global__ void __launch_bounds__(THREADS, 1)
-skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ CUtensorMap mapA, SkParams P) {
+skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint32_t* a_hi = reinterpret_cast<uint32_t*>(smem + STAGES * STAGE_BYTES);  // [16 rows][A_STRIDE] fp16 pairs
+  uint32_t* a_lo = a_hi + A_ROWS * A_STRIDE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(a_lo + A_ROWS * A_STRIDE);
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * STAGES;
 
@@ -126,7 +139,6 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&mapB);
-      tma_prefetch_desc(&mapA);
       int64_t issued = 0;
       for (int64_t i = 0; i < nst; ++i) {
         const int s = static_cast<int>(i % STAGES);
@@ -142,7 +154,6 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
 #pragma unroll
         for (int b = 0; b < NBOX; ++b)
           tma_load_2d(dst + b * (KS * BOX_J * 2), &mapB, fb, static_cast<int32_t>(j_base + b * BOX_J), krow);
-        tma_load_2d(dst + B_STAGE_BYTES, &mapA, fb, krow, 0);
         ++issued;
       }
       const int64_t first = issued > STAGES ? issued - STAGES : 0;
@@ -153,12 +164,36 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
   }
 
   // ------------------------------------------------------------ consumers
+  // Split this CTA's slice of A once: rows 0..15 (zero beyond m), reduction indices
+  // k0 .. k0 + KS*nst (zero beyond k), as packed fp16 pairs of the high and low limbs.
+  {
+    const int64_t k0 = st_begin * KS;
+    const int pairs = static_cast<int>(nst * KS / 2);
+    for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
+      const int row = idx / pairs;
+      const int kp = idx - row * pairs;
+      const int64_t k = k0 + 2 * kp;
+      uint32_t x = 0;
+      if (row < P.m) {
+        const int16_t* src = P.A + row * P.lda + k;
+        const uint32_t v0 = k < P.k ? static_cast<uint16_t>(src[0]) : 0u;
+        const uint32_t v1 = k + 1 < P.k ? static_cast<uint16_t>(src[1]) : 0u;
+        x = v0 | (v1 << 16);
+      }
+      uint32_t hi, lo;
+      split_pair(x, hi, lo);
+      a_hi[row * A_STRIDE + kp] = hi;
+      a_lo[row * A_STRIDE + kp] = lo;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // consumer warps only
+  }
   const int g = lane >> 2;
   const int t = lane & 3;
-  float hh[2][NT][4], xx[2][NT][4], ll[2][NT][4];
-  uint64_t acc[2][NT][4];
+  constexpr int MT = 1;  // m16 tiles (of 16 columns) per warp
+  float hh[MT][NT][4], xx[MT][NT][4], ll[MT][NT][4];
+  uint64_t acc[MT][NT][4];
 #pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
+  for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -166,13 +201,20 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
         hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
         acc[mt][nt][c] = 0;
       }
-  // this warp's 32 columns live in box warp/2, 16-byte chunks (warp%2)*4 .. +3 of each 128-byte row
-  const int box = warp >> 1;
-  const int chunk_base = (warp & 1) * 4;
+  // this warp's 16 columns live in box warp/4, 16-byte chunks (warp%4)*2 .. +1 of each 128-byte row
+  const int box = warp >> 2;
+  const int chunk_base = (warp & 3) * 2;
   // ldmatrix lanes: 0-7 rows 0-7 / cols 0-7, 8-15 rows 0-7 / cols 8-15, 16-23 rows 8-15 / cols 0-7,
   // 24-31 rows 8-15 / cols 8-15 of a 16x16 (reduction x column) slab
   const int lrow = (lane & 7) + ((lane >> 4) << 3);
   const int lchunk = (lane >> 3) & 1;
+  // 128-byte swizzle: 16-byte chunk c of row r is stored at chunk c ^ (r & 7); the rows a lane
+  // addresses differ by multiples of 16, so its swizzled offset inside a row never changes
+  uint32_t lane_off[MT];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt)
+    lane_off[mt] = box * (KS * BOX_J * 2) + lrow * 128 + (((chunk_base + mt * 2 + lchunk) ^ (lrow & 7)) << 4);
+  const uint32_t a_hi_s = smem_u32(a_hi), a_lo_s = smem_u32(a_lo);
   for (int64_t i = 0; i < nst; ++i) {
     const int s = static_cast<int>(i % STAGES);
     const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
@@ -181,26 +223,24 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
       if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 12);
       return;
     }
-    const uint32_t bbox = smem_u32(smem + s * STAGE_BYTES) + box * (KS * BOX_J * 2);
-    const uint32_t abase = smem_u32(smem + s * STAGE_BYTES + B_STAGE_BYTES);  // [16 rows][32 indices] int16
+    const uint32_t sbase = smem_u32(smem + s * STAGE_BYTES);
 #pragma unroll
     for (int ks = 0; ks < KS / 16; ++ks) {
-      // A fragments (the mma's B operand: 16 reduction indices x 8 rows of A)
+      // A fragments (the mma's B operand: 16 reduction indices x 8 rows of A), already split
       uint32_t ahi[NT][2], alo[NT][2];
+      const int kp = static_cast<int>(i) * (KS / 2) + ks * 8 + t;  // pair index of reduction index 2kp
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const uint32_t arow = abase + (nt * 8 + g) * (KS * 2) + (ks * 16 + 2 * t) * 2;
-        split_pair(lds32(arow), ahi[nt][0], alo[nt][0]);
-        split_pair(lds32(arow + 16), ahi[nt][1], alo[nt][1]);
+        const uint32_t off = static_cast<uint32_t>(((nt * 8 + g) * A_STRIDE + kp) * 4);
+        ahi[nt][0] = lds32(a_hi_s + off);
+        ahi[nt][1] = lds32(a_hi_s + off + 16);
+        alo[nt][0] = lds32(a_lo_s + off);
+        alo[nt][1] = lds32(a_lo_s + off + 16);
       }
-      const int row = ks * 16 + lrow;
 #pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        // 128-byte swizzle: 16-byte chunk c of row r is stored at chunk c ^ (r & 7)
-        const int chunk = chunk_base + mt * 2 + lchunk;
-        const uint32_t addr = bbox + row * 128 + ((chunk ^ (row & 7)) << 4);
+      for (int mt = 0; mt < MT; ++mt) {
         uint32_t b[4], bhi[4], blo[4];
-        ldsm_x4_trans(addr, b);
+        ldsm_x4_trans(sbase + ks * (16 * 128) + lane_off[mt], b);
 #pragma unroll
         for (int q = 0; q < 4; ++q) split_pair(b[q], bhi[q], blo[q]);
 #pragma unroll
@@ -216,7 +256,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
     if (lane == 0) mbar_arrive(empty0 + 8 * s);
     if ((i + 1) % DRAIN_EVERY == 0 || i + 1 == nst) {
 #pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
+      for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -232,13 +272,13 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
   // C fragment (m16n8): c0 (row g, col 2t), c1 (g, 2t+1), c2 (g+8, 2t), c3 (g+8, 2t+1);
   // the mma's rows are columns j of C, its columns are rows i of C.
 #pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
+  for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const int64_t i = nt * 8 + 2 * t + (c & 1);
-        const int64_t j = j_base + warp * 32 + mt * 16 + g + 8 * (c >> 1);
+        const int64_t j = j_base + warp * (16 * MT) + mt * 16 + g + 8 * (c >> 1);
         if (i < P.m && j < P.n) {
           unsigned long long* dst = reinterpret_cast<unsigned long long*>(P.C + i * P.ldc + j);
           const unsigned long long v = static_cast<unsigned long long>(acc[mt][nt][c]);
@@ -250,12 +290,9 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, const __grid_constant__ 
 
 template <int NT>
 cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
-  CUtensorMap mapB, mapA;
+  CUtensorMap mapB;
   if (!encode_tensor_map_2d(&mapB, 0, a.B, static_cast<uint64_t>(a.n), static_cast<uint64_t>(a.k),
                             static_cast<uint64_t>(a.ldb) * 2, BOX_J, KS, 128, why))
-    return cudaErrorInvalidValue;
-  if (!encode_tensor_map_2d(&mapA, 0, a.A, static_cast<uint64_t>(a.k), static_cast<uint64_t>(a.m),
-                            static_cast<uint64_t>(a.lda) * 2, KS, A_ROWS, 0, why))
     return cudaErrorInvalidValue;
   const int64_t nj = (a.n + JB - 1) / JB;
   const int64_t total_stages = (a.k + KS - 1) / KS;
@@ -268,6 +305,9 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
     const int64_t cap = total_stages / 4 > 0 ? total_stages / 4 : 1;
     if (ksplit > cap) ksplit = cap;
   }
+  // at most KMAX_CTA reduction indices per CTA: its A limbs must fit in shared memory
+  const int64_t min_split = (total_stages + (KMAX_CTA / KS) - 1) / (KMAX_CTA / KS);
+  if (ksplit < min_split) ksplit = min_split;
   if (ksplit > total_stages) ksplit = total_stages;
   if (ksplit < 1) ksplit = 1;
   const int64_t per = (total_stages + ksplit - 1) / ksplit;
@@ -280,6 +320,8 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   P.m = a.m;
   P.n = a.n;
   P.k = a.k;
+  P.A = a.A;
+  P.lda = a.lda;
   P.C = a.C;
   P.ldc = a.ldc;
   P.stages_per_cta = per;
@@ -288,11 +330,18 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
   constexpr size_t smem = sk_smem();
-  cudaError_t e = cudaFuncSetAttribute(skinny_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
+  // the shared-memory opt-in is set once per device for this kernel
+  static bool attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64 || !attr_done[dev]) {
+    const cudaError_t attr = cudaFuncSetAttribute(skinny_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  static_cast<int>(smem));
+    if (attr != cudaSuccess) return attr;
+    if (dev >= 0 && dev < 64) attr_done[dev] = true;
+  }
   dim3 grid(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit));
-  skinny_kernel<NT><<<grid, THREADS, smem, s>>>(mapB, mapA, P);
+  skinny_kernel<NT><<<grid, THREADS, smem, s>>>(mapB, P);
   return cudaGetLastError();
 }
 

@@ -340,3 +340,27 @@ def test_tc_options_keep_results(gm, opts):
     finally:
         for k, v in saved.items():
             gm.set_option(getattr(gm, k), v)
+
+
+def test_calls_captured_in_a_cuda_graph(gm):
+    """Calls captured into a CUDA graph replay exactly, and uncaptured calls still work afterwards."""
+    s = torch.cuda.Stream()
+    for kind, shape in (("i16", (300, 260, 700)), ("i16", (8, 1000, 900)), ("i8", (200, 130, 600))):
+        A, B, C = gi.random_problem(1100 + sum(shape), *shape, kind)
+        dA, dB = torch.from_numpy(A).cuda(), torch.from_numpy(B).cuda()
+        dC = torch.from_numpy(C).cuda()
+        fn = gm.gemm_i16 if kind == "i16" else gm.gemm_i8
+        with torch.cuda.stream(s):
+            fn(dA, dB, torch.from_numpy(C).cuda())  # warm-up outside the capture (workspace growth)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            fn(dA, dB, dC)
+        dC.copy_(torch.from_numpy(C).cuda())
+        g.replay()
+        g.replay()
+        torch.cuda.synchronize()
+        exp = expected(A, B, C)
+        oracle.gemm(A, B, exp)
+        assert_same(dC.cpu().numpy(), exp, f"graph x2 {kind} {shape}")
+        assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"uncaptured after graph {kind} {shape}")
