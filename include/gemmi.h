@@ -157,7 +157,7 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  * gemmi_kernel_time() waits for the recorded events and returns the summed
  * device time (milliseconds) and the number of timed launches of one kernel.
  * gemmi_kernel_timing(0|1) switches recording and resets the sums.
- *   GEMMI_KERNEL_SPLIT   : the limb split / conversion of A and B (one timed pair per call)
+ *   GEMMI_KERNEL_SPLIT   : the limb split / conversion of A and B (one launch per call)
  *   GEMMI_KERNEL_TC_I16  : the tcgen05 int16 GEMM kernel
  *   GEMMI_KERNEL_TC_I8   : the tcgen05 int8 GEMM kernel
  *   GEMMI_KERNEL_SKINNY  : the skinny-M int16 kernel

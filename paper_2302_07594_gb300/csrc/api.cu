@@ -251,11 +251,9 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   cudaError_t e;
   cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
   if (nl == 2) {
-    e = gemmi::split_rows_i16(static_cast<const int16_t*>(A), lda, m, k, pa, s);
-    if (e == cudaSuccess) e = gemmi::split_cols_i16(static_cast<const int16_t*>(B), ldb, k, n, pb, s);
+    e = gemmi::split_i16(static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb, m, n, k, pa, pb, s);
   } else {
-    e = gemmi::convert_rows_i8(static_cast<const int8_t*>(A), lda, m, k, pa, s);
-    if (e == cudaSuccess) e = gemmi::convert_cols_i8(static_cast<const int8_t*>(B), ldb, k, n, pb, s);
+    e = gemmi::convert_i8(static_cast<const int8_t*>(A), lda, static_cast<const int8_t*>(B), ldb, m, n, k, pa, pb, s);
   }
   timer_end(GEMMI_KERNEL_SPLIT, t0, s);
   if (e != cudaSuccess) return cuda_error(e, "limb split launch");

@@ -18,10 +18,11 @@ struct LimbPlanes {
 // ---- split.cu: operands -> fp16 limb planes (K-major).
 // int16: two centred 8-bit limbs, a = 256*h + l, h in [-128,128], l in [-128,127].
 // int8: one plane holding the value itself.
-cudaError_t split_rows_i16(const int16_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s);
-cudaError_t split_cols_i16(const int16_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s);
-cudaError_t convert_rows_i8(const int8_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s);
-cudaError_t convert_cols_i8(const int8_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s);
+// One launch converts both operands: A (m x k, lda) -> pa (rows m), B (k x n, ldb) -> pb (rows n).
+cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s);
+cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s);
 
 // ---- gemm_tc.cu: tcgen05 GEMM on limb planes, C (int64 for NL=2, int32 for NL=1) += combine(limb products).
 struct TcGemmArgs {

@@ -110,8 +110,7 @@ extern "C" int gemm_i16_noalloc(int64_t m, int64_t n, int64_t k, const int16_t* 
   gemmi::LimbPlanes pb{{planes + 2 * a_plane, planes + 2 * a_plane + b_plane}, n, pitch};
   // every plane byte the GEMM reads is written here first (pitch padding included), so nothing
   // left over from an earlier call is ever read
-  e = gemmi::split_rows_i16(A, lda, m, k, pa, s);
-  if (e == cudaSuccess) e = gemmi::split_cols_i16(B, ldb, k, n, pb, s);
+  e = gemmi::split_i16(A, lda, B, ldb, m, n, k, pa, pb, s);
   if (e != cudaSuccess) return fail(GEMMI_ECUDA, std::string("limb split launch: ") + cudaGetErrorString(e));
   gemmi::TcGemmArgs ta;
   ta.m = m;

@@ -13,6 +13,11 @@
 // its row-major layout; B (k x n, row-major) is transposed to n x k.  Plane
 // rows have a pitch that is a multiple of 8 elements (16 bytes), which the TMA
 // tensor maps require.  Pitch columns at and beyond k are written as zero.
+//
+// One launch converts both operands: the first blocks of the grid stream A
+// (16-byte loads, 2 x 16-byte stores per 8 elements), the rest transpose B in
+// 64 x 64 tiles through shared memory (16-byte loads and stores on both sides).
+// The kernel is bound by HBM: per int16 element 2 bytes are read and 4 written.
 #include <cuda_fp16.h>
 
 #include "internal.h"
@@ -30,124 +35,147 @@ __device__ __forceinline__ void limbs16(int a, __half& h, __half& l) {
   l = to_half_exact(lo);
 }
 
-// A: m x k (lda) -> planes m x pitch.  One thread per 8 consecutive elements of a row.
-template <typename T, int NL>
-__global__ void split_rows_kernel(const T* __restrict__ A, int64_t lda, int64_t m, int64_t k,
-                                  __half* __restrict__ P0, __half* __restrict__ P1, int64_t pitch, bool vec) {
-  const int64_t groups_per_row = pitch / 8;
-  const int64_t total = m * groups_per_row;
-  for (int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = g / groups_per_row;
-    const int64_t p0 = (g - r * groups_per_row) * 8;
-    const T* src = A + r * lda + p0;
-    int v[8];
-    if (vec && p0 + 8 <= k) {
-      if constexpr (sizeof(T) == 2) {
-        const uint4 u = *reinterpret_cast<const uint4*>(src);
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+template <typename T>
+struct Part {
+  const T* src;
+  int64_t ld;
+  int64_t rows;   // A: m;  B: k (rows of B)
+  int64_t cols;   // A: k;  B: n
+  __half* p0;
+  __half* p1;
+  int64_t pitch;  // plane row pitch (elements)
+  bool vec;       // 16-byte (int16) / 8-byte (int8) loads of 8 elements are aligned
+};
+
+template <typename T>
+__device__ __forceinline__ void load8(const T* src, bool vec, int64_t valid, int (&v)[8]) {
+  if (vec && valid >= 8) {
+    if constexpr (sizeof(T) == 2) {
+      const uint4 u = __ldg(reinterpret_cast<const uint4*>(src));
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          v[2 * i] = static_cast<int16_t>(w[i] & 0xFFFFu);
-          v[2 * i + 1] = static_cast<int16_t>(w[i] >> 16);
-        }
-      } else {
-        const uint2 u = *reinterpret_cast<const uint2*>(src);
-        const uint32_t w[2] = {u.x, u.y};
-#pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = static_cast<int8_t>((w[i / 4] >> (8 * (i % 4))) & 0xFFu);
+      for (int i = 0; i < 4; ++i) {
+        v[2 * i] = static_cast<int16_t>(w[i] & 0xFFFFu);
+        v[2 * i + 1] = static_cast<int16_t>(w[i] >> 16);
       }
     } else {
+      const uint2 u = __ldg(reinterpret_cast<const uint2*>(src));
+      const uint32_t w[2] = {u.x, u.y};
 #pragma unroll
-      for (int i = 0; i < 8; ++i) v[i] = (p0 + i < k) ? static_cast<int>(src[i]) : 0;
+      for (int i = 0; i < 8; ++i) v[i] = static_cast<int8_t>((w[i / 4] >> (8 * (i % 4))) & 0xFFu);
     }
-    __align__(16) __half h[8];
-    __align__(16) __half l[8];
+  } else {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      if constexpr (NL == 2) {
-        limbs16(v[i], h[i], l[i]);
+    for (int i = 0; i < 8; ++i) v[i] = (i < valid) ? static_cast<int>(src[i]) : 0;
+  }
+}
+
+template <int NL>
+__device__ __forceinline__ void store8(__half* p0, __half* p1, const int (&v)[8]) {
+  __align__(16) __half h[8];
+  __align__(16) __half l[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if constexpr (NL == 2) {
+      limbs16(v[i], h[i], l[i]);
+    } else {
+      h[i] = to_half_exact(v[i]);
+    }
+  }
+  *reinterpret_cast<uint4*>(p0) = *reinterpret_cast<const uint4*>(h);
+  if constexpr (NL == 2) *reinterpret_cast<uint4*>(p1) = *reinterpret_cast<const uint4*>(l);
+}
+
+constexpr int TT = 64;      // transpose tile edge
+constexpr int THREADS = 256;
+
+template <typename T, int NL>
+__global__ void __launch_bounds__(THREADS)
+split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_tiles) {
+  __shared__ int16_t tile[TT][TT + 8];
+  if (static_cast<int>(blockIdx.x) < a_blocks) {
+    // ---- A: m x k (lda) -> planes m x pitch, 8 consecutive elements per thread
+    const int64_t groups_per_row = a.pitch / 8;
+    const int64_t total = a.rows * groups_per_row;
+    for (int64_t g = blockIdx.x * static_cast<int64_t>(THREADS) + threadIdx.x; g < total;
+         g += static_cast<int64_t>(a_blocks) * THREADS) {
+      const int64_t r = g / groups_per_row;
+      const int64_t p0 = (g - r * groups_per_row) * 8;
+      int v[8];
+      load8(a.src + r * a.ld + p0, a.vec, a.cols - p0, v);
+      store8<NL>(a.p0 + r * a.pitch + p0, a.p1 + r * a.pitch + p0, v);
+    }
+    return;
+  }
+  // ---- B: k x n (ldb) -> planes n x pitch (transposed), 64 x 64 tiles
+  const int64_t nblk = gridDim.x - a_blocks;
+  for (int64_t t = blockIdx.x - a_blocks; t < b_tiles; t += nblk) {
+    const int64_t p_base = (t / b_tiles_j) * TT;  // reduction index = row of B
+    const int64_t j_base = (t % b_tiles_j) * TT;  // column of B
+#pragma unroll
+    for (int q = threadIdx.x; q < TT * TT / 8; q += THREADS) {
+      const int r = q >> 3;
+      const int c8 = (q & 7) * 8;
+      const int64_t p = p_base + r, j = j_base + c8;
+      int v[8];
+      if (p < b.rows) {
+        load8(b.src + p * b.ld + j, b.vec, b.cols - j, v);
       } else {
-        h[i] = to_half_exact(v[i]);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = 0;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) tile[r][c8 + i] = static_cast<int16_t>(v[i]);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = threadIdx.x; q < TT * TT / 8; q += THREADS) {
+      const int jj = q >> 3;
+      const int pc = (q & 7) * 8;
+      const int64_t j = j_base + jj, p = p_base + pc;
+      if (j < b.cols && p < b.pitch) {
+        int v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = tile[pc + i][jj];
+        store8<NL>(b.p0 + j * b.pitch + p, b.p1 + j * b.pitch + p, v);
       }
     }
-    *reinterpret_cast<uint4*>(P0 + r * pitch + p0) = *reinterpret_cast<const uint4*>(h);
-    if constexpr (NL == 2) *reinterpret_cast<uint4*>(P1 + r * pitch + p0) = *reinterpret_cast<const uint4*>(l);
+    __syncthreads();
   }
 }
 
-// B: k x n (ldb) -> planes n x pitch (transposed).  64 x 64 tiles through shared memory.
-constexpr int TT = 64;
-
 template <typename T, int NL>
-__global__ void split_cols_kernel(const T* __restrict__ B, int64_t ldb, int64_t k, int64_t n,
-                                  __half* __restrict__ P0, __half* __restrict__ P1, int64_t pitch) {
-  __shared__ int16_t tile[TT][TT + 2];
-  const int64_t p_base = static_cast<int64_t>(blockIdx.x) * TT;  // reduction index (rows of B)
-  const int64_t j_base = static_cast<int64_t>(blockIdx.y) * TT;  // column of B
-  const int tx = threadIdx.x % TT;
-  const int ty = threadIdx.x / TT;  // 0..3
-  for (int r = ty; r < TT; r += 4) {
-    const int64_t p = p_base + r, j = j_base + tx;
-    tile[r][tx] = (p < k && j < n) ? static_cast<int16_t>(B[p * ldb + j]) : static_cast<int16_t>(0);
-  }
-  __syncthreads();
-  // write: row j of the planes, columns p (zero beyond k up to the pitch)
-  for (int r = ty; r < TT; r += 4) {
-    const int64_t j = j_base + r, p = p_base + tx;
-    if (j < n && p < pitch) {
-      const int v = tile[tx][r];
-      if constexpr (NL == 2) {
-        __half h, l;
-        limbs16(v, h, l);
-        P0[j * pitch + p] = h;
-        P1[j * pitch + p] = l;
-      } else {
-        P0[j * pitch + p] = to_half_exact(v);
-      }
-    }
-  }
-}
-
-int grid_for(int64_t work, int threads) {
-  int64_t b = (work + threads - 1) / threads;
-  if (b < 1) b = 1;
-  if (b > 152 * 32) b = 152 * 32;
-  return static_cast<int>(b);
-}
-
-template <typename T, int NL>
-cudaError_t rows_impl(const T* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s) {
-  const bool vec = (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * static_cast<int64_t>(sizeof(T))) % 16 == 0);
-  const int64_t work = m * (out.pitch / 8);
-  split_rows_kernel<T, NL><<<grid_for(work, 256), 256, 0, s>>>(A, lda, m, k, static_cast<__half*>(out.plane[0]),
-                                                               static_cast<__half*>(out.plane[1]), out.pitch, vec);
-  return cudaGetLastError();
-}
-
-template <typename T, int NL>
-cudaError_t cols_impl(const T* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s) {
-  const int64_t gp = (out.pitch + TT - 1) / TT;  // cover the zero padding up to the pitch too
-  const int64_t gj = (n + TT - 1) / TT;
-  if (gp > 0x7FFFFFFF || gj > 65535) return cudaErrorInvalidValue;
-  dim3 grid(static_cast<unsigned>(gp), static_cast<unsigned>(gj));
-  split_cols_kernel<T, NL><<<grid, 256, 0, s>>>(B, ldb, k, n, static_cast<__half*>(out.plane[0]),
-                                                static_cast<__half*>(out.plane[1]), out.pitch);
+cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                   LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
+  constexpr int64_t esz = sizeof(T);
+  Part<T> a{A, lda, m, k, static_cast<__half*>(pa.plane[0]), static_cast<__half*>(pa.plane[NL - 1]), pa.pitch,
+            reinterpret_cast<uintptr_t>(A) % (8 * esz) == 0 && (lda * esz) % (8 * esz) == 0};
+  Part<T> b{B, ldb, k, n, static_cast<__half*>(pb.plane[0]), static_cast<__half*>(pb.plane[NL - 1]), pb.pitch,
+            reinterpret_cast<uintptr_t>(B) % (8 * esz) == 0 && (ldb * esz) % (8 * esz) == 0};
+  // A: about 8 elements per thread per grid-stride step; B: one 64 x 64 tile per block step
+  const int64_t a_work = m * (pa.pitch / 8);
+  int64_t a_blocks = (a_work + THREADS - 1) / THREADS;
+  if (a_blocks > 152 * 8) a_blocks = 152 * 8;
+  const int64_t tiles_p = (pb.pitch + TT - 1) / TT;  // cover the zero padding up to the pitch too
+  const int64_t tiles_j = (n + TT - 1) / TT;
+  const int64_t b_tiles = tiles_p * tiles_j;
+  int64_t b_blocks = b_tiles < 152 * 8 ? b_tiles : 152 * 8;
+  if (a_blocks < 1 || b_blocks < 1) return cudaErrorInvalidValue;
+  split_kernel<T, NL><<<static_cast<unsigned>(a_blocks + b_blocks), THREADS, 0, s>>>(
+      a, b, static_cast<int>(a_blocks), tiles_j, b_tiles);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t split_rows_i16(const int16_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s) {
-  return rows_impl<int16_t, 2>(A, lda, m, k, out, s);
+cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
+  return launch<int16_t, 2>(A, lda, B, ldb, m, n, k, pa, pb, s);
 }
-cudaError_t split_cols_i16(const int16_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s) {
-  return cols_impl<int16_t, 2>(B, ldb, k, n, out, s);
-}
-cudaError_t convert_rows_i8(const int8_t* A, int64_t lda, int64_t m, int64_t k, LimbPlanes out, cudaStream_t s) {
-  return rows_impl<int8_t, 1>(A, lda, m, k, out, s);
-}
-cudaError_t convert_cols_i8(const int8_t* B, int64_t ldb, int64_t k, int64_t n, LimbPlanes out, cudaStream_t s) {
-  return cols_impl<int8_t, 1>(B, ldb, k, n, out, s);
+
+cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
+  return launch<int8_t, 1>(A, lda, B, ldb, m, n, k, pa, pb, s);
 }
 
 }  // namespace gemmi
