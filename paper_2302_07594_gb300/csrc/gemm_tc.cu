@@ -55,7 +55,7 @@ namespace gemmi {
 namespace {
 
 constexpr int BM = 128;
-constexpr int BN = 128;
+constexpr int UMMA_N = 128;                  // N of one tcgen05.mma (an accumulator is 128 columns)
 constexpr int UMMA_K = 16;                   // K of one tcgen05.mma kind::f16
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int PRODUCER_WARP = 8;
@@ -76,11 +76,16 @@ struct Scheme;
 //   issuer 0 owns HH and LL (products 0, 3), issuer 1 owns X (products 1, 2): 8 MMAs each per K block.
 template <>
 struct Scheme<2> {
+  static constexpr int BN = 128;          // output tile width
   static constexpr int NACC = 3;
   static constexpr int NPROD = 4;
-  static constexpr int EMPTY_COUNT = 2;  // both issuers read every stage
+  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
+  static constexpr int COLS = 64;         // C columns per epilogue thread (two warps per lane quadrant)
+  static constexpr int DRAIN_WARPS = 8;   // every epilogue warp drains every accumulator (its 64 columns)
+  __device__ static constexpr bool drains(int, int) { return true; }
   __device__ static constexpr int a_limb(int p) { return p >> 1; }
   __device__ static constexpr int b_limb(int p) { return p & 1; }
+  __device__ static constexpr int b_row0(int) { return 0; }  // first row (output column) of the B tile used
   __device__ static constexpr int acc(int p, int) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
   __device__ static constexpr int issuer(int p, int) { return (p == 0 || p == 3) ? 0 : 1; }
   __device__ static constexpr int owner(int a) { return a == 1 ? 1 : 0; }
@@ -99,25 +104,29 @@ struct Scheme<2> {
   }
 };
 
-// int8: the value itself in one fp16 plane, one product per K block.  Two accumulators take the
-// even and the odd K blocks (issuer 0 and 1), each with chunks of 512*CS of its own reduction
-// indices, |sum| <= 512*CS * 2^14; their chunk ends are staggered by half a chunk.
+// int8: the value itself in one fp16 plane, one product per K block and output column half.
+// The tile is 128 x 256: each issuer owns one 128-column half (its own accumulator), so both
+// halves reuse the same A tile.  Chunks of 512*CS reduction indices, |sum| <= 512*CS * 2^14;
+// the two accumulators' chunk ends are staggered by half a chunk.
 template <>
 struct Scheme<1> {
+  static constexpr int BN = 256;
   static constexpr int NACC = 2;
-  static constexpr int NPROD = 1;
-  static constexpr int EMPTY_COUNT = 1;  // each stage is read by one issuer
+  static constexpr int NPROD = 2;         // product p: column half p
+  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
+  static constexpr int COLS = 128;        // C columns per epilogue thread: warp (quad, half) owns half h
+  static constexpr int DRAIN_WARPS = 4;   // an accumulator is drained by the four warps of its half
+  __device__ static constexpr bool drains(int half, int a) { return half == a; }
   __device__ static constexpr int a_limb(int) { return 0; }
   __device__ static constexpr int b_limb(int) { return 0; }
-  __device__ static constexpr int acc(int, int kb) { return kb & 1; }
-  __device__ static constexpr int issuer(int, int kb) { return kb & 1; }
+  __device__ static constexpr int b_row0(int p) { return p * 128; }
+  __device__ static constexpr int acc(int p, int) { return p; }
+  __device__ static constexpr int issuer(int p, int) { return p; }
   __device__ static constexpr int owner(int a) { return a; }
   __device__ static constexpr int shift(int) { return 0; }
   template <int CS>
   __device__ static bool chunk_ends(int a, int kb, int nkb) {
-    if ((kb & 1) != a) return false;
-    const int own = (kb >> 1) + 1;  // K blocks this accumulator has taken, including kb
-    return kb + 2 >= nkb || ((own * 64 + a * 256 * CS) % (512 * CS)) == 0;
+    return kb == nkb - 1 || (((kb + 1) * 64 + a * 256 * CS) % (512 * CS)) == 0;
   }
 };
 
@@ -158,8 +167,10 @@ struct SlotRing {
 constexpr int BK = 64;
 template <int NL>
 struct Geom {
-  static constexpr int TILE_BYTES = BM * BK * 2;          // one limb tile (BM == BN)
-  static constexpr int SB = 2 * NL * TILE_BYTES;          // one stage: NL tiles of A and of B
+  static constexpr int BN = Scheme<NL>::BN;
+  static constexpr int TILE_A = BM * BK * 2;              // one limb tile of A
+  static constexpr int TILE_B = BN * BK * 2;              // one limb tile of B
+  static constexpr int SB = NL * (TILE_A + TILE_B);       // one stage: NL tiles of A, then NL of B
   static constexpr int STAGES = (192 * 1024) / SB;        // 192 KB of stages
   static constexpr int SWIZZLE = BK * 2;                  // bytes per swizzled row
   static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + 8 * (2 * STAGES + 2 * NSLOT + 1) + 16;
@@ -223,7 +234,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   using G = Geom<NL>;
   constexpr int STAGES = G::STAGES;
   constexpr int SB = G::SB;
-  constexpr int TILE_BYTES = G::TILE_BYTES;
+  constexpr int TILE_A = G::TILE_A;
+  constexpr int TILE_B = G::TILE_B;
+  constexpr int BN = S::BN;
+  constexpr int COLS = S::COLS;
   // C element type and the unsigned type of the running sum (wrap-around is modular, never UB)
   using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
   using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
@@ -249,7 +263,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     }
     for (int s = 0; s < NSLOT; ++s) {
       mbar_init(sfull0 + 8 * s, 1);
-      mbar_init(sempty0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(sempty0 + 8 * s, S::DRAIN_WARPS);
     }
     mbar_init(final_bar, NISSUE);
     *abort_flag = 0;
@@ -297,9 +311,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           mbar_arrive_expect_tx(fb, SB);
           const uint32_t base = smem_u32(smem + stage * SB);
           tma_load_2d_hint(base, &mapA0, fb, kb * BK, mt * BM, P.hint_a, pol_a);
-          if (NL == 2) tma_load_2d_hint(base + TILE_BYTES, &mapA1, fb, kb * BK, mt * BM, P.hint_a, pol_a);
-          tma_load_2d_hint(base + NL * TILE_BYTES, &mapB0, fb, kb * BK, nt * BN, P.hint_b, pol_b);
-          if (NL == 2) tma_load_2d_hint(base + (NL + 1) * TILE_BYTES, &mapB1, fb, kb * BK, nt * BN, P.hint_b, pol_b);
+          if (NL == 2) tma_load_2d_hint(base + TILE_A, &mapA1, fb, kb * BK, mt * BM, P.hint_a, pol_a);
+          tma_load_2d_hint(base + NL * TILE_A, &mapB0, fb, kb * BK, nt * BN, P.hint_b, pol_b);
+          if (NL == 2) tma_load_2d_hint(base + NL * TILE_A + TILE_B, &mapB1, fb, kb * BK, nt * BN, P.hint_b, pol_b);
           ++issued;
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -316,7 +330,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     // ------------------------------------------------------------ MMA issuers (one thread each)
     const int me = warp - MMA_WARP0;
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+      constexpr uint32_t idesc = idesc_f16_f32(BM, UMMA_N);
       int stage = 0;
       uint32_t phase = 0;
       SlotRing<S::NACC> ring;
@@ -360,8 +374,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
                 tc_fence_after();
               }
               const uint32_t d = tmem_base + static_cast<uint32_t>(ring.slot_of[a] * SLOT_COLS);
-              const uint64_t adesc = smem_desc_kmajor<G::SWIZZLE>(base + S::a_limb(p) * TILE_BYTES);
-              const uint64_t bdesc = smem_desc_kmajor<G::SWIZZLE>(base + (NL + S::b_limb(p)) * TILE_BYTES);
+              const uint64_t adesc = smem_desc_kmajor<G::SWIZZLE>(base + S::a_limb(p) * TILE_A);
+              const uint64_t bdesc = smem_desc_kmajor<G::SWIZZLE>(base + NL * TILE_A + S::b_limb(p) * TILE_B +
+                                                                  S::b_row0(p) * (BK * 2));
 #pragma unroll
               for (int kk = 0; kk < BK / UMMA_K; ++kk) {
                 // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
@@ -395,32 +410,32 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const int quad = warp & 3;       // TMEM lanes 32*quad .. 32*quad+31 (hardware lane quadrant)
-    const int half = warp >> 2;      // column half of the tile: 0..63 or 64..127
+    const int half = warp >> 2;      // column half of the tile: columns half*COLS .. +COLS-1
     SlotRing<S::NACC> ring;
     ring.init();
     uint32_t drain_parity = 0;  // bit s: parity of the number of drains of slot s
     bool ok = true;
-    UT acc[64];
+    UT acc[COLS];
     for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
       int mt, nt;
       tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
       const int64_t row = static_cast<int64_t>(mt) * BM + quad * 32 + lane;
-      const int64_t col0 = static_cast<int64_t>(nt) * BN + half * 64;
+      const int64_t col0 = static_cast<int64_t>(nt) * BN + half * COLS;
       CT* crow = static_cast<CT*>(P.C) + row * P.ldc + col0;
       const bool row_ok = row < P.m;
-      const bool full_cols = col0 + 64 <= P.n;
+      const bool full_cols = col0 + COLS <= P.n;
       // running sum starts from C itself, so the tile ends with a plain store
       if (row_ok && full_cols && P.c_vec) {
         if constexpr (NL == 2) {
 #pragma unroll
-          for (int c = 0; c < 64; c += 2) {
+          for (int c = 0; c < COLS; c += 2) {
             const longlong2 v = *reinterpret_cast<const longlong2*>(crow + c);
             acc[c] = static_cast<UT>(v.x);
             acc[c + 1] = static_cast<UT>(v.y);
           }
         } else {
 #pragma unroll
-          for (int c = 0; c < 64; c += 4) {
+          for (int c = 0; c < COLS; c += 4) {
             const int4 v = *reinterpret_cast<const int4*>(crow + c);
             acc[c] = static_cast<UT>(v.x);
             acc[c + 1] = static_cast<UT>(v.y);
@@ -430,7 +445,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 64; ++c) acc[c] = (row_ok && col0 + c < P.n) ? static_cast<UT>(crow[c]) : UT(0);
+        for (int c = 0; c < COLS; ++c) acc[c] = (row_ok && col0 + c < P.n) ? static_cast<UT>(crow[c]) : UT(0);
       }
       {
         // warm L2 with this thread's C row segment of the next tile it will process
@@ -439,10 +454,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           int mn, nn;
           tile_coords(tn, P.num_m_tiles, P.num_n_tiles, P.group_m, mn, nn);
           const int64_t prow = static_cast<int64_t>(mn) * BM + quad * 32 + lane;
-          const int64_t pcol = static_cast<int64_t>(nn) * BN + half * 64;
+          const int64_t pcol = static_cast<int64_t>(nn) * BN + half * COLS;
           if (prow < P.m && pcol < P.n) {
             const CT* pc = static_cast<const CT*>(P.C) + prow * P.ldc + pcol;
-            const int64_t cols = min(static_cast<int64_t>(64), P.n - pcol);
+            const int64_t cols = min(static_cast<int64_t>(COLS), P.n - pcol);
             for (int64_t c = 0; c < cols; c += 128 / static_cast<int64_t>(sizeof(CT)))
               asm volatile("prefetch.global.L2 [%0];" ::"l"(pc + c));
           }
@@ -452,6 +467,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 #pragma unroll
         for (int a = 0; a < S::NACC; ++a) {
           if (!S::template chunk_ends<CS>(a, kb, nkb)) continue;
+          if (!S::drains(half, a)) {
+            // another half's accumulator: its chunk still completes one phase of this slot's full
+            // barrier (slots pass between accumulators), so keep that parity and the ring in step
+            drain_parity ^= 1u << ring.slot_of[a];
+            ring.rotate(a);
+            continue;
+          }
           const int s = ring.slot_of[a];
           // every lane waits; the warp then decides together (tcgen05.ld needs a converged warp)
           const bool got = bounded_wait(sfull0 + 8 * s, (drain_parity >> s) & 1u, P.timeout_ns);
@@ -463,10 +485,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           }
           drain_parity ^= 1u << s;
           tc_fence_after();
+          // this warp's columns of the accumulator: all 128 (int8, one accumulator per half)
+          // or its 64-column half (int16)
           const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                                 static_cast<uint32_t>(s * SLOT_COLS + half * 64);
+                                 static_cast<uint32_t>(s * SLOT_COLS + (NL == 2 ? half * COLS : 0));
 #pragma unroll
-          for (int c = 0; c < 64; c += 32) {
+          for (int c = 0; c < COLS; c += 32) {
             uint32_t r0[16], r1[16];
             tc_ld_32x32b_x16(taddr + c, r0);
             tc_ld_32x32b_x16(taddr + c + 16, r1);
@@ -488,19 +512,19 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       if (row_ok && full_cols && P.c_vec) {
         if constexpr (NL == 2) {
 #pragma unroll
-          for (int c = 0; c < 64; c += 2)
+          for (int c = 0; c < COLS; c += 2)
             *reinterpret_cast<longlong2*>(crow + c) =
                 make_longlong2(static_cast<long long>(acc[c]), static_cast<long long>(acc[c + 1]));
         } else {
 #pragma unroll
-          for (int c = 0; c < 64; c += 4)
+          for (int c = 0; c < COLS; c += 4)
             *reinterpret_cast<int4*>(crow + c) =
                 make_int4(static_cast<int>(acc[c]), static_cast<int>(acc[c + 1]), static_cast<int>(acc[c + 2]),
                           static_cast<int>(acc[c + 3]));
         }
       } else if (row_ok) {
 #pragma unroll
-        for (int c = 0; c < 64; ++c)
+        for (int c = 0; c < COLS; ++c)
           if (col0 + c < P.n) crow[c] = static_cast<CT>(acc[c]);
       }
     }
@@ -529,7 +553,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
       const void* base = ops[o]->plane[l < NL ? l : 0];
       if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
                                 static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
-                                o == 0 ? BM : BN, G::SWIZZLE, why))
+                                o == 0 ? BM : G::BN, G::SWIZZLE, why))
         return cudaErrorInvalidValue;
     }
   }
@@ -540,7 +564,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   P.C = a.C;
   P.ldc = a.ldc;
   P.num_m_tiles = static_cast<int>((a.m + BM - 1) / BM);
-  P.num_n_tiles = static_cast<int>((a.n + BN - 1) / BN);
+  P.num_n_tiles = static_cast<int>((a.n + G::BN - 1) / G::BN);
   P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
   const size_t esz = NL == 2 ? 8 : 4;
   P.c_vec = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && ((a.ldc * esz) % 16 == 0);
