@@ -99,6 +99,33 @@ int gemm_i8_host(int64_t m, int64_t n, int64_t k,
                  const int8_t* B, int64_t ldb,
                  int32_t* C, int64_t ldc);
 
+/*
+ * Weight pre-packing.  Section 5.1 of the paper keeps the weight operand packed,
+ * off-line, in fast memory, because a deployed model runs many inputs through
+ * the same weights; only the activations are packed at run time.  Here the
+ * weights are the B operand: gemmi_pack_b_* converts B (k x n, row-major,
+ * DEVICE pointer, only read) once into the library's internal limb planes,
+ * held in device memory the handle owns (allocated by this call), on `stream`.
+ * gemm_*_packed then computes C += A * B for any A (m x k) with that B,
+ * converting only A per call; the result is bit-identical to gemm_i16/gemm_i8.
+ * Packed GEMMs always take the tensor-core path (for m <= 16, gemm_i16 on the
+ * raw B streams fewer bytes).  The handle belongs to the device that was
+ * current when it was made; gemmi_packed_b_free() synchronises that device and
+ * frees it.  Errors as for gemm_i16 (a null handle or one of another device:
+ * GEMMI_EINVAL).
+ */
+typedef struct gemmi_packed_b gemmi_packed_b;
+int gemmi_pack_b_i16(int64_t k, int64_t n, const int16_t* B, int64_t ldb, void* stream, gemmi_packed_b** out);
+int gemmi_pack_b_i8(int64_t k, int64_t n, const int8_t* B, int64_t ldb, void* stream, gemmi_packed_b** out);
+int gemm_i16_packed(int64_t m, const int16_t* A, int64_t lda, const gemmi_packed_b* B, int64_t* C, int64_t ldc,
+                    void* stream);
+int gemm_i8_packed(int64_t m, const int8_t* A, int64_t lda, const gemmi_packed_b* B, int32_t* C, int64_t ldc,
+                   void* stream);
+int gemmi_packed_b_free(gemmi_packed_b* packed);
+/* k and n of a packed operand (0 for a null handle). */
+int64_t gemmi_packed_b_k(const gemmi_packed_b* packed);
+int64_t gemmi_packed_b_n(const gemmi_packed_b* packed);
+
 /* Stream used by gemm_i16 / gemm_i8 / *_host (a cudaStream_t as void*). */
 void gemmi_set_stream(void* stream);
 

@@ -29,7 +29,8 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_detail",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
-            "gemm_i16_noalloc")
+            "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
+            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY = 0, 1, 2, 3
 
@@ -81,6 +82,17 @@ def lib():
         L.gemmi_kernel_time.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
         L.gemmi_kernel_time.restype = ctypes.c_int
         L.gemmi_version.restype = ctypes.c_char_p
+        for name in ("gemmi_pack_b_i16", "gemmi_pack_b_i8"):
+            getattr(L, name).argtypes = [i64, i64, vp, i64, vp, ctypes.POINTER(vp)]
+            getattr(L, name).restype = ctypes.c_int
+        for name in ("gemm_i16_packed", "gemm_i8_packed"):
+            getattr(L, name).argtypes = [i64, vp, i64, vp, vp, i64, vp]
+            getattr(L, name).restype = ctypes.c_int
+        L.gemmi_packed_b_free.argtypes = [vp]
+        L.gemmi_packed_b_free.restype = ctypes.c_int
+        for name in ("gemmi_packed_b_k", "gemmi_packed_b_n"):
+            getattr(L, name).argtypes = [vp]
+            getattr(L, name).restype = i64
         _lib = L
     return _lib
 
@@ -149,6 +161,90 @@ def gemm_i8(A, B, C, stream=None):
     """C += A @ B on the GPU: int8 A, int8 B, int32 C; exact modulo 2^32."""
     import torch
     return _torch_call("gemm_i8_ex", A, B, C, torch.int8, torch.int32, stream)
+
+
+# ------------------------------------------------------------------ pre-packed weights
+class PackedB:
+    """B (k x n) packed once on the device for repeated GEMMs (Section 5.1: weights are packed
+    off-line, only activations at run time).  Frees its device memory when closed or collected."""
+
+    def __init__(self, handle, kind, k, n, device):
+        self._h = handle
+        self.kind, self.k, self.n, self.device = kind, k, n, device
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise ValueError("packed operand was freed")
+        return self._h
+
+    def close(self):
+        if self._h is not None:
+            h, self._h = self._h, None
+            _check(lib().gemmi_packed_b_free(h))
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # interpreter shutdown
+            pass
+
+
+def _pack(fn_name, kind, B, dtype, stream):
+    import torch
+    if not isinstance(B, torch.Tensor) or not B.is_cuda or B.dtype != dtype:
+        raise TypeError(f"B must be a CUDA {dtype} tensor")
+    k, n = B.shape
+    if stream is None:
+        stream = torch.cuda.current_stream(B.device)
+    out = ctypes.c_void_p(0)
+    with torch.cuda.device(B.device):
+        rc = getattr(lib(), fn_name)(k, n, B.data_ptr(), _dev_ld(B, "B"), stream.cuda_stream, ctypes.byref(out))
+    _check(rc)
+    return PackedB(out.value, kind, k, n, B.device)
+
+
+def pack_b_i16(B, stream=None) -> PackedB:
+    """Pack an int16 B (k x n) for gemm_i16_packed."""
+    import torch
+    return _pack("gemmi_pack_b_i16", "i16", B, torch.int16, stream)
+
+
+def pack_b_i8(B, stream=None) -> PackedB:
+    """Pack an int8 B (k x n) for gemm_i8_packed."""
+    import torch
+    return _pack("gemmi_pack_b_i8", "i8", B, torch.int8, stream)
+
+
+def _packed_call(fn_name, kind, A, Bp, C, op_dtype, c_dtype, stream):
+    import torch
+    if not isinstance(Bp, PackedB) or Bp.kind != kind:
+        raise TypeError(f"B must be a PackedB of kind {kind}")
+    for t, nm, dt in ((A, "A", op_dtype), (C, "C", c_dtype)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dtype != dt:
+            raise TypeError(f"{nm} must be a CUDA {dt} tensor")
+    m, k = A.shape
+    if k != Bp.k or tuple(C.shape) != (m, Bp.n):
+        raise ValueError(f"shape mismatch: A {tuple(A.shape)}, packed B {(Bp.k, Bp.n)}, C {tuple(C.shape)}")
+    if stream is None:
+        stream = torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = getattr(lib(), fn_name)(m, A.data_ptr(), _dev_ld(A, "A"), Bp.handle, C.data_ptr(), _dev_ld(C, "C"),
+                                     stream.cuda_stream)
+    _check(rc)
+    return C
+
+
+def gemm_i16_packed(A, Bp, C, stream=None):
+    """C += A @ B with B pre-packed by pack_b_i16 (bit-identical to gemm_i16)."""
+    import torch
+    return _packed_call("gemm_i16_packed", "i16", A, Bp, C, torch.int16, torch.int64, stream)
+
+
+def gemm_i8_packed(A, Bp, C, stream=None):
+    """C += A @ B with B pre-packed by pack_b_i8 (bit-identical to gemm_i8)."""
+    import torch
+    return _packed_call("gemm_i8_packed", "i8", A, Bp, C, torch.int8, torch.int32, stream)
 
 
 # ------------------------------------------------------------------ host-buffer entry points

@@ -238,16 +238,19 @@ Layout plane_layout(int64_t m, int64_t n, int64_t pitch, int nl) {
   return L;
 }
 
+// The tensor-core path: split A (and B, unless `packed_b` already holds its planes) into the
+// workspace, then run the tcgen05 GEMM.
 int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B,
-           int64_t ldb, void* C, int64_t ldc, cudaStream_t s) {
+           int64_t ldb, void* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b = nullptr) {
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
-  const Layout L = plane_layout(m, n, pitch, nl);
+  const Layout L = plane_layout(m, packed_b ? 0 : n, pitch, nl);
   int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
   if (rc != GEMMI_OK) return rc;
   if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
   char* ws = static_cast<char*>(d.ws);
   LimbPlanes pa{{ws + L.a0, ws + L.a1}, m, pitch};
-  LimbPlanes pb{{ws + L.b0, ws + L.b1}, n, pitch};
+  LimbPlanes pb = packed_b ? *packed_b : LimbPlanes{{ws + L.b0, ws + L.b1}, n, pitch};
+  if (packed_b) B = nullptr;  // nothing to convert for B
   cudaError_t e;
   cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
   if (nl == 2) {
@@ -470,6 +473,111 @@ int gemm_i8_host(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, 
                  int32_t* C, int64_t ldc) {
   return host_gemm(m, n, k, A, lda, B, ldb, C, ldc, gemm_i8_locked);
 }
+
+}  // extern "C"
+
+struct gemmi_packed_b {
+  int nl;        // 2: int16 limb planes, 1: int8 values as fp16
+  int device;
+  int64_t k, n, pitch;
+  void* mem;     // the planes, owned by the handle
+};
+
+namespace {
+
+int pack_b(int nl, int64_t k, int64_t n, const void* B, int64_t ldb, void* stream, gemmi_packed_b** out) {
+  if (out == nullptr) return set_error(GEMMI_EINVAL, "null output handle");
+  *out = nullptr;
+  if (k < 1 || n < 1) return set_error(GEMMI_EINVAL, "packed operand needs k >= 1 and n >= 1");
+  if (ldb < n) return set_error(GEMMI_EINVAL, "ldb < n");
+  if (B == nullptr) return set_error(GEMMI_EINVAL, "B is null");
+  if (k > (int64_t(1) << 31) || n > (int64_t(1) << 31)) return set_error(GEMMI_EINVAL, "matrix dimension too large");
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const size_t plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
+  void* mem = nullptr;
+  if (cudaMalloc(&mem, plane * nl) != cudaSuccess) {
+    cudaGetLastError();
+    return set_error(GEMMI_ENOMEM, "cannot allocate the packed operand");
+  }
+  char* base = static_cast<char*>(mem);
+  LimbPlanes pb{{base, base + (nl == 2 ? plane : 0)}, n, pitch};
+  LimbPlanes none{{nullptr, nullptr}, 0, pitch};
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = nl == 2 ? gemmi::split_i16(nullptr, k, static_cast<const int16_t*>(B), ldb, 0, n, k, none, pb, s)
+                          : gemmi::convert_i8(nullptr, k, static_cast<const int8_t*>(B), ldb, 0, n, k, none, pb, s);
+  if (e != cudaSuccess) {
+    cudaFree(mem);
+    return cuda_error(e, "packing launch");
+  }
+  *out = new gemmi_packed_b{nl, dev, k, n, pitch, mem};
+  return GEMMI_OK;
+}
+
+int gemm_packed(int nl, int64_t m, const void* A, int64_t lda, const gemmi_packed_b* Bp, void* C, int64_t ldc,
+                void* stream) {
+  if (Bp == nullptr) return set_error(GEMMI_EINVAL, "null packed operand");
+  if (Bp->nl != nl) return set_error(GEMMI_EINVAL, "packed operand has the other element type");
+  const int64_t n = Bp->n, k = Bp->k;
+  const size_t op = nl == 2 ? 2 : 1, cs = nl == 2 ? 8 : 4;
+  // the packed planes stand in for B in the overlap check (C must not overlap them either)
+  const int pre = check_args(m, n, k, A, lda, Bp->mem, n, C, ldc, op, cs);
+  if (pre >= 0) return pre;
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != Bp->device) return set_error(GEMMI_EINVAL, "packed operand belongs to another device");
+  const size_t plane = round_up(static_cast<size_t>(n) * Bp->pitch * 2, kAlign);
+  char* base = static_cast<char*>(Bp->mem);
+  LimbPlanes pb{{base, base + (nl == 2 ? plane : 0)}, n, Bp->pitch};
+  return run_tc(*d, nl, m, n, k, A, lda, nullptr, n, C, ldc, static_cast<cudaStream_t>(stream), &pb);
+}
+
+}  // namespace
+
+extern "C" {
+
+int gemmi_pack_b_i16(int64_t k, int64_t n, const int16_t* B, int64_t ldb, void* stream, gemmi_packed_b** out) {
+  return pack_b(2, k, n, B, ldb, stream, out);
+}
+
+int gemmi_pack_b_i8(int64_t k, int64_t n, const int8_t* B, int64_t ldb, void* stream, gemmi_packed_b** out) {
+  return pack_b(1, k, n, B, ldb, stream, out);
+}
+
+int gemm_i16_packed(int64_t m, const int16_t* A, int64_t lda, const gemmi_packed_b* B, int64_t* C, int64_t ldc,
+                    void* stream) {
+  return gemm_packed(2, m, A, lda, B, C, ldc, stream);
+}
+
+int gemm_i8_packed(int64_t m, const int8_t* A, int64_t lda, const gemmi_packed_b* B, int32_t* C, int64_t ldc,
+                   void* stream) {
+  return gemm_packed(1, m, A, lda, B, C, ldc, stream);
+}
+
+int gemmi_packed_b_free(gemmi_packed_b* packed) {
+  if (packed == nullptr) return GEMMI_OK;
+  int prev = 0;
+  cudaGetDevice(&prev);
+  cudaSetDevice(packed->device);
+  cudaDeviceSynchronize();
+  cudaError_t e = cudaFree(packed->mem);
+  cudaSetDevice(prev);
+  delete packed;
+  if (e != cudaSuccess) return cuda_error(e, "cudaFree(packed operand)");
+  return GEMMI_OK;
+}
+
+int64_t gemmi_packed_b_k(const gemmi_packed_b* packed) { return packed ? packed->k : 0; }
+int64_t gemmi_packed_b_n(const gemmi_packed_b* packed) { return packed ? packed->n : 0; }
 
 void gemmi_set_stream(void* stream) {
   std::lock_guard<std::mutex> lock(g_mutex);

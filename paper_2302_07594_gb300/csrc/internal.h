@@ -19,6 +19,7 @@ struct LimbPlanes {
 // int16: two centred 8-bit limbs, a = 256*h + l, h in [-128,128], l in [-128,127].
 // int8: one plane holding the value itself.
 // One launch converts both operands: A (m x k, lda) -> pa (rows m), B (k x n, ldb) -> pb (rows n).
+// A null A (or B) skips that operand.
 cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s);
 cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,

@@ -14,7 +14,7 @@
 // rows have a pitch that is a multiple of 8 elements (16 bytes), which the TMA
 // tensor maps require.  Pitch columns at and beyond k are written as zero.
 //
-// One launch converts both operands: the first blocks of the grid stream A
+// One launch converts both operands (or just one: a null operand is skipped): the first blocks of the grid stream A
 // (16-byte loads, 2 x 16-byte stores per 8 elements), the rest transpose B in
 // 64 x 64 tiles through shared memory (16-byte loads and stores on both sides).
 // The kernel is bound by HBM: per int16 element 2 bytes are read and 4 written.
@@ -152,15 +152,16 @@ cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, 
             reinterpret_cast<uintptr_t>(A) % (8 * esz) == 0 && (lda * esz) % (8 * esz) == 0};
   Part<T> b{B, ldb, k, n, static_cast<__half*>(pb.plane[0]), static_cast<__half*>(pb.plane[NL - 1]), pb.pitch,
             reinterpret_cast<uintptr_t>(B) % (8 * esz) == 0 && (ldb * esz) % (8 * esz) == 0};
-  // A: about 8 elements per thread per grid-stride step; B: one 64 x 64 tile per block step
-  const int64_t a_work = m * (pa.pitch / 8);
+  // A: about 8 elements per thread per grid-stride step; B: one 64 x 64 tile per block step.
+  // A null operand is skipped (packing only the weights, or only the activations).
+  const int64_t a_work = A != nullptr ? m * (pa.pitch / 8) : 0;
   int64_t a_blocks = (a_work + THREADS - 1) / THREADS;
   if (a_blocks > 152 * 8) a_blocks = 152 * 8;
   const int64_t tiles_p = (pb.pitch + TT - 1) / TT;  // cover the zero padding up to the pitch too
-  const int64_t tiles_j = (n + TT - 1) / TT;
+  const int64_t tiles_j = B != nullptr ? (n + TT - 1) / TT : 0;
   const int64_t b_tiles = tiles_p * tiles_j;
   int64_t b_blocks = b_tiles < 152 * 8 ? b_tiles : 152 * 8;
-  if (a_blocks < 1 || b_blocks < 1) return cudaErrorInvalidValue;
+  if (a_blocks + b_blocks < 1) return cudaSuccess;
   split_kernel<T, NL><<<static_cast<unsigned>(a_blocks + b_blocks), THREADS, 0, s>>>(
       a, b, static_cast<int>(a_blocks), tiles_j, b_tiles);
   return cudaGetLastError();
