@@ -35,6 +35,14 @@ import gemm_inputs as gi  # noqa: E402
 
 L2_BYTES = 129 * 2 ** 20
 PROFILES = os.path.join(ROOT, "profiles")
+# per kernel of the library: its CUDA symbol, the sources it is built from, and its bound
+KERNEL_INFO = {
+    "split": ("split_kernel", ("split.cu",), "hbm"),
+    "tc_i16": ("tc_gemm_kernel<2>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
+    "tc_i8": ("tc_gemm_kernel<1>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
+    "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh"), "hbm"),
+    "fused_i16": ("fused_kernel", ("gemm_fused.cu", "tc_common.cuh", "ptx.cuh"), "hbm"),
+}
 
 
 def parse_args():
@@ -234,9 +242,7 @@ def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_se
     e1.record()
     torch.cuda.synchronize()
     eager_ms = e0.elapsed_time(e1) / steps
-    kt = {name: gm.kernel_time(kid) for name, kid in
-          (("split", gm.KERNEL_SPLIT), ("tc_i16", gm.KERNEL_TC_I16), ("tc_i8", gm.KERNEL_TC_I8),
-           ("skinny", gm.KERNEL_SKINNY))}
+    kt = {name: gm.kernel_time(kid) for name, kid in gm.KERNELS}
     gm.kernel_timing(False)
     # CUDA-graph replay of the same calls
     ncap = min(steps, 64)
@@ -320,9 +326,7 @@ def run_gemmi(args):
         dist.barrier()
     clocks = sampler.stop()
     ms = e0.elapsed_time(e1) / args.steps
-    kt = {name: gm.kernel_time(kid) for name, kid in
-          (("split", gm.KERNEL_SPLIT), ("tc_i16", gm.KERNEL_TC_I16), ("tc_i8", gm.KERNEL_TC_I8),
-           ("skinny", gm.KERNEL_SKINNY))}
+    kt = {name: gm.kernel_time(kid) for name, kid in gm.KERNELS}
     gm.kernel_timing(False)
     assert gm.device_status() == gm.OK
     if world > 1:
@@ -331,35 +335,33 @@ def run_gemmi(args):
         ms = float(t.item())
     value = world * w.ops / (ms * 1e-3) / 1e12
 
-    # ---- dominant kernel and its roofline
-    launches = kt["split"][1] + kt["tc_i16"][1] + kt["tc_i8"][1] + kt["skinny"][1]
-    if w.kind == "i16" and w.m > gm.get_option(gm.OPT_SKINNY_MAX_M):
-        kname, (kms, kn), src = "tc_gemm_kernel<2>", kt["tc_i16"], ("gemm_tc.cu", "ptx.cuh")
-        per_launch_ms = kms / max(kn, 1)
+    # ---- dominant kernel (most device time in the timed region) and its roofline
+    launches = sum(kn for _, kn in kt.values())
+    kname = max((name for name in KERNEL_INFO if kt[name][1] > 0), key=lambda name: kt[name][0])
+    sym, src, bound = KERNEL_INFO[kname]
+    kms, kn = kt[kname]
+    per_launch_ms = kms / max(kn, 1)
+    if bound == "tensor" and w.kind == "i16":
         achieved = w.ops / (per_launch_ms * 1e-3) / 1e12
         peak = peaks["bf16_tflops"] / 4.0
-        roof = {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak, "unit": "TOPS",
+        roof = {"bound": "tensor", "kernel": sym, "achieved": achieved, "peak": peak, "unit": "TOPS",
                 "frac": achieved / peak,
                 "peak_note": f"fp16 dense tensor peak ({peaks['source']} bf16 burst {peaks['bf16_tflops']} TFLOP/s, "
                              "fp16 = bf16 rate) / 4 limb products per int16 multiply-add",
                 "frac_of_sustained": achieved / (peaks["bf16_tflops_sustained"] / 4.0),
                 "kernel_ms": per_launch_ms}
-    elif w.kind == "i8":
-        kname, (kms, kn), src = "tc_gemm_kernel<1>", kt["tc_i8"], ("gemm_tc.cu", "ptx.cuh")
-        per_launch_ms = kms / max(kn, 1)
+    elif bound == "tensor":
         achieved = w.ops / (per_launch_ms * 1e-3) / 1e12
         peak = peaks["bf16_tflops"]
-        roof = {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak, "unit": "TOPS",
+        roof = {"bound": "tensor", "kernel": sym, "achieved": achieved, "peak": peak, "unit": "TOPS",
                 "frac": achieved / peak, "peak_note": "fp16 dense tensor peak (one fp16 product per int8 product)",
                 "kernel_ms": per_launch_ms}
     else:
-        kname, (kms, kn), src = "skinny_kernel", kt["skinny"], ("skinny.cu", "ptx.cuh")
-        per_launch_ms = kms / max(kn, 1)
         achieved = workload_bytes(w) / (per_launch_ms * 1e-3) / 1e9
-        roof = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        roof = {"bound": "hbm", "kernel": sym, "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / peaks["hbm_gbs"], "kernel_ms": per_launch_ms}
     src_hash = kernel_source_hash(src)
-    traffic = recorded_traffic(kname, src_hash)
+    traffic = recorded_traffic(sym, src_hash)
     roof["traffic"] = traffic
     roof["source_hash"] = src_hash
     roof["peak_source"] = peaks["source"]
@@ -408,19 +410,13 @@ def run_gemmi(args):
             ent = {"ms": oms, "timing": "CUDA-graph replay, per call", "eager_ms": eager_ms,
                    "TOPS": ow.ops / (oms * 1e-3) / 1e12,
                    "GB_per_s": workload_bytes(ow) / (oms * 1e-3) / 1e9, "input_sets_rotated": nsets}
-            if ow.kind == "i16" and ow.m > gm.get_option(gm.OPT_SKINNY_MAX_M):
-                ent["kernel_ms"] = {"split": okt["split"][0] / max(okt["split"][1], 1),
-                                    "tc_gemm_kernel<2>": okt["tc_i16"][0] / max(okt["tc_i16"][1], 1)}
-                ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
-                ent["frac_of_hbm"] = ent["GB_per_s"] / peaks["hbm_gbs"]
-            elif ow.kind == "i8":
-                ent["kernel_ms"] = {"split": okt["split"][0] / max(okt["split"][1], 1),
-                                    "tc_gemm_kernel<1>": okt["tc_i8"][0] / max(okt["tc_i8"][1], 1)}
+            ent["kernel_ms"] = {KERNEL_INFO[name][0]: okt[name][0] / okt[name][1]
+                                for name in KERNEL_INFO if okt[name][1] > 0}
+            if ow.kind == "i8":
                 ent["frac_of_fp16_tensor_peak"] = ent["TOPS"] / peaks["bf16_tflops"]
             else:
-                ent["kernel_ms"] = {"skinny_kernel": okt["skinny"][0] / max(okt["skinny"][1], 1)}
+                ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
                 ent["frac_of_hbm"] = ent["GB_per_s"] / peaks["hbm_gbs"]
-                ent["B_GB_per_s"] = ow.k * ow.n * 2 / (oms * 1e-3) / 1e9
             if int8_peak:
                 ent["frac_of_int8_roofline_div4" if ow.kind == "i16" else "frac_of_int8_roofline"] = (
                     ent["TOPS"] / (int8_peak / 4 if ow.kind == "i16" else int8_peak))

@@ -161,10 +161,14 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_TC_GROUP_M   : tile raster band height in 128-row tiles (default 16).
  *   GEMMI_OPT_TC_L2_HINTS  : L2 eviction policy of the operand tile loads, bits 0-1 for A,
  *                            bits 2-3 for B: 0 normal, 1 evict_last, 2 evict_first (default 0).
+ *   GEMMI_OPT_FUSED_MAX_N  : int16 GEMMs with n <= this value (and an A whose base is 16-byte
+ *                            aligned with lda % 8 == 0) take the kernel that reads A raw and
+ *                            splits it on chip (default 64; 0 disables it; at most 4096).
  * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
 enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
-       GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6 };
+       GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6,
+       GEMMI_OPT_FUSED_MAX_N = 7 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 
@@ -188,9 +192,10 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_TC_I16  : the tcgen05 int16 GEMM kernel
  *   GEMMI_KERNEL_TC_I8   : the tcgen05 int8 GEMM kernel
  *   GEMMI_KERNEL_SKINNY  : the skinny-M int16 kernel
+ *   GEMMI_KERNEL_FUSED_I16 : the narrow-n int16 kernel that splits A on chip
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
-       GEMMI_KERNEL_COUNT = 4 };
+       GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_COUNT = 5 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

@@ -113,6 +113,7 @@ int64_t g_skinny_ksplit = 0;
 int64_t g_tc_chunk_scale = 2;
 int64_t g_tc_group_m = 16;
 int64_t g_tc_l2_hints = 0;
+int64_t g_fused_max_n = 64;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -240,8 +241,59 @@ Layout plane_layout(int64_t m, int64_t n, int64_t pitch, int nl) {
 
 // The tensor-core path: split A (and B, unless `packed_b` already holds its planes) into the
 // workspace, then run the tcgen05 GEMM.
+// The narrow-n int16 path: only B is split (unless packed); A is read raw by the kernel, which
+// splits it on chip.  TMA reads A, so its base must be 16-byte aligned and lda a multiple of 8.
+bool fused_applies(int nl, int64_t n, const void* A, int64_t lda) {
+  return nl == 2 && n <= g_fused_max_n && reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 8 == 0;
+}
+
+int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
+              int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b) {
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const bool split_b = packed_b == nullptr;
+  LimbPlanes pb{};
+  if (split_b) {
+    const Layout L = plane_layout(0, n, pitch, 2);
+    int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
+    if (rc != GEMMI_OK) return rc;
+    if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+    char* ws = static_cast<char*>(d.ws);
+    pb = LimbPlanes{{ws + L.b0, ws + L.b1}, n, pitch};
+    const LimbPlanes none{{nullptr, nullptr}, 0, pitch};
+    cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+    const cudaError_t e = gemmi::split_i16(nullptr, lda, B, ldb, m, n, k, none, pb, s);
+    timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+    if (e != cudaSuccess) return cuda_error(e, "limb split launch");
+  } else {
+    pb = *packed_b;
+  }
+  gemmi::FusedArgs fa;
+  fa.m = m;
+  fa.n = n;
+  fa.k = k;
+  fa.A = A;
+  fa.lda = lda;
+  fa.b = pb;
+  fa.C = C;
+  fa.ldc = ldc;
+  fa.status = d.status;
+  fa.timeout_ns = timeout_ns();
+  fa.num_sms = d.sm_count;
+  fa.chunk_scale = static_cast<int>(g_tc_chunk_scale);
+  fa.group_m = static_cast<int>(g_tc_group_m);
+  const char* why = "fused tcgen05 GEMM launch";
+  cudaEvent_t t1 = timer_begin(GEMMI_KERNEL_FUSED_I16, s);
+  const cudaError_t e = gemmi::tc_gemm_fused_i16(fa, s, &why);
+  timer_end(GEMMI_KERNEL_FUSED_I16, t1, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return split_b ? end_workspace_use(d, s) : GEMMI_OK;
+}
+
 int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B,
            int64_t ldb, void* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b = nullptr) {
+  if (fused_applies(nl, n, A, lda))
+    return run_fused(d, m, n, k, static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb,
+                     static_cast<int64_t*>(C), ldc, s, packed_b);
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
   const Layout L = plane_layout(m, packed_b ? 0 : n, pitch, nl);
   int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
@@ -654,6 +706,10 @@ int gemmi_set_option(int option, int64_t value) {
         return set_error(GEMMI_EINVAL, "L2 hints: 2 bits each for A and B, values 0..2");
       g_tc_l2_hints = value;
       return GEMMI_OK;
+    case GEMMI_OPT_FUSED_MAX_N:
+      if (value < 0 || value > 4096) return set_error(GEMMI_EINVAL, "fused-kernel n limit must be in [0, 4096]");
+      g_fused_max_n = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -668,6 +724,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_TC_CHUNK_SCALE: return g_tc_chunk_scale;
     case GEMMI_OPT_TC_GROUP_M: return g_tc_group_m;
     case GEMMI_OPT_TC_L2_HINTS: return g_tc_l2_hints;
+    case GEMMI_OPT_FUSED_MAX_N: return g_fused_max_n;
     default: return -1;
   }
 }

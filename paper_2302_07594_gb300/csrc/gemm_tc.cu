@@ -11,8 +11,8 @@
 // Each limb product is an integer of magnitude <= 2^14 that fp16 x fp16 forms
 // exactly, and an fp32 accumulator sums integers exactly while every partial
 // sum stays below 2^24.  So each accumulator is only allowed a bounded run of
-// the reduction dimension (a "chunk": 512 indices for HH and LL, 256 for X,
-// keeping every partial sum within 2^23), after which it is drained:
+// the reduction dimension (a "chunk": by default 1024 indices for HH and LL,
+// 512 for X, keeping every partial sum within 2^24), after which it is drained:
 // converted to an integer and added, shifted by its weight (16, 8, 0 bits),
 // into a 64-bit running sum held in registers.  This plays the role of the
 // AIE's 48-bit accumulators (Section 6.2): wide accumulation so nothing
@@ -50,13 +50,13 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace gemmi {
 namespace {
 
-constexpr int BM = 128;
+using namespace tc;
 constexpr int UMMA_N = 128;                  // N of one tcgen05.mma (an accumulator is 128 columns)
-constexpr int UMMA_K = 16;                   // K of one tcgen05.mma kind::f16
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int PRODUCER_WARP = 8;
 constexpr int MMA_WARP0 = 9;                  // issuer warps 9 and 10; warp 9 also owns the TMEM allocation
@@ -65,106 +65,8 @@ constexpr int NUM_THREADS = (NUM_EPI_WARPS + 1 + NISSUE) * 32;
 constexpr int NSLOT = 4;
 constexpr int SLOT_COLS = 128;
 constexpr int TMEM_COLS = NSLOT * SLOT_COLS;  // 512
-constexpr uint32_t STATUS_TIMEOUT = 4;
-
-template <int NL>
-struct Scheme;
-
-// int16: two limbs per operand, four products, three accumulators.
-//   product p: (A limb, B limb) = (h,h), (h,l), (l,h), (l,l); limb 0 = high, 1 = low
-//   accumulators: 0 = HH (weight 2^16), 1 = X (2^8), 2 = LL (1)
-//   issuer 0 owns HH and LL (products 0, 3), issuer 1 owns X (products 1, 2): 8 MMAs each per K block.
-template <>
-struct Scheme<2> {
-  static constexpr int BN = 128;          // output tile width
-  static constexpr int NACC = 3;
-  static constexpr int NPROD = 4;
-  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
-  static constexpr int COLS = 64;         // C columns per epilogue thread (two warps per lane quadrant)
-  static constexpr int DRAIN_WARPS = 8;   // every epilogue warp drains every accumulator (its 64 columns)
-  __device__ static constexpr bool drains(int, int) { return true; }
-  __device__ static constexpr int a_limb(int p) { return p >> 1; }
-  __device__ static constexpr int b_limb(int p) { return p & 1; }
-  __device__ static constexpr int b_row0(int) { return 0; }  // first row (output column) of the B tile used
-  __device__ static constexpr int acc(int p, int) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
-  __device__ static constexpr int issuer(int p, int) { return (p == 0 || p == 3) ? 0 : 1; }
-  __device__ static constexpr int owner(int a) { return a == 1 ? 1 : 0; }
-  __device__ static constexpr int shift(int a) { return a == 0 ? 16 : a == 1 ? 8 : 0; }
-  // Chunk schedule, in reduction indices, for chunk scale CS (1 or 2): accumulator a ends a
-  // chunk after the K block that ends at index e when (e + PHASE[a]) % PERIOD[a] == 0, or at
-  // the last block of the tile.  HH, LL: 512*CS indices, |sum| <= 512*CS * 2^14;  X: 256*CS
-  // indices, |sum| <= 256*CS * 2^15.  CS = 1 keeps every partial sum within 2^23 (one bit below
-  // the 2^24 limit of exact fp32 integer sums), CS = 2 within 2^24.  The phases stagger the
-  // three chunk ends 128*CS indices apart (HH at 128*CS, X at 256*CS, LL at 384*CS, X at 512*CS, ...).
-  template <int CS>
-  __device__ static bool chunk_ends(int a, int kb, int nkb) {
-    const int period = (a == 1 ? 256 : 512) * CS;
-    const int phase = (a == 0 ? 384 : a == 1 ? 0 : 128) * CS;
-    return kb == nkb - 1 || (((kb + 1) * 64 + phase) % period) == 0;
-  }
-};
-
-// int8: the value itself in one fp16 plane, one product per K block and output column half.
-// The tile is 128 x 256: each issuer owns one 128-column half (its own accumulator), so both
-// halves reuse the same A tile.  Chunks of 512*CS reduction indices, |sum| <= 512*CS * 2^14;
-// the two accumulators' chunk ends are staggered by half a chunk.
-template <>
-struct Scheme<1> {
-  static constexpr int BN = 256;
-  static constexpr int NACC = 2;
-  static constexpr int NPROD = 2;         // product p: column half p
-  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
-  static constexpr int COLS = 128;        // C columns per epilogue thread: warp (quad, half) owns half h
-  static constexpr int DRAIN_WARPS = 4;   // an accumulator is drained by the four warps of its half
-  __device__ static constexpr bool drains(int half, int a) { return half == a; }
-  __device__ static constexpr int a_limb(int) { return 0; }
-  __device__ static constexpr int b_limb(int) { return 0; }
-  __device__ static constexpr int b_row0(int p) { return p * 128; }
-  __device__ static constexpr int acc(int p, int) { return p; }
-  __device__ static constexpr int issuer(int p, int) { return p; }
-  __device__ static constexpr int owner(int a) { return a; }
-  __device__ static constexpr int shift(int) { return 0; }
-  template <int CS>
-  __device__ static bool chunk_ends(int a, int kb, int nkb) {
-    return kb == nkb - 1 || (((kb + 1) * 64 + a * 256 * CS) % (512 * CS)) == 0;
-  }
-};
-
-// Assignment of accumulators to the four TMEM slots, replayed identically by every role.
-// Spare slots form a FIFO: a chunk end moves the accumulator into the oldest spare and queues
-// its old slot.  rotate() returns the parity to wait on (the slot's empty barrier) before the
-// new slot may be written: the n-th assignment of a slot waits for its (n-1)-th drain.
-template <int NACC>
-struct SlotRing {
-  int slot_of[NACC];
-  int spares[NSLOT - NACC];
-  uint32_t assign_parity;  // bit s: parity of the number of assignments of slot s so far
-
-  __device__ __forceinline__ void init() {
-    assign_parity = 0;
-#pragma unroll
-    for (int a = 0; a < NACC; ++a) {
-      slot_of[a] = a;
-      assign_parity ^= 1u << a;
-    }
-#pragma unroll
-    for (int i = 0; i < NSLOT - NACC; ++i) spares[i] = NACC + i;
-  }
-  __device__ __forceinline__ uint32_t rotate(int a) {
-    const int old = slot_of[a];
-    const int fresh = spares[0];
-#pragma unroll
-    for (int i = 0; i + 1 < NSLOT - NACC; ++i) spares[i] = spares[i + 1];
-    spares[NSLOT - NACC - 1] = old;
-    slot_of[a] = fresh;
-    const uint32_t par = ((assign_parity >> fresh) & 1u) ^ 1u;
-    assign_parity ^= 1u << fresh;
-    return par;
-  }
-};
 
 // Tile geometry: K blocks of 64 fp16 (128-byte rows, the 128-byte swizzle span).
-constexpr int BK = 64;
 template <int NL>
 struct Geom {
   static constexpr int BN = Scheme<NL>::BN;
@@ -189,42 +91,6 @@ struct TcParams {
   uint64_t timeout_ns;
   uint32_t* status;
 };
-
-__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
-  const int per_group = group_m * num_n;
-  const int group = t / per_group;
-  const int first_m = group * group_m;
-  const int rows_here = min(group_m, num_m - first_m);
-  const int in_group = t - group * per_group;
-  mt = first_m + in_group % rows_here;
-  nt = in_group / rows_here;
-}
-
-__device__ __forceinline__ uint64_t l2_policy(int hint) {
-  uint64_t p = 0;
-  if (hint == 1) asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  else if (hint == 2) asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const void* map, uint32_t bar, int32_t x, int32_t y,
-                                                 int hint, uint64_t policy) {
-  if (hint == 0) {
-    tma_load_2d(dst, map, bar, x, y);
-  } else {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%3, %4}], [%2], %5;"
-        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "l"(policy)
-        : "memory");
-  }
-}
-
-__device__ __forceinline__ int32_t f32_to_i32(uint32_t bits) {
-  int32_t v;
-  asm("cvt.rni.s32.f32 %0, %1;" : "=r"(v) : "f"(__uint_as_float(bits)));
-  return v;
-}
 
 template <int NL, int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -333,7 +199,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       constexpr uint32_t idesc = idesc_f16_f32(BM, UMMA_N);
       int stage = 0;
       uint32_t phase = 0;
-      SlotRing<S::NACC> ring;
+      SlotRing<S::NACC, NSLOT> ring;
       ring.init();
       uint32_t wait_par[S::NACC];
       bool need_acquire[S::NACC], fresh[S::NACC];
@@ -411,7 +277,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const int quad = warp & 3;       // TMEM lanes 32*quad .. 32*quad+31 (hardware lane quadrant)
     const int half = warp >> 2;      // column half of the tile: columns half*COLS .. +COLS-1
-    SlotRing<S::NACC> ring;
+    SlotRing<S::NACC, NSLOT> ring;
     ring.init();
     uint32_t drain_parity = 0;  // bit s: parity of the number of drains of slot s
     bool ok = true;

@@ -43,6 +43,22 @@ struct TcGemmArgs {
 cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
 
+// ---- gemm_fused.cu: int16 GEMM, n <= 64 per tile column, A read raw (int16) and split on chip.
+struct FusedArgs {
+  int64_t m, n, k;
+  const int16_t* A;  // m x k row-major; base 16-byte aligned and lda % 8 == 0 (TMA)
+  int64_t lda;
+  LimbPlanes b;      // B's two limb planes (rows = n)
+  int64_t* C;
+  int64_t ldc;
+  uint32_t* status;
+  uint64_t timeout_ns;
+  int num_sms;
+  int chunk_scale;
+  int group_m;
+};
+cudaError_t tc_gemm_fused_i16(const FusedArgs& args, cudaStream_t s, const char** why);
+
 // ---- skinny.cu: m <= 16 int16 GEMM streaming B once.
 struct SkinnyArgs {
   int64_t m, n, k;

@@ -1,0 +1,151 @@
+// tc_common.cuh -- pieces shared by the tcgen05 GEMM kernels (gemm_tc.cu, gemm_fused.cu):
+// the limb-product / accumulator schemes with their exact-chunk schedules, the TMEM slot ring,
+// the tile raster and small device helpers.
+#pragma once
+
+#include <cstdint>
+
+#include "ptx.cuh"
+
+namespace gemmi {
+namespace tc {
+
+constexpr int BM = 128;                      // output tile rows (= TMEM lanes)
+constexpr int BK = 64;                       // K block: 64 fp16 = 128 bytes = one swizzle row
+constexpr int UMMA_K = 16;                   // K of one tcgen05.mma kind::f16
+constexpr uint32_t STATUS_TIMEOUT = 4;
+
+template <int NL>
+struct Scheme;
+
+// int16: two limbs per operand, four products, three accumulators.
+//   product p: (A limb, B limb) = (h,h), (h,l), (l,h), (l,l); limb 0 = high, 1 = low
+//   accumulators: 0 = HH (weight 2^16), 1 = X (2^8), 2 = LL (1)
+//   issuer 0 owns HH and LL (products 0, 3), issuer 1 owns X (products 1, 2): 8 MMAs each per K block.
+template <>
+struct Scheme<2> {
+  static constexpr int BN = 128;          // output tile width
+  static constexpr int NACC = 3;
+  static constexpr int NPROD = 4;
+  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
+  static constexpr int COLS = 64;         // C columns per epilogue thread (two warps per lane quadrant)
+  static constexpr int DRAIN_WARPS = 8;   // every epilogue warp drains every accumulator (its 64 columns)
+  __device__ static constexpr bool drains(int, int) { return true; }
+  __device__ static constexpr int a_limb(int p) { return p >> 1; }
+  __device__ static constexpr int b_limb(int p) { return p & 1; }
+  __device__ static constexpr int b_row0(int) { return 0; }  // first row (output column) of the B tile used
+  __device__ static constexpr int acc(int p, int) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
+  __device__ static constexpr int issuer(int p, int) { return (p == 0 || p == 3) ? 0 : 1; }
+  __device__ static constexpr int owner(int a) { return a == 1 ? 1 : 0; }
+  __device__ static constexpr int shift(int a) { return a == 0 ? 16 : a == 1 ? 8 : 0; }
+  // Chunk schedule, in reduction indices, for chunk scale CS (1 or 2): accumulator a ends a
+  // chunk after the K block that ends at index e when (e + PHASE[a]) % PERIOD[a] == 0, or at
+  // the last block of the tile.  HH, LL: 512*CS indices, |sum| <= 512*CS * 2^14;  X: 256*CS
+  // indices, |sum| <= 256*CS * 2^15.  CS = 1 keeps every partial sum within 2^23 (one bit below
+  // the 2^24 limit of exact fp32 integer sums), CS = 2 within 2^24.  The phases stagger the
+  // three chunk ends 128*CS indices apart (HH at 128*CS, X at 256*CS, LL at 384*CS, X at 512*CS, ...).
+  template <int CS>
+  __device__ static bool chunk_ends(int a, int kb, int nkb) {
+    const int period = (a == 1 ? 256 : 512) * CS;
+    const int phase = (a == 0 ? 384 : a == 1 ? 0 : 128) * CS;
+    return kb == nkb - 1 || (((kb + 1) * 64 + phase) % period) == 0;
+  }
+};
+
+// int8: the value itself in one fp16 plane, one product per K block and output column half.
+// The tile is 128 x 256: each issuer owns one 128-column half (its own accumulator), so both
+// halves reuse the same A tile.  Chunks of 512*CS reduction indices, |sum| <= 512*CS * 2^14;
+// the two accumulators' chunk ends are staggered by half a chunk.
+template <>
+struct Scheme<1> {
+  static constexpr int BN = 256;
+  static constexpr int NACC = 2;
+  static constexpr int NPROD = 2;         // product p: column half p
+  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
+  static constexpr int COLS = 128;        // C columns per epilogue thread: warp (quad, half) owns half h
+  static constexpr int DRAIN_WARPS = 4;   // an accumulator is drained by the four warps of its half
+  __device__ static constexpr bool drains(int half, int a) { return half == a; }
+  __device__ static constexpr int a_limb(int) { return 0; }
+  __device__ static constexpr int b_limb(int) { return 0; }
+  __device__ static constexpr int b_row0(int p) { return p * 128; }
+  __device__ static constexpr int acc(int p, int) { return p; }
+  __device__ static constexpr int issuer(int p, int) { return p; }
+  __device__ static constexpr int owner(int a) { return a; }
+  __device__ static constexpr int shift(int) { return 0; }
+  template <int CS>
+  __device__ static bool chunk_ends(int a, int kb, int nkb) {
+    return kb == nkb - 1 || (((kb + 1) * 64 + a * 256 * CS) % (512 * CS)) == 0;
+  }
+};
+
+// Assignment of accumulators to the four TMEM slots, replayed identically by every role.
+// Spare slots form a FIFO: a chunk end moves the accumulator into the oldest spare and queues
+// its old slot.  rotate() returns the parity to wait on (the slot's empty barrier) before the
+// new slot may be written: the n-th assignment of a slot waits for its (n-1)-th drain.
+template <int NACC, int NSLOT>
+struct SlotRing {
+  int slot_of[NACC];
+  int spares[NSLOT - NACC];
+  uint32_t assign_parity;  // bit s: parity of the number of assignments of slot s so far
+
+  __device__ __forceinline__ void init() {
+    assign_parity = 0;
+#pragma unroll
+    for (int a = 0; a < NACC; ++a) {
+      slot_of[a] = a;
+      assign_parity ^= 1u << a;
+    }
+#pragma unroll
+    for (int i = 0; i < NSLOT - NACC; ++i) spares[i] = NACC + i;
+  }
+  __device__ __forceinline__ uint32_t rotate(int a) {
+    const int old = slot_of[a];
+    const int fresh = spares[0];
+#pragma unroll
+    for (int i = 0; i + 1 < NSLOT - NACC; ++i) spares[i] = spares[i + 1];
+    spares[NSLOT - NACC - 1] = old;
+    slot_of[a] = fresh;
+    const uint32_t par = ((assign_parity >> fresh) & 1u) ^ 1u;
+    assign_parity ^= 1u << fresh;
+    return par;
+  }
+};
+
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
+  const int per_group = group_m * num_n;
+  const int group = t / per_group;
+  const int first_m = group * group_m;
+  const int rows_here = min(group_m, num_m - first_m);
+  const int in_group = t - group * per_group;
+  mt = first_m + in_group % rows_here;
+  nt = in_group / rows_here;
+}
+
+__device__ __forceinline__ uint64_t l2_policy(int hint) {
+  uint64_t p = 0;
+  if (hint == 1) asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  else if (hint == 2) asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const void* map, uint32_t bar, int32_t x, int32_t y,
+                                                 int hint, uint64_t policy) {
+  if (hint == 0) {
+    tma_load_2d(dst, map, bar, x, y);
+  } else {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%3, %4}], [%2], %5;"
+        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "l"(policy)
+        : "memory");
+  }
+}
+
+__device__ __forceinline__ int32_t f32_to_i32(uint32_t bits) {
+  int32_t v;
+  asm("cvt.rni.s32.f32 %0, %1;" : "=r"(v) : "f"(__uint_as_float(bits)));
+  return v;
+}
+
+}  // namespace tc
+}  // namespace gemmi

@@ -92,6 +92,29 @@ def test_options(L):
         gm.set_option(99, 1)
 
 
+def test_fused_option(L):
+    old = gm.get_option(gm.OPT_FUSED_MAX_N)
+    assert old == 64
+    gm.set_option(gm.OPT_FUSED_MAX_N, 0)
+    assert gm.get_option(gm.OPT_FUSED_MAX_N) == 0
+    gm.set_option(gm.OPT_FUSED_MAX_N, old)
+    for bad in (-1, 4097):
+        with pytest.raises(gm.GemmiError):
+            gm.set_option(gm.OPT_FUSED_MAX_N, bad)
+
+
+def test_header_constants_match_binding():
+    text = open(HEADER).read()
+    consts = dict((name, int(v)) for name, v in re.findall(r"GEMMI_((?:OPT|KERNEL)_[A-Z0-9_]+)\s*=\s*(\d+)", text))
+    assert consts, "no option or kernel constants found in the header"
+    for name, value in consts.items():
+        if name == "KERNEL_COUNT":
+            assert value == len(gm.KERNELS)
+            continue
+        assert getattr(gm, name) == value, name
+    assert sorted(kid for _, kid in gm.KERNELS) == list(range(consts["KERNEL_COUNT"]))
+
+
 def test_missing_library_fails_loudly(tmp_path, monkeypatch):
     monkeypatch.setattr(gm, "LIB_PATH", str(tmp_path / "absent.so"))
     monkeypatch.setattr(gm, "_lib", None)
