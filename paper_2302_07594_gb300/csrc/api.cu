@@ -242,9 +242,11 @@ Layout plane_layout(int64_t m, int64_t n, int64_t pitch, int nl) {
 // The tensor-core path: split A (and B, unless `packed_b` already holds its planes) into the
 // workspace, then run the tcgen05 GEMM.
 // The narrow-n int16 path: only B is split (unless packed); A is read raw by the kernel, which
-// splits it on chip.  TMA reads A, so its base must be 16-byte aligned and lda a multiple of 8.
-bool fused_applies(int nl, int64_t n, const void* A, int64_t lda) {
-  return nl == 2 && n <= g_fused_max_n && reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 8 == 0;
+// splits it on chip.  TMA reads A, so its base must be 16-byte aligned and lda a multiple of 8;
+// the kernel adds into C with 64-bit reductions, so C must be 8-byte aligned.
+bool fused_applies(int nl, int64_t n, const void* A, int64_t lda, const void* C) {
+  return nl == 2 && n <= g_fused_max_n && reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 8 == 0 &&
+         reinterpret_cast<uintptr_t>(C) % 8 == 0;
 }
 
 int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
@@ -291,7 +293,7 @@ int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A,
 
 int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B,
            int64_t ldb, void* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b = nullptr) {
-  if (fused_applies(nl, n, A, lda))
+  if (fused_applies(nl, n, A, lda, C))
     return run_fused(d, m, n, k, static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb,
                      static_cast<int64_t*>(C), ldc, s, packed_b);
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));

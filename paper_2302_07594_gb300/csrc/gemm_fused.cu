@@ -3,32 +3,48 @@
 // Convolutions lowered with IM2COL/IM2ROW give GEMMs with one very large and
 // two small dimensions (Section 2 of the paper): m = batch*H*W rows of
 // activations, n = output channels, k = C_in*3*3.  Such a GEMM is bound by
-// reading A once from HBM; a separate limb-split pass (split.cu) would read A,
-// write its two fp16 limb planes (twice A's bytes) and read them again.  Here
-// A is streamed raw (int16) and split on chip, the way the paper packs the
-// activation operand at run time while the weights stay packed (Section 5.1):
+// reading A once and C twice from HBM.  A separate limb-split pass (split.cu)
+// would read A, write its two fp16 limb planes (twice A's bytes) and read them
+// again; here A is streamed raw (int16) and split on chip, the way the paper
+// packs the activation operand at run time while the weights stay packed
+// (Section 5.1).  C is never loaded into the SM: each tile's A*B is added into
+// C by bulk reductions that L2 carries out.
 //
+// Roles (one CTA per SM, 128 x 64 output tiles, K blocks of 64):
 //   warp 8      TMA producer of raw A tiles (128 rows x 64 reduction indices of
-//               int16, 128-byte swizzle) into a ring of RAW_STAGES smem slots;
-//   warp 9      TMA producer of B's limb tiles (64 x 64 fp16, from the split or
-//               packed planes) into the limb stages;
-//   warps 10-11 MMA issuers, as in gemm_tc.cu: tcgen05.mma kind::f16, M=128,
-//               N=64, issuer 0 owns HH and LL, issuer 1 owns X;
-//   warps 0-7   epilogue: they split each raw A tile into the fp16 limb tiles
-//               AH, AL of a limb stage -- the raw and the limb tiles share one
-//               swizzled layout, so every 16-byte chunk converts in place --
-//               running LOOKAHEAD K blocks ahead of their main job, which is to
-//               drain the accumulators (staggered exact chunks, as in gemm_tc.cu)
-//               into int64 registers and read-modify-write C once per tile.
+//               int16, 128-byte swizzle) into a ring of RAW_STAGES slots.  A slot
+//               is free again once its tile has been converted, so the HBM
+//               stream never waits for the tensor cores; the ring is deep
+//               because nothing else of A lives in shared memory.
+//   warp 9      TMA producer of B's two limb tiles (64 x 64 fp16 each, stacked
+//               into one 128-row tile) into a ring of B_STAGES slots.
+//   warps 10-11 MMA issuers.  Issuer p multiplies A limb p (0 high, 1 low),
+//               which sits in tensor memory, by the stacked B tile with one
+//               tcgen05.mma of N = 128: columns 0-63 of its accumulator get
+//               A_p * B_high, columns 64-127 get A_p * B_low.
+//   warps 0-7   epilogue.  Warp (quadrant q = w % 4, half h = w / 4), lane t,
+//               owns row 32q + t of the tile.  It splits K-block halves of its
+//               row (32 reduction indices) from the raw slot into the two fp16
+//               limbs and writes them into the A limb stage in tensor memory
+//               (tcgen05.st), LOOKAHEAD K blocks ahead of its main job: draining
+//               the accumulators (staggered exact chunks) into int64 registers
+//               for output columns 32h .. 32h + 31.  At the end of a tile the
+//               two warps of a quadrant write their 32 rows into a dense
+//               staging block that goes out as one bulk reduction
+//               (cp.reduce.async.bulk .add.u64) when C's rows are 64 wide and
+//               contiguous, or as one reduction per row otherwise.
 //
 // Limb split of a packed int16 pair x = (a1 << 16) | a0 with centred limbs
 // h = floor((a + 128) / 256), l = a - 256 h, done on both halves at once:
 //   l + 128 = lo_byte ^ 0x80,   h + 128 = (hi_byte ^ 0x80) + (lo_byte >> 7),
 // each placed under the fp16 exponent of 1024 (bits 0x6400) and recovered
-// exactly by one fp16 subtraction of 1152.
+// exactly by one fp16 subtraction of 1152.  Every limb product is at most 2^14
+// in magnitude, so a chunk of 512 * CS reduction indices sums exactly in fp32.
 //
-// TMEM: eight 64-column accumulator slots (three live, five spare).  Every
-// mbarrier wait is bounded; a wait that runs out records GEMMI_ETIMEOUT.
+// TMEM (512 columns): two A limb stages of 64 columns (high limb 0-31, low
+// 32-63; K packed two fp16 per column) and three 128-column accumulator slots
+// (two live, one spare).  Every mbarrier wait is bounded; a wait that runs out
+// records GEMMI_ETIMEOUT.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -40,37 +56,56 @@ namespace gemmi {
 namespace {
 
 using namespace tc;
-using S = Scheme<2>;
 
-constexpr int BN = 64;
+constexpr int BN = 64;                        // output tile width
+constexpr int UMMA_N = 2 * BN;                // B's two limbs stacked
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int A_PRODUCER_WARP = 8;
 constexpr int B_PRODUCER_WARP = 9;
 constexpr int MMA_WARP0 = 10;
 constexpr int NISSUE = 2;
 constexpr int NUM_THREADS = (NUM_EPI_WARPS + 2 + NISSUE) * 32;
-constexpr int NSLOT = 8;
-constexpr int SLOT_COLS = 64;
-constexpr int TMEM_COLS = NSLOT * SLOT_COLS;  // 512
-constexpr int STAGES = 3;                     // limb stages
-constexpr int RAW_STAGES = 4;                 // raw A stages
-constexpr int TILE_A = BM * BK * 2;           // 16 KB: a raw int16 A tile, and each A limb tile
-constexpr int TILE_B = BN * BK * 2;           // 8 KB: each B limb tile
-constexpr int SB = 2 * TILE_A + 2 * TILE_B;   // limb stage: AH, AL, BH, BL
-constexpr int LOOKAHEAD = 2;                  // conversions run ahead of drains (< STAGES)
+constexpr int NACC = 2;                       // accumulator p: A limb p times both B limbs
+constexpr int NSLOT = 3;
+constexpr int SLOT_COLS = UMMA_N;             // 128
+constexpr int A_STAGES = 2;                   // A limb stages in TMEM
+constexpr int A_STAGE_COLS = BK;              // 2 limbs x 64 fp16 / 2 per column
+constexpr int ACC_COL0 = A_STAGES * A_STAGE_COLS;
+constexpr int TMEM_COLS = 512;
+static_assert(ACC_COL0 + NSLOT * SLOT_COLS <= TMEM_COLS, "tensor memory budget");
+constexpr int TILE_RAW = BM * BK * 2;         // 16 KB: a raw int16 A tile
+constexpr int TILE_B = UMMA_N * BK * 2;       // 16 KB: the stacked B limb tiles
+constexpr int RAW_STAGES = 7;
+constexpr int B_STAGES = 3;
+constexpr int LOOKAHEAD = 1;                  // conversions run ahead of drains (< A_STAGES)
 constexpr int COLS = 32;                      // C columns per epilogue thread
-constexpr int CHUNKS_PER_WARP = TILE_A / 16 / NUM_EPI_WARPS;  // 16-byte chunks converted per warp
-constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + static_cast<size_t>(RAW_STAGES) * TILE_A +
-                        8 * (2 * STAGES + 2 * RAW_STAGES + 2 * NSLOT + 1) + 16;
+constexpr int STG_ROW = BN * 8;               // staging: dense int64 rows of the C tile
+constexpr int STG_QUAD = 32 * STG_ROW;        // the 32 rows of one TMEM lane quadrant (16 KB)
+constexpr int OFF_B = RAW_STAGES * TILE_RAW;
+constexpr int OFF_STG = OFF_B + B_STAGES * TILE_B;
+constexpr int OFF_BAR = OFF_STG + 4 * STG_QUAD;
+constexpr int NBAR = 2 * RAW_STAGES + 2 * A_STAGES + 2 * B_STAGES + 2 * NSLOT + 1 + 2 * 4;
+constexpr size_t SMEM = 1024 + static_cast<size_t>(OFF_BAR) + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
-static_assert(LOOKAHEAD < STAGES, "conversions may not wait on MMAs that wait on later drains");
+static_assert(LOOKAHEAD < A_STAGES, "conversions may not wait on MMAs that wait on later drains");
+static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0, "swizzled tiles start on 1024-byte boundaries");
+
+// The two accumulators' exact chunks: 512 * CS reduction indices, staggered by half a chunk.
+template <int CS>
+__device__ __forceinline__ bool chunk_ends(int a, int kb, int nkb) {
+  return kb == nkb - 1 || (((kb + 1) * BK + a * 256 * CS) % (512 * CS)) == 0;
+}
+// weights of accumulator a's two column halves: A limb a times B limb 0 (high) and 1 (low)
+__device__ __forceinline__ int shift_left_half(int a) { return a == 0 ? 16 : 8; }
+__device__ __forceinline__ int shift_right_half(int a) { return a == 0 ? 8 : 0; }
 
 struct FusedParams {
   int64_t m, n, k;
   int64_t* C;
   int64_t ldc;
   int num_m_tiles, num_n_tiles, num_k_blocks;
-  int c_vec;
+  int c_bulk;   // C base 16-byte aligned and ldc even: the tile goes out as bulk reductions
+  int c_dense;  // also n == ldc == 64: the 32 rows of a lane quadrant are one 16 KB block of C
   int group_m;
   uint64_t timeout_ns;
   uint32_t* status;
@@ -98,41 +133,96 @@ __device__ __forceinline__ void split_centred(uint32_t x, uint32_t& hi, uint32_t
   hi = *reinterpret_cast<const uint32_t*>(&h);
 }
 
+// Writes this thread's 32 accumulated values (one C row segment) into its row of the dense
+// staging block.  Row segments of consecutive lanes are 512 bytes apart, so storing the same
+// 16-byte chunk on every lane would hit one bank group eight times per quarter warp; instead
+// step c stores chunk c ^ (lane % 8), and the values are first permuted to match by three
+// conditional swaps of register pairs (static indexing keeps them in registers).
+__device__ __forceinline__ void stage_row(uint32_t row_addr, uint64_t (&acc)[COLS], uint32_t lane) {
+  const uint32_t x = lane & 7u;
+#pragma unroll
+  for (int b = 0; b < 3; ++b) {
+    const bool sw = (x >> b) & 1u;
+#pragma unroll
+    for (int j = 0; j < COLS / 2; ++j) {
+      if (j & (1 << b)) continue;
+      const int j2 = j | (1 << b);
+      const uint64_t a0 = acc[2 * j], a1 = acc[2 * j + 1], b0 = acc[2 * j2], b1 = acc[2 * j2 + 1];
+      acc[2 * j] = sw ? b0 : a0;
+      acc[2 * j + 1] = sw ? b1 : a1;
+      acc[2 * j2] = sw ? a0 : b0;
+      acc[2 * j2 + 1] = sw ? a1 : b1;
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < COLS / 2; ++c) {
+    uint4 v;
+    v.x = static_cast<uint32_t>(acc[2 * c]);
+    v.y = static_cast<uint32_t>(acc[2 * c] >> 32);
+    v.z = static_cast<uint32_t>(acc[2 * c + 1]);
+    v.w = static_cast<uint32_t>(acc[2 * c + 1] >> 32);
+    sts128(row_addr + ((static_cast<uint32_t>(c) ^ x) << 4), v);
+  }
+}
+
+// Adds `count` staged columns of one row into C: the even part as one bulk reduction, an odd
+// last column by an atomic add read back from the staging row.
+__device__ __forceinline__ void reduce_row(int64_t* dst, uint32_t stage_row, int count) {
+  const int even = count & ~1;
+  if (even > 0) bulk_reduce_add_u64(dst, stage_row, static_cast<uint32_t>(even * 8));
+  if (count & 1) {
+    unsigned long long last;
+    asm volatile("ld.shared.u64 %0, [%1];" : "=l"(last) : "r"(stage_row + (count - 1) * 8));
+    atomicAdd(reinterpret_cast<unsigned long long*>(dst + count - 1), last);
+  }
+}
+
 template <int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapBH,
              const __grid_constant__ CUtensorMap mapBL, FusedParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* raw = smem + STAGES * SB;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(raw + RAW_STAGES * TILE_A);
-  const uint32_t full0 = smem_u32(bars);
-  const uint32_t empty0 = full0 + 8 * STAGES;
-  const uint32_t rfull0 = empty0 + 8 * STAGES;
-  const uint32_t rempty0 = rfull0 + 8 * RAW_STAGES;
-  const uint32_t sfull0 = rempty0 + 8 * RAW_STAGES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  const uint32_t raw_full0 = smem_u32(bars);                 // raw A tile landed
+  const uint32_t raw_empty0 = raw_full0 + 8 * RAW_STAGES;    // raw A tile converted by the 8 epilogue warps
+  const uint32_t a_ready0 = raw_empty0 + 8 * RAW_STAGES;     // A limbs stored in TMEM by the 8 epilogue warps
+  const uint32_t a_empty0 = a_ready0 + 8 * A_STAGES;         // both issuers' MMAs on the A limb stage completed
+  const uint32_t b_full0 = a_empty0 + 8 * A_STAGES;          // B limb tiles landed
+  const uint32_t b_empty0 = b_full0 + 8 * B_STAGES;          // both issuers' MMAs on the B limbs completed
+  const uint32_t sfull0 = b_empty0 + 8 * B_STAGES;
   const uint32_t sempty0 = sfull0 + 8 * NSLOT;
   const uint32_t final_bar = sempty0 + 8 * NSLOT;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2 * RAW_STAGES + 2 * NSLOT + 1);
+  const uint32_t stg_free0 = final_bar + 8;        // per quadrant: its staging block has been read
+  const uint32_t stg_full0 = stg_free0 + 8 * 4;    // per quadrant: both warps have staged their rows
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + NBAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(full0 + 8 * s, 1 + NUM_EPI_WARPS);  // B producer's expect_tx arrival + 8 converter warps
-      mbar_init(empty0 + 8 * s, NISSUE);
-    }
     for (int s = 0; s < RAW_STAGES; ++s) {
-      mbar_init(rfull0 + 8 * s, 1);
-      mbar_init(rempty0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(raw_full0 + 8 * s, 1);
+      mbar_init(raw_empty0 + 8 * s, NUM_EPI_WARPS);
+    }
+    for (int s = 0; s < A_STAGES; ++s) {
+      mbar_init(a_ready0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(a_empty0 + 8 * s, NISSUE);
+    }
+    for (int s = 0; s < B_STAGES; ++s) {
+      mbar_init(b_full0 + 8 * s, 1);
+      mbar_init(b_empty0 + 8 * s, NISSUE);
     }
     for (int s = 0; s < NSLOT; ++s) {
       mbar_init(sfull0 + 8 * s, 1);
       mbar_init(sempty0 + 8 * s, NUM_EPI_WARPS);
     }
     mbar_init(final_bar, NISSUE);
+    for (int qd = 0; qd < 4; ++qd) {
+      mbar_init(stg_free0 + 8 * qd, 1);
+      mbar_init(stg_full0 + 8 * qd, 2);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -153,118 +243,94 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
                            : 0;
   const int64_t total_q = static_cast<int64_t>(my_tiles) * nkb;  // this CTA's K blocks, over its tiles
 
-  if (warp == A_PRODUCER_WARP) {
-    // ------------------------------------------------------------ raw A tiles
+  if (warp == A_PRODUCER_WARP || warp == B_PRODUCER_WARP) {
+    // ------------------------------------------------------------ TMA producers
+    const bool is_a = warp == A_PRODUCER_WARP;
+    const int nst = is_a ? RAW_STAGES : B_STAGES;
+    const uint32_t full0 = is_a ? raw_full0 : b_full0;
+    const uint32_t empty0 = is_a ? raw_empty0 : b_empty0;
     if (lane == 0) {
-      tma_prefetch_desc(&mapA);
-      int64_t issued = 0;
-      for (int64_t q = 0; q < total_q; ++q) {
-        const int i = static_cast<int>(q / nkb), kb = static_cast<int>(q % nkb);
-        int mt, nt;
-        tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
-                    P.group_m, mt, nt);
-        const int r = static_cast<int>(q % RAW_STAGES);
-        const uint32_t par = static_cast<uint32_t>((q / RAW_STAGES) & 1);
-        if (!bounded_wait(rempty0 + 8 * r, par ^ 1u, P.timeout_ns) || *abort_flag) {
-          report_status(P.status, STATUS_TIMEOUT, 21);
-          *abort_flag = 1;
-          break;
-        }
-        mbar_arrive_expect_tx(rfull0 + 8 * r, TILE_A);
-        tma_load_2d(smem_u32(raw + r * TILE_A), &mapA, rfull0 + 8 * r, kb * BK, mt * BM);
-        ++issued;
+      if (is_a) {
+        tma_prefetch_desc(&mapA);
+      } else {
+        tma_prefetch_desc(&mapBH);
+        tma_prefetch_desc(&mapBL);
       }
-      for (int64_t q = issued > RAW_STAGES ? issued - RAW_STAGES : 0; q < issued; ++q)
-        bounded_wait(rfull0 + 8 * static_cast<int>(q % RAW_STAGES), static_cast<uint32_t>((q / RAW_STAGES) & 1),
-                     P.timeout_ns);
-    }
-  } else if (warp == B_PRODUCER_WARP) {
-    // ------------------------------------------------------------ B limb tiles
-    if (lane == 0) {
-      tma_prefetch_desc(&mapBH);
-      tma_prefetch_desc(&mapBL);
       int64_t issued = 0;
       for (int64_t q = 0; q < total_q; ++q) {
         const int i = static_cast<int>(q / nkb), kb = static_cast<int>(q % nkb);
         int mt, nt;
         tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
                     P.group_m, mt, nt);
-        const int s = static_cast<int>(q % STAGES);
-        const uint32_t par = static_cast<uint32_t>((q / STAGES) & 1);
+        const int s = static_cast<int>(q % nst);
+        const uint32_t par = static_cast<uint32_t>((q / nst) & 1);
         if (!bounded_wait(empty0 + 8 * s, par ^ 1u, P.timeout_ns) || *abort_flag) {
-          report_status(P.status, STATUS_TIMEOUT, 22);
+          report_status(P.status, STATUS_TIMEOUT, is_a ? 21 : 22);
           *abort_flag = 1;
           break;
         }
         const uint32_t fb = full0 + 8 * s;
-        const uint32_t base = smem_u32(smem + s * SB);
-        mbar_arrive_expect_tx(fb, 2 * TILE_B);
-        tma_load_2d(base + 2 * TILE_A, &mapBH, fb, kb * BK, nt * BN);
-        tma_load_2d(base + 2 * TILE_A + TILE_B, &mapBL, fb, kb * BK, nt * BN);
+        if (is_a) {
+          mbar_arrive_expect_tx(fb, TILE_RAW);
+          tma_load_2d(smem_u32(smem + s * TILE_RAW), &mapA, fb, kb * BK, mt * BM);
+        } else {
+          const uint32_t base = smem_u32(smem + OFF_B + s * TILE_B);
+          mbar_arrive_expect_tx(fb, TILE_B);
+          tma_load_2d(base, &mapBH, fb, kb * BK, nt * BN);
+          tma_load_2d(base + TILE_B / 2, &mapBL, fb, kb * BK, nt * BN);
+        }
         ++issued;
       }
-      for (int64_t q = issued > STAGES ? issued - STAGES : 0; q < issued; ++q)
-        bounded_wait(full0 + 8 * static_cast<int>(q % STAGES), static_cast<uint32_t>((q / STAGES) & 1), P.timeout_ns);
+      for (int64_t q = issued > nst ? issued - nst : 0; q < issued; ++q)
+        bounded_wait(full0 + 8 * static_cast<int>(q % nst), static_cast<uint32_t>((q / nst) & 1), P.timeout_ns);
     }
   } else if (warp >= MMA_WARP0) {
-    // ------------------------------------------------------------ MMA issuers
+    // ------------------------------------------------------------ MMA issuers (issuer me owns accumulator me)
     const int me = warp - MMA_WARP0;
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
-      SlotRing<S::NACC, NSLOT> ring;
+      constexpr uint32_t idesc = idesc_f16_f32(BM, UMMA_N);
+      SlotRing<NACC, NSLOT> ring;
       ring.init();
-      uint32_t wait_par[S::NACC];
-      bool need_acquire[S::NACC], fresh[S::NACC];
-#pragma unroll
-      for (int a = 0; a < S::NACC; ++a) {
-        wait_par[a] = 1u;
-        need_acquire[a] = true;
-        fresh[a] = true;
-      }
+      uint32_t wait_par = 1u;
+      bool need_acquire = true, fresh = true;
       bool ok = true;
       for (int64_t q = 0; q < total_q && ok; ++q) {
         const int kb = static_cast<int>(q % nkb);
-        const int s = static_cast<int>(q % STAGES);
-        if (!bounded_wait(full0 + 8 * s, static_cast<uint32_t>((q / STAGES) & 1), P.timeout_ns)) {
+        const int sa = static_cast<int>(q % A_STAGES);
+        const int sb = static_cast<int>(q % B_STAGES);
+        if (!bounded_wait(a_ready0 + 8 * sa, static_cast<uint32_t>((q / A_STAGES) & 1), P.timeout_ns) ||
+            !bounded_wait(b_full0 + 8 * sb, static_cast<uint32_t>((q / B_STAGES) & 1), P.timeout_ns)) {
           report_status(P.status, STATUS_TIMEOUT, 23);
           *abort_flag = 1;
           break;
         }
-        tc_fence_after();
-        const uint32_t base = smem_u32(smem + s * SB);
-#pragma unroll
-        for (int p = 0; p < S::NPROD; ++p) {
-          if (S::issuer(p, kb) != me) continue;
-          const int a = S::acc(p, kb);
-          if (need_acquire[a]) {
-            if (!bounded_wait(sempty0 + 8 * ring.slot_of[a], wait_par[a], P.timeout_ns)) {
-              report_status(P.status, STATUS_TIMEOUT, 24);
-              *abort_flag = 1;
-              ok = false;
-              break;
-            }
-            need_acquire[a] = false;
-            tc_fence_after();
+        if (need_acquire) {
+          if (!bounded_wait(sempty0 + 8 * ring.slot_of[me], wait_par, P.timeout_ns)) {
+            report_status(P.status, STATUS_TIMEOUT, 24);
+            *abort_flag = 1;
+            break;
           }
-          const uint32_t d = tmem_base + static_cast<uint32_t>(ring.slot_of[a] * SLOT_COLS);
-          const uint64_t adesc = smem_desc_kmajor<128>(base + S::a_limb(p) * TILE_A);
-          const uint64_t bdesc = smem_desc_kmajor<128>(base + 2 * TILE_A + S::b_limb(p) * TILE_B);
-#pragma unroll
-          for (int kk = 0; kk < BK / UMMA_K; ++kk)
-            tc_mma_f16(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (fresh[a] && kk == 0) ? 0u : 1u);
-          fresh[a] = false;
+          need_acquire = false;
         }
-        if (!ok) break;
-        tc_commit(empty0 + 8 * s);
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(ACC_COL0 + ring.slot_of[me] * SLOT_COLS);
+        const uint32_t a_tmem = tmem_base + static_cast<uint32_t>(sa * A_STAGE_COLS + me * (BK / 2));
+        const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + sb * TILE_B));
 #pragma unroll
-        for (int a = 0; a < S::NACC; ++a) {
-          if (!S::template chunk_ends<CS>(a, kb, nkb)) continue;
-          if (S::owner(a) == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);
+        for (int kk = 0; kk < BK / UMMA_K; ++kk)
+          tc_mma_f16_ts(d, a_tmem + kk * (UMMA_K / 2), bdesc + 2 * kk, idesc, (fresh && kk == 0) ? 0u : 1u);
+        fresh = false;
+        tc_commit(a_empty0 + 8 * sa);
+        tc_commit(b_empty0 + 8 * sb);
+#pragma unroll
+        for (int a = 0; a < NACC; ++a) {
+          if (!chunk_ends<CS>(a, kb, nkb)) continue;
+          if (a == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);
           const uint32_t par = ring.rotate(a);
-          if (S::owner(a) == me) {
-            wait_par[a] = par;
-            need_acquire[a] = true;
-            fresh[a] = true;
+          if (a == me) {
+            wait_par = par;
+            need_acquire = true;
+            fresh = true;
           }
         }
       }
@@ -272,79 +338,76 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       bounded_wait(final_bar, 0, P.timeout_ns);
     }
   } else {
-    // ------------------------------------------------------------ epilogue: convert A, drain, C
+    // ------------------------------------------------------------ epilogue: convert A, drain, reduce into C
     const int quad = warp & 3;
     const int half = warp >> 2;
-    SlotRing<S::NACC, NSLOT> ring;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;  // TMEM lane field of this quadrant
+    SlotRing<NACC, NSLOT> ring;
     ring.init();
     uint32_t drain_parity = 0;
     bool ok = true;
     int64_t cq = 0;  // next K block (over this CTA's tiles) whose A tile this warp converts
 
-    // Converts this warp's share of raw A tile qq into the A limb tiles of its limb stage.
+    // Splits this thread's half K block (32 indices of row 32*quad + lane) of K block qq into its
+    // two limbs and stores them in the A limb stage of qq.
     auto convert = [&](int64_t qq) -> bool {
       const int r = static_cast<int>(qq % RAW_STAGES);
-      const int s = static_cast<int>(qq % STAGES);
-      const bool got_raw = bounded_wait(rfull0 + 8 * r, static_cast<uint32_t>((qq / RAW_STAGES) & 1), P.timeout_ns);
-      const bool got_stage =
-          got_raw && bounded_wait(empty0 + 8 * s, static_cast<uint32_t>(((qq / STAGES) & 1) ^ 1), P.timeout_ns);
-      if (!__all_sync(0xFFFFFFFFu, got_stage)) {
+      const int sa = static_cast<int>(qq % A_STAGES);
+      const bool got_raw =
+          bounded_wait(raw_full0 + 8 * r, static_cast<uint32_t>((qq / RAW_STAGES) & 1), P.timeout_ns);
+      const bool got = got_raw && bounded_wait(a_empty0 + 8 * sa, static_cast<uint32_t>(((qq / A_STAGES) & 1) ^ 1),
+                                               P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, got)) {
         if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
         *abort_flag = 1;
         return false;
       }
-      const uint32_t src = smem_u32(raw + r * TILE_A);
-      const uint32_t dst_h = smem_u32(smem + s * SB);
-      const uint32_t dst_l = dst_h + TILE_A;
+      tc_fence_after();
+      // the raw tile's row `row` is 128 bytes; 16-byte chunk c sits at chunk c ^ (row % 8) (128-byte swizzle)
+      const uint32_t row = static_cast<uint32_t>(quad * 32 + lane);
+      const uint32_t src = smem_u32(smem + r * TILE_RAW) + row * 128;
+      uint32_t hi[16], lo[16];
 #pragma unroll
-      for (int c = 0; c < CHUNKS_PER_WARP / 32; ++c) {
-        const uint32_t off = static_cast<uint32_t>((warp * CHUNKS_PER_WARP + c * 32 + lane) * 16);
-        const uint4 x = lds128(src + off);
-        uint4 h, l;
-        split_centred(x.x, h.x, l.x);
-        split_centred(x.y, h.y, l.y);
-        split_centred(x.z, h.z, l.z);
-        split_centred(x.w, h.w, l.w);
-        sts128(dst_h + off, h);
-        sts128(dst_l + off, l);
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t c = static_cast<uint32_t>(half * 4 + i);
+        const uint4 x = lds128(src + ((c ^ (row & 7u)) << 4));
+        split_centred(x.x, hi[4 * i + 0], lo[4 * i + 0]);
+        split_centred(x.y, hi[4 * i + 1], lo[4 * i + 1]);
+        split_centred(x.z, hi[4 * i + 2], lo[4 * i + 2]);
+        split_centred(x.w, hi[4 * i + 3], lo[4 * i + 3]);
       }
-      fence_proxy_async_smem();  // the tensor core reads these tiles through the async proxy
+      const uint32_t t = tmem_base + lane_base + static_cast<uint32_t>(sa * A_STAGE_COLS + half * 16);
+      tc_st_32x32b_x16(t, hi);
+      tc_st_32x32b_x16(t + BK / 2, lo);
+      tc_wait_st();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        mbar_arrive(full0 + 8 * s);
-        mbar_arrive(rempty0 + 8 * r);
+        mbar_arrive(raw_empty0 + 8 * r);
+        mbar_arrive(a_ready0 + 8 * sa);
       }
       return true;
     };
+
+    uint64_t acc[COLS];
+    const uint32_t quad_stage = smem_u32(smem + OFF_STG + quad * STG_QUAD);
+    uint32_t tile_ends = 0;  // staged tile ends so far (the quadrant barriers' phase)
 
     int64_t q = 0;
     for (int i = 0; i < my_tiles && ok; ++i) {
       int mt, nt;
       tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
                   P.group_m, mt, nt);
-      const int64_t row = static_cast<int64_t>(mt) * BM + quad * 32 + lane;
-      const int64_t col0 = static_cast<int64_t>(nt) * BN + half * COLS;
-      int64_t* crow = P.C + row * P.ldc + col0;
-      const bool row_ok = row < P.m;
-      const bool full_cols = col0 + COLS <= P.n;
-      uint64_t acc[COLS];
-      if (row_ok && full_cols && P.c_vec) {
-#pragma unroll
-        for (int c = 0; c < COLS; c += 2) {
-          const longlong2 v = *reinterpret_cast<const longlong2*>(crow + c);
-          acc[c] = static_cast<uint64_t>(v.x);
-          acc[c + 1] = static_cast<uint64_t>(v.y);
-        }
-      } else {
-#pragma unroll
-        for (int c = 0; c < COLS; ++c) acc[c] = (row_ok && col0 + c < P.n) ? static_cast<uint64_t>(crow[c]) : 0ull;
-      }
       for (int kb = 0; kb < nkb && ok; ++kb, ++q) {
         while (ok && cq <= q + LOOKAHEAD && cq < total_q) ok = convert(cq++);
         if (!ok) break;
+        if (kb == 0) {
 #pragma unroll
-        for (int a = 0; a < S::NACC; ++a) {
-          if (!S::template chunk_ends<CS>(a, kb, nkb)) continue;
+          for (int c = 0; c < COLS; ++c) acc[c] = 0;
+        }
+#pragma unroll
+        for (int a = 0; a < NACC; ++a) {
+          if (!chunk_ends<CS>(a, kb, nkb)) continue;
           const int s = ring.slot_of[a];
           const bool got = bounded_wait(sfull0 + 8 * s, (drain_parity >> s) & 1u, P.timeout_ns);
           if (!__all_sync(0xFFFFFFFFu, got)) {
@@ -355,16 +418,20 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
           }
           drain_parity ^= 1u << s;
           tc_fence_after();
-          const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                                 static_cast<uint32_t>(s * SLOT_COLS + half * COLS);
-          uint32_t r0[16], r1[16];
-          tc_ld_32x32b_x16(taddr, r0);
-          tc_ld_32x32b_x16(taddr + 16, r1);
+          const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(ACC_COL0 + s * SLOT_COLS + half * COLS);
+          uint32_t l0[16], l1[16], r0[16], r1[16];
+          tc_ld_32x32b_x16(taddr, l0);
+          tc_ld_32x32b_x16(taddr + 16, l1);
+          tc_ld_32x32b_x16(taddr + BN, r0);
+          tc_ld_32x32b_x16(taddr + BN + 16, r1);
           tc_wait_ld();
+          const int sl = shift_left_half(a), sr = shift_right_half(a);
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            acc[j] += static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r0[j]))) << S::shift(a);
-            acc[16 + j] += static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r1[j]))) << S::shift(a);
+            acc[j] += (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(l0[j]))) << sl) +
+                      (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r0[j]))) << sr);
+            acc[16 + j] += (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(l1[j]))) << sl) +
+                           (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r1[j]))) << sr);
           }
           tc_fence_before();
           __syncwarp();
@@ -373,17 +440,58 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
         }
       }
       if (!ok) break;
-      if (row_ok && full_cols && P.c_vec) {
-#pragma unroll
-        for (int c = 0; c < COLS; c += 2)
-          *reinterpret_cast<longlong2*>(crow + c) =
-              make_longlong2(static_cast<long long>(acc[c]), static_cast<long long>(acc[c + 1]));
-      } else if (row_ok) {
+      // ---- C tile += acc, through the staging block and bulk reductions
+      const int64_t row0 = static_cast<int64_t>(mt) * BM + quad * 32;
+      const int64_t row = row0 + lane;
+      const int64_t tcol0 = static_cast<int64_t>(nt) * BN;
+      const int64_t left = P.n - tcol0;
+      const int tile_cols = left >= BN ? BN : static_cast<int>(left);
+      if (P.c_bulk) {
+        const uint32_t par = tile_ends & 1u;
+        if (half == 0) {  // this warp issues the quadrant's reductions: they must have read the block
+          bulk_wait_read_all();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(stg_free0 + 8 * quad);
+        } else if (!__all_sync(0xFFFFFFFFu, bounded_wait(stg_free0 + 8 * quad, par, P.timeout_ns))) {
+          if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 27);
+          *abort_flag = 1;
+          ok = false;
+          break;
+        }
+        const uint32_t my_row = quad_stage + static_cast<uint32_t>(lane * STG_ROW + half * COLS * 8);
+        stage_row(my_row, acc, lane);
+        fence_proxy_async_smem();  // the bulk reductions read the block through the async proxy
+        __syncwarp();
+        if (lane == 0) mbar_arrive(stg_full0 + 8 * quad);
+        if (half == 0) {
+          if (!__all_sync(0xFFFFFFFFu, bounded_wait(stg_full0 + 8 * quad, par, P.timeout_ns))) {
+            if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 28);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          if (P.c_dense) {
+            const int64_t rows = P.m - row0 < 32 ? P.m - row0 : 32;
+            if (lane == 0 && rows > 0) {
+              bulk_reduce_add_u64(P.C + row0 * BN, quad_stage, static_cast<uint32_t>(rows * STG_ROW));
+              bulk_commit();
+            }
+          } else if (row < P.m) {
+            reduce_row(P.C + row * P.ldc + tcol0, quad_stage + static_cast<uint32_t>(lane * STG_ROW), tile_cols);
+            bulk_commit();
+          }
+        }
+        ++tile_ends;
+      } else if (row < P.m) {
+        int64_t* crow = P.C + row * P.ldc + tcol0 + half * COLS;
+        const int valid = tile_cols - half * COLS;
 #pragma unroll
         for (int c = 0; c < COLS; ++c)
-          if (col0 + c < P.n) crow[c] = static_cast<int64_t>(acc[c]);
+          if (c < valid)
+            atomicAdd(reinterpret_cast<unsigned long long*>(crow + c), static_cast<unsigned long long>(acc[c]));
       }
     }
+    bulk_wait_all();
   }
 
   tc_fence_before();
@@ -414,7 +522,8 @@ cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
   P.num_m_tiles = static_cast<int>((a.m + BM - 1) / BM);
   P.num_n_tiles = static_cast<int>((a.n + BN - 1) / BN);
   P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
-  P.c_vec = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && (a.ldc % 2 == 0);
+  P.c_bulk = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && (a.ldc % 2 == 0);
+  P.c_dense = P.c_bulk && a.n == BN && a.ldc == BN;
   P.group_m = a.group_m > 0 ? a.group_m : 16;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;

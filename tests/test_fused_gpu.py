@@ -166,17 +166,36 @@ def test_fused_dispatch_rules(gm):
     assert_same(dC.cpu().numpy(), expected(A, B, C), "lda=104")
 
 
-def test_fused_padded_c(gm):
-    A, B, C = gi.random_problem(724, 300, 40, 577, "i16")
-    Cpad = gi.uniform_int(725, (300, 45), -(1 << 50), 1 << 50, np.int64)
-    Cpad[:, :40] = C
+# ldc odd: element-wise atomic adds; ldc even: one bulk reduction per row (n < 64 or ldc > n)
+@pytest.mark.parametrize("n,ldc", [(40, 45), (40, 48), (64, 72), (33, 34)])
+def test_fused_padded_c(gm, n, ldc):
+    A, B, C = gi.random_problem(724 + ldc, 300, n, 577, "i16")
+    Cpad = gi.uniform_int(725, (300, ldc), -(1 << 50), 1 << 50, np.int64)
+    Cpad[:, :n] = C
     dA, dB = device_a(A), torch.from_numpy(B).cuda()
     dCp = torch.from_numpy(Cpad).cuda()
-    counts = launches(gm, lambda: gm.gemm_i16(dA, dB, dCp[:, :40]))
+    counts = launches(gm, lambda: gm.gemm_i16(dA, dB, dCp[:, :n]))
     assert counts["fused_i16"] == 1, counts
     got = dCp.cpu().numpy()
-    assert_same(got[:, :40], expected(A, B, C), "ldc=45")
-    assert np.array_equal(got[:, 40:], Cpad[:, 40:]), "columns beyond n were written"
+    assert_same(got[:, :n], expected(A, B, C), f"ldc={ldc}")
+    assert np.array_equal(got[:, n:], Cpad[:, n:]), "columns beyond n were written"
+
+
+def test_fused_c_not_16_byte_aligned(gm):
+    # C starts 8 bytes into a buffer: row segments cannot go out as 16-byte bulk reductions,
+    # the kernel adds them element by element
+    A, B, C = gi.random_problem(728, 400, 64, 300, "i16")
+    Cbuf = gi.uniform_int(729, (400, 66), -(1 << 50), 1 << 50, np.int64)
+    Cbuf[:, 1:65] = C
+    dA, dB = device_a(A), torch.from_numpy(B).cuda()
+    dCb = torch.from_numpy(Cbuf).cuda()
+    view = dCb[:, 1:65]
+    assert view.data_ptr() % 16 == 8
+    counts = launches(gm, lambda: gm.gemm_i16(dA, dB, view))
+    assert counts["fused_i16"] == 1, counts
+    got = dCb.cpu().numpy()
+    assert_same(got[:, 1:65], expected(A, B, C), "C offset by 8 bytes")
+    assert np.array_equal(got[:, [0, 65]], Cbuf[:, [0, 65]]), "columns outside C were written"
 
 
 def test_fused_with_packed_weights(gm):
