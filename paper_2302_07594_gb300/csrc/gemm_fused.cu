@@ -13,7 +13,7 @@
 // Roles (one CTA per SM, 128 x 64 output tiles, K blocks of 64):
 //   warp 8      TMA producer of raw A tiles (128 rows x 64 reduction indices of
 //               int16, 128-byte swizzle) into a ring of RAW_STAGES slots.  A slot
-//               is free again once its tile has been converted, so the HBM
+//               is free again as soon as the converters have read it, so the HBM
 //               stream never waits for the tensor cores; the ring is deep
 //               because nothing else of A lives in shared memory.
 //   warp 9      TMA producer of B's two limb tiles (64 x 64 fp16 each, stacked
@@ -22,15 +22,14 @@
 //               which sits in tensor memory, by the stacked B tile with one
 //               tcgen05.mma of N = 128: columns 0-63 of its accumulator get
 //               A_p * B_high, columns 64-127 get A_p * B_low.
+//   warps 12-15 converters.  Thread (warp 12 + j, lane t) splits row 32j + t of
+//               each raw tile into the two fp16 limbs and stores them in its
+//               TMEM lane of the A limb stage (tcgen05.st).
 //   warps 0-7   epilogue.  Warp (quadrant q = w % 4, half h = w / 4), lane t,
-//               owns row 32q + t of the tile.  It splits K-block halves of its
-//               row (32 reduction indices) from the raw slot into the two fp16
-//               limbs and writes them into the A limb stage in tensor memory
-//               (tcgen05.st), LOOKAHEAD K blocks ahead of its main job: draining
-//               the accumulators (staggered exact chunks) into int64 registers
-//               for output columns 32h .. 32h + 31.  At the end of a tile the
-//               two warps of a quadrant write their 32 rows into a dense
-//               staging block that goes out as one bulk reduction
+//               drains row 32q + t, output columns 32h .. 32h + 31, of the
+//               accumulators (staggered exact chunks) into int64 registers.  At
+//               the end of a tile the two warps of a quadrant write their 32 rows
+//               into a dense staging block that goes out as one bulk reduction
 //               (cp.reduce.async.bulk .add.u64) when C's rows are 64 wide and
 //               contiguous, or as one reduction per row otherwise.
 //
@@ -64,7 +63,10 @@ constexpr int A_PRODUCER_WARP = 8;
 constexpr int B_PRODUCER_WARP = 9;
 constexpr int MMA_WARP0 = 10;
 constexpr int NISSUE = 2;
-constexpr int NUM_THREADS = (NUM_EPI_WARPS + 2 + NISSUE) * 32;
+constexpr int CONV_WARP0 = 12;                // converter warpgroup: warp 12 + j serves TMEM lanes 32j .. 32j + 31
+constexpr int NUM_CONV_WARPS = 4;
+constexpr int NUM_THREADS = (CONV_WARP0 + NUM_CONV_WARPS) * 32;
+static_assert(CONV_WARP0 % 4 == 0, "a warp reaches the TMEM lane quadrant of its warp index modulo 4");
 constexpr int NACC = 2;                       // accumulator p: A limb p times both B limbs
 constexpr int NSLOT = 3;
 constexpr int SLOT_COLS = UMMA_N;             // 128
@@ -77,7 +79,6 @@ constexpr int TILE_RAW = BM * BK * 2;         // 16 KB: a raw int16 A tile
 constexpr int TILE_B = UMMA_N * BK * 2;       // 16 KB: the stacked B limb tiles
 constexpr int RAW_STAGES = 7;
 constexpr int B_STAGES = 3;
-constexpr int LOOKAHEAD = 1;                  // conversions run ahead of drains (< A_STAGES)
 constexpr int COLS = 32;                      // C columns per epilogue thread
 constexpr int STG_ROW = BN * 8;               // staging: dense int64 rows of the C tile
 constexpr int STG_QUAD = 32 * STG_ROW;        // the 32 rows of one TMEM lane quadrant (16 KB)
@@ -87,7 +88,6 @@ constexpr int OFF_BAR = OFF_STG + 4 * STG_QUAD;
 constexpr int NBAR = 2 * RAW_STAGES + 2 * A_STAGES + 2 * B_STAGES + 2 * NSLOT + 1 + 2 * 4;
 constexpr size_t SMEM = 1024 + static_cast<size_t>(OFF_BAR) + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
-static_assert(LOOKAHEAD < A_STAGES, "conversions may not wait on MMAs that wait on later drains");
 static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0, "swizzled tiles start on 1024-byte boundaries");
 
 // The two accumulators' exact chunks: 512 * CS reduction indices, staggered by half a chunk.
@@ -185,8 +185,8 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   const uint32_t raw_full0 = smem_u32(bars);                 // raw A tile landed
-  const uint32_t raw_empty0 = raw_full0 + 8 * RAW_STAGES;    // raw A tile converted by the 8 epilogue warps
-  const uint32_t a_ready0 = raw_empty0 + 8 * RAW_STAGES;     // A limbs stored in TMEM by the 8 epilogue warps
+  const uint32_t raw_empty0 = raw_full0 + 8 * RAW_STAGES;    // raw A tile read by the 4 converter warps
+  const uint32_t a_ready0 = raw_empty0 + 8 * RAW_STAGES;     // A limbs stored in TMEM by the 4 converter warps
   const uint32_t a_empty0 = a_ready0 + 8 * A_STAGES;         // both issuers' MMAs on the A limb stage completed
   const uint32_t b_full0 = a_empty0 + 8 * A_STAGES;          // B limb tiles landed
   const uint32_t b_empty0 = b_full0 + 8 * B_STAGES;          // both issuers' MMAs on the B limbs completed
@@ -204,10 +204,10 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
   if (threadIdx.x == 0) {
     for (int s = 0; s < RAW_STAGES; ++s) {
       mbar_init(raw_full0 + 8 * s, 1);
-      mbar_init(raw_empty0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(raw_empty0 + 8 * s, NUM_CONV_WARPS);
     }
     for (int s = 0; s < A_STAGES; ++s) {
-      mbar_init(a_ready0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(a_ready0 + 8 * s, NUM_CONV_WARPS);
       mbar_init(a_empty0 + 8 * s, NISSUE);
     }
     for (int s = 0; s < B_STAGES; ++s) {
@@ -256,34 +256,94 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
         tma_prefetch_desc(&mapBH);
         tma_prefetch_desc(&mapBL);
       }
+      RingPos pos;
       int64_t issued = 0;
-      for (int64_t q = 0; q < total_q; ++q) {
-        const int i = static_cast<int>(q / nkb), kb = static_cast<int>(q % nkb);
+      bool stop = false;
+      for (int i = 0; i < my_tiles && !stop; ++i) {
         int mt, nt;
         tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
                     P.group_m, mt, nt);
-        const int s = static_cast<int>(q % nst);
-        const uint32_t par = static_cast<uint32_t>((q / nst) & 1);
-        if (!bounded_wait(empty0 + 8 * s, par ^ 1u, P.timeout_ns) || *abort_flag) {
-          report_status(P.status, STATUS_TIMEOUT, is_a ? 21 : 22);
-          *abort_flag = 1;
-          break;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!bounded_wait(empty0 + 8 * pos.slot, pos.phase ^ 1u, P.timeout_ns) || *abort_flag) {
+            report_status(P.status, STATUS_TIMEOUT, is_a ? 21 : 22);
+            *abort_flag = 1;
+            stop = true;
+            break;
+          }
+          const uint32_t fb = full0 + 8 * pos.slot;
+          if (is_a) {
+            mbar_arrive_expect_tx(fb, TILE_RAW);
+            tma_load_2d(smem_u32(smem + pos.slot * TILE_RAW), &mapA, fb, kb * BK, mt * BM);
+          } else {
+            const uint32_t base = smem_u32(smem + OFF_B + pos.slot * TILE_B);
+            mbar_arrive_expect_tx(fb, TILE_B);
+            tma_load_2d(base, &mapBH, fb, kb * BK, nt * BN);
+            tma_load_2d(base + TILE_B / 2, &mapBL, fb, kb * BK, nt * BN);
+          }
+          pos.advance(nst);
+          ++issued;
         }
-        const uint32_t fb = full0 + 8 * s;
-        if (is_a) {
-          mbar_arrive_expect_tx(fb, TILE_RAW);
-          tma_load_2d(smem_u32(smem + s * TILE_RAW), &mapA, fb, kb * BK, mt * BM);
-        } else {
-          const uint32_t base = smem_u32(smem + OFF_B + s * TILE_B);
-          mbar_arrive_expect_tx(fb, TILE_B);
-          tma_load_2d(base, &mapBH, fb, kb * BK, nt * BN);
-          tma_load_2d(base + TILE_B / 2, &mapBL, fb, kb * BK, nt * BN);
-        }
-        ++issued;
       }
-      for (int64_t q = issued > nst ? issued - nst : 0; q < issued; ++q)
-        bounded_wait(full0 + 8 * static_cast<int>(q % nst), static_cast<uint32_t>((q / nst) & 1), P.timeout_ns);
+      // the copies still in flight: slots below pos.slot in this round, the others in the last one
+      for (int x = 0; x < nst; ++x) {
+        if (x < pos.slot)
+          bounded_wait(full0 + 8 * x, pos.phase, P.timeout_ns);
+        else if (issued >= nst)
+          bounded_wait(full0 + 8 * x, pos.phase ^ 1u, P.timeout_ns);
+      }
     }
+  } else if (warp >= CONV_WARP0) {
+    // ------------------------------------------------------------ converters: raw A -> limbs in TMEM
+    // Thread (warp 12 + j, lane t) converts row 32j + t of every raw tile: it loads the row's eight
+    // 16-byte chunks (128-byte swizzle: chunk c sits at c ^ (row % 8)), hands the raw slot back at
+    // once, splits the 64 values into their two limbs and stores them in its TMEM lane.
+    const int quad = warp - CONV_WARP0;
+    const uint32_t row = static_cast<uint32_t>(quad * 32 + lane);
+    const uint32_t lane_field = static_cast<uint32_t>(quad * 32) << 16;
+    RingPos craw, cstage;
+    bool ok = true;
+    for (int64_t q = 0; q < total_q && ok; ++q) {
+      const bool got = bounded_wait(raw_full0 + 8 * craw.slot, craw.phase, P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, got)) {
+        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
+        *abort_flag = 1;
+        break;
+      }
+      const uint32_t src = smem_u32(smem + craw.slot * TILE_RAW) + row * 128;
+      uint4 x[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) x[c] = lds128(src + ((static_cast<uint32_t>(c) ^ (row & 7u)) << 4));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(raw_empty0 + 8 * craw.slot);
+      craw.advance(RAW_STAGES);
+      const bool free_stage = bounded_wait(a_empty0 + 8 * cstage.slot, cstage.phase ^ 1u, P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, free_stage)) {
+        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 29);
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t t = tmem_base + lane_field + static_cast<uint32_t>(cstage.slot * A_STAGE_COLS);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {  // 32 reduction indices per TMEM store of 16 columns per limb
+        uint32_t hi[16], lo[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          split_centred(x[4 * h + i].x, hi[4 * i + 0], lo[4 * i + 0]);
+          split_centred(x[4 * h + i].y, hi[4 * i + 1], lo[4 * i + 1]);
+          split_centred(x[4 * h + i].z, hi[4 * i + 2], lo[4 * i + 2]);
+          split_centred(x[4 * h + i].w, hi[4 * i + 3], lo[4 * i + 3]);
+        }
+        tc_st_32x32b_x16(t + h * 16, hi);
+        tc_st_32x32b_x16(t + BK / 2 + h * 16, lo);
+      }
+      tc_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(a_ready0 + 8 * cstage.slot);
+      cstage.advance(A_STAGES);
+    }
+    (void)ok;
   } else if (warp >= MMA_WARP0) {
     // ------------------------------------------------------------ MMA issuers (issuer me owns accumulator me)
     const int me = warp - MMA_WARP0;
@@ -294,43 +354,47 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       uint32_t wait_par = 1u;
       bool need_acquire = true, fresh = true;
       bool ok = true;
-      for (int64_t q = 0; q < total_q && ok; ++q) {
-        const int kb = static_cast<int>(q % nkb);
-        const int sa = static_cast<int>(q % A_STAGES);
-        const int sb = static_cast<int>(q % B_STAGES);
-        if (!bounded_wait(a_ready0 + 8 * sa, static_cast<uint32_t>((q / A_STAGES) & 1), P.timeout_ns) ||
-            !bounded_wait(b_full0 + 8 * sb, static_cast<uint32_t>((q / B_STAGES) & 1), P.timeout_ns)) {
-          report_status(P.status, STATUS_TIMEOUT, 23);
-          *abort_flag = 1;
-          break;
-        }
-        if (need_acquire) {
-          if (!bounded_wait(sempty0 + 8 * ring.slot_of[me], wait_par, P.timeout_ns)) {
-            report_status(P.status, STATUS_TIMEOUT, 24);
+      RingPos pa, pb;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!bounded_wait(a_ready0 + 8 * pa.slot, pa.phase, P.timeout_ns) ||
+              !bounded_wait(b_full0 + 8 * pb.slot, pb.phase, P.timeout_ns)) {
+            report_status(P.status, STATUS_TIMEOUT, 23);
             *abort_flag = 1;
+            ok = false;
             break;
           }
-          need_acquire = false;
-        }
-        tc_fence_after();
-        const uint32_t d = tmem_base + static_cast<uint32_t>(ACC_COL0 + ring.slot_of[me] * SLOT_COLS);
-        const uint32_t a_tmem = tmem_base + static_cast<uint32_t>(sa * A_STAGE_COLS + me * (BK / 2));
-        const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + sb * TILE_B));
+          if (need_acquire) {
+            if (!bounded_wait(sempty0 + 8 * ring.slot_of[me], wait_par, P.timeout_ns)) {
+              report_status(P.status, STATUS_TIMEOUT, 24);
+              *abort_flag = 1;
+              ok = false;
+              break;
+            }
+            need_acquire = false;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem_base + static_cast<uint32_t>(ACC_COL0 + ring.slot_of[me] * SLOT_COLS);
+          const uint32_t a_tmem = tmem_base + static_cast<uint32_t>(pa.slot * A_STAGE_COLS + me * (BK / 2));
+          const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + pb.slot * TILE_B));
 #pragma unroll
-        for (int kk = 0; kk < BK / UMMA_K; ++kk)
-          tc_mma_f16_ts(d, a_tmem + kk * (UMMA_K / 2), bdesc + 2 * kk, idesc, (fresh && kk == 0) ? 0u : 1u);
-        fresh = false;
-        tc_commit(a_empty0 + 8 * sa);
-        tc_commit(b_empty0 + 8 * sb);
+          for (int kk = 0; kk < BK / UMMA_K; ++kk)
+            tc_mma_f16_ts(d, a_tmem + kk * (UMMA_K / 2), bdesc + 2 * kk, idesc, (fresh && kk == 0) ? 0u : 1u);
+          fresh = false;
+          tc_commit(a_empty0 + 8 * pa.slot);
+          tc_commit(b_empty0 + 8 * pb.slot);
+          pa.advance(A_STAGES);
+          pb.advance(B_STAGES);
 #pragma unroll
-        for (int a = 0; a < NACC; ++a) {
-          if (!chunk_ends<CS>(a, kb, nkb)) continue;
-          if (a == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);
-          const uint32_t par = ring.rotate(a);
-          if (a == me) {
-            wait_par = par;
-            need_acquire = true;
-            fresh = true;
+          for (int a = 0; a < NACC; ++a) {
+            if (!chunk_ends<CS>(a, kb, nkb)) continue;
+            if (a == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);
+            const uint32_t par = ring.rotate(a);
+            if (a == me) {
+              wait_par = par;
+              need_acquire = true;
+              fresh = true;
+            }
           }
         }
       }
@@ -338,7 +402,7 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       bounded_wait(final_bar, 0, P.timeout_ns);
     }
   } else {
-    // ------------------------------------------------------------ epilogue: convert A, drain, reduce into C
+    // ------------------------------------------------------------ epilogue: drain, reduce into C
     const int quad = warp & 3;
     const int half = warp >> 2;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;  // TMEM lane field of this quadrant
@@ -346,49 +410,6 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
     ring.init();
     uint32_t drain_parity = 0;
     bool ok = true;
-    int64_t cq = 0;  // next K block (over this CTA's tiles) whose A tile this warp converts
-
-    // Splits this thread's half K block (32 indices of row 32*quad + lane) of K block qq into its
-    // two limbs and stores them in the A limb stage of qq.
-    auto convert = [&](int64_t qq) -> bool {
-      const int r = static_cast<int>(qq % RAW_STAGES);
-      const int sa = static_cast<int>(qq % A_STAGES);
-      const bool got_raw =
-          bounded_wait(raw_full0 + 8 * r, static_cast<uint32_t>((qq / RAW_STAGES) & 1), P.timeout_ns);
-      const bool got = got_raw && bounded_wait(a_empty0 + 8 * sa, static_cast<uint32_t>(((qq / A_STAGES) & 1) ^ 1),
-                                               P.timeout_ns);
-      if (!__all_sync(0xFFFFFFFFu, got)) {
-        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
-        *abort_flag = 1;
-        return false;
-      }
-      tc_fence_after();
-      // the raw tile's row `row` is 128 bytes; 16-byte chunk c sits at chunk c ^ (row % 8) (128-byte swizzle)
-      const uint32_t row = static_cast<uint32_t>(quad * 32 + lane);
-      const uint32_t src = smem_u32(smem + r * TILE_RAW) + row * 128;
-      uint32_t hi[16], lo[16];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint32_t c = static_cast<uint32_t>(half * 4 + i);
-        const uint4 x = lds128(src + ((c ^ (row & 7u)) << 4));
-        split_centred(x.x, hi[4 * i + 0], lo[4 * i + 0]);
-        split_centred(x.y, hi[4 * i + 1], lo[4 * i + 1]);
-        split_centred(x.z, hi[4 * i + 2], lo[4 * i + 2]);
-        split_centred(x.w, hi[4 * i + 3], lo[4 * i + 3]);
-      }
-      const uint32_t t = tmem_base + lane_base + static_cast<uint32_t>(sa * A_STAGE_COLS + half * 16);
-      tc_st_32x32b_x16(t, hi);
-      tc_st_32x32b_x16(t + BK / 2, lo);
-      tc_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(raw_empty0 + 8 * r);
-        mbar_arrive(a_ready0 + 8 * sa);
-      }
-      return true;
-    };
-
     uint64_t acc[COLS];
     const uint32_t quad_stage = smem_u32(smem + OFF_STG + quad * STG_QUAD);
     uint32_t tile_ends = 0;  // staged tile ends so far (the quadrant barriers' phase)
@@ -399,8 +420,6 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
                   P.group_m, mt, nt);
       for (int kb = 0; kb < nkb && ok; ++kb, ++q) {
-        while (ok && cq <= q + LOOKAHEAD && cq < total_q) ok = convert(cq++);
-        if (!ok) break;
         if (kb == 0) {
 #pragma unroll
           for (int c = 0; c < COLS; ++c) acc[c] = 0;
@@ -419,19 +438,17 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
           drain_parity ^= 1u << s;
           tc_fence_after();
           const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(ACC_COL0 + s * SLOT_COLS + half * COLS);
-          uint32_t l0[16], l1[16], r0[16], r1[16];
-          tc_ld_32x32b_x16(taddr, l0);
-          tc_ld_32x32b_x16(taddr + 16, l1);
-          tc_ld_32x32b_x16(taddr + BN, r0);
-          tc_ld_32x32b_x16(taddr + BN + 16, r1);
-          tc_wait_ld();
           const int sl = shift_left_half(a), sr = shift_right_half(a);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            acc[j] += (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(l0[j]))) << sl) +
-                      (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r0[j]))) << sr);
-            acc[16 + j] += (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(l1[j]))) << sl) +
-                           (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(r1[j]))) << sr);
+          for (int g = 0; g < 2; ++g) {  // 16 output columns at a time: B high limb part, B low limb part
+            uint32_t lv[16], rv[16];
+            tc_ld_32x32b_x16(taddr + g * 16, lv);
+            tc_ld_32x32b_x16(taddr + BN + g * 16, rv);
+            tc_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              acc[16 * g + j] += (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(lv[j]))) << sl) +
+                                 (static_cast<uint64_t>(static_cast<int64_t>(f32_to_i32(rv[j]))) << sr);
           }
           tc_fence_before();
           __syncwarp();

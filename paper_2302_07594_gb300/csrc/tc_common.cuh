@@ -111,6 +111,20 @@ struct SlotRing {
   }
 };
 
+// Position in a ring of n slots: the slot and the parity of its current use.  Pipeline loops
+// advance it by one per K block instead of dividing a running counter (64-bit division is a
+// long software routine on the GPU, and it sat on every producer's critical path).
+struct RingPos {
+  int slot = 0;
+  uint32_t phase = 0;
+  __device__ __forceinline__ void advance(int n) {
+    if (++slot == n) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
 __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
   const int per_group = group_m * num_n;
   const int group = t / per_group;
