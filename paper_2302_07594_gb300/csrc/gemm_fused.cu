@@ -177,6 +177,34 @@ __device__ __forceinline__ void reduce_row(int64_t* dst, uint32_t stage_row, int
   }
 }
 
+// This CTA's share of the work: the K-block units (tile t, K block kb), numbered t * nkb + kb with
+// the tiles in raster order, split into gridDim.x contiguous ranges of equal length (within one).
+// A tile whose K blocks straddle two ranges is computed in two parts that are both added into C,
+// which the bulk reductions do anyway; so every CTA finishes at the same time however the tile
+// count divides by the SM count.
+struct Span {
+  int64_t u, first, end;  // current unit, this CTA's first unit, one past its last
+  int t, kb, nkb;         // current tile and K block
+  __device__ __forceinline__ void init(int64_t total_units, int nkb_) {
+    nkb = nkb_;
+    first = static_cast<int64_t>(blockIdx.x) * total_units / gridDim.x;
+    end = (static_cast<int64_t>(blockIdx.x) + 1) * total_units / gridDim.x;
+    u = first;
+    t = static_cast<int>(u / nkb);
+    kb = static_cast<int>(u - static_cast<int64_t>(t) * nkb);
+  }
+  __device__ __forceinline__ bool done() const { return u >= end; }
+  __device__ __forceinline__ bool part_first() const { return kb == 0 || u == first; }
+  __device__ __forceinline__ bool part_last() const { return kb == nkb - 1 || u + 1 == end; }
+  __device__ __forceinline__ void next() {
+    ++u;
+    if (++kb == nkb) {
+      kb = 0;
+      ++t;
+    }
+  }
+};
+
 template <int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapBH,
@@ -235,13 +263,10 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
-  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
   const int nkb = P.num_k_blocks;
-  const int my_tiles = total_tiles > static_cast<int>(blockIdx.x)
-                           ? (total_tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                                 static_cast<int>(gridDim.x)
-                           : 0;
-  const int64_t total_q = static_cast<int64_t>(my_tiles) * nkb;  // this CTA's K blocks, over its tiles
+  const int64_t total_units = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles * nkb;
+  Span span;
+  span.init(total_units, nkb);
 
   if (warp == A_PRODUCER_WARP || warp == B_PRODUCER_WARP) {
     // ------------------------------------------------------------ TMA producers
@@ -259,11 +284,11 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       RingPos pos;
       int64_t issued = 0;
       bool stop = false;
-      for (int i = 0; i < my_tiles && !stop; ++i) {
-        int mt, nt;
-        tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
-                    P.group_m, mt, nt);
-        for (int kb = 0; kb < nkb; ++kb) {
+      int mt = 0, nt = 0;
+      for (Span sp = span; !sp.done() && !stop; sp.next()) {
+        const int kb = sp.kb;
+        if (sp.part_first()) tile_coords(sp.t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+        {
           if (!bounded_wait(empty0 + 8 * pos.slot, pos.phase ^ 1u, P.timeout_ns) || *abort_flag) {
             report_status(P.status, STATUS_TIMEOUT, is_a ? 21 : 22);
             *abort_flag = 1;
@@ -302,7 +327,7 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
     const uint32_t lane_field = static_cast<uint32_t>(quad * 32) << 16;
     RingPos craw, cstage;
     bool ok = true;
-    for (int64_t q = 0; q < total_q && ok; ++q) {
+    for (int64_t q = span.first; q < span.end && ok; ++q) {
       const bool got = bounded_wait(raw_full0 + 8 * craw.slot, craw.phase, P.timeout_ns);
       if (!__all_sync(0xFFFFFFFFu, got)) {
         if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
@@ -355,8 +380,9 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       bool need_acquire = true, fresh = true;
       bool ok = true;
       RingPos pa, pb;
-      for (int i = 0; i < my_tiles && ok; ++i) {
-        for (int kb = 0; kb < nkb; ++kb) {
+      for (Span sp = span; !sp.done() && ok; sp.next()) {
+        const int kb = sp.kb;
+        {
           if (!bounded_wait(a_ready0 + 8 * pa.slot, pa.phase, P.timeout_ns) ||
               !bounded_wait(b_full0 + 8 * pb.slot, pb.phase, P.timeout_ns)) {
             report_status(P.status, STATUS_TIMEOUT, 23);
@@ -385,9 +411,10 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
           tc_commit(b_empty0 + 8 * pb.slot);
           pa.advance(A_STAGES);
           pb.advance(B_STAGES);
+          const bool part_last = sp.part_last();
 #pragma unroll
           for (int a = 0; a < NACC; ++a) {
-            if (!chunk_ends<CS>(a, kb, nkb)) continue;
+            if (!part_last && !chunk_ends<CS>(a, kb, nkb)) continue;
             if (a == me) tc_commit(sfull0 + 8 * ring.slot_of[a]);
             const uint32_t par = ring.rotate(a);
             if (a == me) {
@@ -414,19 +441,19 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
     const uint32_t quad_stage = smem_u32(smem + OFF_STG + quad * STG_QUAD);
     uint32_t tile_ends = 0;  // staged tile ends so far (the quadrant barriers' phase)
 
-    int64_t q = 0;
-    for (int i = 0; i < my_tiles && ok; ++i) {
-      int mt, nt;
-      tile_coords(static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x), P.num_m_tiles, P.num_n_tiles,
-                  P.group_m, mt, nt);
-      for (int kb = 0; kb < nkb && ok; ++kb, ++q) {
-        if (kb == 0) {
+    int mt = 0, nt = 0;
+    for (Span sp = span; !sp.done() && ok; sp.next()) {
+      const int kb = sp.kb;
+      const bool part_last = sp.part_last();
+      if (sp.part_first()) {
+        tile_coords(sp.t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
 #pragma unroll
-          for (int c = 0; c < COLS; ++c) acc[c] = 0;
-        }
+        for (int c = 0; c < COLS; ++c) acc[c] = 0;
+      }
+      {
 #pragma unroll
         for (int a = 0; a < NACC; ++a) {
-          if (!chunk_ends<CS>(a, kb, nkb)) continue;
+          if (!part_last && !chunk_ends<CS>(a, kb, nkb)) continue;
           const int s = ring.slot_of[a];
           const bool got = bounded_wait(sfull0 + 8 * s, (drain_parity >> s) & 1u, P.timeout_ns);
           if (!__all_sync(0xFFFFFFFFu, got)) {
@@ -457,7 +484,9 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
         }
       }
       if (!ok) break;
-      // ---- C tile += acc, through the staging block and bulk reductions
+      if (!part_last) continue;
+      // ---- C tile += acc (this CTA's part of the tile's K blocks), through the staging block and
+      //      bulk reductions
       const int64_t row0 = static_cast<int64_t>(mt) * BM + quad * 32;
       const int64_t row = row0 + lane;
       const int64_t tcol0 = static_cast<int64_t>(nt) * BN;
@@ -544,8 +573,8 @@ cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
   P.group_m = a.group_m > 0 ? a.group_m : 16;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
-  const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
-  const int grid = static_cast<int>(tiles < a.num_sms ? tiles : a.num_sms);
+  const int64_t units = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles * P.num_k_blocks;
+  const int grid = static_cast<int>(units < a.num_sms ? units : a.num_sms);
   static bool attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
