@@ -90,9 +90,13 @@ constexpr size_t SMEM = 1024 + static_cast<size_t>(OFF_BAR) + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
 static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0, "swizzled tiles start on 1024-byte boundaries");
 
-// The two accumulators' exact chunks: 512 * CS reduction indices, staggered by half a chunk.
+// The two accumulators' exact chunks: at most 512 * CS reduction indices, staggered by half a
+// chunk so that their drains alternate.  When a whole tile fits in one chunk (k <= 512 * CS) there
+// is no chunk end inside a tile: both accumulators are drained once, where the tile (or this CTA's
+// part of it) ends.
 template <int CS>
 __device__ __forceinline__ bool chunk_ends(int a, int kb, int nkb) {
+  if (nkb * BK <= 512 * CS) return kb == nkb - 1;
   return kb == nkb - 1 || (((kb + 1) * BK + a * 256 * CS) % (512 * CS)) == 0;
 }
 // weights of accumulator a's two column halves: A limb a times B limb 0 (high) and 1 (low)
