@@ -5,38 +5,40 @@
 //
 // How.  The operands arrive as fp16 limb planes (split.cu): a = 256*h + l with
 // |h|, |l| <= 128, so for one reduction index
-//     a*b = 2^16 * (h_a h_b) + 2^8 * (h_a l_b + l_a h_b) + (l_a l_b),
-// and the GEMM is four limb GEMMs summed into three accumulators
-//     HH = Ah*Bh,   X = Ah*Bl + Al*Bh,   LL = Al*Bl.
-// Each limb product is an integer of magnitude <= 2^14 that fp16 x fp16 forms
-// exactly, and an fp32 accumulator sums integers exactly while every partial
-// sum stays below 2^24.  So each accumulator is only allowed a bounded run of
-// the reduction dimension (a "chunk": by default 1024 indices for HH and LL,
-// 512 for X, keeping every partial sum within 2^24), after which it is drained:
-// converted to an integer and added, shifted by its weight (16, 8, 0 bits),
-// into a 64-bit running sum held in registers.  This plays the role of the
-// AIE's 48-bit accumulators (Section 6.2): wide accumulation so nothing
-// overflows, here built from exact fp32 chunks and int64 registers.  The int8
-// path is the same with one plane, one product and one accumulator (int32 sum).
+//     a*b = 2^16 * (h_a h_b) + 2^8 * (h_a l_b + l_a h_b) + (l_a l_b).
+// B's two limb tiles sit one above the other in shared memory, so one
+// tcgen05.mma of N = 256 multiplies an A limb by both B limbs at once: the
+// accumulator of A_high holds HH | HL, the accumulator of A_low holds LH | LL
+// (column halves).  Each limb product is an integer of magnitude <= 2^14 that
+// fp16 x fp16 forms exactly, and an fp32 accumulator sums integers exactly
+// while every partial sum stays below 2^24.  So an accumulator is only allowed
+// a bounded run of the reduction dimension (a "chunk": by default 1024
+// indices), after which it is drained: converted to an integer and added,
+// shifted by its weight (16, 8 or 0 bits), into a 64-bit running sum held in
+// registers.  This plays the role of the AIE's 48-bit accumulators (Section
+// 6.2): wide accumulation so nothing overflows, here built from exact fp32
+// chunks and int64 registers.  The int8 path multiplies the values themselves
+// (one plane) into one accumulator per 128-column half of a 128 x 256 tile.
 //
-// Structure (one persistent CTA per SM, 352 threads, 128x128 output tiles):
+// Structure (one persistent CTA per SM, 352 threads, 128x128 output tiles for
+// int16):
 //   warp 8      TMA producer: 2-D tiled bulk-tensor loads of 64-wide K blocks of
 //               the limb planes (128-byte swizzle) into a ring of smem stages;
-//   warps 9-10  MMA issuers: tcgen05.mma kind::f16 (M=128, N=128, K=16) from smem
-//               descriptors into fp32 accumulators in tensor memory (TMEM).  A
-//               single issuing thread leaves the tensor pipe idle for every cycle
-//               it spends waiting or book-keeping (the pipe buffers almost no
-//               instructions), so two warps issue concurrently, each owning its
-//               own accumulators: HH+LL and X for int16; even and odd K blocks
-//               for int8;
+//   warps 9-10  MMA issuers: tcgen05.mma kind::f16 (M=128, K=16, N=256 for
+//               int16, N=128 for int8) from smem descriptors into fp32
+//               accumulators in tensor memory (TMEM).  A single issuing thread
+//               leaves the tensor pipe idle for every cycle it spends waiting or
+//               book-keeping (the pipe buffers almost no instructions), so two
+//               warps issue concurrently, each owning its own accumulator;
 //   warps 0-7   epilogue: drain accumulators (tcgen05.ld) into int64 registers,
 //               and read-modify-write C once per tile.
-// TMEM holds four 128-column accumulator slots: the live accumulators plus
-// spares.  Chunk ends are staggered, so at every chunk end the owning issuer
-// moves that accumulator into the oldest spare slot and keeps issuing while the
-// epilogue drains the old one.  Every role replays the same deterministic
-// chunk schedule, so slot assignments need no communication beyond the
-// full/empty barriers of each slot.  This takes the place of the
+// TMEM holds the accumulators: two 256-column slots for int16 (chunk ends
+// staggered by half a chunk, so while one issuer waits for the drain of its
+// slot the other keeps the tensor pipe busy), four 128-column slots for int8
+// (two live, two spare: at a chunk end the owning issuer moves its accumulator
+// into the oldest spare and keeps issuing).  Every role replays the same
+// deterministic chunk schedule, so slot assignments need no communication
+// beyond the full/empty barriers of each slot.  This takes the place of the
 // paper's loop L6 / micro-kernel (Figure 1, Section 5.2); the smem stage ring
 // takes the place of the B_r copies into local memory (Section 5.1).
 //
@@ -56,15 +58,12 @@ namespace gemmi {
 namespace {
 
 using namespace tc;
-constexpr int UMMA_N = 128;                  // N of one tcgen05.mma (an accumulator is 128 columns)
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int PRODUCER_WARP = 8;
 constexpr int MMA_WARP0 = 9;                  // issuer warps 9 and 10; warp 9 also owns the TMEM allocation
 constexpr int NISSUE = 2;
 constexpr int NUM_THREADS = (NUM_EPI_WARPS + 1 + NISSUE) * 32;
-constexpr int NSLOT = 4;
-constexpr int SLOT_COLS = 128;
-constexpr int TMEM_COLS = NSLOT * SLOT_COLS;  // 512
+constexpr int TMEM_COLS = 512;
 
 // Tile geometry: K blocks of 64 fp16 (128-byte rows, the 128-byte swizzle span).
 template <int NL>
@@ -75,7 +74,9 @@ struct Geom {
   static constexpr int SB = NL * (TILE_A + TILE_B);       // one stage: NL tiles of A, then NL of B
   static constexpr int STAGES = (192 * 1024) / SB;        // 192 KB of stages
   static constexpr int SWIZZLE = BK * 2;                  // bytes per swizzled row
+  static constexpr int NSLOT = Scheme<NL>::NSLOT;
   static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + 8 * (2 * STAGES + 2 * NSLOT + 1) + 16;
+  static_assert(NSLOT * Scheme<NL>::SLOT_COLS <= TMEM_COLS, "tensor memory budget");
   static_assert(SMEM <= 227 * 1024, "shared memory budget");
 };
 
@@ -104,6 +105,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   constexpr int TILE_B = G::TILE_B;
   constexpr int BN = S::BN;
   constexpr int COLS = S::COLS;
+  constexpr int NSLOT = S::NSLOT;
+  constexpr int SLOT_COLS = S::SLOT_COLS;
+  constexpr int UMMA_N = S::UMMA_N;
   // C element type and the unsigned type of the running sum (wrap-around is modular, never UB)
   using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
   using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
@@ -353,19 +357,38 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           tc_fence_after();
           // this warp's columns of the accumulator: all 128 (int8, one accumulator per half)
           // or its 64-column half (int16)
-          const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                                 static_cast<uint32_t>(s * SLOT_COLS + (NL == 2 ? half * COLS : 0));
+          if constexpr (NL == 2) {
+            // this warp's 64 output columns: the B-high part (accumulator columns 0-127) and the
+            // B-low part (columns 128-255) of each, 16 columns at a time
+            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                                   static_cast<uint32_t>(s * SLOT_COLS + half * COLS);
 #pragma unroll
-          for (int c = 0; c < COLS; c += 32) {
-            uint32_t r0[16], r1[16];
-            tc_ld_32x32b_x16(taddr + c, r0);
-            tc_ld_32x32b_x16(taddr + c + 16, r1);
-            tc_wait_ld();
+            for (int c = 0; c < COLS; c += 16) {
+              uint32_t rh[16], rl[16];
+              tc_ld_32x32b_x16(taddr + c, rh);
+              tc_ld_32x32b_x16(taddr + BN + c, rl);
+              tc_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              // sign-extend to the unsigned running-sum type, then weight by 2^shift (modular)
-              acc[c + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r0[i]))) << S::shift(a);
-              acc[c + 16 + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r1[i]))) << S::shift(a);
+              for (int i = 0; i < 16; ++i)
+                acc[c + i] += (static_cast<UT>(static_cast<CT>(f32_to_i32(rh[i]))) << S::shift(a)) +
+                              (static_cast<UT>(static_cast<CT>(f32_to_i32(rl[i]))) << S::shift_low(a));
+            }
+          } else {
+            // this warp's 128 columns: the accumulator of its half
+            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                                   static_cast<uint32_t>(s * SLOT_COLS);
+#pragma unroll
+            for (int c = 0; c < COLS; c += 32) {
+              uint32_t r0[16], r1[16];
+              tc_ld_32x32b_x16(taddr + c, r0);
+              tc_ld_32x32b_x16(taddr + c + 16, r1);
+              tc_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                // sign-extend to the unsigned running-sum type (modular)
+                acc[c + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r0[i])));
+                acc[c + 16 + i] += static_cast<UT>(static_cast<CT>(f32_to_i32(r1[i])));
+              }
             }
           }
           tc_fence_before();

@@ -18,37 +18,40 @@ constexpr uint32_t STATUS_TIMEOUT = 4;
 template <int NL>
 struct Scheme;
 
-// int16: two limbs per operand, four products, three accumulators.
-//   product p: (A limb, B limb) = (h,h), (h,l), (l,h), (l,l); limb 0 = high, 1 = low
-//   accumulators: 0 = HH (weight 2^16), 1 = X (2^8), 2 = LL (1)
-//   issuer 0 owns HH and LL (products 0, 3), issuer 1 owns X (products 1, 2): 8 MMAs each per K block.
+// int16: two limbs per operand.  B's two limb tiles are stacked into one 256-row tile, so one
+// tcgen05.mma of N = 256 multiplies an A limb by both B limbs: accumulator p (owned by issuer p)
+// holds A_p * B_high in its columns 0-127 and A_p * B_low in columns 128-255 (limb 0 = high,
+// 1 = low), weights 2^16 | 2^8 for p = 0 and 2^8 | 1 for p = 1.  Compared with four N = 128
+// products this halves the MMA count and the times each A tile is read from shared memory.
+// The two accumulators fill TMEM (two 256-column slots, no spare): at a chunk end the owning
+// issuer waits for the drain of its slot, while the other issuer -- whose chunk ends half a
+// chunk later -- keeps the tensor pipe busy.
 template <>
 struct Scheme<2> {
   static constexpr int BN = 128;          // output tile width
-  static constexpr int NACC = 3;
-  static constexpr int NPROD = 4;
+  static constexpr int UMMA_N = 256;      // B's two limbs stacked
+  static constexpr int NACC = 2;
+  static constexpr int NPROD = 2;         // product p: A limb p times the stacked B
+  static constexpr int NSLOT = 2;
+  static constexpr int SLOT_COLS = 256;
   static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
   static constexpr int COLS = 64;         // C columns per epilogue thread (two warps per lane quadrant)
   static constexpr int DRAIN_WARPS = 8;   // every epilogue warp drains every accumulator (its 64 columns)
   __device__ static constexpr bool drains(int, int) { return true; }
-  __device__ static constexpr int a_limb(int p) { return p >> 1; }
-  __device__ static constexpr int b_limb(int p) { return p & 1; }
-  __device__ static constexpr int b_row0(int) { return 0; }  // first row (output column) of the B tile used
-  __device__ static constexpr int acc(int p, int) { return p == 0 ? 0 : p == 3 ? 2 : 1; }
-  __device__ static constexpr int issuer(int p, int) { return (p == 0 || p == 3) ? 0 : 1; }
-  __device__ static constexpr int owner(int a) { return a == 1 ? 1 : 0; }
-  __device__ static constexpr int shift(int a) { return a == 0 ? 16 : a == 1 ? 8 : 0; }
-  // Chunk schedule, in reduction indices, for chunk scale CS (1 or 2): accumulator a ends a
-  // chunk after the K block that ends at index e when (e + PHASE[a]) % PERIOD[a] == 0, or at
-  // the last block of the tile.  HH, LL: 512*CS indices, |sum| <= 512*CS * 2^14;  X: 256*CS
-  // indices, |sum| <= 256*CS * 2^15.  CS = 1 keeps every partial sum within 2^23 (one bit below
-  // the 2^24 limit of exact fp32 integer sums), CS = 2 within 2^24.  The phases stagger the
-  // three chunk ends 128*CS indices apart (HH at 128*CS, X at 256*CS, LL at 384*CS, X at 512*CS, ...).
+  __device__ static constexpr int a_limb(int p) { return p; }
+  __device__ static constexpr int b_limb(int) { return 0; }  // the stacked B starts at the high limb
+  __device__ static constexpr int b_row0(int) { return 0; }
+  __device__ static constexpr int acc(int p, int) { return p; }
+  __device__ static constexpr int issuer(int p, int) { return p; }
+  __device__ static constexpr int owner(int a) { return a; }
+  __device__ static constexpr int shift(int a) { return a == 0 ? 16 : 8; }       // columns 0-127
+  __device__ static constexpr int shift_low(int a) { return a == 0 ? 8 : 0; }    // columns 128-255
+  // Chunks of 512 * CS reduction indices, |sum| <= 512 * CS * 2^14 (within 2^23 for CS = 1,
+  // 2^24 for CS = 2, the limit of exact fp32 integer sums); the two accumulators' chunk ends
+  // are staggered by half a chunk.
   template <int CS>
   __device__ static bool chunk_ends(int a, int kb, int nkb) {
-    const int period = (a == 1 ? 256 : 512) * CS;
-    const int phase = (a == 0 ? 384 : a == 1 ? 0 : 128) * CS;
-    return kb == nkb - 1 || (((kb + 1) * 64 + phase) % period) == 0;
+    return kb == nkb - 1 || (((kb + 1) * 64 + a * 256 * CS) % (512 * CS)) == 0;
   }
 };
 
@@ -59,6 +62,9 @@ struct Scheme<2> {
 template <>
 struct Scheme<1> {
   static constexpr int BN = 256;
+  static constexpr int UMMA_N = 128;      // one column half per MMA
+  static constexpr int NSLOT = 4;
+  static constexpr int SLOT_COLS = 128;
   static constexpr int NACC = 2;
   static constexpr int NPROD = 2;         // product p: column half p
   static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
@@ -107,6 +113,29 @@ struct SlotRing {
     slot_of[a] = fresh;
     const uint32_t par = ((assign_parity >> fresh) & 1u) ^ 1u;
     assign_parity ^= 1u << fresh;
+    return par;
+  }
+};
+
+// No spare slots: accumulator a keeps slot a, and each new chunk waits for the previous chunk's
+// drain of that slot.
+template <int NACC>
+struct SlotRing<NACC, NACC> {
+  int slot_of[NACC];
+  uint32_t assign_parity;
+
+  __device__ __forceinline__ void init() {
+    assign_parity = 0;
+#pragma unroll
+    for (int a = 0; a < NACC; ++a) {
+      slot_of[a] = a;
+      assign_parity ^= 1u << a;
+    }
+  }
+  __device__ __forceinline__ uint32_t rotate(int a) {
+    const int slot = slot_of[a];
+    const uint32_t par = ((assign_parity >> slot) & 1u) ^ 1u;
+    assign_parity ^= 1u << slot;
     return par;
   }
 };
