@@ -6,16 +6,16 @@
 // large and two small dimensions (Section 2, IM2COL lowering).  This kernel is
 // built around the stream of B:
 //
-//   * B is cut into column blocks of 256 (512 contiguous bytes of every row)
-//     and the reduction dimension into ranges, one (column block, range) per
-//     CTA, about one CTA per SM; a producer warp streams 32-row x 256-column
-//     stages of B (four 2-D TMA boxes, 128-byte swizzle) into a ring of
-//     shared-memory stages.  The CTA's slice of A (m <= 16 rows, at most 1024
+//   * B is cut into column blocks of 512 (1 KB contiguous of every row, which
+//     DRAM streams markedly better than 512-byte runs) and the reduction
+//     dimension into ranges, one (column block, range) per CTA, about one CTA
+//     per SM; a producer warp streams 32-row x 512-column stages of B (eight
+//     2-D TMA boxes, 128-byte swizzle) into a ring of shared-memory stages.  The CTA's slice of A (m <= 16 rows, at most 1024
 //     reduction indices) is split into fp16 limbs once, into shared memory, when
 //     the CTA starts, so the inner loop converts only B;
-//   * sixteen consumer warps each own 16 columns of the block (four warps per
-//     scheduler, so the latencies of one warp's dependent ldmatrix / mma chains
-//     are covered by the others).  Per 16-row step a
+//   * sixteen consumer warps each own 32 columns of the block, two m16 tiles
+//     (four warps per scheduler, so the latencies of one warp's dependent
+//     ldmatrix / mma chains are covered by the others).  Per 16-row step a
 //     warp reads its B slab transposed with ldmatrix (the "A" operand of
 //     C^T = B^T A^T), splits every int16 into 8-bit limbs
 //         b = 256*hi + lo,  hi = b >> 8 in [-128,127],  lo = b & 255 in [0,255],
@@ -37,18 +37,20 @@
 namespace gemmi {
 namespace {
 
-constexpr int JB = 256;                 // columns of B per CTA
+constexpr int JB = 512;                 // columns of B per CTA (1 KB of every row: long DRAM runs)
 constexpr int BOX_J = 64;               // columns per TMA box (128 bytes, the swizzle span)
-constexpr int NBOX = JB / BOX_J;        // 4 boxes per stage
+constexpr int NBOX = JB / BOX_J;        // 8 boxes per stage
 constexpr int KS = 32;                  // rows of B per stage (two 16-row mma steps)
-constexpr int STAGES = 8;
-constexpr int STAGE_BYTES = KS * JB * 2;         // 16 KB of B per stage
+constexpr int STAGES = 4;
+constexpr int STAGE_BYTES = KS * JB * 2;         // 32 KB of B per stage
 constexpr int A_ROWS = 16;
 constexpr int KMAX_CTA = 1024;                   // reduction indices per CTA (bounds the A limbs in smem)
 constexpr int A_PAIRS = KMAX_CTA / 2;            // packed fp16 pairs per A row
 constexpr int A_STRIDE = A_PAIRS + 4;            // words per A limb row (+4 words: conflict-free fragment reads)
 constexpr int A_LIMB_BYTES = A_ROWS * A_STRIDE * 4;  // one limb (hi or lo) of the CTA's A slice
-constexpr int NCONS = 16;               // consumer warps, 16 columns (one m16 tile) each
+constexpr int NCONS = 16;               // consumer warps
+constexpr int MT = JB / (16 * NCONS);   // m16 tiles (of 16 columns) per consumer warp
+static_assert(MT * 16 * NCONS == JB, "the consumer warps cover the column block");
 constexpr int THREADS = (NCONS + 1) * 32;
 constexpr int DRAIN_EVERY = 4;          // stages per drain: 4 x 32 = 128 reduction indices
 constexpr uint32_t STATUS_TIMEOUT = 4;
@@ -107,6 +109,8 @@ __device__ __forceinline__ int32_t f2i(float f) {
   return v;
 }
 
+// 17 warps: one of the four schedulers hosts five of them, and its quarter of the register file
+// (16,384) caps every thread at 96 registers.
 template <int NT>
 __global__ void __launch_bounds__(THREADS, 1)
 skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
@@ -189,7 +193,6 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   }
   const int g = lane >> 2;
   const int t = lane & 3;
-  constexpr int MT = 1;  // m16 tiles (of 16 columns) per warp
   float hh[MT][NT][4], xx[MT][NT][4], ll[MT][NT][4];
   uint64_t acc[MT][NT][4];
 #pragma unroll
@@ -201,9 +204,10 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
         acc[mt][nt][c] = 0;
       }
-  // this warp's 16 columns live in box warp/4, 16-byte chunks (warp%4)*2 .. +1 of each 128-byte row
-  const int box = warp >> 2;
-  const int chunk_base = (warp & 3) * 2;
+  // this warp's 16*MT columns start in box (warp*16*MT)/64, at 16-byte chunk ((warp*16*MT)%64)/8
+  // of each 128-byte row (two chunks per m16 tile)
+  const int box = (warp * 16 * MT) / BOX_J;
+  const int chunk_base = ((warp * 16 * MT) % BOX_J) / 8;
   // ldmatrix lanes: 0-7 rows 0-7 / cols 0-7, 8-15 rows 0-7 / cols 8-15, 16-23 rows 8-15 / cols 0-7,
   // 24-31 rows 8-15 / cols 8-15 of a 16x16 (reduction x column) slab
   const int lrow = (lane & 7) + ((lane >> 4) << 3);
