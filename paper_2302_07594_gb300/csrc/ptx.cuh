@@ -106,6 +106,17 @@ __device__ __forceinline__ void report_status(uint32_t* status, uint32_t code, u
   atomicCAS(status, 0u, word);
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Lets the next kernel in the stream (launched with programmatic stream serialization) start its
+// prologue on SMs as this grid's CTAs retire.  A no-op without such a dependent.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// Waits until the grids this one depends on have completed and their memory is visible; every
+// access to global memory that earlier kernels may have written must come after it.  A no-op
+// for a grid launched without a programmatic dependency.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- TMA
 // Asks L2 to fetch [src, src + bytes) from global memory: a hint with nothing to wait for.
 // src 16-byte aligned, bytes a multiple of 16, the range inside one allocation.

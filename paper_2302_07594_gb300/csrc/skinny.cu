@@ -130,6 +130,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   if (st_end > P.total_stages) st_end = P.total_stages;
   const int64_t nst = st_end > st_begin ? st_end - st_begin : 0;
 
+  pdl_launch_dependents();
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -138,6 +139,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     fence_mbar_init();
   }
   __syncthreads();
+  pdl_wait();  // A, B and C may come from the previous kernel in the stream
 
   if (warp == NCONS) {
     // ------------------------------------------------------------ producer
@@ -344,9 +346,19 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
     if (attr != cudaSuccess) return attr;
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
   }
-  dim3 grid(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit));
-  skinny_kernel<NT><<<grid, THREADS, smem, s>>>(mapB, P);
-  return cudaGetLastError();
+  // programmatic stream serialization: the kernel may be scheduled while the previous kernel in
+  // the stream drains; it waits (griddepcontrol.wait) before its first global memory access
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit));
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, skinny_kernel<NT>, mapB, P);
 }
 
 }  // namespace

@@ -305,6 +305,27 @@ def test_repeated_calls_accumulate(gm):
     assert_same(dC.cpu().numpy(), exp, "3x accumulate")
 
 
+@pytest.mark.parametrize("m", [1, 8, 16])
+def test_skinny_back_to_back_dependencies(gm, m):
+    """Skinny launches may start while the previous kernel in the stream drains (programmatic
+    dependent launch); each still has to see everything earlier kernels wrote.  Calls accumulate
+    into one C, and between calls a torch kernel rewrites A in place, with no host
+    synchronisation anywhere."""
+    n, k = 700, 2000
+    A, B, C = gi.random_problem(905 + m, m, n, k, "i16", a_range=(-1000, 1000))
+    dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+    exp = C.copy()
+    a_host = A.copy()
+    for r in range(6):
+        gm.gemm_i16(dA, dB, dC)
+        oracle.gemm(a_host, B, exp)
+        dA.add_(r + 1)  # a torch kernel writes the next call's input
+        a_host = (a_host.astype(np.int32) + r + 1).astype(np.int16)
+    torch.cuda.synchronize()
+    assert gm.device_status() == gm.OK
+    assert_same(dC.cpu().numpy(), exp, f"m={m}: back-to-back skinny calls")
+
+
 def test_bounded_wait_reports_timeout(gm):
     """A pipeline wait that can never complete gives up, reports, and leaves the context usable."""
     assert gm.selftest_wait_timeout(2000) == gm.ETIMEOUT
