@@ -50,6 +50,8 @@ def _bind(lib):
         f = getattr(lib, name)
         f.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int]
         f.restype = ctypes.c_int
+    lib.gemm_oracle_i16_srs.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int, ctypes.c_int]
+    lib.gemm_oracle_i16_srs.restype = ctypes.c_int
     lib.gemm_oracle_max_threads.restype = ctypes.c_int
     return lib
 
@@ -94,6 +96,23 @@ def gemm(A: np.ndarray, B: np.ndarray, C: np.ndarray, nthreads: int = 1, lib=Non
             _ptr(C), _ld(C, C.itemsize), int(nthreads))
     if rc != 0:
         raise ValueError(f"oracle rejected the arguments (rc={rc})")
+    return C
+
+
+def gemm_srs(A: np.ndarray, B: np.ndarray, C: np.ndarray, shift: int, nthreads: int = 1, lib=None) -> np.ndarray:
+    """In place: C (int16) = wrap16(C + sat16(round_half_up(A @ B / 2^shift))), the paper's
+    shift-round-saturate micro-kernel output (see gemm_oracle.c for the readings)."""
+    lib = lib or load()
+    if A.dtype != np.int16 or B.dtype != np.int16 or C.dtype != np.int16:
+        raise TypeError("gemm_srs takes int16 A, B and C")
+    m, k = A.shape
+    k2, n = B.shape
+    if k2 != k or C.shape != (m, n):
+        raise ValueError(f"shape mismatch: A {A.shape}, B {B.shape}, C {C.shape}")
+    rc = lib.gemm_oracle_i16_srs(m, n, k, _ptr(A), _ld(A, 2), _ptr(B), _ld(B, 2), _ptr(C), _ld(C, 2),
+                                 int(shift), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments")
     return C
 
 

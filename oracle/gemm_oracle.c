@@ -101,6 +101,54 @@ int gemm_oracle_i8(int64_t m, int64_t n, int64_t k,
   return 0;
 }
 
+/*
+ * The paper's micro-kernel output (Section 5.2, the simplified AIE micro-kernel listing): the
+ * wide accumulator is shifted, rounded and saturated to 16 bits ("srs") and added to the int16
+ * C block with a plain 16-bit vector addition.  The paper is silent on the rounding of the shift
+ * (its listing uses shift 0, where there is none), on how wide the accumulated reduction is when
+ * k_c < k, and on whether the addition saturates.  The readings taken here:
+ *   - the accumulator holds the full reduction, S = sum_p A[i][p] * B[p][j] (k_c = k, the
+ *     configuration of the paper's best result);
+ *   - the shift rounds half up: R = floor((S + 2^(shift-1)) / 2^shift) for shift >= 1, R = S
+ *     for shift 0;
+ *   - saturation clamps R to [-32768, 32767];
+ *   - the addition wraps modulo 2^16.
+ * S is formed exactly: |S| <= k * 2^30 < 2^62 for every k below 2^31, so no step wraps.
+ */
+static int64_t oracle_floor_div_pow2(int64_t v, int shift) {
+  /* floor(v / 2^shift) written with non-negative operands only */
+  const int64_t d = (int64_t)1 << shift;
+  if (v >= 0) return v / d;
+  return -((-v + d - 1) / d);
+}
+
+int gemm_oracle_i16_srs(int64_t m, int64_t n, int64_t k,
+                        const int16_t* A, int64_t lda,
+                        const int16_t* B, int64_t ldb,
+                        int16_t* C, int64_t ldc, int shift, int nthreads) {
+  if (oracle_check(m, n, k, A, lda, B, ldb, C, ldc)) return 1;
+  if (shift < 0 || shift > 62) return 1;
+  if (m == 0 || n == 0) return 0;
+#ifdef _OPENMP
+  if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads)
+#else
+  (void)nthreads;
+#endif
+  for (int64_t i = 0; i < m; ++i) {
+    for (int64_t j = 0; j < n; ++j) {
+      int64_t s = 0;
+      for (int64_t p = 0; p < k; ++p) s += (int64_t)A[i * lda + p] * (int64_t)B[p * ldb + j];
+      int64_t r = shift == 0 ? s : oracle_floor_div_pow2(s + ((int64_t)1 << (shift - 1)), shift);
+      if (r > 32767) r = 32767;
+      if (r < -32768) r = -32768;
+      const uint16_t sum = (uint16_t)((uint16_t)C[i * ldc + j] + (uint16_t)r);
+      C[i * ldc + j] = (int16_t)sum;
+    }
+  }
+  return 0;
+}
+
 /* Threads the library was built to use (1 without OpenMP). */
 int gemm_oracle_max_threads(void) {
 #ifdef _OPENMP

@@ -223,8 +223,73 @@ def check_transpose(lib):
     return [] if np.array_equal(X, Y.T) else ["transpose identity (AB)^T = B^T A^T"]
 
 
+# ---- the paper's micro-kernel output: C16 += srs(A*B, shift)  (gemm_oracle_i16_srs)
+SRS_GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "srs_cases.json")
+
+
+def _run_srs(lib, A, B, C, shift):
+    X = C.copy()
+    oracle.gemm_srs(A, B, X, shift, lib=lib)
+    return X
+
+
+def check_srs_golden(lib):
+    """Worked examples (tests/golden/srs_cases.json): rounding, saturation, wrapping add."""
+    bad = []
+    with open(SRS_GOLDEN) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        m, n, k = c["m"], c["n"], c["k"]
+        A = np.array(c["A"], dtype=np.int16).reshape(m, k)
+        B = np.array(c["B"], dtype=np.int16).reshape(k, n)
+        C = np.array(c["C_in"], dtype=np.int16).reshape(m, n)
+        E = np.array(c["C_out"], dtype=np.int16).reshape(m, n)
+        got = _run_srs(lib, A, B, C, c["shift"])
+        if not np.array_equal(got, E):
+            bad.append(f"srs golden {c['name']}: got {got.tolist()} want {E.tolist()}")
+    return bad
+
+
+def check_srs_reduces_to_gemm(lib):
+    """Shift 0 with sums inside int16: srs is the identity, so C16 + S taken modulo 2^16 must match
+    the exact GEMM (numpy's integer matmul) -- on every entry, with values chosen so that no sum
+    saturates."""
+    bad = []
+    for seed, (m, n, k) in enumerate(((3, 5, 7), (17, 9, 40), (40, 33, 64))):
+        A = gi.uniform_int(700 + seed, (m, k), -11, 11, np.int16)
+        B = gi.uniform_int(710 + seed, (k, n), -11, 11, np.int16)
+        C = gi.uniform_int(720 + seed, (m, n), -32768, 32767, np.int16)
+        S = np.matmul(A.astype(np.int64), B.astype(np.int64))
+        assert np.abs(S).max() <= 32767
+        want = ((C.astype(np.int64) + S) & 0xFFFF).astype(np.uint16).view(np.int16)
+        if not np.array_equal(_run_srs(lib, A, B, C, 0), want):
+            bad.append(f"srs shift 0 != exact GEMM mod 2^16 on {(m, n, k)}")
+    return bad
+
+
+def check_srs_closed_forms(lib):
+    """All-ones operands give S = k on every entry: srs is then known in closed form."""
+    bad = []
+    for k, shift, want in ((5, 1, 3), (6, 2, 2), (7, 1, 4), (40000, 0, 32767), (40000, 1, 20000),
+                           (65535, 1, 32767), (9, 3, 1), (12, 3, 2)):
+        A = np.ones((2, k), np.int16)
+        B = np.ones((k, 3), np.int16)
+        got = _run_srs(lib, A, B, np.zeros((2, 3), np.int16), shift)
+        if not (got == want).all():
+            bad.append(f"srs all-ones k={k} shift={shift}: got {got[0, 0]} want {want}")
+        got = _run_srs(lib, -A, B, np.zeros((2, 3), np.int16), shift)
+        # -k/2^shift rounded half up: e.g. -2.5 -> -2; -40000 saturates at -32768
+        wn = {(5, 1): -2, (6, 2): -1, (7, 1): -3, (40000, 0): -32768, (40000, 1): -20000,
+              (65535, 1): -32767, (9, 3): -1, (12, 3): -1}[(k, shift)]
+        if not (got == wn).all():
+            bad.append(f"srs all-minus-ones k={k} shift={shift}: got {got[0, 0]} want {wn}")
+    return bad
+
+
+SRS_CHECKS = (check_srs_golden, check_srs_reduces_to_gemm, check_srs_closed_forms)
+
 ALL_CHECKS = (check_golden, check_extreme_bruteforce, check_closed_forms, check_identity_permutation,
-              check_blocked, check_padding, check_linearity, check_transpose, check_numpy)
+              check_blocked, check_padding, check_linearity, check_transpose, check_numpy) + SRS_CHECKS
 
 
 def pin_failures(lib, bruteforce_shapes=None):

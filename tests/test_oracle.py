@@ -34,6 +34,26 @@ def test_numpy_integer_matmul(lib):
     assert pins.check_numpy(lib) == []
 
 
+def test_srs_golden(lib):
+    assert pins.check_srs_golden(lib) == []
+
+
+def test_srs_reduces_to_gemm(lib):
+    assert pins.check_srs_reduces_to_gemm(lib) == []
+
+
+def test_srs_closed_forms(lib):
+    assert pins.check_srs_closed_forms(lib) == []
+
+
+def test_srs_rejects_bad_shift(lib):
+    A = np.ones((2, 3), np.int16)
+    B = np.ones((3, 2), np.int16)
+    for shift in (-1, 63):
+        with pytest.raises(ValueError):
+            oracle.gemm_srs(A, B, np.zeros((2, 2), np.int16), shift, lib=lib)
+
+
 def test_closed_forms(lib):
     assert pins.check_closed_forms(lib) == []
 
@@ -104,7 +124,8 @@ def test_workload_small_case_matches_numpy(lib):
 MUTANTS = {
     "drop_last_rank1_term": ("for (int64_t p = 0; p < k; ++p) {", "for (int64_t p = 0; p < k - 1; ++p) {"),
     "wrong_sign": ("c[j] += (uint64_t)(a * (int64_t)b[j]);", "c[j] -= (uint64_t)(a * (int64_t)b[j]);"),
-    "transposed_A_index": ("const int64_t a = (int64_t)A[i * lda + p];", "const int64_t a = (int64_t)A[p * lda + i];"),
+    # an indexing mistake that stays inside A (a transposed index can read past it and crash)
+    "reversed_A_index": ("const int64_t a = (int64_t)A[i * lda + p];", "const int64_t a = (int64_t)A[i * lda + (k - 1 - p)];"),
     "int32_accumulator": ("c[j] += (uint64_t)(a * (int64_t)b[j]);",
                           "c[j] = (uint64_t)(int64_t)(int32_t)(uint32_t)(c[j] + (uint64_t)(a * (int64_t)b[j]));"),
     "overwrites_C": ("uint64_t* c = (uint64_t*)(C + i * ldc);",
@@ -113,6 +134,18 @@ MUTANTS = {
     "off_by_one_column": ("for (int64_t j = 0; j < n; ++j)\n        c[j] +=", "for (int64_t j = 1; j < n; ++j)\n        c[j] +="),
     "i8_truncates_to_16_bits": ("c[j] = (int32_t)(uint32_t)s;", "c[j] = (int32_t)(int16_t)s;"),
     "i8_transposed_B": ("(int64_t)B[p * ldb + j]", "(int64_t)B[j * ldb + p]"),
+    # the micro-kernel output C16 += srs(A*B, shift)
+    "srs_rounds_half_down": ("oracle_floor_div_pow2(s + ((int64_t)1 << (shift - 1)), shift)",
+                             "oracle_floor_div_pow2(s + ((int64_t)1 << (shift - 1)) - 1, shift)"),
+    "srs_truncates_toward_zero": ("  if (v >= 0) return v / d;\n  return -((-v + d - 1) / d);", "  return v / d;"),
+    "srs_no_positive_saturation": ("if (r > 32767) r = 32767;", "if (r > 65535) r = 65535;"),
+    "srs_no_negative_saturation": ("if (r < -32768) r = -32768;", "if (r < -65536) r = -65536;"),
+    "srs_saturating_add": ("const uint16_t sum = (uint16_t)((uint16_t)C[i * ldc + j] + (uint16_t)r);",
+                           "int64_t t = (int64_t)C[i * ldc + j] + r; if (t > 32767) t = 32767; "
+                           "if (t < -32768) t = -32768; const uint16_t sum = (uint16_t)t;"),
+    "srs_overwrites_C": ("(uint16_t)((uint16_t)C[i * ldc + j] + (uint16_t)r)", "(uint16_t)r"),
+    "srs_shift_off_by_one": ("const int64_t d = (int64_t)1 << shift;", "const int64_t d = (int64_t)1 << (shift + 1);"),
+    "srs_drops_last_term": ("for (int64_t p = 0; p < k; ++p) s +=", "for (int64_t p = 0; p + 1 < k; ++p) s +="),
 }
 
 
