@@ -42,6 +42,7 @@ KERNEL_INFO = {
     "tc_i8": ("tc_gemm_kernel<1>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
     "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh"), "hbm"),
     "fused_i16": ("fused_kernel", ("gemm_fused.cu", "tc_common.cuh", "ptx.cuh"), "hbm"),
+    "srs": ("srs_add_kernel", ("requant.cu",), "hbm"),
 }
 
 

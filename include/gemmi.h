@@ -100,6 +100,31 @@ int gemm_i8_host(int64_t m, int64_t n, int64_t k,
                  int32_t* C, int64_t ldc);
 
 /*
+ * gemm_i16_srs -- the output of the paper's AIE micro-kernel (Section 5.2, the
+ * simplified micro-kernel listing): the wide accumulator is shifted, rounded and
+ * saturated to 16 bits ("srs") and added to an int16 C with a 16-bit addition.
+ *
+ *   S = A * B (exact), R = S for shift == 0,
+ *   R = floor((S + 2^(shift-1)) / 2^shift) for shift >= 1 (round half up),
+ *   C[i,j] = (C[i,j] + clamp(R, -32768, 32767)) mod 2^16.
+ *
+ * The paper leaves the rounding and the kind of addition unstated (its listing
+ * shifts by 0); these are this library's readings.  The saturation sees the full
+ * reduction (k_c = k).  A, B: int16 device matrices as for gemm_i16; C: int16,
+ * row-major with leading dimension ldc, updated in place.  shift in [0, 62].
+ * The exact sums pass through a library-owned int64 scratch of m x roundup(n, 8)
+ * entries (released by gemmi_release_workspace).  Errors as for gemm_i16.
+ */
+int gemm_i16_srs(int64_t m, int64_t n, int64_t k,
+                 const int16_t* A, int64_t lda,
+                 const int16_t* B, int64_t ldb,
+                 int16_t* C, int64_t ldc, int shift);
+int gemm_i16_srs_ex(int64_t m, int64_t n, int64_t k,
+                    const int16_t* A, int64_t lda,
+                    const int16_t* B, int64_t ldb,
+                    int16_t* C, int64_t ldc, int shift, void* stream);
+
+/*
  * Weight pre-packing.  Section 5.1 of the paper keeps the weight operand packed,
  * off-line, in fast memory, because a deployed model runs many inputs through
  * the same weights; only the activations are packed at run time.  Here the
@@ -193,9 +218,10 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_TC_I8   : the tcgen05 int8 GEMM kernel
  *   GEMMI_KERNEL_SKINNY  : the skinny-M int16 kernel
  *   GEMMI_KERNEL_FUSED_I16 : the narrow-n int16 kernel that splits A on chip
+ *   GEMMI_KERNEL_SRS     : the requantising pass of gemm_i16_srs
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
-       GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_COUNT = 5 };
+       GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_COUNT = 6 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

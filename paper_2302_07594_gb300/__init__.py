@@ -30,11 +30,11 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
-            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n")
+            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
-KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16 = 0, 1, 2, 3, 4
+KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
 KERNELS = (("split", KERNEL_SPLIT), ("tc_i16", KERNEL_TC_I16), ("tc_i8", KERNEL_TC_I8), ("skinny", KERNEL_SKINNY),
-           ("fused_i16", KERNEL_FUSED_I16))
+           ("fused_i16", KERNEL_FUSED_I16), ("srs", KERNEL_SRS))
 
 _lib = None
 
@@ -66,6 +66,10 @@ def lib():
         for name in ("gemm_i16_ex", "gemm_i8_ex", "gemm_i16_noalloc"):
             getattr(L, name).argtypes = core + [vp]
             getattr(L, name).restype = ctypes.c_int
+        L.gemm_i16_srs.argtypes = core + [ctypes.c_int]
+        L.gemm_i16_srs.restype = ctypes.c_int
+        L.gemm_i16_srs_ex.argtypes = core + [ctypes.c_int, vp]
+        L.gemm_i16_srs_ex.restype = ctypes.c_int
         L.gemmi_set_stream.argtypes = [vp]
         L.gemmi_set_stream.restype = None
         L.gemmi_last_error.restype = ctypes.c_char_p
@@ -157,6 +161,33 @@ def gemm_i16_noalloc(A, B, C, stream=None):
     """
     import torch
     return _torch_call("gemm_i16_noalloc", A, B, C, torch.int16, torch.int64, stream)
+
+
+def gemm_i16_srs(A, B, C, shift, stream=None):
+    """The paper's micro-kernel output on the GPU: int16 C += srs(A @ B, shift).
+
+    The exact int16 product is shifted right by `shift` (rounding half up), saturated to int16
+    and added to C modulo 2^16 (see gemm_i16_srs in include/gemmi.h).  C is int16.
+    """
+    import torch
+    for t, nm in ((A, "A"), (B, "B"), (C, "C")):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda:
+            raise TypeError(f"{nm} must be a CUDA tensor")
+        if t.dtype != torch.int16:
+            raise TypeError(f"{nm} must be torch.int16, got {t.dtype}")
+    if not (A.device == B.device == C.device):
+        raise ValueError("A, B and C must be on the same device")
+    m, k = A.shape
+    k2, n = B.shape
+    if k2 != k or tuple(C.shape) != (m, n):
+        raise ValueError(f"shape mismatch: A {tuple(A.shape)}, B {tuple(B.shape)}, C {tuple(C.shape)}")
+    if stream is None:
+        stream = torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = lib().gemm_i16_srs_ex(m, n, k, A.data_ptr(), _dev_ld(A, "A"), B.data_ptr(), _dev_ld(B, "B"),
+                                   C.data_ptr(), _dev_ld(C, "C"), int(shift), stream.cuda_stream)
+    _check(rc)
+    return C
 
 
 def gemm_i8(A, B, C, stream=None):

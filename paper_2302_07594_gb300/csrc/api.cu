@@ -45,6 +45,8 @@ struct DeviceState {
   size_t ws_bytes = 0;
   void* host_buf = nullptr;     // device staging for the *_host entry points
   size_t host_buf_bytes = 0;
+  void* sum_buf = nullptr;      // exact int64 sums for the requantising entry point
+  size_t sum_buf_bytes = 0;
   cudaEvent_t last_use = nullptr;
   cudaStream_t last_stream = nullptr;
   bool used = false;
@@ -403,6 +405,34 @@ int gemm_i16_locked(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t l
   return run_tc(*d, 2, m, n, k, A, lda, B, ldb, C, ldc, s);
 }
 
+// The paper's micro-kernel output (Section 5.2): C16 += srs(A*B, shift).  The exact product goes
+// into a zeroed int64 scratch through the regular int16 paths, then requant.cu applies the
+// shift (rounding half up), the int16 saturation and the wrapping 16-bit addition.
+int gemm_i16_srs_locked(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
+                        int64_t ldb, int16_t* C, int64_t ldc, int shift, cudaStream_t s) {
+  if (shift < 0 || shift > 62) return set_error(GEMMI_EINVAL, "shift must be in [0, 62]");
+  const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, 2, 2);
+  if (pre >= 0) return pre;  // includes m == 0, n == 0 and k == 0 (srs of an empty sum adds 0)
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const int64_t lds = static_cast<int64_t>(round_up(static_cast<size_t>(n), 8));
+  const size_t bytes = static_cast<size_t>(m) * static_cast<size_t>(lds) * 8;
+  if ((rc = ensure_buffer(&d->sum_buf, &d->sum_buf_bytes, bytes)) != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(*d, s)) != GEMMI_OK) return rc;
+  int64_t* S = static_cast<int64_t*>(d->sum_buf);
+  cudaError_t e = cudaMemsetAsync(S, 0, bytes, s);
+  if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(sums)");
+  rc = m <= g_skinny_max_m ? run_skinny(*d, m, n, k, A, lda, B, ldb, S, lds, s)
+                           : run_tc(*d, 2, m, n, k, A, lda, B, ldb, S, lds, s);
+  if (rc != GEMMI_OK) return rc;
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SRS, s);
+  e = gemmi::srs_add_i16(S, lds, C, ldc, m, n, shift, s);
+  timer_end(GEMMI_KERNEL_SRS, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, "srs launch");
+  return end_workspace_use(*d, s);
+}
+
 int gemm_i8_locked(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
                    int32_t* C, int64_t ldc, cudaStream_t s) {
   const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, 1, 4);
@@ -504,6 +534,18 @@ int gemm_i16(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, con
              int64_t* C, int64_t ldc) {
   std::lock_guard<std::mutex> lock(g_mutex);
   return gemm_i16_locked(m, n, k, A, lda, B, ldb, C, ldc, g_stream);
+}
+
+int gemm_i16_srs_ex(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
+                    int64_t ldb, int16_t* C, int64_t ldc, int shift, void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i16_srs_locked(m, n, k, A, lda, B, ldb, C, ldc, shift, static_cast<cudaStream_t>(stream));
+}
+
+int gemm_i16_srs(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,
+                 int16_t* C, int64_t ldc, int shift) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i16_srs_locked(m, n, k, A, lda, B, ldb, C, ldc, shift, g_stream);
 }
 
 int gemm_i8_ex(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
@@ -662,12 +704,14 @@ int gemmi_release_workspace(void) {
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices) return set_error(GEMMI_EINVAL, "device ordinal out of range");
   DeviceState& d = g_dev[dev];
-  if (d.ws == nullptr && d.host_buf == nullptr) return GEMMI_OK;
+  if (d.ws == nullptr && d.host_buf == nullptr && d.sum_buf == nullptr) return GEMMI_OK;
   e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
   if (d.ws) cudaFree(d.ws);
   if (d.host_buf) cudaFree(d.host_buf);
-  d.ws = d.host_buf = nullptr;
+  if (d.sum_buf) cudaFree(d.sum_buf);
+  d.ws = d.host_buf = d.sum_buf = nullptr;
+  d.sum_buf_bytes = 0;
   d.ws_bytes = d.host_buf_bytes = 0;
   d.used = false;
   return GEMMI_OK;
@@ -677,7 +721,7 @@ size_t gemmi_workspace_bytes(void) {
   std::lock_guard<std::mutex> lock(g_mutex);
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
-  return g_dev[dev].ws_bytes + g_dev[dev].host_buf_bytes;
+  return g_dev[dev].ws_bytes + g_dev[dev].host_buf_bytes + g_dev[dev].sum_buf_bytes;
 }
 
 int gemmi_set_option(int option, int64_t value) {

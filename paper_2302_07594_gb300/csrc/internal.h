@@ -78,6 +78,10 @@ cudaError_t skinny_gemm_i16(const SkinnyArgs& args, cudaStream_t s, const char**
 // ---- error text of the calling thread, as returned by gemmi_last_error().
 void record_error(const char* msg);
 
+// ---- requant.cu: C16 += srs(S, shift), S an int64 m x n matrix with row pitch lds (a multiple of 8).
+cudaError_t srs_add_i16(const int64_t* S, int64_t lds, int16_t* C, int64_t ldc, int64_t m, int64_t n, int shift,
+                        cudaStream_t s);
+
 // ---- selftest of the bounded wait.
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
 

@@ -92,6 +92,19 @@ def test_options(L):
         gm.set_option(99, 1)
 
 
+def test_srs_argument_checks(L):
+    dummy = ctypes.c_void_p(0x1000)
+    # shift outside [0, 62] is rejected before any device work
+    for shift in (-1, 63):
+        assert L.gemm_i16_srs(4, 4, 4, dummy, 4, ctypes.c_void_p(0x2000), 4, ctypes.c_void_p(0x3000), 4,
+                              shift) == gm.EINVAL
+        assert "shift" in gm.last_error()
+    assert L.gemm_i16_srs(-1, 4, 4, dummy, 4, dummy, 4, dummy, 4, 0) == gm.EINVAL
+    # empty problems are no-ops
+    assert L.gemm_i16_srs(0, 4, 4, None, 4, None, 4, None, 4, 3) == gm.OK
+    assert L.gemm_i16_srs(3, 3, 0, None, 1, None, 3, ctypes.c_void_p(0x3000), 3, 3) == gm.OK
+
+
 def test_fused_option(L):
     old = gm.get_option(gm.OPT_FUSED_MAX_N)
     assert old == 64
