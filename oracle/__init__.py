@@ -52,6 +52,8 @@ def _bind(lib):
         f.restype = ctypes.c_int
     lib.gemm_oracle_i16_srs.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int, ctypes.c_int]
     lib.gemm_oracle_i16_srs.restype = ctypes.c_int
+    lib.gemm_oracle_conv2d_i16.argtypes = [i64] * 9 + [vp, vp, vp, ctypes.c_int]
+    lib.gemm_oracle_conv2d_i16.restype = ctypes.c_int
     lib.gemm_oracle_max_threads.restype = ctypes.c_int
     return lib
 
@@ -114,6 +116,31 @@ def gemm_srs(A: np.ndarray, B: np.ndarray, C: np.ndarray, shift: int, nthreads: 
     if rc != 0:
         raise ValueError("oracle rejected the arguments")
     return C
+
+
+def conv2d(X: np.ndarray, Wt: np.ndarray, Y: np.ndarray, R: int, S: int, pad_h: int, pad_w: int,
+           nthreads: int = 1, lib=None) -> np.ndarray:
+    """In place: Y += conv(X, Wt), stride 1, zero padding (see gemm_oracle.c).
+
+    X: int16 (N, H, W, Cin); Wt: int16 (R*S*Cin, Cout) in (r, s, c) row order; Y: int64
+    (N, Ho, Wo, Cout) with Ho = H + 2*pad_h - R + 1, Wo = W + 2*pad_w - S + 1.  All C-contiguous.
+    """
+    lib = lib or load()
+    N, H, W, Cin = X.shape
+    K, Cout = Wt.shape
+    Ho, Wo = H + 2 * pad_h - R + 1, W + 2 * pad_w - S + 1
+    if X.dtype != np.int16 or Wt.dtype != np.int16 or Y.dtype != np.int64:
+        raise TypeError("conv2d takes int16 X and Wt and an int64 Y")
+    if K != R * S * Cin or Y.shape != (N, Ho, Wo, Cout):
+        raise ValueError(f"shape mismatch: X {X.shape}, Wt {Wt.shape}, Y {Y.shape}")
+    for t in (X, Wt, Y):
+        if not t.flags.c_contiguous:
+            raise ValueError("conv2d operands must be C-contiguous")
+    rc = lib.gemm_oracle_conv2d_i16(N, H, W, Cin, Cout, R, S, pad_h, pad_w, _ptr(X), _ptr(Wt), _ptr(Y),
+                                    int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments")
+    return Y
 
 
 def max_threads() -> int:

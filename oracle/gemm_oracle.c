@@ -149,6 +149,58 @@ int gemm_oracle_i16_srs(int64_t m, int64_t n, int64_t k,
   return 0;
 }
 
+/*
+ * A convolution lowered to the GEMM (Sections 2 and 3 of the paper: the IM2COL / IM2ROW
+ * transform turns the convolution operator into one large GEMM, and the transform can be applied
+ * on the fly as part of the packing).  The oracle is the convolution itself, written out from its
+ * definition rather than through a lowered matrix:
+ *   Y[n][ho][wo][co] += sum over r < R, s < S, c < Cin of
+ *                       X[n][ho + r - pad_h][wo + s - pad_w][c] * Wt[(r*S + s)*Cin + c][co],
+ * with X taken as 0 outside 0 <= h < H, 0 <= w < W (zero padding), stride 1, and
+ * Ho = H + 2*pad_h - R + 1, Wo = W + 2*pad_w - S + 1.  X is NHWC (N x H x W x Cin), Wt is the
+ * weight matrix of the lowered GEMM (R*S*Cin rows in (r, s, c) order, Cout columns), Y is NHWC
+ * (N x Ho x Wo x Cout); all dense, all HOST pointers.  Sums modulo 2^64 as in the GEMM.
+ * Returns 0, or 1 on an invalid argument.
+ */
+int gemm_oracle_conv2d_i16(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout,
+                           int64_t R, int64_t S, int64_t pad_h, int64_t pad_w,
+                           const int16_t* X, const int16_t* Wt, int64_t* Y, int nthreads) {
+  if (N < 0 || H < 0 || W < 0 || Cin < 0 || Cout < 0 || R < 1 || S < 1 || pad_h < 0 || pad_w < 0) return 1;
+  const int64_t Ho = H + 2 * pad_h - R + 1, Wo = W + 2 * pad_w - S + 1;
+  if (Ho < 0 || Wo < 0) return 1;
+  if (N == 0 || Ho == 0 || Wo == 0 || Cout == 0) return 0;
+  if (Y == NULL) return 1;
+  if (Cin == 0) return 0;
+  if (X == NULL || Wt == NULL) return 1;
+#ifdef _OPENMP
+  if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads)
+#else
+  (void)nthreads;
+#endif
+  for (int64_t row = 0; row < N * Ho; ++row) {
+    const int64_t n = row / Ho, ho = row % Ho;
+    for (int64_t wo = 0; wo < Wo; ++wo) {
+      uint64_t* y = (uint64_t*)(Y + ((n * Ho + ho) * Wo + wo) * Cout);
+      for (int64_t r = 0; r < R; ++r) {
+        const int64_t h = ho + r - pad_h;
+        if (h < 0 || h >= H) continue;
+        for (int64_t s = 0; s < S; ++s) {
+          const int64_t w = wo + s - pad_w;
+          if (w < 0 || w >= W) continue;
+          const int16_t* x = X + ((n * H + h) * W + w) * Cin;
+          for (int64_t c = 0; c < Cin; ++c) {
+            const int64_t a = (int64_t)x[c];
+            const int16_t* wt = Wt + ((r * S + s) * Cin + c) * Cout;
+            for (int64_t co = 0; co < Cout; ++co) y[co] += (uint64_t)(a * (int64_t)wt[co]);
+          }
+        }
+      }
+    }
+  }
+  return 0;
+}
+
 /* Threads the library was built to use (1 without OpenMP). */
 int gemm_oracle_max_threads(void) {
 #ifdef _OPENMP

@@ -288,8 +288,95 @@ def check_srs_closed_forms(lib):
 
 SRS_CHECKS = (check_srs_golden, check_srs_reduces_to_gemm, check_srs_closed_forms)
 
+
+# ---- convolution through the lowered GEMM: Y += conv(X, Wt)  (gemm_oracle_conv2d_i16)
+CONV_GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "conv_cases.json")
+
+
+def _conv(lib, X, Wt, Y, R, S, ph, pw):
+    Z = Y.copy()
+    oracle.conv2d(X, Wt, Z, R, S, ph, pw, lib=lib)
+    return Z
+
+
+def check_conv_golden(lib):
+    bad = []
+    with open(CONV_GOLDEN) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        N, H, W, Ci, Co, R, S, ph, pw = (c[x] for x in ("N", "H", "W", "Cin", "Cout", "R", "S", "pad_h", "pad_w"))
+        Ho, Wo = H + 2 * ph - R + 1, W + 2 * pw - S + 1
+        X = np.array(c["X"], np.int16).reshape(N, H, W, Ci)
+        Wt = np.array(c["Wt"], np.int16).reshape(R * S * Ci, Co)
+        Y = np.array(c["Y_in"], np.int64).reshape(N, Ho, Wo, Co)
+        E = np.array(c["Y_out"], np.int64).reshape(N, Ho, Wo, Co)
+        got = _conv(lib, X, Wt, Y, R, S, ph, pw)
+        if not np.array_equal(got, E):
+            bad.append(f"conv golden {c['name']}: got {got.ravel().tolist()} want {E.ravel().tolist()}")
+    return bad
+
+
+def check_conv_1x1_is_gemm(lib):
+    """A 1x1 convolution is the GEMM of the pixels (N*H*W x Cin) by the weights: numpy's matmul."""
+    bad = []
+    for seed, (N, H, W, Ci, Co) in enumerate(((2, 3, 5, 4, 6), (1, 7, 2, 9, 3))):
+        X = gi.uniform_int(730 + seed, (N, H, W, Ci), -32768, 32767, np.int16)
+        Wt = gi.uniform_int(740 + seed, (Ci, Co), -32768, 32767, np.int16)
+        Y = gi.uniform_int(750 + seed, (N, H, W, Co), -(1 << 40), 1 << 40, np.int64)
+        want = Y + np.matmul(X.reshape(-1, Ci).astype(np.int64), Wt.astype(np.int64)).reshape(N, H, W, Co)
+        if not np.array_equal(_conv(lib, X, Wt, Y, 1, 1, 0, 0), want):
+            bad.append(f"conv 1x1 != GEMM on {(N, H, W, Ci, Co)}")
+    return bad
+
+
+def check_conv_delta_kernels(lib):
+    """A kernel that is 1 at one tap and the identity across channels copies the input, shifted by
+    that tap's offset, with zeros where the shifted pixel lies outside the image."""
+    bad = []
+    N, H, W, C = 2, 5, 4, 3
+    X = gi.uniform_int(760, (N, H, W, C), -32768, 32767, np.int16)
+    Xp = np.pad(X.astype(np.int64), ((0, 0), (1, 1), (1, 1), (0, 0)))
+    for r in range(3):
+        for s in range(3):
+            Wt = np.zeros((9 * C, C), np.int16)
+            for c in range(C):
+                Wt[(r * 3 + s) * C + c, c] = 1
+            want = Xp[:, r:r + H, s:s + W, :]  # Y[h][w] = X[h + r - 1][w + s - 1], zero outside
+            got = _conv(lib, X, Wt, np.zeros((N, H, W, C), np.int64), 3, 3, 1, 1)
+            if not np.array_equal(got, want):
+                bad.append(f"conv delta at tap ({r},{s})")
+    return bad
+
+
+def check_conv_im2col_lowering(lib):
+    """The IM2COL transform (Section 2 of the paper): build the lowered matrix element by element
+    and multiply it by the weights with numpy's integer matmul."""
+    bad = []
+    for seed, (N, H, W, Ci, Co, R, S, ph, pw) in enumerate(((1, 4, 5, 2, 3, 3, 3, 1, 1),
+                                                            (2, 3, 6, 3, 2, 2, 3, 0, 1))):
+        Ho, Wo = H + 2 * ph - R + 1, W + 2 * pw - S + 1
+        X = gi.uniform_int(770 + seed, (N, H, W, Ci), -32768, 32767, np.int16)
+        Wt = gi.uniform_int(780 + seed, (R * S * Ci, Co), -32768, 32767, np.int16)
+        low = np.zeros((N * Ho * Wo, R * S * Ci), np.int64)
+        for n in range(N):
+            for ho in range(Ho):
+                for wo in range(Wo):
+                    for r in range(R):
+                        for s in range(S):
+                            h, w = ho + r - ph, wo + s - pw
+                            if 0 <= h < H and 0 <= w < W:
+                                for c in range(Ci):
+                                    low[(n * Ho + ho) * Wo + wo, (r * S + s) * Ci + c] = X[n, h, w, c]
+        want = np.matmul(low, Wt.astype(np.int64)).reshape(N, Ho, Wo, Co)
+        if not np.array_equal(_conv(lib, X, Wt, np.zeros((N, Ho, Wo, Co), np.int64), R, S, ph, pw), want):
+            bad.append(f"conv != IM2COL lowering on {(N, H, W, Ci, Co, R, S, ph, pw)}")
+    return bad
+
+
+CONV_CHECKS = (check_conv_golden, check_conv_1x1_is_gemm, check_conv_delta_kernels, check_conv_im2col_lowering)
+
 ALL_CHECKS = (check_golden, check_extreme_bruteforce, check_closed_forms, check_identity_permutation,
-              check_blocked, check_padding, check_linearity, check_transpose, check_numpy) + SRS_CHECKS
+              check_blocked, check_padding, check_linearity, check_transpose, check_numpy) + SRS_CHECKS + CONV_CHECKS
 
 
 def pin_failures(lib, bruteforce_shapes=None):

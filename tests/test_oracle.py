@@ -54,6 +54,22 @@ def test_srs_rejects_bad_shift(lib):
             oracle.gemm_srs(A, B, np.zeros((2, 2), np.int16), shift, lib=lib)
 
 
+def test_conv_golden(lib):
+    assert pins.check_conv_golden(lib) == []
+
+
+def test_conv_1x1_is_gemm(lib):
+    assert pins.check_conv_1x1_is_gemm(lib) == []
+
+
+def test_conv_delta_kernels(lib):
+    assert pins.check_conv_delta_kernels(lib) == []
+
+
+def test_conv_im2col_lowering(lib):
+    assert pins.check_conv_im2col_lowering(lib) == []
+
+
 def test_closed_forms(lib):
     assert pins.check_closed_forms(lib) == []
 
@@ -146,6 +162,16 @@ MUTANTS = {
     "srs_overwrites_C": ("(uint16_t)((uint16_t)C[i * ldc + j] + (uint16_t)r)", "(uint16_t)r"),
     "srs_shift_off_by_one": ("const int64_t d = (int64_t)1 << shift;", "const int64_t d = (int64_t)1 << (shift + 1);"),
     "srs_drops_last_term": ("for (int64_t p = 0; p < k; ++p) s +=", "for (int64_t p = 0; p + 1 < k; ++p) s +="),
+    # the convolution through the lowered GEMM
+    "conv_swaps_r_and_s": ("const int16_t* wt = Wt + ((r * S + s) * Cin + c) * Cout;",
+                           "const int16_t* wt = Wt + ((s * R + r) * Cin + c) * Cout;"),
+    "conv_padding_off_by_one": ("const int64_t h = ho + r - pad_h;", "const int64_t h = ho + r - pad_h + 1;"),
+    "conv_wraps_instead_of_zero_padding": ("const int64_t w = wo + s - pad_w;",
+                                           "const int64_t w = (wo + s - pad_w + W) % W;"),
+    "conv_drops_last_channel": ("for (int64_t c = 0; c < Cin; ++c) {\n            const int64_t a = (int64_t)x[c];",
+                                "for (int64_t c = 0; c + 1 < Cin; ++c) {\n            const int64_t a = (int64_t)x[c];"),
+    "conv_channel_stride_is_cout": ("const int16_t* x = X + ((n * H + h) * W + w) * Cin;",
+                                    "const int16_t* x = X + ((n * H + h) * W + w) * Cout;"),
 }
 
 
