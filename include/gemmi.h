@@ -125,6 +125,31 @@ int gemm_i16_srs_ex(int64_t m, int64_t n, int64_t k,
                     int16_t* C, int64_t ldc, int shift, void* stream);
 
 /*
+ * gemmi_conv2d_i16 -- a convolution through the lowered GEMM.  Sections 2 and 3 of
+ * the paper cast a convolution as one large GEMM with the IM2COL / IM2ROW transform,
+ * and note that the transform may be applied on the fly as part of the packing.
+ *
+ *   Y[n][ho][wo][co] += sum over r < R, s < S, c < Cin of
+ *                       X[n][ho + r - pad_h][wo + s - pad_w][c] * Wt[(r*S + s)*Cin + c][co],
+ * stride 1, X read as 0 outside the image, Ho = H + 2*pad_h - R + 1,
+ * Wo = W + 2*pad_w - S + 1; exact, modulo 2^64 as gemm_i16.
+ *
+ * X: int16 NHWC (N x H x W x Cin), dense.  Wt: int16, the lowered weight matrix,
+ * R*S*Cin rows in (r, s, c) order by Cout columns, dense.  Y: int64 NHWC
+ * (N x Ho x Wo x Cout), dense, updated in place.  All device pointers, owned by
+ * the caller; Y may not overlap X or Wt.  When Ho == H, Wo == W (a "same"
+ * convolution), Cin % 64 == 0, Cout <= 256 and X is 16-byte aligned, the GEMM
+ * reads X directly (no lowered matrix is formed); other shapes lower X into
+ * library-owned memory first (released by gemmi_release_workspace).
+ * Errors: GEMMI_EINVAL for negative sizes or paddings, R or S below 1, a filter
+ * larger than the padded input, null pointers with non-zero sizes, overlapping Y;
+ * otherwise as gemm_i16.  Empty outputs return GEMMI_OK.
+ */
+int gemmi_conv2d_i16(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout,
+                     int64_t R, int64_t S, int64_t pad_h, int64_t pad_w,
+                     const int16_t* X, const int16_t* Wt, int64_t* Y, void* stream);
+
+/*
  * Weight pre-packing.  Section 5.1 of the paper keeps the weight operand packed,
  * off-line, in fast memory, because a deployed model runs many inputs through
  * the same weights; only the activations are packed at run time.  Here the

@@ -30,7 +30,7 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
-            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex")
+            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex", "gemmi_conv2d_i16")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
 KERNELS = (("split", KERNEL_SPLIT), ("tc_i16", KERNEL_TC_I16), ("tc_i8", KERNEL_TC_I8), ("skinny", KERNEL_SKINNY),
@@ -70,6 +70,8 @@ def lib():
         L.gemm_i16_srs.restype = ctypes.c_int
         L.gemm_i16_srs_ex.argtypes = core + [ctypes.c_int, vp]
         L.gemm_i16_srs_ex.restype = ctypes.c_int
+        L.gemmi_conv2d_i16.argtypes = [i64] * 9 + [vp, vp, vp, vp]
+        L.gemmi_conv2d_i16.restype = ctypes.c_int
         L.gemmi_set_stream.argtypes = [vp]
         L.gemmi_set_stream.restype = None
         L.gemmi_last_error.restype = ctypes.c_char_p
@@ -188,6 +190,37 @@ def gemm_i16_srs(A, B, C, shift, stream=None):
                                    C.data_ptr(), _dev_ld(C, "C"), int(shift), stream.cuda_stream)
     _check(rc)
     return C
+
+
+def conv2d_i16(X, Wt, Y, R, S, pad_h, pad_w, stream=None):
+    """Y += conv(X, Wt) on the GPU: a stride-1, zero-padded convolution through the lowered GEMM.
+
+    X: int16 (N, H, W, Cin) NHWC; Wt: int16 (R*S*Cin, Cout), rows in (r, s, c) order; Y: int64
+    (N, Ho, Wo, Cout) with Ho = H + 2*pad_h - R + 1, Wo = W + 2*pad_w - S + 1.  All CUDA tensors,
+    C-contiguous.  See gemmi_conv2d_i16 in include/gemmi.h.
+    """
+    import torch
+    for t, nm, dt in ((X, "X", torch.int16), (Wt, "Wt", torch.int16), (Y, "Y", torch.int64)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda:
+            raise TypeError(f"{nm} must be a CUDA tensor")
+        if t.dtype != dt:
+            raise TypeError(f"{nm} must be {dt}, got {t.dtype}")
+        if not t.is_contiguous():
+            raise ValueError(f"{nm} must be contiguous")
+    if not (X.device == Wt.device == Y.device):
+        raise ValueError("X, Wt and Y must be on the same device")
+    N, H, W, Cin = X.shape
+    K, Cout = Wt.shape
+    Ho, Wo = H + 2 * pad_h - R + 1, W + 2 * pad_w - S + 1
+    if K != R * S * Cin or tuple(Y.shape) != (N, Ho, Wo, Cout):
+        raise ValueError(f"shape mismatch: X {tuple(X.shape)}, Wt {tuple(Wt.shape)}, Y {tuple(Y.shape)}")
+    if stream is None:
+        stream = torch.cuda.current_stream(X.device)
+    with torch.cuda.device(X.device):
+        rc = lib().gemmi_conv2d_i16(N, H, W, Cin, Cout, R, S, pad_h, pad_w, X.data_ptr(), Wt.data_ptr(),
+                                    Y.data_ptr(), stream.cuda_stream)
+    _check(rc)
+    return Y
 
 
 def gemm_i8(A, B, C, stream=None):

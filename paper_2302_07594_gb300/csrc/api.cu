@@ -47,6 +47,8 @@ struct DeviceState {
   size_t host_buf_bytes = 0;
   void* sum_buf = nullptr;      // exact int64 sums for the requantising entry point
   size_t sum_buf_bytes = 0;
+  void* conv_buf = nullptr;     // explicitly lowered convolution operand (fallback path)
+  size_t conv_buf_bytes = 0;
   cudaEvent_t last_use = nullptr;
   cudaStream_t last_stream = nullptr;
   bool used = false;
@@ -251,8 +253,15 @@ bool fused_applies(int nl, int64_t n, const void* A, int64_t lda, const void* C)
          reinterpret_cast<uintptr_t>(C) % 8 == 0;
 }
 
+// A stride-1 convolution whose output has the input's height and width, read as an implicit
+// IM2COL operand by the fused kernel (see FusedArgs).
+struct ConvShape {
+  int64_t N, H, W, Cin, S, ph, pw;
+};
+
 int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
-              int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b) {
+              int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b,
+              const ConvShape* conv = nullptr) {
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
   const bool split_b = packed_b == nullptr;
   LimbPlanes pb{};
@@ -285,6 +294,16 @@ int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A,
   fa.num_sms = d.sm_count;
   fa.chunk_scale = static_cast<int>(g_tc_chunk_scale);
   fa.group_m = static_cast<int>(g_tc_group_m);
+  if (conv != nullptr) {
+    fa.conv = 1;
+    fa.conv_pixels = conv->N * conv->H * conv->W;
+    fa.conv_cin = static_cast<int>(conv->Cin);
+    fa.conv_h = static_cast<int>(conv->H);
+    fa.conv_w = static_cast<int>(conv->W);
+    fa.conv_s = static_cast<int>(conv->S);
+    fa.conv_ph = static_cast<int>(conv->ph);
+    fa.conv_pw = static_cast<int>(conv->pw);
+  }
   const char* why = "fused tcgen05 GEMM launch";
   cudaEvent_t t1 = timer_begin(GEMMI_KERNEL_FUSED_I16, s);
   const cudaError_t e = gemmi::tc_gemm_fused_i16(fa, s, &why);
@@ -433,6 +452,54 @@ int gemm_i16_srs_locked(int64_t m, int64_t n, int64_t k, const int16_t* A, int64
   return end_workspace_use(*d, s);
 }
 
+// A convolution through the lowered GEMM (Sections 2 and 3 of the paper: the IM2COL transform
+// casts the convolution as one large GEMM, and the transform may be applied on the fly as part of
+// the packing).  "Same" stride-1 convolutions with Cin % 64 == 0 run the fused kernel straight
+// from the NHWC tensor (each 64-wide K block is one filter tap of 64 channels, a shifted box of
+// 128 pixels, with the converters zeroing the taps that fall outside the image); other shapes
+// materialise the lowered matrix with im2col.cu and run the regular int16 path.
+int conv2d_locked(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout, int64_t R, int64_t S, int64_t ph,
+                  int64_t pw, const int16_t* X, const int16_t* Wt, int64_t* Y, cudaStream_t s) {
+  if (N < 0 || H < 0 || W < 0 || Cin < 0 || Cout < 0) return set_error(GEMMI_EINVAL, "negative tensor dimension");
+  if (R < 1 || S < 1) return set_error(GEMMI_EINVAL, "filter height and width must be at least 1");
+  if (ph < 0 || pw < 0) return set_error(GEMMI_EINVAL, "negative padding");
+  const int64_t Ho = H + 2 * ph - R + 1, Wo = W + 2 * pw - S + 1;
+  if (Ho < 0 || Wo < 0) return set_error(GEMMI_EINVAL, "filter larger than the padded input");
+  const int64_t M = N * Ho * Wo, K = R * S * Cin;
+  if (M == 0 || Cout == 0 || K == 0) return GEMMI_OK;
+  if (X == nullptr || Wt == nullptr || Y == nullptr) return set_error(GEMMI_EINVAL, "X, Wt or Y is null");
+  if (N > (int64_t(1) << 31) || H > (int64_t(1) << 20) || W > (int64_t(1) << 20) || Cin > (int64_t(1) << 20) ||
+      Cout > (int64_t(1) << 20) || R > 64 || S > 64 || M > (int64_t(1) << 40) || K > (int64_t(1) << 31))
+    return set_error(GEMMI_EINVAL, "tensor dimension too large");
+  const size_t x_bytes = static_cast<size_t>(N * H * W * Cin) * 2;
+  const size_t w_bytes = static_cast<size_t>(K * Cout) * 2;
+  const size_t y_bytes = static_cast<size_t>(M * Cout) * 8;
+  if (overlaps(Y, y_bytes, X, x_bytes) || overlaps(Y, y_bytes, Wt, w_bytes))
+    return set_error(GEMMI_EINVAL, "Y overlaps X or Wt");
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const bool implicit = Ho == H && Wo == W && Cin % 64 == 0 && M > g_skinny_max_m && Cout <= 256 &&
+                        N * H * W < (int64_t(1) << 31) && reinterpret_cast<uintptr_t>(X) % 16 == 0 &&
+                        reinterpret_cast<uintptr_t>(Y) % 8 == 0;
+  if (implicit) {
+    const ConvShape cs{N, H, W, Cin, S, ph, pw};
+    return run_fused(*d, M, Cout, K, X, K, Wt, Cout, Y, Cout, s, nullptr, &cs);
+  }
+  // explicit lowering into library-owned memory, then the int16 GEMM
+  const int64_t lda = static_cast<int64_t>(round_up(static_cast<size_t>(K), 8));
+  const size_t a_bytes = static_cast<size_t>(M) * static_cast<size_t>(lda) * 2;
+  if ((rc = ensure_buffer(&d->conv_buf, &d->conv_buf_bytes, a_bytes)) != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(*d, s)) != GEMMI_OK) return rc;
+  int16_t* A = static_cast<int16_t*>(d->conv_buf);
+  cudaError_t e = gemmi::im2col_i16(X, A, lda, N, H, W, Cin, R, S, ph, pw, s);
+  if (e != cudaSuccess) return cuda_error(e, "im2col launch");
+  rc = M <= g_skinny_max_m ? run_skinny(*d, M, Cout, K, A, lda, Wt, Cout, Y, Cout, s)
+                           : run_tc(*d, 2, M, Cout, K, A, lda, Wt, Cout, Y, Cout, s);
+  if (rc != GEMMI_OK) return rc;
+  return end_workspace_use(*d, s);
+}
+
 int gemm_i8_locked(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
                    int32_t* C, int64_t ldc, cudaStream_t s) {
   const int pre = check_args(m, n, k, A, lda, B, ldb, C, ldc, 1, 4);
@@ -546,6 +613,12 @@ int gemm_i16_srs(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda,
                  int16_t* C, int64_t ldc, int shift) {
   std::lock_guard<std::mutex> lock(g_mutex);
   return gemm_i16_srs_locked(m, n, k, A, lda, B, ldb, C, ldc, shift, g_stream);
+}
+
+int gemmi_conv2d_i16(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout, int64_t R, int64_t S,
+                     int64_t pad_h, int64_t pad_w, const int16_t* X, const int16_t* Wt, int64_t* Y, void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return conv2d_locked(N, H, W, Cin, Cout, R, S, pad_h, pad_w, X, Wt, Y, static_cast<cudaStream_t>(stream));
 }
 
 int gemm_i8_ex(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
@@ -704,14 +777,15 @@ int gemmi_release_workspace(void) {
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices) return set_error(GEMMI_EINVAL, "device ordinal out of range");
   DeviceState& d = g_dev[dev];
-  if (d.ws == nullptr && d.host_buf == nullptr && d.sum_buf == nullptr) return GEMMI_OK;
+  if (d.ws == nullptr && d.host_buf == nullptr && d.sum_buf == nullptr && d.conv_buf == nullptr) return GEMMI_OK;
   e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
   if (d.ws) cudaFree(d.ws);
   if (d.host_buf) cudaFree(d.host_buf);
   if (d.sum_buf) cudaFree(d.sum_buf);
-  d.ws = d.host_buf = d.sum_buf = nullptr;
-  d.sum_buf_bytes = 0;
+  if (d.conv_buf) cudaFree(d.conv_buf);
+  d.ws = d.host_buf = d.sum_buf = d.conv_buf = nullptr;
+  d.sum_buf_bytes = d.conv_buf_bytes = 0;
   d.ws_bytes = d.host_buf_bytes = 0;
   d.used = false;
   return GEMMI_OK;
@@ -721,7 +795,7 @@ size_t gemmi_workspace_bytes(void) {
   std::lock_guard<std::mutex> lock(g_mutex);
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
-  return g_dev[dev].ws_bytes + g_dev[dev].host_buf_bytes + g_dev[dev].sum_buf_bytes;
+  return g_dev[dev].ws_bytes + g_dev[dev].host_buf_bytes + g_dev[dev].sum_buf_bytes + g_dev[dev].conv_buf_bytes;
 }
 
 int gemmi_set_option(int option, int64_t value) {

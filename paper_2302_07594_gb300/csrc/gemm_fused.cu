@@ -22,9 +22,12 @@
 //               which sits in tensor memory, by the stacked B tile with one
 //               tcgen05.mma of N = 128: columns 0-63 of its accumulator get
 //               A_p * B_high, columns 64-127 get A_p * B_low.
-//   warps 12-15 converters.  Thread (warp 12 + j, lane t) splits row 32j + t of
-//               each raw tile into the two fp16 limbs and stores them in its
-//               TMEM lane of the A limb stage (tcgen05.st).
+//   warps 12-19 converters, two warpgroups.  Thread (warp 12 + 4h + j, lane t)
+//               splits half h (32 reduction indices) of row 32j + t of each raw
+//               tile into the two fp16 limbs and stores them in its TMEM lane of
+//               the A limb stage (tcgen05.st).  A warp's chain of shared-memory
+//               loads, byte logic and TMEM stores is latency-bound, so two warps
+//               per scheduler convert each K block.
 //   warps 0-7   epilogue.  Warp (quadrant q = w % 4, half h = w / 4), lane t,
 //               drains row 32q + t, output columns 32h .. 32h + 31, of the
 //               accumulators (staggered exact chunks) into int64 registers.  At
@@ -42,8 +45,17 @@
 //
 // TMEM (512 columns): two A limb stages of 64 columns (high limb 0-31, low
 // 32-63; K packed two fp16 per column) and three 128-column accumulator slots
-// (two live, one spare).  Every mbarrier wait is bounded; a wait that runs out
-// records GEMMI_ETIMEOUT.
+// (two live, one spare).  Registers: 640 threads are launched with 96 each;
+// the warpgroups then re-split them with setmaxnreg (epilogue 136, producers
+// and issuers 56, converters 72), within the launch allocation, which the host
+// checks against the compiled kernel before every launch.  Every mbarrier wait
+// is bounded; a wait that runs out records GEMMI_ETIMEOUT.
+//
+// Implicit IM2COL (FusedArgs::conv): for a "same" stride-1 convolution with
+// Cin % 64 == 0, K block kb is filter tap (r, s) of 64 channels, and its A tile
+// is the box of 128 input pixels starting (r - pad_h) * W + (s - pad_w) pixels
+// from the tile's first output pixel; the converters zero the taps that fall
+// outside the image.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -63,10 +75,17 @@ constexpr int A_PRODUCER_WARP = 8;
 constexpr int B_PRODUCER_WARP = 9;
 constexpr int MMA_WARP0 = 10;
 constexpr int NISSUE = 2;
-constexpr int CONV_WARP0 = 12;                // converter warpgroup: warp 12 + j serves TMEM lanes 32j .. 32j + 31
-constexpr int NUM_CONV_WARPS = 4;
+constexpr int CONV_WARP0 = 12;                // converter warpgroups: warp 12 + 4h + j serves TMEM lanes 32j .. 32j + 31
+constexpr int NUM_CONV_WARPS = 8;            // two warpgroups: warp 12 + 4h + j converts K-block half h of quadrant j
+// per-role register budgets (setmaxnreg), per thread: epilogue, producers and issuers, converters
+constexpr int EPI_REGS = 136, CTRL_REGS = 56, CONV_REGS = 72;
+
 constexpr int NUM_THREADS = (CONV_WARP0 + NUM_CONV_WARPS) * 32;
 static_assert(CONV_WARP0 % 4 == 0, "a warp reaches the TMEM lane quadrant of its warp index modulo 4");
+static_assert((2 * EPI_REGS + CTRL_REGS + 2 * CONV_REGS) * 128 <= NUM_THREADS * 96,
+              "the split must fit what 640 threads are launched with (96 registers each)");
+static_assert((2 * EPI_REGS + CTRL_REGS + 2 * CONV_REGS) * 32 <= 16384,
+              "each scheduler holds one warp of every warpgroup: its quarter of the register file");
 constexpr int NACC = 2;                       // accumulator p: A limb p times both B limbs
 constexpr int NSLOT = 3;
 constexpr int SLOT_COLS = UMMA_N;             // 128
@@ -113,6 +132,29 @@ struct FusedParams {
   int group_m;
   uint64_t timeout_ns;
   uint32_t* status;
+  // implicit IM2COL (see FusedArgs): image height and width, filter width, paddings, channel blocks
+  int conv, conv_h, conv_w, conv_s, conv_ph, conv_pw, conv_cb;
+};
+
+// The filter tap (r, s) and channel block cb of K block kb of an implicit-IM2COL GEMM, advanced
+// one K block at a time (the division happens once, where a CTA's part of a tile starts).
+struct TapPos {
+  int cb, s, r;
+  __device__ __forceinline__ void set(int kb, const FusedParams& P) {
+    const int tap = kb / P.conv_cb;
+    cb = kb - tap * P.conv_cb;
+    r = tap / P.conv_s;
+    s = tap - r * P.conv_s;
+  }
+  __device__ __forceinline__ void advance(const FusedParams& P) {
+    if (++cb == P.conv_cb) {
+      cb = 0;
+      if (++s == P.conv_s) {
+        s = 0;
+        ++r;
+      }
+    }
+  }
 };
 
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
@@ -272,7 +314,84 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
   Span span;
   span.init(total_units, nkb);
 
-  if (warp == A_PRODUCER_WARP || warp == B_PRODUCER_WARP) {
+  if (warp >= CONV_WARP0) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(CONV_REGS) : "memory");
+    // ------------------------------------------------------------ converters: raw A -> limbs in TMEM
+    // Thread (warp 12 + 4h + j, lane t) converts half h of row 32j + t of every raw tile: it loads
+    // the half's four 16-byte chunks (128-byte swizzle: chunk c sits at c ^ (row % 8)), hands the
+    // raw slot back at once, splits the 32 values into their two limbs and stores them in its TMEM
+    // lane.
+    const int quad = (warp - CONV_WARP0) & 3;
+    const int khalf = (warp - CONV_WARP0) >> 2;  // reduction indices 32*khalf .. +31 of each K block
+    const uint32_t row = static_cast<uint32_t>(quad * 32 + lane);
+    const uint32_t lane_field = static_cast<uint32_t>(quad * 32) << 16;
+    RingPos craw, cstage;
+    bool ok = true;
+    TapPos tap;
+    int ho = 0, wo = 0;  // implicit IM2COL: this row's output pixel
+    for (Span sp = span; !sp.done() && ok; sp.next()) {
+      if (P.conv && sp.part_first()) {
+        int mt, nt;
+        tile_coords(sp.t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+        const int64_t m = static_cast<int64_t>(mt) * BM + row;
+        const int64_t img_row = m / P.conv_w;
+        wo = static_cast<int>(m - img_row * P.conv_w);
+        ho = static_cast<int>(img_row % P.conv_h);
+        tap.set(sp.kb, P);
+      }
+      const bool got = bounded_wait(raw_full0 + 8 * craw.slot, craw.phase, P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, got)) {
+        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
+        *abort_flag = 1;
+        break;
+      }
+      const uint32_t src = smem_u32(smem + craw.slot * TILE_RAW) + row * 128;
+      uint4 x[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        x[c] = lds128(src + ((static_cast<uint32_t>(4 * khalf + c) ^ (row & 7u)) << 4));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(raw_empty0 + 8 * craw.slot);
+      craw.advance(RAW_STAGES);
+      if (P.conv) {
+        // zero padding: the tap reads outside the image for this output pixel
+        const int h = ho + tap.r - P.conv_ph, w = wo + tap.s - P.conv_pw;
+        if (h < 0 || h >= P.conv_h || w < 0 || w >= P.conv_w) {
+#pragma unroll
+          for (int c = 0; c < 4; ++c) x[c] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        tap.advance(P);
+      }
+      const bool free_stage = bounded_wait(a_empty0 + 8 * cstage.slot, cstage.phase ^ 1u, P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, free_stage)) {
+        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 29);
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t t = tmem_base + lane_field + static_cast<uint32_t>(cstage.slot * A_STAGE_COLS);
+      {  // 32 reduction indices: one TMEM store of 16 columns per limb
+        uint32_t hi[16], lo[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          split_centred(x[i].x, hi[4 * i + 0], lo[4 * i + 0]);
+          split_centred(x[i].y, hi[4 * i + 1], lo[4 * i + 1]);
+          split_centred(x[i].z, hi[4 * i + 2], lo[4 * i + 2]);
+          split_centred(x[i].w, hi[4 * i + 3], lo[4 * i + 3]);
+        }
+        tc_st_32x32b_x16(t + khalf * 16, hi);
+        tc_st_32x32b_x16(t + BK / 2 + khalf * 16, lo);
+      }
+      tc_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(a_ready0 + 8 * cstage.slot);
+      cstage.advance(A_STAGES);
+    }
+    (void)ok;
+  } else if (warp >= NUM_EPI_WARPS) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(CTRL_REGS) : "memory");
+    if (warp == A_PRODUCER_WARP || warp == B_PRODUCER_WARP) {
     // ------------------------------------------------------------ TMA producers
     const bool is_a = warp == A_PRODUCER_WARP;
     const int nst = is_a ? RAW_STAGES : B_STAGES;
@@ -289,9 +408,13 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       int64_t issued = 0;
       bool stop = false;
       int mt = 0, nt = 0;
+      TapPos tap;
       for (Span sp = span; !sp.done() && !stop; sp.next()) {
         const int kb = sp.kb;
-        if (sp.part_first()) tile_coords(sp.t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+        if (sp.part_first()) {
+          tile_coords(sp.t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+          if (P.conv) tap.set(kb, P);
+        }
         {
           if (!bounded_wait(empty0 + 8 * pos.slot, pos.phase ^ 1u, P.timeout_ns) || *abort_flag) {
             report_status(P.status, STATUS_TIMEOUT, is_a ? 21 : 22);
@@ -301,8 +424,17 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
           }
           const uint32_t fb = full0 + 8 * pos.slot;
           if (is_a) {
+            // implicit IM2COL: the tap's 128 input pixels start (r - pad_h) rows and (s - pad_w)
+            // columns away from the tile's first output pixel (pixels outside the tensor read as 0;
+            // the converters zero those that fall outside the image)
+            int32_t x = kb * BK, y = mt * BM;
+            if (P.conv) {
+              x = tap.cb * BK;
+              y += (tap.r - P.conv_ph) * P.conv_w + (tap.s - P.conv_pw);
+              tap.advance(P);
+            }
             mbar_arrive_expect_tx(fb, TILE_RAW);
-            tma_load_2d(smem_u32(smem + pos.slot * TILE_RAW), &mapA, fb, kb * BK, mt * BM);
+            tma_load_2d(smem_u32(smem + pos.slot * TILE_RAW), &mapA, fb, x, y);
           } else {
             const uint32_t base = smem_u32(smem + OFF_B + pos.slot * TILE_B);
             mbar_arrive_expect_tx(fb, TILE_B);
@@ -321,59 +453,7 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
           bounded_wait(full0 + 8 * x, pos.phase ^ 1u, P.timeout_ns);
       }
     }
-  } else if (warp >= CONV_WARP0) {
-    // ------------------------------------------------------------ converters: raw A -> limbs in TMEM
-    // Thread (warp 12 + j, lane t) converts row 32j + t of every raw tile: it loads the row's eight
-    // 16-byte chunks (128-byte swizzle: chunk c sits at c ^ (row % 8)), hands the raw slot back at
-    // once, splits the 64 values into their two limbs and stores them in its TMEM lane.
-    const int quad = warp - CONV_WARP0;
-    const uint32_t row = static_cast<uint32_t>(quad * 32 + lane);
-    const uint32_t lane_field = static_cast<uint32_t>(quad * 32) << 16;
-    RingPos craw, cstage;
-    bool ok = true;
-    for (int64_t q = span.first; q < span.end && ok; ++q) {
-      const bool got = bounded_wait(raw_full0 + 8 * craw.slot, craw.phase, P.timeout_ns);
-      if (!__all_sync(0xFFFFFFFFu, got)) {
-        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 25);
-        *abort_flag = 1;
-        break;
-      }
-      const uint32_t src = smem_u32(smem + craw.slot * TILE_RAW) + row * 128;
-      uint4 x[8];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) x[c] = lds128(src + ((static_cast<uint32_t>(c) ^ (row & 7u)) << 4));
-      __syncwarp();
-      if (lane == 0) mbar_arrive(raw_empty0 + 8 * craw.slot);
-      craw.advance(RAW_STAGES);
-      const bool free_stage = bounded_wait(a_empty0 + 8 * cstage.slot, cstage.phase ^ 1u, P.timeout_ns);
-      if (!__all_sync(0xFFFFFFFFu, free_stage)) {
-        if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 29);
-        *abort_flag = 1;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t t = tmem_base + lane_field + static_cast<uint32_t>(cstage.slot * A_STAGE_COLS);
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {  // 32 reduction indices per TMEM store of 16 columns per limb
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          split_centred(x[4 * h + i].x, hi[4 * i + 0], lo[4 * i + 0]);
-          split_centred(x[4 * h + i].y, hi[4 * i + 1], lo[4 * i + 1]);
-          split_centred(x[4 * h + i].z, hi[4 * i + 2], lo[4 * i + 2]);
-          split_centred(x[4 * h + i].w, hi[4 * i + 3], lo[4 * i + 3]);
-        }
-        tc_st_32x32b_x16(t + h * 16, hi);
-        tc_st_32x32b_x16(t + BK / 2 + h * 16, lo);
-      }
-      tc_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(a_ready0 + 8 * cstage.slot);
-      cstage.advance(A_STAGES);
-    }
-    (void)ok;
-  } else if (warp >= MMA_WARP0) {
+    } else {
     // ------------------------------------------------------------ MMA issuers (issuer me owns accumulator me)
     const int me = warp - MMA_WARP0;
     if (lane == 0) {
@@ -432,7 +512,9 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       tc_commit(final_bar);
       bounded_wait(final_bar, 0, P.timeout_ns);
     }
+    }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(EPI_REGS) : "memory");
     // ------------------------------------------------------------ epilogue: drain, reduce into C
     const int quad = warp & 3;
     const int half = warp >> 2;
@@ -543,7 +625,6 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
     }
     bulk_wait_all();
   }
-
   tc_fence_before();
   __syncthreads();
   if (warp == MMA_WARP0) {
@@ -556,8 +637,11 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
 template <int CS>
 cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
   CUtensorMap mapA, mapBH, mapBL;
-  if (!encode_tensor_map_2d(&mapA, 0, a.A, static_cast<uint64_t>(a.k), static_cast<uint64_t>(a.m),
-                            static_cast<uint64_t>(a.lda) * 2, BK, BM, 128, why) ||
+  // A: the lowered matrix, or for an implicit IM2COL the NHWC tensor as (pixels x channels)
+  const uint64_t a_inner = a.conv ? static_cast<uint64_t>(a.conv_cin) : static_cast<uint64_t>(a.k);
+  const uint64_t a_outer = a.conv ? static_cast<uint64_t>(a.conv_pixels) : static_cast<uint64_t>(a.m);
+  const uint64_t a_row_bytes = a.conv ? static_cast<uint64_t>(a.conv_cin) * 2 : static_cast<uint64_t>(a.lda) * 2;
+  if (!encode_tensor_map_2d(&mapA, 0, a.A, a_inner, a_outer, a_row_bytes, BK, BM, 128, why) ||
       !encode_tensor_map_2d(&mapBH, 1, a.b.plane[0], static_cast<uint64_t>(a.k), static_cast<uint64_t>(a.b.rows),
                             static_cast<uint64_t>(a.b.pitch) * 2, BK, BN, 128, why) ||
       !encode_tensor_map_2d(&mapBL, 1, a.b.plane[1], static_cast<uint64_t>(a.k), static_cast<uint64_t>(a.b.rows),
@@ -577,6 +661,13 @@ cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
   P.group_m = a.group_m > 0 ? a.group_m : 16;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
+  P.conv = a.conv;
+  P.conv_h = a.conv_h;
+  P.conv_w = a.conv_w;
+  P.conv_s = a.conv_s;
+  P.conv_ph = a.conv_ph;
+  P.conv_pw = a.conv_pw;
+  P.conv_cb = a.conv ? a.conv_cin / BK : 1;
   const int64_t units = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles * P.num_k_blocks;
   const int grid = static_cast<int>(units < a.num_sms ? units : a.num_sms);
   static bool attr_done[64] = {};
@@ -587,6 +678,18 @@ cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
                                                   static_cast<int>(SMEM));
     if (attr != cudaSuccess) return attr;
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
+  }
+  // setmaxnreg.inc waits for registers the CTA was launched with: never launch a split that the
+  // launch allocation cannot cover (it would wait forever)
+  {
+    cudaFuncAttributes fattr;
+    const cudaError_t ae = cudaFuncGetAttributes(&fattr, fused_kernel<CS>);
+    if (ae != cudaSuccess) return ae;
+    constexpr int need = (2 * EPI_REGS + CTRL_REGS + 2 * CONV_REGS) * 128;
+    if (fattr.numRegs * NUM_THREADS < need) {
+      *why = "fused kernel: per-role register split exceeds the launch allocation";
+      return cudaErrorInvalidConfiguration;
+    }
   }
   fused_kernel<CS><<<grid, NUM_THREADS, SMEM, s>>>(mapA, mapBH, mapBL, P);
   return cudaGetLastError();

@@ -56,6 +56,13 @@ struct FusedArgs {
   int num_sms;
   int chunk_scale;
   int group_m;
+  // Implicit IM2COL (conv != 0): A is not a matrix but an NHWC tensor of conv_pixels pixels of
+  // conv_cin channels (base 16-byte aligned, conv_cin % 64 == 0); row m of the lowered matrix is
+  // output pixel m of a stride-1 convolution with Ho == H and Wo == W, and its K block kb is the
+  // 64 channels cb = kb % (cin / 64) of filter tap (r, s) = (tap / S, tap % S), tap = kb / (cin / 64).
+  int conv = 0;
+  int64_t conv_pixels = 0;
+  int conv_cin = 0, conv_h = 0, conv_w = 0, conv_s = 0, conv_ph = 0, conv_pw = 0;
 };
 cudaError_t tc_gemm_fused_i16(const FusedArgs& args, cudaStream_t s, const char** why);
 
@@ -81,6 +88,10 @@ void record_error(const char* msg);
 // ---- requant.cu: C16 += srs(S, shift), S an int64 m x n matrix with row pitch lds (a multiple of 8).
 cudaError_t srs_add_i16(const int64_t* S, int64_t lds, int16_t* C, int64_t ldc, int64_t m, int64_t n, int shift,
                         cudaStream_t s);
+
+// ---- im2col.cu: the explicit IM2COL lowering of a stride-1 convolution (lda % 8 == 0, Aout 16-byte aligned).
+cudaError_t im2col_i16(const int16_t* X, int16_t* Aout, int64_t lda, int64_t N, int64_t H, int64_t W, int64_t Cin,
+                       int64_t R, int64_t S, int64_t ph, int64_t pw, cudaStream_t s);
 
 // ---- selftest of the bounded wait.
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
