@@ -218,20 +218,10 @@ def run_reference(args):
 
 
 # ------------------------------------------------------------------ the GPU leg
-def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_sets=64):
-    """Device-resident timing of one workload; rotates input sets so the working set exceeds L2.
-
-    Returns (ms per call under CUDA-graph replay, ms per call issued eagerly, kernel timers, sets).
-    The graph replay removes the host's per-call cost (Python, argument checks, launches), which
-    is larger than the GPU time of the small workloads.
-    """
-    per_set = workload_bytes(w)
-    nsets = int(min(max_sets, max(1, math.ceil(rotate_bytes / per_set))))
-    A, B, C = gi.make_inputs(w)
-    sets = []
-    for _ in range(nsets):
-        sets.append(tuple(torch.from_numpy(x).cuda() for x in (A, B, C)))
-    fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
+def _time_calls(gm, torch, sets, fn, steps, warmup):
+    """(ms per call under CUDA-graph replay, ms per call issued eagerly, kernel timers) of fn(*set),
+    rotating over the input sets."""
+    nsets = len(sets)
     for i in range(warmup):
         fn(*sets[i % nsets])
     torch.cuda.synchronize()
@@ -262,7 +252,51 @@ def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_se
     torch.cuda.synchronize()
     graph_ms = e0.elapsed_time(e1) / (reps * ncap)
     assert gm.device_status() == gm.OK
-    del sets, graph
+    del graph
+    return graph_ms, eager_ms, kt
+
+
+def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_sets=64):
+    """Device-resident timing of one workload; rotates input sets so the working set exceeds L2.
+
+    Returns (ms per call under CUDA-graph replay, ms per call issued eagerly, kernel timers, sets).
+    The graph replay removes the host's per-call cost (Python, argument checks, launches), which
+    is larger than the GPU time of the small workloads.
+    """
+    per_set = workload_bytes(w)
+    nsets = int(min(max_sets, max(1, math.ceil(rotate_bytes / per_set))))
+    A, B, C = gi.make_inputs(w)
+    sets = [tuple(torch.from_numpy(x).cuda() for x in (A, B, C)) for _ in range(nsets)]
+    fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
+    graph_ms, eager_ms, kt = _time_calls(gm, torch, sets, fn, steps, warmup)
+    del sets
+    torch.cuda.empty_cache()
+    return graph_ms, eager_ms, kt, nsets
+
+
+# The convolution behind the im2col workload, computed from its NHWC activations
+# (gemmi_conv2d_i16): batch 32, 56x56, 64 -> 64 channels, 3x3, stride 1, pad 1.
+CONV = dict(N=32, H=56, W=56, Cin=64, Cout=64, R=3, S=3, ph=1, pw=1)
+
+
+def conv_bytes():
+    c = CONV
+    return (c["N"] * c["H"] * c["W"] * c["Cin"] * 2 + c["R"] * c["S"] * c["Cin"] * c["Cout"] * 2
+            + 2 * c["N"] * c["H"] * c["W"] * c["Cout"] * 8)
+
+
+def time_conv(gm, torch, steps, warmup, rotate_bytes=4 * L2_BYTES):
+    """Like time_workload, for the implicit convolution: X with the workload's activation
+    distribution (half exact zeros, else [0, 4095]), weights in [-2048, 2047], Y = 0."""
+    c = CONV
+    nsets = int(max(1, math.ceil(rotate_bytes / conv_bytes())))
+    X = gi.half_zero_uniform(1003, (c["N"], c["H"], c["W"], c["Cin"]), 4095, np.int16)
+    Wt = gi.uniform_int(1006, (c["R"] * c["S"] * c["Cin"], c["Cout"]), -2048, 2047, np.int16)
+    Y = np.zeros((c["N"], c["H"], c["W"], c["Cout"]), np.int64)
+    sets = [tuple(torch.from_numpy(x).cuda() for x in (X, Wt, Y)) for _ in range(nsets)]
+    fn = lambda x, wt, y: gm.conv2d_i16(x, wt, y, c["R"], c["S"], c["ph"], c["pw"])
+    graph_ms, eager_ms, kt = _time_calls(gm, torch, sets, fn, steps, warmup)
+    del sets
     torch.cuda.empty_cache()
     return graph_ms, eager_ms, kt, nsets
 
@@ -422,6 +456,18 @@ def run_gemmi(args):
                 ent["frac_of_int8_roofline_div4" if ow.kind == "i16" else "frac_of_int8_roofline"] = (
                     ent["TOPS"] / (int8_peak / 4 if ow.kind == "i16" else int8_peak))
             extra[name] = ent
+        try:
+            cms, ceager, ckt, cn = time_conv(gm, torch, steps=128, warmup=5)
+            ops = 2 * CONV["N"] * CONV["H"] * CONV["W"] * CONV["Cout"] * CONV["R"] * CONV["S"] * CONV["Cin"]
+            extra["conv3x3_implicit"] = {
+                "ms": cms, "timing": "CUDA-graph replay, per call", "eager_ms": ceager,
+                "what": "gemmi_conv2d_i16 on NHWC activations: the im2col workload's convolution "
+                        "without forming the lowered matrix", "shape": CONV,
+                "TOPS": ops / (cms * 1e-3) / 1e12, "GB_per_s": conv_bytes() / (cms * 1e-3) / 1e9,
+                "frac_of_hbm": conv_bytes() / (cms * 1e-3) / 1e9 / peaks["hbm_gbs"], "input_sets_rotated": cn,
+                "kernel_ms": {KERNEL_INFO[k][0]: ckt[k][0] / ckt[k][1] for k in KERNEL_INFO if ckt[k][1] > 0}}
+        except Exception as ex:  # pragma: no cover
+            extra["conv3x3_implicit"] = {"error": str(ex)}
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
