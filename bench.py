@@ -47,6 +47,10 @@ KERNEL_INFO = {
 
 
 def parse_args():
+    return parse_args_list(None)
+
+
+def parse_args_list(argv):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=200)
@@ -56,7 +60,7 @@ def parse_args():
     p.add_argument("--no-extra", action="store_true", help="skip the per-workload table")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU budget of the oracle baseline")
-    return p.parse_args()
+    return p.parse_args(argv)
 
 
 def measured_peaks():
@@ -145,6 +149,22 @@ def workload_bytes(w):
     op = 2 if w.kind == "i16" else 1
     cb = 8 if w.kind == "i16" else 4
     return w.m * w.k * op + w.k * w.n * op + 2 * w.m * w.n * cb
+
+
+def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
+    """The largest value of x over all ranks (the slowest replica sets the job's time)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, seconds: float, world: int) -> float:
+    """Whole-job rate: every rank processed units_per_rank in the (max-over-ranks) time."""
+    return world * units_per_rank / seconds
 
 
 def dist_setup():
@@ -364,11 +384,8 @@ def run_gemmi(args):
     kt = {name: gm.kernel_time(kid) for name, kid in gm.KERNELS}
     gm.kernel_timing(False)
     assert gm.device_status() == gm.OK
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * w.ops / (ms * 1e-3) / 1e12
+    ms = max_over_ranks(ms, world)
+    value = job_throughput(w.ops, ms * 1e-3, world) / 1e12
 
     # ---- dominant kernel (most device time in the timed region) and its roofline
     launches = sum(kn for _, kn in kt.values())
@@ -422,11 +439,8 @@ def run_gemmi(args):
     for _ in range(e2e_steps):
         host_fn(hA, hB, hC)
     e2e_s = (time.perf_counter() - t0) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e = {"value": world * w.ops / e2e_s / 1e12, "unit": "TOPS", "ms_per_step": e2e_s * 1e3,
+    e2e_s = max_over_ranks(e2e_s, world)
+    e2e = {"value": job_throughput(w.ops, e2e_s, world) / 1e12, "unit": "TOPS", "ms_per_step": e2e_s * 1e3,
            "h2d_bytes_per_step": int(A.nbytes + B.nbytes + C.nbytes), "d2h_bytes_per_step": int(C.nbytes),
            "steps": e2e_steps, "api": "gemm_i16_host" if w.kind == "i16" else "gemm_i8_host"}
     del hA, hB, hC
