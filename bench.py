@@ -43,6 +43,8 @@ KERNEL_INFO = {
     "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh"), "hbm"),
     "fused_i16": ("fused_kernel", ("gemm_fused.cu", "tc_common.cuh", "ptx.cuh"), "hbm"),
     "srs": ("srs_add_kernel", ("requant.cu",), "hbm"),
+    "tc_pair_i16": ("tc_pair_kernel<2>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "tensor"),
+    "tc_pair_i8": ("tc_pair_kernel<1>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "tensor"),
 }
 
 

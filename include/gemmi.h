@@ -214,11 +214,14 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_FUSED_MAX_N  : int16 GEMMs with n <= this value (and an A whose base is 16-byte
  *                            aligned with lda % 8 == 0) take the kernel that reads A raw and
  *                            splits it on chip (default 64; 0 disables it; at most 4096).
+ *   GEMMI_OPT_TC_PAIR      : 1 (default): tensor-core GEMMs run on pairs of SMs (tcgen05
+ *                            cta_group::2, clusters of two CTAs) whenever C is 16-byte aligned
+ *                            with ldc * sizeof(element) a multiple of 16; 0: one SM per tile.
  * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
 enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
        GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6,
-       GEMMI_OPT_FUSED_MAX_N = 7 };
+       GEMMI_OPT_FUSED_MAX_N = 7, GEMMI_OPT_TC_PAIR = 8 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 
@@ -244,9 +247,12 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_SKINNY  : the skinny-M int16 kernel
  *   GEMMI_KERNEL_FUSED_I16 : the narrow-n int16 kernel that splits A on chip
  *   GEMMI_KERNEL_SRS     : the requantising pass of gemm_i16_srs
+ *   GEMMI_KERNEL_TC_PAIR_I16 : the tcgen05 int16 GEMM kernel on SM pairs
+ *   GEMMI_KERNEL_TC_PAIR_I8  : the tcgen05 int8 GEMM kernel on SM pairs
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
-       GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_COUNT = 6 };
+       GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_TC_PAIR_I16 = 6, GEMMI_KERNEL_TC_PAIR_I8 = 7,
+       GEMMI_KERNEL_COUNT = 8 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

@@ -118,6 +118,7 @@ int64_t g_tc_chunk_scale = 2;
 int64_t g_tc_group_m = 16;
 int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
+int64_t g_tc_pair = 1;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -351,9 +352,14 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
   ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
   const char* why = "tcgen05 GEMM launch";
-  const int kind = nl == 2 ? GEMMI_KERNEL_TC_I16 : GEMMI_KERNEL_TC_I8;
+  // SM pairs (cta_group::2) unless switched off or C cannot take 16-byte bulk reductions
+  const int64_t esz = nl == 2 ? 8 : 4;
+  const bool pair = g_tc_pair != 0 && reinterpret_cast<uintptr_t>(C) % 16 == 0 && (ldc * esz) % 16 == 0;
+  const int kind = pair ? (nl == 2 ? GEMMI_KERNEL_TC_PAIR_I16 : GEMMI_KERNEL_TC_PAIR_I8)
+                        : (nl == 2 ? GEMMI_KERNEL_TC_I16 : GEMMI_KERNEL_TC_I8);
   cudaEvent_t t1 = timer_begin(kind, s);
-  e = nl == 2 ? gemmi::tc_gemm_i16(ta, s, &why) : gemmi::tc_gemm_i8(ta, s, &why);
+  if (pair) e = nl == 2 ? gemmi::tc_pair_gemm_i16(ta, s, &why) : gemmi::tc_pair_gemm_i8(ta, s, &why);
+  else e = nl == 2 ? gemmi::tc_gemm_i16(ta, s, &why) : gemmi::tc_gemm_i8(ta, s, &why);
   timer_end(kind, t1, s);
   if (e != cudaSuccess) return cuda_error(e, why);
   return end_workspace_use(d, s);
@@ -830,6 +836,10 @@ int gemmi_set_option(int option, int64_t value) {
       if (value < 0 || value > 4096) return set_error(GEMMI_EINVAL, "fused-kernel n limit must be in [0, 4096]");
       g_fused_max_n = value;
       return GEMMI_OK;
+    case GEMMI_OPT_TC_PAIR:
+      if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "SM-pair option must be 0 or 1");
+      g_tc_pair = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -845,6 +855,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_TC_GROUP_M: return g_tc_group_m;
     case GEMMI_OPT_TC_L2_HINTS: return g_tc_l2_hints;
     case GEMMI_OPT_FUSED_MAX_N: return g_fused_max_n;
+    case GEMMI_OPT_TC_PAIR: return g_tc_pair;
     default: return -1;
   }
 }

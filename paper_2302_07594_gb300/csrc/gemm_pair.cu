@@ -1,0 +1,462 @@
+// gemm_pair.cu -- exact integer GEMM on SM pairs: tcgen05.mma with cta_group::2 (sm_103a).
+//
+// What it computes: C += A*B (Section 4.1 of the paper) for int16 operands and an int64 C, or int8
+// operands and an int32 C, bit-exactly -- the same operation as gemm_tc.cu, from the same fp16
+// limb planes (split.cu), with the same exact-chunk accumulation (fp32 sums of at most 512 * CS
+// limb products of magnitude <= 2^14, drained into 64-bit registers; the role of the AIE's wide
+// accumulators, Section 6.2).
+//
+// How it differs.  Two CTAs of a cluster, on two SMs, form a pair.  One thread of the even CTA
+// issues tcgen05.mma.cta_group::2 of M = 256, N = 256, K = 16: rows 0-127 of the A operand and
+// of the accumulator live in the even CTA, rows 128-255 in the odd one, and each CTA holds half
+// of the (K-major) B operand.  The pair gives every SM a single 256-column accumulator, so the
+// other 256 TMEM columns are a spare slot: at a chunk end the MMAs move on into the spare while
+// the epilogue drains the full slot, and the tensor pipe does not wait for drains.
+//   int16: the even CTA holds the high limb of A's 128 rows, the odd CTA the low limb of the same
+//          rows; B's high limb tile is the even CTA's half of B, the low limb tile the odd CTA's.
+//          So the even SM accumulates A_high * [B_high | B_low] (weights 2^16 | 2^8) and the odd
+//          SM A_low * [B_high | B_low] (weights 2^8 | 1) for one 128 x 128 output tile.
+//   int8:  a 256 x 256 output tile; each SM holds 128 rows of A and 128 rows (output columns)
+//          of B, and accumulates its 128 rows x all 256 columns.
+// Per K block of 64 each SM loads 32 KB (its A tile and its B tile) for 512 tensor cycles: 64 B
+// per cycle from L2, where a single-SM 128 x 256 int8 tile needs 96.
+//
+// The running int64 (int32) sums of a tile are added into C with bulk asynchronous reductions
+// (cp.reduce.async.bulk .add) from a small per-thread staging area, so the two SMs of an int16
+// tile add their weighted halves into C independently and C is never read by the SMs.
+//
+// Structure (one CTA per SM, clusters of two, 320 threads per CTA):
+//   warp 8   TMA producer: both CTAs load their halves; every load completes on the full
+//            barrier of the even CTA, which expects the bytes of both;
+//   warp 9   TMEM allocation (both CTAs) and, in the even CTA, the single MMA-issuing thread;
+//            its commits arrive on the barriers of both CTAs (multicast);
+//   warps 0-7 epilogue: drain this SM's accumulator (tcgen05.ld), release the slot on the even
+//            CTA's barrier (a remote arrival from the odd CTA), and reduce finished tiles into C.
+// Every wait is bounded (a timeout records GEMMI_ETIMEOUT in the status word); a final handshake
+// between the two CTAs keeps each alive until its peer no longer signals it.
+#include <cuda.h>
+#include <cuda_fp16.h>
+
+#include <type_traits>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "ptx_pair.cuh"
+#include "tc_common.cuh"
+
+namespace gemmi {
+namespace {
+
+using tc::BK;
+using tc::UMMA_K;
+
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int PRODUCER_WARP = 8;
+constexpr int MMA_WARP = 9;
+constexpr int NUM_THREADS = 10 * 32;
+constexpr int TMEM_COLS = 512;
+constexpr int NSLOT = 2;                      // accumulator slots of 256 columns
+constexpr int SLOT_COLS = 256;
+constexpr int UMMA_M = 256;
+constexpr int UMMA_N = 256;
+constexpr int HALF = 128;                     // rows of A, and of K-major B, per CTA and stage
+constexpr int TILE_A = HALF * BK * 2;         // 16 KB
+constexpr int TILE_B = HALF * BK * 2;         // 16 KB
+constexpr int SB = TILE_A + TILE_B;           // one CTA's part of a stage
+constexpr int STAGES = 5;
+constexpr int SWIZZLE = BK * 2;               // 128-byte rows
+constexpr int RED_BYTES = 128;                // bytes of one C row segment per bulk reduction
+constexpr int STG_LANE = RED_BYTES + 16;      // staging stride per thread (the 16 spread the banks)
+constexpr int STG_BYTES = NUM_EPI_WARPS * 32 * STG_LANE;
+constexpr int NBAR = 2 * STAGES + 2 * NSLOT + 2;  // full, empty, slot full, slot empty, final, bye
+constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + STG_BYTES + 8 * NBAR + 16;
+static_assert(SMEM <= 227 * 1024, "shared memory budget");
+static_assert(NSLOT * SLOT_COLS <= TMEM_COLS, "tensor memory budget");
+
+// Output tile of one pair and where each CTA's operand rows start inside it.
+template <int NL>
+struct PairGeom;
+template <>
+struct PairGeom<2> {
+  static constexpr int TM = 128, TN = 128;           // output tile
+  static constexpr int A_STEP = 0, B_STEP = 0;       // both CTAs read the same rows (other limb)
+  static constexpr int COLS = 64;                    // output columns per epilogue thread
+};
+template <>
+struct PairGeom<1> {
+  static constexpr int TM = 256, TN = 256;
+  static constexpr int A_STEP = 128, B_STEP = 128;   // the odd CTA's rows / columns
+  static constexpr int COLS = 128;
+};
+
+struct PairParams {
+  int64_t m, n, k;
+  void* C;
+  int64_t ldc;
+  int num_m_tiles, num_n_tiles, num_k_blocks;
+  int group_m;
+  int hint_a, hint_b;
+  uint64_t timeout_ns;
+  uint32_t* status;
+};
+
+__device__ __forceinline__ void load_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y, int hint,
+                                          uint64_t policy) {
+  if (hint == 0) tma_load_2d_pair(dst, map, bar, x, y);
+  else tma_load_2d_pair_hint(dst, map, bar, x, y, policy);
+}
+
+// The epilogue of one CTA.  For int16 the weights of accumulator columns 0-127 and 128-255 depend
+// on the CTA's A limb: 2^16 | 2^8 in the even CTA, 2^8 | 1 in the odd one.  Both CTAs drain
+// with the odd CTA's weights (one code path, constant shifts) and the even CTA scales its tile's
+// sums by 2^8 when it adds them into C: shifting commutes with addition modulo 2^64.
+template <int NL, int CS>
+__device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uint32_t tmem_base, uint32_t sfull0,
+                                         uint32_t sempty_leader0, uint8_t* stg, int pair, int npairs, int nchunks) {
+  const uint32_t tile_shift = (NL == 2 && rank == 0) ? 8u : 0u;
+  using G = PairGeom<NL>;
+  using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
+  using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
+  constexpr int COLS = G::COLS;
+  constexpr int EPR = RED_BYTES / static_cast<int>(sizeof(CT));  // elements per reduction
+  constexpr int ROUNDS = COLS / EPR;
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  const int quad = warp & 3;   // TMEM lanes 32*quad .. +31 (the warp's hardware lane quadrant)
+  const int half = warp >> 2;  // output columns half*COLS .. +COLS-1 of the tile
+  uint8_t* my_stg = stg + (warp * 32 + lane) * STG_LANE;
+  const uint32_t my_stg_s = smem_u32(my_stg);
+  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
+  int chunk = 0;
+  bool ok = true;
+  UT acc[COLS];
+  for (int t = pair; t < total_tiles && ok; t += npairs) {
+    int mt, nt;
+    tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+    const int64_t row = static_cast<int64_t>(mt) * G::TM + rank * G::A_STEP + quad * 32 + lane;
+    const int64_t col0 = static_cast<int64_t>(nt) * G::TN + half * COLS;
+#pragma unroll
+    for (int c = 0; c < COLS; ++c) acc[c] = 0;
+    for (int ch = 0; ch < nchunks; ++ch, ++chunk) {
+      const int slot = chunk & 1;
+      const uint32_t use = static_cast<uint32_t>(chunk >> 1);
+      // every lane waits; the warp then decides together (tcgen05.ld needs a converged warp)
+      const bool got = bounded_wait(sfull0 + 8 * slot, use & 1u, P.timeout_ns);
+      if (!__all_sync(0xFFFFFFFFu, got)) {
+        if (lane == 0) report_status(P.status, tc::STATUS_TIMEOUT, 24);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                             static_cast<uint32_t>(slot * SLOT_COLS + half * COLS);
+      if constexpr (NL == 2) {
+        // this thread's 64 output columns: weight 2^8 from accumulator columns 0-127 (B high
+        // limb), 1 from columns 128-255 (B low limb), before the tile shift
+#pragma unroll
+        for (int c = 0; c < COLS; c += 8) {
+          uint32_t rh[8], rl[8];  // eight columns at a time: the 64 running sums take 128 registers
+          tc_ld_32x32b_x8(taddr + c, rh);
+          tc_ld_32x32b_x8(taddr + 128 + c, rl);
+          tc_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            acc[c + i] += (static_cast<UT>(static_cast<CT>(tc::f32_to_i32(rh[i]))) << 8) +
+                          static_cast<UT>(static_cast<CT>(tc::f32_to_i32(rl[i])));
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < COLS; c += 32) {
+          uint32_t r0[16], r1[16];
+          tc_ld_32x32b_x16(taddr + c, r0);
+          tc_ld_32x32b_x16(taddr + c + 16, r1);
+          tc_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            acc[c + i] += static_cast<UT>(tc::f32_to_i32(r0[i]));
+            acc[c + 16 + i] += static_cast<UT>(tc::f32_to_i32(r1[i]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(sempty_leader0 + 8 * slot);
+    }
+    if (!ok) break;
+    // add the tile's running sums into C, one 128-byte row segment per bulk reduction
+    if (row < P.m) {
+      CT* crow = static_cast<CT*>(P.C) + row * P.ldc + col0;
+#pragma unroll
+      for (int j = 0; j < ROUNDS; ++j) {
+        const int64_t valid = P.n - (col0 + j * EPR);
+        if (valid <= 0) break;
+        bulk_wait_read_all();  // the previous reduction has finished reading the staging area
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if constexpr (NL == 2) {
+            *reinterpret_cast<ulonglong2*>(my_stg + 16 * q) =
+                make_ulonglong2(acc[j * EPR + 2 * q] << tile_shift, acc[j * EPR + 2 * q + 1] << tile_shift);
+          } else {
+            *reinterpret_cast<uint4*>(my_stg + 16 * q) = make_uint4(acc[j * EPR + 4 * q], acc[j * EPR + 4 * q + 1],
+                                                                    acc[j * EPR + 4 * q + 2], acc[j * EPR + 4 * q + 3]);
+          }
+        }
+        fence_proxy_async_smem();
+        CT* dst = crow + j * EPR;
+        const int v = valid >= EPR ? EPR : static_cast<int>(valid);
+        const int bulk_elems = (v * static_cast<int>(sizeof(CT))) / 16 * 16 / static_cast<int>(sizeof(CT));
+        if (bulk_elems > 0) {
+          if constexpr (NL == 2) bulk_reduce_add_u64(dst, my_stg_s, static_cast<uint32_t>(bulk_elems * 8));
+          else bulk_reduce_add_u32(dst, my_stg_s, static_cast<uint32_t>(bulk_elems * 4));
+          bulk_commit();
+        }
+        // a ragged right edge: the last few elements one by one (read back from the staging area)
+        for (int i = bulk_elems; i < v; ++i) {
+          if constexpr (NL == 2)
+            atomicAdd(reinterpret_cast<unsigned long long*>(dst + i),
+                      static_cast<unsigned long long>(reinterpret_cast<const UT*>(my_stg)[i]));
+          else
+            atomicAdd(reinterpret_cast<unsigned int*>(dst + i), reinterpret_cast<const UT*>(my_stg)[i]);
+        }
+      }
+    }
+  }
+  bulk_wait_all();
+}
+
+template <int NL, int CS>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
+               const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1, PairParams P) {
+  using G = PairGeom<NL>;
+  constexpr int KPC = 8 * CS;  // K blocks per exact chunk: 512 * CS reduction indices
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* stg = smem + STAGES * SB;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(stg + STG_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t sfull0 = empty0 + 8 * STAGES;
+  const uint32_t sempty0 = sfull0 + 8 * NSLOT;
+  const uint32_t final_bar = sempty0 + 8 * NSLOT;
+  const uint32_t bye_bar = final_bar + 8;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + NBAR);
+
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);   // the even CTA's producer arrives (with both CTAs' bytes)
+      mbar_init(empty0 + 8 * s, 1);  // one commit of the MMA thread
+    }
+    for (int s = 0; s < NSLOT; ++s) {
+      mbar_init(sfull0 + 8 * s, 1);
+      mbar_init(sempty0 + 8 * s, 2 * NUM_EPI_WARPS);  // every epilogue warp of both CTAs
+    }
+    mbar_init(final_bar, 1);
+    mbar_init(bye_bar, 1);
+    fence_mbar_init();
+  }
+  if (warp == MMA_WARP) {
+    tmem_alloc_pair(smem_u32(tmem_holder), TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const int pair = static_cast<int>(cluster_id_x());
+  const int npairs = static_cast<int>(cluster_count_x());
+  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
+  const int nkb = P.num_k_blocks;
+  const int nchunks = (nkb + KPC - 1) / KPC;
+
+  if (warp == PRODUCER_WARP) {
+    // ------------------------------------------------------------ TMA producer (both CTAs)
+    if (lane == 0) {
+      const CUtensorMap* ma = (NL == 2 && rank == 1) ? &mapA1 : &mapA0;
+      const CUtensorMap* mb = (NL == 2 && rank == 1) ? &mapB1 : &mapB0;
+      tma_prefetch_desc(ma);
+      tma_prefetch_desc(mb);
+      const uint64_t pol_a = tc::l2_policy(P.hint_a);
+      const uint64_t pol_b = tc::l2_policy(P.hint_b);
+      const uint32_t full_leader0 = map_to_rank(full0, 0);
+      tc::RingPos st;
+      int64_t issued = 0;
+      bool ok = true;
+      for (int t = pair; t < total_tiles && ok; t += npairs) {
+        int mt, nt;
+        tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+        const int arow = mt * G::TM + static_cast<int>(rank) * G::A_STEP;
+        const int brow = nt * G::TN + static_cast<int>(rank) * G::B_STEP;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
+            report_status(P.status, tc::STATUS_TIMEOUT, 21);
+            ok = false;
+            break;
+          }
+          if (leader) mbar_arrive_expect_tx(full0 + 8 * st.slot, 2 * SB);
+          const uint32_t fb = full_leader0 + 8 * st.slot;
+          const uint32_t base = smem_u32(smem + st.slot * SB);
+          load_pair(base, ma, fb, kb * BK, arow, P.hint_a, pol_a);
+          load_pair(base + TILE_A, mb, fb, kb * BK, brow, P.hint_b, pol_b);
+          ++issued;
+          st.advance(STAGES);
+        }
+      }
+      // no copy of this CTA may still be landing when it exits: the last stages must have been
+      // consumed by the MMAs (which waited for every byte of them)
+      const int64_t first = issued > STAGES ? issued - STAGES : 0;
+      for (int64_t i = first; i < issued; ++i)
+        bounded_wait(empty0 + 8 * static_cast<int>(i % STAGES), static_cast<uint32_t>((i / STAGES) & 1), P.timeout_ns);
+    }
+  } else if (warp == MMA_WARP) {
+    // ------------------------------------------------------------ MMA issue (even CTA, one thread)
+    if (lane == 0) {
+      if (leader) {
+        constexpr uint32_t idesc = idesc_f16_f32(UMMA_M, UMMA_N);
+        tc::RingPos st;
+        int chunk = 0;
+        bool ok = true;
+        for (int t = pair; t < total_tiles && ok; t += npairs) {
+          for (int ch = 0; ch < nchunks; ++ch, ++chunk) {
+            const int slot = chunk & 1;
+            const uint32_t use = static_cast<uint32_t>(chunk >> 1);
+            // the slot's previous chunk must have been drained by both CTAs
+            if (!bounded_wait_cluster(sempty0 + 8 * slot, (use & 1u) ^ 1u, P.timeout_ns)) {
+              report_status(P.status, tc::STATUS_TIMEOUT, 22);
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS);
+            const int kb0 = ch * KPC;
+            const int kb1 = min(nkb, kb0 + KPC);
+            for (int kb = kb0; kb < kb1; ++kb) {
+              if (!bounded_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns)) {
+                report_status(P.status, tc::STATUS_TIMEOUT, 23);
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t base = smem_u32(smem + st.slot * SB);
+              const uint64_t adesc = smem_desc_kmajor<SWIZZLE>(base);
+              const uint64_t bdesc = smem_desc_kmajor<SWIZZLE>(base + TILE_A);
+#pragma unroll
+              for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+                // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
+                tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb == kb0 && kk == 0) ? 0u : 1u);
+              }
+              tc_commit_pair(empty0 + 8 * st.slot, 0x3);  // stage free in both CTAs once read
+              st.advance(STAGES);
+            }
+            if (!ok) break;
+            tc_commit_pair(sfull0 + 8 * slot, 0x3);  // chunk ready to drain in both CTAs
+          }
+        }
+        tc_commit_pair(final_bar, 0x3);
+      }
+      // both CTAs: every MMA of the pair, and every commit arrival, has landed
+      bounded_wait(final_bar, 0, P.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 0..7)
+    const uint32_t sempty_leader0 = map_to_rank(sempty0, 0);
+    epilogue<NL, CS>(P, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs, nchunks);
+  }
+
+  // Pair handshake: neither CTA exits (or frees tensor memory) while its peer may still signal it.
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    mbar_arrive_cluster(map_to_rank(bye_bar, rank ^ 1u));
+    if (!bounded_wait_cluster(bye_bar, 0, P.timeout_ns)) report_status(P.status, tc::STATUS_TIMEOUT, 25);
+  }
+  __syncthreads();
+  if (warp == MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+template <int NL, int CS>
+cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
+  using G = PairGeom<NL>;
+  CUtensorMap maps[4];
+  const LimbPlanes* ops[2] = {&a.a, &a.b};
+  for (int o = 0; o < 2; ++o) {
+    for (int l = 0; l < 2; ++l) {
+      const void* base = ops[o]->plane[l < NL ? l : 0];
+      if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
+                                static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
+                                HALF, SWIZZLE, why))
+        return cudaErrorInvalidValue;
+    }
+  }
+  PairParams P;
+  P.m = a.m;
+  P.n = a.n;
+  P.k = a.k;
+  P.C = a.C;
+  P.ldc = a.ldc;
+  P.num_m_tiles = static_cast<int>((a.m + G::TM - 1) / G::TM);
+  P.num_n_tiles = static_cast<int>((a.n + G::TN - 1) / G::TN);
+  P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
+  P.group_m = a.group_m > 0 ? a.group_m : 16;
+  P.hint_a = a.hint_a;
+  P.hint_b = a.hint_b;
+  P.timeout_ns = a.timeout_ns;
+  P.status = a.status;
+  const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
+
+  auto kernel = tc_pair_kernel<NL, CS>;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = SMEM;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // the shared-memory opt-in and the number of co-resident pairs, once per device
+  static int max_pairs[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int pairs_here = (dev >= 0 && dev < 64) ? max_pairs[dev] : 0;
+  if (pairs_here == 0) {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(SMEM));
+    if (e != cudaSuccess) return e;
+    cfg.gridDim = dim3(2 * static_cast<unsigned>(a.num_sms / 2), 1, 1);
+    e = cudaOccupancyMaxActiveClusters(&pairs_here, kernel, &cfg);
+    if (e != cudaSuccess) return e;
+    if (pairs_here <= 0) {
+      *why = "no two SMs can host a CTA pair of the tcgen05 pair GEMM";
+      return cudaErrorInvalidConfiguration;
+    }
+    if (dev >= 0 && dev < 64) max_pairs[dev] = pairs_here;
+  }
+  const int npairs = static_cast<int>(tiles < pairs_here ? tiles : pairs_here);
+  cfg.gridDim = dim3(2 * static_cast<unsigned>(npairs), 1, 1);
+  *why = "tcgen05 pair GEMM launch";
+  return cudaLaunchKernelEx(&cfg, kernel, maps[0], maps[1], maps[2], maps[3], P);
+}
+
+}  // namespace
+
+cudaError_t tc_pair_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch_pair<2, 2>(args, s, why) : launch_pair<2, 1>(args, s, why);
+}
+cudaError_t tc_pair_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch_pair<1, 2>(args, s, why) : launch_pair<1, 1>(args, s, why);
+}
+
+}  // namespace gemmi

@@ -43,6 +43,11 @@ struct TcGemmArgs {
 cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
 
+// ---- gemm_pair.cu: the same GEMM on SM pairs (tcgen05 cta_group::2).  The kernel adds into C with
+// bulk reductions: C 16-byte aligned and ldc * sizeof(C element) a multiple of 16.
+cudaError_t tc_pair_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
+cudaError_t tc_pair_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
+
 // ---- gemm_fused.cu: int16 GEMM, n <= 64 per tile column, A read raw (int16) and split on chip.
 struct FusedArgs {
   int64_t m, n, k;

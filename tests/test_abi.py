@@ -116,6 +116,16 @@ def test_fused_option(L):
             gm.set_option(gm.OPT_FUSED_MAX_N, bad)
 
 
+def test_pair_option(L):
+    assert gm.get_option(gm.OPT_TC_PAIR) == 1
+    gm.set_option(gm.OPT_TC_PAIR, 0)
+    assert gm.get_option(gm.OPT_TC_PAIR) == 0
+    gm.set_option(gm.OPT_TC_PAIR, 1)
+    for bad in (-1, 2):
+        with pytest.raises(gm.GemmiError):
+            gm.set_option(gm.OPT_TC_PAIR, bad)
+
+
 def test_header_constants_match_binding():
     text = open(HEADER).read()
     consts = dict((name, int(v)) for name, v in re.findall(r"GEMMI_((?:OPT|KERNEL)_[A-Z0-9_]+)\s*=\s*(\d+)", text))
