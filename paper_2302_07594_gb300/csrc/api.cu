@@ -275,7 +275,7 @@ int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A,
     pb = LimbPlanes{{ws + L.b0, ws + L.b1}, n, pitch};
     const LimbPlanes none{{nullptr, nullptr}, 0, pitch};
     cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
-    const cudaError_t e = gemmi::split_i16(nullptr, lda, B, ldb, m, n, k, none, pb, s);
+    const cudaError_t e = gemmi::split_i16(nullptr, lda, B, ldb, m, n, k, none, pb, s, d.status, timeout_ns());
     timer_end(GEMMI_KERNEL_SPLIT, t0, s);
     if (e != cudaSuccess) return cuda_error(e, "limb split launch");
   } else {
@@ -330,9 +330,11 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   cudaError_t e;
   cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
   if (nl == 2) {
-    e = gemmi::split_i16(static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb, m, n, k, pa, pb, s);
+    e = gemmi::split_i16(static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb, m, n, k, pa, pb, s,
+                         d.status, timeout_ns());
   } else {
-    e = gemmi::convert_i8(static_cast<const int8_t*>(A), lda, static_cast<const int8_t*>(B), ldb, m, n, k, pa, pb, s);
+    e = gemmi::convert_i8(static_cast<const int8_t*>(A), lda, static_cast<const int8_t*>(B), ldb, m, n, k, pa, pb, s,
+                          d.status, timeout_ns());
   }
   timer_end(GEMMI_KERNEL_SPLIT, t0, s);
   if (e != cudaSuccess) return cuda_error(e, "limb split launch");

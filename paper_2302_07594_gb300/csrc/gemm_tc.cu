@@ -481,7 +481,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
 
 }  // namespace
 
-bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, uint64_t inner, uint64_t outer,
+bool encode_tensor_map_2d(void* map, int dtype, const void* base, uint64_t inner, uint64_t outer,
                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes,
                           const char** why) {
   std::call_once(g_encode_once, [] {
@@ -496,8 +496,9 @@ bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, ui
     *why = "cuTensorMapEncodeTiled is not available from the driver";
     return false;
   }
-  const CUtensorMapDataType dt =
-      dtype_fp16_or_i16 == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
+  const CUtensorMapDataType dt = dtype == 1   ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                 : dtype == 2 ? CU_TENSOR_MAP_DATA_TYPE_UINT8
+                                              : CU_TENSOR_MAP_DATA_TYPE_UINT16;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};

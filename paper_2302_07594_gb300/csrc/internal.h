@@ -20,10 +20,15 @@ struct LimbPlanes {
 // int8: one plane holding the value itself.
 // One launch converts both operands: A (m x k, lda) -> pa (rows m), B (k x n, ldb) -> pb (rows n).
 // A null A (or B) skips that operand.
+// Operands whose base is 16-byte aligned with a row stride that is a multiple of 16 bytes are
+// streamed through shared memory by TMA (every wait bounded by timeout_ns; a timeout is recorded
+// in *status when status is not null); others take a plain-load kernel.
 cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
-                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s);
+                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status = nullptr,
+                      uint64_t timeout_ns = 4000000000ull);
 cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
-                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s);
+                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status = nullptr,
+                       uint64_t timeout_ns = 4000000000ull);
 
 // ---- gemm_tc.cu: tcgen05 GEMM on limb planes, C (int64 for NL=2, int32 for NL=1) += combine(limb products).
 struct TcGemmArgs {
@@ -101,8 +106,9 @@ cudaError_t im2col_i16(const int16_t* X, int16_t* Aout, int64_t lda, int64_t N, 
 // ---- selftest of the bounded wait.
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
 
-// Tensor-map encoder from the driver (resolved once through the runtime).
-bool encode_tensor_map_2d(void* map, int dtype_fp16_or_i16, const void* base, uint64_t inner, uint64_t outer,
+// Tensor-map encoder from the driver (resolved once through the runtime).  dtype: 0 = 16-bit
+// integer, 1 = fp16, 2 = 8-bit integer.  row_bytes is the byte stride between rows (outer index).
+bool encode_tensor_map_2d(void* map, int dtype, const void* base, uint64_t inner, uint64_t outer,
                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes,
                           const char** why);
 

@@ -14,13 +14,17 @@
 // rows have a pitch that is a multiple of 8 elements (16 bytes), which the TMA
 // tensor maps require.  Pitch columns at and beyond k are written as zero.
 //
-// One launch converts both operands (or just one: a null operand is skipped): the first blocks of the grid stream A
-// (16-byte loads, 2 x 16-byte stores per 8 elements), the rest transpose B in
-// 64 x 64 tiles through shared memory (16-byte loads and stores on both sides).
-// The kernel is bound by HBM: per int16 element 2 bytes are read and 4 written.
+// One launch converts both operands (or just one: a null operand is skipped): the first blocks
+// of the grid stream A, one warp per row (16-byte loads, 16-byte stores per plane and 8
+// elements), the rest transpose B in 64 x 64 tiles through shared memory (16-byte accesses on
+// both sides, swizzled so neither side has bank conflicts).  The kernel is bound by HBM: per
+// int16 element 2 bytes are read and 4 written; per int8 element 1 and 2.
+#include <cuda.h>
 #include <cuda_fp16.h>
 
 #include "internal.h"
+#include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace gemmi {
 namespace {
@@ -86,37 +90,56 @@ __device__ __forceinline__ void store8(__half* p0, __half* p1, const int (&v)[8]
   if constexpr (NL == 2) *reinterpret_cast<uint4*>(p1) = *reinterpret_cast<const uint4*>(l);
 }
 
-constexpr int TT = 64;      // transpose tile edge
+constexpr int TT = 64;      // transpose tile edge: 64 reduction indices x 64 columns of B
 constexpr int THREADS = 256;
+constexpr int WARPS = THREADS / 32;
 
+// A: m x k (lda) -> planes m x pitch.  One warp per row at a time; each lane converts U groups of
+// 8 elements per step, all loads issued before the stores (U * 16 bytes of int16 in flight).
 template <typename T, int NL>
-__global__ void __launch_bounds__(THREADS)
-split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_tiles) {
-  __shared__ int16_t tile[TT][TT + 8];
-  if (static_cast<int>(blockIdx.x) < a_blocks) {
-    // ---- A: m x k (lda) -> planes m x pitch, 8 consecutive elements per thread
-    const int64_t groups_per_row = a.pitch / 8;
-    const int64_t total = a.rows * groups_per_row;
-    for (int64_t g = blockIdx.x * static_cast<int64_t>(THREADS) + threadIdx.x; g < total;
-         g += static_cast<int64_t>(a_blocks) * THREADS) {
-      const int64_t r = g / groups_per_row;
-      const int64_t p0 = (g - r * groups_per_row) * 8;
-      int v[8];
-      load8(a.src + r * a.ld + p0, a.vec, a.cols - p0, v);
-      store8<NL>(a.p0 + r * a.pitch + p0, a.p1 + r * a.pitch + p0, v);
+__device__ __forceinline__ void split_rows(const Part<T>& a, int a_blocks) {
+  constexpr int U = sizeof(T) == 2 ? 2 : 4;
+  const int lane = threadIdx.x % 32;
+  const int64_t groups = a.pitch / 8;
+  const int64_t nwarps = static_cast<int64_t>(a_blocks) * WARPS;
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * WARPS + threadIdx.x / 32; r < a.rows; r += nwarps) {
+    const T* src = a.src + r * a.ld;
+    __half* d0 = a.p0 + r * a.pitch;
+    __half* d1 = a.p1 + r * a.pitch;
+    for (int64_t g0 = lane; g0 < groups; g0 += 32 * U) {
+      int v[U][8];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t p = (g0 + 32 * u) * 8;
+        if (p < a.pitch) load8(src + p, a.vec, a.cols - p, v[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t p = (g0 + 32 * u) * 8;
+        if (p < a.pitch) store8<NL>(d0 + p, d1 + p, v[u]);
+      }
     }
-    return;
   }
-  // ---- B: k x n (ldb) -> planes n x pitch (transposed), 64 x 64 tiles
+}
+
+// B: k x n (ldb) -> planes n x pitch (transposed), one 64 x 64 tile per step.  The tile passes
+// through shared memory already converted to fp16, stored untransposed (row = reduction index p,
+// 128 bytes = 64 columns j) with its 16-byte chunks XOR-swizzled by bits 3-5 of p.  Rows are
+// written a 16-byte chunk per thread; the transposed read gathers column j of 8 consecutive rows
+// p, and the swizzle puts the 8 row groups of one read in 8 different bank groups.
+template <typename T, int NL>
+__device__ __forceinline__ void split_cols(const Part<T>& b, int a_blocks, int64_t b_tiles_j, int64_t b_tiles,
+                                           __half (*sm)[TT * TT]) {
   const int64_t nblk = gridDim.x - a_blocks;
   for (int64_t t = blockIdx.x - a_blocks; t < b_tiles; t += nblk) {
     const int64_t p_base = (t / b_tiles_j) * TT;  // reduction index = row of B
     const int64_t j_base = (t % b_tiles_j) * TT;  // column of B
+    // load: 64 rows x 8 groups of 8 columns
 #pragma unroll
     for (int q = threadIdx.x; q < TT * TT / 8; q += THREADS) {
-      const int r = q >> 3;
-      const int c8 = (q & 7) * 8;
-      const int64_t p = p_base + r, j = j_base + c8;
+      const int r = q >> 3;       // p - p_base
+      const int c = q & 7;        // 16-byte chunk = columns 8c .. 8c+7
+      const int64_t p = p_base + r, j = j_base + 8 * c;
       int v[8];
       if (p < b.rows) {
         load8(b.src + p * b.ld + j, b.vec, b.cols - j, v);
@@ -124,20 +147,26 @@ split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_ti
 #pragma unroll
         for (int i = 0; i < 8; ++i) v[i] = 0;
       }
-#pragma unroll
-      for (int i = 0; i < 8; ++i) tile[r][c8 + i] = static_cast<int16_t>(v[i]);
+      const int off = r * TT + ((c ^ ((r >> 3) & 7)) * 8);
+      store8<NL>(&sm[0][off], &sm[NL - 1][off], v);
     }
     __syncthreads();
+    // store: 64 plane rows j x 8 chunks of 8 reduction indices; 8 lanes write one 128-byte row
 #pragma unroll
     for (int q = threadIdx.x; q < TT * TT / 8; q += THREADS) {
-      const int jj = q >> 3;
-      const int pc = (q & 7) * 8;
-      const int64_t j = j_base + jj, p = p_base + pc;
+      const int jj = q >> 3;      // j - j_base
+      const int g = q & 7;        // reduction indices p_base + 8g .. +7
+      const int64_t j = j_base + jj, p = p_base + 8 * g;
       if (j < b.cols && p < b.pitch) {
-        int v[8];
+        const int col = ((jj >> 3) ^ g) * 8 + (jj & 7);  // rows 8g..8g+7 all have swizzle g
 #pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = tile[pc + i][jj];
-        store8<NL>(b.p0 + j * b.pitch + p, b.p1 + j * b.pitch + p, v);
+        for (int l = 0; l < NL; ++l) {
+          __align__(16) __half h[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) h[i] = sm[l][(8 * g + i) * TT + col];
+          __half* dst = (l == 0 ? b.p0 : b.p1) + j * b.pitch + p;
+          *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(h);
+        }
       }
     }
     __syncthreads();
@@ -145,17 +174,306 @@ split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_ti
 }
 
 template <typename T, int NL>
-cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
-                   LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
+__global__ void __launch_bounds__(THREADS)
+split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_tiles) {
+  __shared__ __align__(16) __half sm[NL][TT * TT];
+  if (static_cast<int>(blockIdx.x) < a_blocks) split_rows<T, NL>(a, a_blocks);
+  else split_cols<T, NL>(b, a_blocks, b_tiles_j, b_tiles, sm);
+}
+
+// ---------------------------------------------------------------- TMA-fed variant
+// For operands whose rows TMA can address (16-byte aligned base and row stride), raw tiles of
+// 8 KB stream into a 4-stage shared-memory ring (one producer thread, mbarriers), so each SM
+// keeps about 100 KB of loads in flight; eight consumer warps convert them.
+//   A item: 32 rows x 256 bytes of raw A -> fp16 planes with coalesced 16-byte stores.
+//   B item: 64 reduction indices x 128 bytes of raw B (64 int16 or 128 int8 columns), loaded
+//           with the 128-byte swizzle, so the transposing gather of one column j from 8
+//           consecutive rows touches 8 different bank groups; the fp16 result goes to a staging
+//           tile in the same swizzled layout (row j = 64 reduction indices) and out by a TMA store.
+// Every wait is bounded; there is no hardware barrier after the start, so a timeout in one warp
+// can only make the others time out too.
+namespace tsplit {
+constexpr int CONSUMERS = 256;
+constexpr int THREADS = CONSUMERS + 32;
+constexpr int RAW = 8192;
+constexpr int STAGES = 4;
+constexpr int A_ROWS = 32;
+constexpr int B_P = 64;
+constexpr int STG = 16384;
+constexpr int NBAR = 2 * STAGES + 4;  // full, empty, staging full x2, staging free x2
+constexpr size_t SMEM = 1024 + STAGES * RAW + 2 * STG + 8 * NBAR;
+}  // namespace tsplit
+
+struct TmaSplitParams {
+  int64_t m, a_pitch;
+  __half* a_p0;
+  __half* a_p1;
+  int64_t a_tiles_k, a_items;
+  int64_t b_tiles_j, b_items;
+  uint32_t* status;
+  uint64_t timeout_ns;
+};
+
+__device__ __forceinline__ void tma_store_2d(const void* map, uint32_t src, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+
+template <typename T, int NL>
+__global__ void __launch_bounds__(tsplit::THREADS)
+split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant__ CUtensorMap rawB,
+                 const __grid_constant__ CUtensorMap outB0, const __grid_constant__ CUtensorMap outB1,
+                 TmaSplitParams P) {
+  using namespace tsplit;
+  constexpr int A_COLS = 256 / static_cast<int>(sizeof(T));  // raw A tile: 128 int16 / 256 int8
+  constexpr int JB = 128 / static_cast<int>(sizeof(T));      // raw B tile columns: 64 int16 / 128 int8
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* stg = smem + STAGES * RAW;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(stg + 2 * STG);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t sfull0 = empty0 + 8 * STAGES;  // staging buffer b written by all consumers
+  const uint32_t sfree0 = sfull0 + 16;          // staging buffer b read by its TMA store
+  const int64_t items = P.a_items + P.b_items;
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, CONSUMERS / 32);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(sfull0 + 8 * b, CONSUMERS);
+      mbar_init(sfree0 + 8 * b, 1);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == CONSUMERS / 32) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      if (P.a_items) tma_prefetch_desc(&rawA);
+      if (P.b_items) tma_prefetch_desc(&rawB);
+      tc::RingPos st;
+      for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
+        if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
+          report_status(P.status, tc::STATUS_TIMEOUT, 31);
+          break;
+        }
+        const uint32_t fb = full0 + 8 * st.slot;
+        mbar_arrive_expect_tx(fb, RAW);
+        const uint32_t dst = smem_u32(smem + st.slot * RAW);
+        if (it < P.a_items) {
+          const int64_t rt = it / P.a_tiles_k, kt = it - (it / P.a_tiles_k) * P.a_tiles_k;
+          tma_load_2d(dst, &rawA, fb, static_cast<int32_t>(kt * A_COLS), static_cast<int32_t>(rt * A_ROWS));
+        } else {
+          const int64_t b = it - P.a_items;
+          const int64_t pt = b / P.b_tiles_j, jt = b - (b / P.b_tiles_j) * P.b_tiles_j;
+          tma_load_2d(dst, &rawB, fb, static_cast<int32_t>(jt * JB), static_cast<int32_t>(pt * B_P));
+        }
+        st.advance(STAGES);
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------------- consumers (warps 0-7)
+  const int tid = threadIdx.x;
+  tc::RingPos st;
+  int nb = 0;  // B items processed so far (staging buffer = nb & 1, its use = nb >> 1)
+  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
+    const bool got = bounded_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns);
+    if (!__all_sync(0xFFFFFFFFu, got)) {
+      if (lane == 0) report_status(P.status, tc::STATUS_TIMEOUT, 32);
+      break;
+    }
+    const uint8_t* rawt = smem + st.slot * RAW;
+    if (it < P.a_items) {
+      // ---- A: row = q / 16, 16-byte chunk c = q % 16 of the 256-byte raw row
+      const int64_t rt = it / P.a_tiles_k, kt = it - rt * P.a_tiles_k;
+      uint4 w[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) w[u] = *reinterpret_cast<const uint4*>(rawt + (tid + 256 * u) * 16);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int q = tid + 256 * u;
+        const int64_t row = rt * A_ROWS + (q >> 4);
+        if (row >= P.m) continue;
+        const uint32_t wv[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+        if constexpr (sizeof(T) == 2) {
+          const int64_t col = kt * A_COLS + (q & 15) * 8;
+          if (col >= P.a_pitch) continue;
+          int v[8];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            v[2 * i] = static_cast<int16_t>(wv[i] & 0xFFFFu);
+            v[2 * i + 1] = static_cast<int16_t>(wv[i] >> 16);
+          }
+          store8<NL>(P.a_p0 + row * P.a_pitch + col, P.a_p1 + row * P.a_pitch + col, v);
+        } else {
+          const int64_t col = kt * A_COLS + (q & 15) * 16;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            if (col + 8 * h >= P.a_pitch) continue;
+            int v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = static_cast<int8_t>((wv[2 * h + i / 4] >> (8 * (i % 4))) & 0xFFu);
+            store8<NL>(P.a_p0 + row * P.a_pitch + col + 8 * h, P.a_p1 + row * P.a_pitch + col + 8 * h, v);
+          }
+        }
+      }
+    } else {
+      // ---- B: gather column j of rows 8g .. 8g+7, convert, write 16 bytes per plane to staging
+      const int64_t b = it - P.a_items;
+      const int64_t pt = b / P.b_tiles_j, jt = b - pt * P.b_tiles_j;
+      const int buf = nb & 1;
+      const uint32_t use = static_cast<uint32_t>(nb >> 1);
+      if (use > 0) {
+        const bool freed = bounded_wait(sfree0 + 8 * buf, (use - 1) & 1u, P.timeout_ns);
+        if (!__all_sync(0xFFFFFFFFu, freed)) {
+          if (lane == 0) report_status(P.status, tc::STATUS_TIMEOUT, 33);
+          break;
+        }
+      }
+      uint8_t* sbuf = stg + buf * STG;
+      constexpr int PAIRS = JB * 8 / CONSUMERS;  // (column, 8-row group) pairs per thread
+      int vals[PAIRS][8];
+#pragma unroll
+      for (int u = 0; u < PAIRS; ++u) {
+        const int q = tid + CONSUMERS * u;
+        const int j = q % JB;
+        const int g = q / JB;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int p = 8 * g + i;
+          if constexpr (sizeof(T) == 2) {
+            const int off = p * 128 + ((((j >> 3) ^ (p & 7))) << 4) + ((j & 7) << 1);
+            vals[u][i] = *reinterpret_cast<const int16_t*>(rawt + off);
+          } else {
+            const int off = p * 128 + ((((j >> 4) ^ (p & 7))) << 4) + (j & 15);
+            vals[u][i] = *reinterpret_cast<const int8_t*>(rawt + off);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+#pragma unroll
+      for (int u = 0; u < PAIRS; ++u) {
+        const int q = tid + CONSUMERS * u;
+        const int j = q % JB;
+        const int g = q / JB;
+        const int off = j * 128 + ((g ^ (j & 7)) << 4);
+        store8<NL>(reinterpret_cast<__half*>(sbuf + off), reinterpret_cast<__half*>(sbuf + 8192 + off), vals[u]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(sfull0 + 8 * buf);
+      if (tid == 0) {
+        // all consumers have written the staging tile: store it, then release the other buffer
+        // once its store (issued for the previous B item) has finished reading
+        if (!bounded_wait(sfull0 + 8 * buf, use & 1u, P.timeout_ns)) {
+          report_status(P.status, tc::STATUS_TIMEOUT, 34);
+        } else {
+          const int32_t x = static_cast<int32_t>(pt * B_P), y = static_cast<int32_t>(jt * JB);
+          tma_store_2d(&outB0, smem_u32(sbuf), x, y);
+          if constexpr (NL == 2) tma_store_2d(&outB1, smem_u32(sbuf + 8192), x, y);
+          bulk_commit();
+          if (nb > 0) {
+            bulk_wait_read_1();
+            mbar_arrive(sfree0 + 8 * (buf ^ 1));
+          }
+        }
+      }
+      ++nb;
+    }
+    st.advance(STAGES);
+  }
+  if (tid == 0) bulk_wait_all();
+}
+
+template <typename T, int NL>
+bool launch_tma(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int64_t n, int64_t k, LimbPlanes pa,
+                LimbPlanes pb, cudaStream_t s, uint32_t* status, uint64_t timeout_ns, cudaError_t* err) {
   constexpr int64_t esz = sizeof(T);
+  constexpr int A_COLS = 256 / static_cast<int>(esz);
+  constexpr int JB = 128 / static_cast<int>(esz);
+  const int dt = esz == 2 ? 0 : 2;
+  auto aligned = [](const void* p, int64_t ld_bytes) {
+    return p == nullptr || (reinterpret_cast<uintptr_t>(p) % 16 == 0 && ld_bytes % 16 == 0);
+  };
+  if (!aligned(A, lda * esz) || !aligned(B, ldb * esz)) return false;
+  CUtensorMap maps[4] = {};
+  const char* why = nullptr;
+  TmaSplitParams P = {};
+  P.status = status;
+  P.timeout_ns = timeout_ns;
+  if (A != nullptr) {
+    if (!encode_tensor_map_2d(&maps[0], dt, A, static_cast<uint64_t>(k), static_cast<uint64_t>(m),
+                              static_cast<uint64_t>(lda * esz), A_COLS, tsplit::A_ROWS, 0, &why))
+      return false;
+    P.m = m;
+    P.a_pitch = pa.pitch;
+    P.a_p0 = static_cast<__half*>(pa.plane[0]);
+    P.a_p1 = static_cast<__half*>(pa.plane[NL - 1]);
+    P.a_tiles_k = (pa.pitch + A_COLS - 1) / A_COLS;
+    P.a_items = ((m + tsplit::A_ROWS - 1) / tsplit::A_ROWS) * P.a_tiles_k;
+  }
+  if (B != nullptr) {
+    if (!encode_tensor_map_2d(&maps[1], dt, B, static_cast<uint64_t>(n), static_cast<uint64_t>(k),
+                              static_cast<uint64_t>(ldb * esz), JB, tsplit::B_P, 128, &why))
+      return false;
+    for (int l = 0; l < NL; ++l)
+      if (!encode_tensor_map_2d(&maps[2 + l], 1, pb.plane[l], static_cast<uint64_t>(pb.pitch),
+                                static_cast<uint64_t>(n), static_cast<uint64_t>(pb.pitch * 2), 64, JB, 128, &why))
+        return false;
+    if (NL == 1) maps[3] = maps[2];
+    P.b_tiles_j = (n + JB - 1) / JB;
+    P.b_items = ((pb.pitch + tsplit::B_P - 1) / tsplit::B_P) * P.b_tiles_j;
+  }
+  const int64_t items = P.a_items + P.b_items;
+  if (items == 0) {
+    *err = cudaSuccess;
+    return true;
+  }
+  static bool attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64 || !attr_done[dev]) {
+    const cudaError_t e = cudaFuncSetAttribute(split_tma_kernel<T, NL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(tsplit::SMEM));
+    if (e != cudaSuccess) {
+      *err = e;
+      return true;
+    }
+    if (dev >= 0 && dev < 64) attr_done[dev] = true;
+  }
+  const int64_t grid = items < 152 * 3 ? items : 152 * 3;
+  split_tma_kernel<T, NL><<<static_cast<unsigned>(grid), tsplit::THREADS, tsplit::SMEM, s>>>(maps[0], maps[1], maps[2],
+                                                                                            maps[3], P);
+  *err = cudaGetLastError();
+  return true;
+}
+
+template <typename T, int NL>
+cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                   LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status, uint64_t timeout_ns) {
+  constexpr int64_t esz = sizeof(T);
+  cudaError_t err = cudaSuccess;
+  if (launch_tma<T, NL>(A, lda, B, ldb, m, n, k, pa, pb, s, status, timeout_ns, &err)) return err;
   Part<T> a{A, lda, m, k, static_cast<__half*>(pa.plane[0]), static_cast<__half*>(pa.plane[NL - 1]), pa.pitch,
             reinterpret_cast<uintptr_t>(A) % (8 * esz) == 0 && (lda * esz) % (8 * esz) == 0};
   Part<T> b{B, ldb, k, n, static_cast<__half*>(pb.plane[0]), static_cast<__half*>(pb.plane[NL - 1]), pb.pitch,
             reinterpret_cast<uintptr_t>(B) % (8 * esz) == 0 && (ldb * esz) % (8 * esz) == 0};
-  // A: about 8 elements per thread per grid-stride step; B: one 64 x 64 tile per block step.
+  // A: one warp per row per step; B: one 64 x 64 tile per block step.
   // A null operand is skipped (packing only the weights, or only the activations).
-  const int64_t a_work = A != nullptr ? m * (pa.pitch / 8) : 0;
-  int64_t a_blocks = (a_work + THREADS - 1) / THREADS;
+  const int64_t a_rows = A != nullptr ? m : 0;
+  int64_t a_blocks = (a_rows + WARPS - 1) / WARPS;
   if (a_blocks > 152 * 8) a_blocks = 152 * 8;
   const int64_t tiles_p = (pb.pitch + TT - 1) / TT;  // cover the zero padding up to the pitch too
   const int64_t tiles_j = B != nullptr ? (n + TT - 1) / TT : 0;
@@ -170,13 +488,13 @@ cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, 
 }  // namespace
 
 cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
-                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
-  return launch<int16_t, 2>(A, lda, B, ldb, m, n, k, pa, pb, s);
+                      LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status, uint64_t timeout_ns) {
+  return launch<int16_t, 2>(A, lda, B, ldb, m, n, k, pa, pb, s, status, timeout_ns);
 }
 
 cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
-                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s) {
-  return launch<int8_t, 1>(A, lda, B, ldb, m, n, k, pa, pb, s);
+                       LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status, uint64_t timeout_ns) {
+  return launch<int8_t, 1>(A, lda, B, ldb, m, n, k, pa, pb, s, status, timeout_ns);
 }
 
 }  // namespace gemmi
