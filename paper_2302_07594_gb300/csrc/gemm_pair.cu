@@ -106,13 +106,62 @@ __device__ __forceinline__ void load_pair(uint32_t dst, const CUtensorMap* map, 
   else tma_load_2d_pair_hint(dst, map, bar, x, y, policy);
 }
 
+// The work of one pair.  While a full wave of tiles remains, whole tiles round-robin
+// (t = pair, pair + npairs, ...), so the pairs running at one time share operand rows and
+// columns in L2.  The last, partial wave is split along K ("stream-K"): its K blocks are dealt
+// out evenly to up to npairs pairs, in shares of at least MIN_SHARE K blocks, and a share may
+// start or end inside a tile.  Every segment's sums reach C through the same reductions, so the
+// pieces of a tile need no further combining.  Every role replays the same schedule.
+constexpr int MIN_SHARE = 4;
+struct PairSched {
+  int64_t nkb, full_tiles, next_tile, u, uend;
+  int npairs;
+  __device__ __forceinline__ void init(int pair, int npairs_, int64_t tiles, int64_t nkb_) {
+    nkb = nkb_;
+    npairs = npairs_;
+    full_tiles = (tiles / npairs) * npairs;
+    next_tile = pair;
+    const int64_t tail_units = (tiles - full_tiles) * nkb;
+    const int64_t max_split = nkb / MIN_SHARE > 1 ? nkb / MIN_SHARE : 1;
+    const int64_t sharers = min(static_cast<int64_t>(npairs), (tiles - full_tiles) * max_split);
+    const int64_t base = full_tiles * nkb;
+    u = uend = base;
+    if (pair < sharers) {
+      u = base + tail_units * pair / sharers;
+      uend = base + tail_units * (pair + 1) / sharers;
+    }
+  }
+  // The next segment: a tile and its K blocks [kb0, kb1).  False when the pair's work is done.
+  __device__ __forceinline__ bool next(int& tile, int& kb0, int& kb1) {
+    if (next_tile < full_tiles) {
+      tile = static_cast<int>(next_tile);
+      kb0 = 0;
+      kb1 = static_cast<int>(nkb);
+      next_tile += npairs;
+      return true;
+    }
+    if (u < uend) {
+      const int64_t t = u / nkb;
+      const int64_t k0 = u - t * nkb;
+      const int64_t k1 = min(nkb, k0 + (uend - u));
+      tile = static_cast<int>(t);
+      kb0 = static_cast<int>(k0);
+      kb1 = static_cast<int>(k1);
+      u += k1 - k0;
+      return true;
+    }
+    return false;
+  }
+};
+
 // The epilogue of one CTA.  For int16 the weights of accumulator columns 0-127 and 128-255 depend
 // on the CTA's A limb: 2^16 | 2^8 in the even CTA, 2^8 | 1 in the odd one.  Both CTAs drain
 // with the odd CTA's weights (one code path, constant shifts) and the even CTA scales its tile's
 // sums by 2^8 when it adds them into C: shifting commutes with addition modulo 2^64.
 template <int NL, int CS>
 __device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uint32_t tmem_base, uint32_t sfull0,
-                                         uint32_t sempty_leader0, uint8_t* stg, int pair, int npairs, int nchunks) {
+                                         uint32_t sempty_leader0, uint8_t* stg, int pair, int npairs) {
+  constexpr int KPC = 8 * CS;
   const uint32_t tile_shift = (NL == 2 && rank == 0) ? 8u : 0u;
   using G = PairGeom<NL>;
   using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
@@ -126,13 +175,16 @@ __device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uin
   const int half = warp >> 2;  // output columns half*COLS .. +COLS-1 of the tile
   uint8_t* my_stg = stg + (warp * 32 + lane) * STG_LANE;
   const uint32_t my_stg_s = smem_u32(my_stg);
-  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
+  PairSched sched;
+  sched.init(pair, npairs, static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles, P.num_k_blocks);
   int chunk = 0;
   bool ok = true;
   UT acc[COLS];
-  for (int t = pair; t < total_tiles && ok; t += npairs) {
+  int t, kb0, kb1;
+  while (ok && sched.next(t, kb0, kb1)) {
     int mt, nt;
     tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
+    const int nchunks = (kb1 - kb0 + KPC - 1) / KPC;
     const int64_t row = static_cast<int64_t>(mt) * G::TM + rank * G::A_STEP + quad * 32 + lane;
     const int64_t col0 = static_cast<int64_t>(nt) * G::TN + half * COLS;
 #pragma unroll
@@ -272,9 +324,9 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 
   const int pair = static_cast<int>(cluster_id_x());
   const int npairs = static_cast<int>(cluster_count_x());
-  const int total_tiles = P.num_m_tiles * P.num_n_tiles;
-  const int nkb = P.num_k_blocks;
-  const int nchunks = (nkb + KPC - 1) / KPC;
+  const int64_t total_tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
+  PairSched sched;
+  sched.init(pair, npairs, total_tiles, P.num_k_blocks);
 
   if (warp == PRODUCER_WARP) {
     // ------------------------------------------------------------ TMA producer (both CTAs)
@@ -289,12 +341,13 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       tc::RingPos st;
       int64_t issued = 0;
       bool ok = true;
-      for (int t = pair; t < total_tiles && ok; t += npairs) {
+      int t, kb0, kb1;
+      while (ok && sched.next(t, kb0, kb1)) {
         int mt, nt;
         tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
         const int arow = mt * G::TM + static_cast<int>(rank) * G::A_STEP;
         const int brow = nt * G::TN + static_cast<int>(rank) * G::B_STEP;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
             report_status(P.status, tc::STATUS_TIMEOUT, 21);
             ok = false;
@@ -323,7 +376,9 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         tc::RingPos st;
         int chunk = 0;
         bool ok = true;
-        for (int t = pair; t < total_tiles && ok; t += npairs) {
+        int t, kb0, kb1;
+        while (ok && sched.next(t, kb0, kb1)) {
+          const int nchunks = (kb1 - kb0 + KPC - 1) / KPC;
           for (int ch = 0; ch < nchunks; ++ch, ++chunk) {
             const int slot = chunk & 1;
             const uint32_t use = static_cast<uint32_t>(chunk >> 1);
@@ -335,9 +390,9 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
             }
             tc_fence_after();
             const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS);
-            const int kb0 = ch * KPC;
-            const int kb1 = min(nkb, kb0 + KPC);
-            for (int kb = kb0; kb < kb1; ++kb) {
+            const int cb0 = kb0 + ch * KPC;
+            const int cb1 = min(kb1, cb0 + KPC);
+            for (int kb = cb0; kb < cb1; ++kb) {
               if (!bounded_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns)) {
                 report_status(P.status, tc::STATUS_TIMEOUT, 23);
                 ok = false;
@@ -350,7 +405,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 #pragma unroll
               for (int kk = 0; kk < BK / UMMA_K; ++kk) {
                 // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
-                tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb == kb0 && kk == 0) ? 0u : 1u);
+                tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb == cb0 && kk == 0) ? 0u : 1u);
               }
               tc_commit_pair(empty0 + 8 * st.slot, 0x3);  // stage free in both CTAs once read
               st.advance(STAGES);
@@ -367,7 +422,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const uint32_t sempty_leader0 = map_to_rank(sempty0, 0);
-    epilogue<NL, CS>(P, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs, nchunks);
+    epilogue<NL, CS>(P, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs);
   }
 
   // Pair handshake: neither CTA exits (or frees tensor memory) while its peer may still signal it.
@@ -444,7 +499,10 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
     }
     if (dev >= 0 && dev < 64) max_pairs[dev] = pairs_here;
   }
-  const int npairs = static_cast<int>(tiles < pairs_here ? tiles : pairs_here);
+  // enough pairs for every tile, or for every stream-K share when there are fewer tiles than pairs
+  const int64_t max_split = P.num_k_blocks / MIN_SHARE > 1 ? P.num_k_blocks / MIN_SHARE : 1;
+  const int64_t useful = tiles * max_split;
+  const int npairs = static_cast<int>(useful < pairs_here ? useful : pairs_here);
   cfg.gridDim = dim3(2 * static_cast<unsigned>(npairs), 1, 1);
   *why = "tcgen05 pair GEMM launch";
   return cudaLaunchKernelEx(&cfg, kernel, maps[0], maps[1], maps[2], maps[3], P);

@@ -210,3 +210,16 @@ def test_pair_back_to_back_calls_accumulate(gm):
     for _ in range(3):
         oracle.gemm(A, B, exp, nthreads=8)
     assert_same(dC.cpu().numpy(), exp, "three calls")
+
+
+# Stream-K tails: more tiles than pairs with a partial last wave (its K blocks are shared out, so
+# segments start and end inside tiles), and fewer tiles than pairs (every tile split along K)
+STREAM_K = [("i16", 1408, 896, 2048), ("i16", 600, 300, 4096), ("i16", 130, 130, 1100), ("i8", 2304, 2304, 1024),
+            ("i8", 300, 700, 3000)]
+
+
+@pytest.mark.parametrize("case", STREAM_K)
+def test_pair_stream_k_tails(gm, case, chunk_scale):
+    kind, m, n, k = case
+    A, B, C = gi.random_problem(5800 + m + n + k, m, n, k, kind)
+    assert_same(run(gm, A, B, C), expected(A, B, C), f"stream-K {case}, chunk scale {chunk_scale}")
