@@ -21,9 +21,12 @@
 // Per K block of 64 each SM loads 32 KB (its A tile and its B tile) for 512 tensor cycles: 64 B
 // per cycle from L2, where a single-SM 128 x 256 int8 tile needs 96.
 //
-// The running int64 (int32) sums of a tile are added into C with bulk asynchronous reductions
-// (cp.reduce.async.bulk .add) from a small per-thread staging area, so the two SMs of an int16
-// tile add their weighted halves into C independently and C is never read by the SMs.
+// The running int64 (int32) sums of a tile are added into C with 2-D tensor reductions
+// (cp.reduce.async.bulk.tensor .add, one 32-row x 128-byte box per warp and round, through an
+// unsigned tensor map so the adds wrap modulo 2^64 / 2^32), so the two SMs of an int16 tile add
+// their weighted halves into C independently, C is never read by the SMs, and TMA clips the
+// ragged edges.  Few large reductions matter: the cost of a bulk operation is mostly per
+// operation, and 128-byte ones made the tile ends several times slower.
 //
 // Structure (one CTA per SM, clusters of two, 320 threads per CTA):
 //   warp 8   TMA producer: both CTAs load their halves; every load completes on the full
@@ -62,15 +65,21 @@ constexpr int UMMA_N = 256;
 constexpr int HALF = 128;                     // rows of A, and of K-major B, per CTA and stage
 constexpr int TILE_A = HALF * BK * 2;         // 16 KB
 constexpr int TILE_B = HALF * BK * 2;         // 16 KB
-constexpr int SB = TILE_A + TILE_B;           // one CTA's part of a stage
-constexpr int STAGES = 5;
+constexpr int SBK = TILE_A + TILE_B;          // one CTA's tiles of one K block
+// Two K blocks per pipeline stage: the single MMA thread waits on a stage barrier and commits once
+// per eight MMAs instead of four.  That per-stage work does not overlap the tensor pipe (the
+// thread cannot run far ahead of the MMAs it issues), so halving it raises the pipe's busy time.
+constexpr int KPS = 2;
+constexpr int SB = KPS * SBK;                 // one CTA's part of a stage
+constexpr int STAGES = 3;
 constexpr int SWIZZLE = BK * 2;               // 128-byte rows
-constexpr int RED_BYTES = 128;                // bytes of one C row segment per bulk reduction
-constexpr int STG_LANE = RED_BYTES + 16;      // staging stride per thread (the 16 spread the banks)
-constexpr int STG_BYTES = NUM_EPI_WARPS * 32 * STG_LANE;
+constexpr int RED_BYTES = 128;                // bytes of C per row of one reduction box
+constexpr int STG_WARP = 32 * RED_BYTES;      // one warp's box: 32 rows x 128 bytes, 128-byte swizzle
+constexpr int STG_BYTES = NUM_EPI_WARPS * STG_WARP;
 constexpr int NBAR = 2 * STAGES + 2 * NSLOT + 2;  // full, empty, slot full, slot empty, final, bye
 constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * SB + STG_BYTES + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
+static_assert((8 % KPS) == 0, "exact chunks (multiples of 8 K blocks) must end on stage boundaries");
 static_assert(NSLOT * SLOT_COLS <= TMEM_COLS, "tensor memory budget");
 
 // Output tile of one pair and where each CTA's operand rows start inside it.
@@ -159,8 +168,9 @@ struct PairSched {
 // with the odd CTA's weights (one code path, constant shifts) and the even CTA scales its tile's
 // sums by 2^8 when it adds them into C: shifting commutes with addition modulo 2^64.
 template <int NL, int CS>
-__device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uint32_t tmem_base, uint32_t sfull0,
-                                         uint32_t sempty_leader0, uint8_t* stg, int pair, int npairs) {
+__device__ __forceinline__ void epilogue(const PairParams& P, const CUtensorMap* cmap, uint32_t rank,
+                                         uint32_t tmem_base, uint32_t sfull0, uint32_t sempty_leader0, uint8_t* stg,
+                                         int pair, int npairs) {
   constexpr int KPC = 8 * CS;
   const uint32_t tile_shift = (NL == 2 && rank == 0) ? 8u : 0u;
   using G = PairGeom<NL>;
@@ -173,8 +183,8 @@ __device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uin
   const int lane = threadIdx.x % 32;
   const int quad = warp & 3;   // TMEM lanes 32*quad .. +31 (the warp's hardware lane quadrant)
   const int half = warp >> 2;  // output columns half*COLS .. +COLS-1 of the tile
-  uint8_t* my_stg = stg + (warp * 32 + lane) * STG_LANE;
-  const uint32_t my_stg_s = smem_u32(my_stg);
+  uint8_t* wstg = stg + warp * STG_WARP;
+  const uint32_t wstg_s = smem_u32(wstg);
   PairSched sched;
   sched.init(pair, npairs, static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles, P.num_k_blocks);
   int chunk = 0;
@@ -185,7 +195,7 @@ __device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uin
     int mt, nt;
     tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
     const int nchunks = (kb1 - kb0 + KPC - 1) / KPC;
-    const int64_t row = static_cast<int64_t>(mt) * G::TM + rank * G::A_STEP + quad * 32 + lane;
+    const int64_t row0 = static_cast<int64_t>(mt) * G::TM + rank * G::A_STEP + quad * 32;  // the warp's rows
     const int64_t col0 = static_cast<int64_t>(nt) * G::TN + half * COLS;
 #pragma unroll
     for (int c = 0; c < COLS; ++c) acc[c] = 0;
@@ -235,51 +245,44 @@ __device__ __forceinline__ void epilogue(const PairParams& P, uint32_t rank, uin
       if (lane == 0) mbar_arrive_cluster(sempty_leader0 + 8 * slot);
     }
     if (!ok) break;
-    // add the tile's running sums into C, one 128-byte row segment per bulk reduction
-    if (row < P.m) {
-      CT* crow = static_cast<CT*>(P.C) + row * P.ldc + col0;
+    // add the segment's running sums into C: per round, one 32-row x 128-byte box per warp,
+    // written to the staging area in the box's 128-byte-swizzled layout (row r, 16-byte chunk c
+    // at r * 128 + (c ^ (r % 8)) * 16: the eight chunk stores of a warp hit distinct banks)
+    if (row0 < P.m) {
 #pragma unroll
       for (int j = 0; j < ROUNDS; ++j) {
-        const int64_t valid = P.n - (col0 + j * EPR);
-        if (valid <= 0) break;
-        bulk_wait_read_all();  // the previous reduction has finished reading the staging area
+        const int64_t x = col0 + j * EPR;
+        if (x >= P.n) break;
+        if (lane == 0) bulk_wait_read_all();  // the previous box has left the staging area
+        __syncwarp();
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
+          uint8_t* dst = wstg + lane * RED_BYTES + ((q ^ (lane & 7)) << 4);
           if constexpr (NL == 2) {
-            *reinterpret_cast<ulonglong2*>(my_stg + 16 * q) =
+            *reinterpret_cast<ulonglong2*>(dst) =
                 make_ulonglong2(acc[j * EPR + 2 * q] << tile_shift, acc[j * EPR + 2 * q + 1] << tile_shift);
           } else {
-            *reinterpret_cast<uint4*>(my_stg + 16 * q) = make_uint4(acc[j * EPR + 4 * q], acc[j * EPR + 4 * q + 1],
-                                                                    acc[j * EPR + 4 * q + 2], acc[j * EPR + 4 * q + 3]);
+            *reinterpret_cast<uint4*>(dst) = make_uint4(acc[j * EPR + 4 * q], acc[j * EPR + 4 * q + 1],
+                                                        acc[j * EPR + 4 * q + 2], acc[j * EPR + 4 * q + 3]);
           }
         }
         fence_proxy_async_smem();
-        CT* dst = crow + j * EPR;
-        const int v = valid >= EPR ? EPR : static_cast<int>(valid);
-        const int bulk_elems = (v * static_cast<int>(sizeof(CT))) / 16 * 16 / static_cast<int>(sizeof(CT));
-        if (bulk_elems > 0) {
-          if constexpr (NL == 2) bulk_reduce_add_u64(dst, my_stg_s, static_cast<uint32_t>(bulk_elems * 8));
-          else bulk_reduce_add_u32(dst, my_stg_s, static_cast<uint32_t>(bulk_elems * 4));
+        __syncwarp();
+        if (lane == 0) {
+          tma_reduce_add_2d(cmap, wstg_s, static_cast<int32_t>(x), static_cast<int32_t>(row0));
           bulk_commit();
-        }
-        // a ragged right edge: the last few elements one by one (read back from the staging area)
-        for (int i = bulk_elems; i < v; ++i) {
-          if constexpr (NL == 2)
-            atomicAdd(reinterpret_cast<unsigned long long*>(dst + i),
-                      static_cast<unsigned long long>(reinterpret_cast<const UT*>(my_stg)[i]));
-          else
-            atomicAdd(reinterpret_cast<unsigned int*>(dst + i), reinterpret_cast<const UT*>(my_stg)[i]);
         }
       }
     }
   }
-  bulk_wait_all();
+  if (lane == 0) bulk_wait_all();
 }
 
 template <int NL, int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
-               const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1, PairParams P) {
+               const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1,
+               const __grid_constant__ CUtensorMap mapC, PairParams P) {
   using G = PairGeom<NL>;
   constexpr int KPC = 8 * CS;  // K blocks per exact chunk: 512 * CS reduction indices
 
@@ -347,17 +350,23 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         tc::tile_coords(t, P.num_m_tiles, P.num_n_tiles, P.group_m, mt, nt);
         const int arow = mt * G::TM + static_cast<int>(rank) * G::A_STEP;
         const int brow = nt * G::TN + static_cast<int>(rank) * G::B_STEP;
-        for (int kb = kb0; kb < kb1; ++kb) {
+        // stages hold KPS consecutive K blocks of a segment (its last stage possibly fewer)
+        for (int kb = kb0; kb < kb1; kb += KPS) {
+          const int nsub = min(KPS, kb1 - kb);
           if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
             report_status(P.status, tc::STATUS_TIMEOUT, 21);
             ok = false;
             break;
           }
-          if (leader) mbar_arrive_expect_tx(full0 + 8 * st.slot, 2 * SB);
+          if (leader) mbar_arrive_expect_tx(full0 + 8 * st.slot, 2 * nsub * SBK);
           const uint32_t fb = full_leader0 + 8 * st.slot;
-          const uint32_t base = smem_u32(smem + st.slot * SB);
-          load_pair(base, ma, fb, kb * BK, arow, P.hint_a, pol_a);
-          load_pair(base + TILE_A, mb, fb, kb * BK, brow, P.hint_b, pol_b);
+#pragma unroll
+          for (int j = 0; j < KPS; ++j) {
+            if (j >= nsub) break;
+            const uint32_t base = smem_u32(smem + st.slot * SB + j * SBK);
+            load_pair(base, ma, fb, (kb + j) * BK, arow, P.hint_a, pol_a);
+            load_pair(base + TILE_A, mb, fb, (kb + j) * BK, brow, P.hint_b, pol_b);
+          }
           ++issued;
           st.advance(STAGES);
         }
@@ -392,20 +401,26 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
             const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS);
             const int cb0 = kb0 + ch * KPC;
             const int cb1 = min(kb1, cb0 + KPC);
-            for (int kb = cb0; kb < cb1; ++kb) {
+            // chunk lengths are multiples of KPS, so chunks and stages share boundaries
+            for (int kb = cb0; kb < cb1; kb += KPS) {
+              const int nsub = min(KPS, cb1 - kb);
               if (!bounded_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns)) {
                 report_status(P.status, tc::STATUS_TIMEOUT, 23);
                 ok = false;
                 break;
               }
               tc_fence_after();
-              const uint32_t base = smem_u32(smem + st.slot * SB);
-              const uint64_t adesc = smem_desc_kmajor<SWIZZLE>(base);
-              const uint64_t bdesc = smem_desc_kmajor<SWIZZLE>(base + TILE_A);
 #pragma unroll
-              for (int kk = 0; kk < BK / UMMA_K; ++kk) {
-                // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
-                tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb == cb0 && kk == 0) ? 0u : 1u);
+              for (int j = 0; j < KPS; ++j) {
+                if (j >= nsub) break;
+                const uint32_t base = smem_u32(smem + st.slot * SB + j * SBK);
+                const uint64_t adesc = smem_desc_kmajor<SWIZZLE>(base);
+                const uint64_t bdesc = smem_desc_kmajor<SWIZZLE>(base + TILE_A);
+#pragma unroll
+                for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+                  // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
+                  tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb + j == cb0 && kk == 0) ? 0u : 1u);
+                }
               }
               tc_commit_pair(empty0 + 8 * st.slot, 0x3);  // stage free in both CTAs once read
               st.advance(STAGES);
@@ -422,7 +437,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const uint32_t sempty_leader0 = map_to_rank(sempty0, 0);
-    epilogue<NL, CS>(P, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs);
+    epilogue<NL, CS>(P, &mapC, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs);
   }
 
   // Pair handshake: neither CTA exits (or frees tensor memory) while its peer may still signal it.
@@ -454,6 +469,12 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
         return cudaErrorInvalidValue;
     }
   }
+  // C as the target of the tile reductions: an unsigned integer tensor of its element width
+  CUtensorMap mapC;
+  constexpr int ESZ = NL == 2 ? 8 : 4;
+  if (!encode_tensor_map_2d(&mapC, NL == 2 ? 3 : 4, a.C, static_cast<uint64_t>(a.n), static_cast<uint64_t>(a.m),
+                            static_cast<uint64_t>(a.ldc) * ESZ, RED_BYTES / ESZ, 32, 128, why))
+    return cudaErrorInvalidValue;
   PairParams P;
   P.m = a.m;
   P.n = a.n;
@@ -505,7 +526,7 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   const int npairs = static_cast<int>(useful < pairs_here ? useful : pairs_here);
   cfg.gridDim = dim3(2 * static_cast<unsigned>(npairs), 1, 1);
   *why = "tcgen05 pair GEMM launch";
-  return cudaLaunchKernelEx(&cfg, kernel, maps[0], maps[1], maps[2], maps[3], P);
+  return cudaLaunchKernelEx(&cfg, kernel, maps[0], maps[1], maps[2], maps[3], mapC, P);
 }
 
 }  // namespace

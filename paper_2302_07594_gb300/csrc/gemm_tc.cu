@@ -498,6 +498,8 @@ bool encode_tensor_map_2d(void* map, int dtype, const void* base, uint64_t inner
   }
   const CUtensorMapDataType dt = dtype == 1   ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
                                  : dtype == 2 ? CU_TENSOR_MAP_DATA_TYPE_UINT8
+                                 : dtype == 3 ? CU_TENSOR_MAP_DATA_TYPE_UINT64
+                                 : dtype == 4 ? CU_TENSOR_MAP_DATA_TYPE_UINT32
                                               : CU_TENSOR_MAP_DATA_TYPE_UINT16;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};

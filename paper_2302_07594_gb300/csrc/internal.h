@@ -107,7 +107,8 @@ cudaError_t im2col_i16(const int16_t* X, int16_t* Aout, int64_t lda, int64_t N, 
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
 
 // Tensor-map encoder from the driver (resolved once through the runtime).  dtype: 0 = 16-bit
-// integer, 1 = fp16, 2 = 8-bit integer.  row_bytes is the byte stride between rows (outer index).
+// integer, 1 = fp16, 2 = 8-bit integer, 3 = 64-bit integer, 4 = 32-bit integer (unsigned types:
+// reductions through them add modulo 2^64 / 2^32).  row_bytes is the byte stride between rows.
 bool encode_tensor_map_2d(void* map, int dtype, const void* base, uint64_t inner, uint64_t outer,
                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes,
                           const char** why);

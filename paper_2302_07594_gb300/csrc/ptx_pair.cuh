@@ -130,10 +130,14 @@ __device__ __forceinline__ void tc_ld_32x32b_x8(uint32_t taddr, uint32_t (&r)[8]
                : "r"(taddr));
 }
 
-// Bulk (non-tensor) reduction into global memory of unsigned 32-bit elements (see bulk_reduce_add_u64).
-__device__ __forceinline__ void bulk_reduce_add_u32(void* dst, uint32_t src, uint32_t bytes) {
-  asm volatile("cp.reduce.async.bulk.global.shared::cta.bulk_group.add.u32 [%0], [%1], %2;" ::"l"(dst), "r"(src),
-               "r"(bytes)
+// 2-D tiled bulk-tensor reduction: global[box at (x, y)] += shared[src], element type and
+// wrap-around from the tensor map (an unsigned integer type adds modulo 2^bits), elements outside
+// the tensor skipped.  x * element size a multiple of 16 bytes, x and y not negative; completion
+// tracked by this thread's bulk async-groups.
+__device__ __forceinline__ void tma_reduce_add_2d(const void* map, uint32_t src, int32_t x, int32_t y) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
                : "memory");
 }
 
