@@ -51,6 +51,9 @@ struct DeviceState {
   size_t conv_buf_bytes = 0;
   cudaEvent_t last_use = nullptr;
   cudaStream_t last_stream = nullptr;
+  cudaStream_t h2d = nullptr;          // copy streams of the pipelined host-buffer path
+  cudaStream_t d2h = nullptr;
+  cudaEvent_t pipe_ev[12] = {};
   bool used = false;
   uint32_t last_detail = 0;
 };
@@ -537,6 +540,110 @@ int read_status_locked(DeviceState& d, bool clear) {
   return set_error(code, buf);
 }
 
+int ensure_pipeline(DeviceState& d) {
+  if (d.h2d != nullptr) return GEMMI_OK;
+  cudaError_t e = cudaStreamCreateWithFlags(&d.h2d, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&d.d2h, cudaStreamNonBlocking);
+  for (auto& ev : d.pipe_ev)
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+  return e == cudaSuccess ? GEMMI_OK : cuda_error(e, "creating the copy streams of the host-buffer path");
+}
+
+constexpr int kPipeSlots = 3;
+constexpr int64_t kPanelMin = 512;
+
+// Host-buffer GEMM of m >= 2 * kPanelMin rows as a pipeline over row panels of A and C.  B is
+// copied and split into limb planes once; then each panel's copy in (A and C rows), GEMM and
+// copy out run on three streams (copy in, the caller's stream, copy out) through a ring of
+// kPipeSlots device slots, so the host-link copies in both directions overlap each other and the
+// tensor cores.  The link, not the GPU, bounds this path: about 0.2 TB/s each way.
+template <typename OP, typename CT>
+int host_gemm_pipelined(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda,
+                        const OP* B, int64_t ldb, CT* C, int64_t ldc) {
+  int rc = ensure_pipeline(d);
+  if (rc != GEMMI_OK) return rc;
+  cudaStream_t s = g_stream;
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 7) / 8), 128)));
+  const int64_t panels = (m + mb - 1) / mb;
+  const size_t b_raw = round_up(static_cast<size_t>(k) * n * sizeof(OP), kAlign);
+  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
+  const size_t a_slot = round_up(static_cast<size_t>(mb) * k * sizeof(OP), kAlign);
+  const size_t c_slot = round_up(static_cast<size_t>(mb) * n * sizeof(CT), kAlign);
+  if ((rc = ensure_buffer(&d.host_buf, &d.host_buf_bytes, b_raw + nl * b_plane + kPipeSlots * (a_slot + c_slot))) !=
+      GEMMI_OK)
+    return rc;
+  // the A planes of one panel, sized now so no panel has to grow the workspace mid-pipeline
+  if ((rc = ensure_buffer(&d.ws, &d.ws_bytes, plane_layout(mb, 0, pitch, nl).total)) != GEMMI_OK) return rc;
+  char* base = static_cast<char*>(d.host_buf);
+  OP* dB = reinterpret_cast<OP*>(base);
+  LimbPlanes pb{{base + b_raw, base + b_raw + (nl == 2 ? b_plane : 0)}, n, pitch};
+  char* slots = base + b_raw + nl * b_plane;
+  cudaEvent_t* ev = d.pipe_ev;  // 0 start, 1 B copied, 2-4 panel in, 5-7 panel done, 8-10 panel out, 11 end
+  // on an error, let the copies already queued finish before the buffers can be reused
+  auto settle = [&]() {
+    cudaStreamSynchronize(d.h2d);
+    cudaStreamSynchronize(s);
+    cudaStreamSynchronize(d.d2h);
+  };
+  auto fail = [&](cudaError_t e, const char* what) {
+    settle();
+    return cuda_error(e, what);
+  };
+  cudaError_t e = cudaEventRecord(ev[0], s);  // after earlier work of the caller's stream
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(d.h2d, ev[0], 0);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(d.d2h, ev[0], 0);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2DAsync(dB, n * sizeof(OP), B, ldb * sizeof(OP), n * sizeof(OP), k, cudaMemcpyHostToDevice, d.h2d);
+  if (e == cudaSuccess) e = cudaEventRecord(ev[1], d.h2d);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[1], 0);
+  if (e != cudaSuccess) return fail(e, "host-to-device copy of B");
+  {
+    const LimbPlanes none{{nullptr, nullptr}, 0, pitch};
+    cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+    e = nl == 2 ? gemmi::split_i16(nullptr, k, reinterpret_cast<const int16_t*>(dB), n, 0, n, k, none, pb, s, d.status,
+                                   timeout_ns())
+                : gemmi::convert_i8(nullptr, k, reinterpret_cast<const int8_t*>(dB), n, 0, n, k, none, pb, s, d.status,
+                                    timeout_ns());
+    timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+    if (e != cudaSuccess) return fail(e, "split of B");
+  }
+  for (int64_t p = 0; p < panels; ++p) {
+    const int r = static_cast<int>(p % kPipeSlots);
+    const int64_t r0 = p * mb, mi = std::min(mb, m - r0);
+    OP* dA = reinterpret_cast<OP*>(slots + r * (a_slot + c_slot));
+    CT* dC = reinterpret_cast<CT*>(slots + r * (a_slot + c_slot) + a_slot);
+    e = p >= kPipeSlots ? cudaStreamWaitEvent(d.h2d, ev[8 + r], 0) : cudaSuccess;  // slot's last copy out
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(dA, k * sizeof(OP), A + r0 * lda, lda * sizeof(OP), k * sizeof(OP), mi,
+                            cudaMemcpyHostToDevice, d.h2d);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(dC, n * sizeof(CT), C + r0 * ldc, ldc * sizeof(CT), n * sizeof(CT), mi,
+                            cudaMemcpyHostToDevice, d.h2d);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[2 + r], d.h2d);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[2 + r], 0);
+    if (e != cudaSuccess) return fail(e, "host-to-device copy of a panel");
+    rc = run_tc(d, nl, mi, n, k, dA, k, nullptr, n, dC, n, s, &pb);
+    if (rc != GEMMI_OK) {
+      settle();
+      return rc;
+    }
+    e = cudaEventRecord(ev[5 + r], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(d.d2h, ev[5 + r], 0);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(C + r0 * ldc, ldc * sizeof(CT), dC, n * sizeof(CT), n * sizeof(CT), mi,
+                            cudaMemcpyDeviceToHost, d.d2h);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[8 + r], d.d2h);
+    if (e != cudaSuccess) return fail(e, "device-to-host copy of a panel");
+  }
+  // the caller's stream continues after the last copy out
+  e = cudaEventRecord(ev[11], d.d2h);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[11], 0);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return fail(e, "cudaStreamSynchronize");
+  return GEMMI_OK;
+}
+
 template <typename OP, typename CT, typename F>
 int host_gemm(int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda, const OP* B, int64_t ldb, CT* C,
               int64_t ldc, F device_call) {
@@ -546,6 +653,16 @@ int host_gemm(int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda, const O
   DeviceState* d = nullptr;
   int rc = device_state(&d);
   if (rc != GEMMI_OK) return rc;
+  constexpr int nl = sizeof(OP) == 2 ? 2 : 1;
+  if (m >= 2 * kPanelMin && m > (nl == 2 ? g_skinny_max_m : 0)) {
+    rc = host_gemm_pipelined(*d, nl, m, n, k, A, lda, B, ldb, C, ldc);
+    if (rc != GEMMI_OK) return rc;
+    uint32_t word = 0;
+    const cudaError_t e = cudaMemcpy(&word, d->status, sizeof(word), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
+    if (word != 0) return read_status_locked(*d, true);
+    return GEMMI_OK;
+  }
   const size_t a_bytes = round_up(static_cast<size_t>(m) * k * sizeof(OP), kAlign);
   const size_t b_bytes = round_up(static_cast<size_t>(k) * n * sizeof(OP), kAlign);
   const size_t c_bytes = round_up(static_cast<size_t>(m) * n * sizeof(CT), kAlign);

@@ -282,6 +282,28 @@ def test_host_api_padded(gm):
     assert (big[:, n:] == 7).all()
 
 
+# m >= 1024: the host path pipelines row panels of A and C (a ring of three device slots, so
+# panels reuse slots) with B copied and split once; the last panel is ragged here
+@pytest.mark.parametrize("kind,m,n,k", [("i16", 2000, 300, 500), ("i8", 2000, 300, 500), ("i16", 1024, 64, 200),
+                                        ("i16", 5000, 130, 96)])
+def test_host_api_pipelined_panels(gm, kind, m, n, k):
+    A, B, C = gi.random_problem(905 + m + n, m, n, k, kind)
+    # host operands with padded rows: the panel copies must honour the leading dimensions
+    Ap = np.full((m, k + 5), 3, A.dtype)
+    Ap[:, :k] = A
+    Bp = np.full((k, n + 2), -3, B.dtype)
+    Bp[:, :n] = B
+    Cp = np.full((m, n + 1), 11, C.dtype)
+    Cp[:, :n] = C
+    (gm.gemm_i16_host if kind == "i16" else gm.gemm_i8_host)(Ap[:, :k], Bp[:, :n], Cp[:, :n])
+    assert_same(Cp[:, :n], expected(A, B, C), f"host pipelined {kind} {m}x{n}x{k}")
+    assert (Cp[:, n:] == 11).all()
+    # a second call accumulates on top of the first (the slots and the split B are reused)
+    (gm.gemm_i16_host if kind == "i16" else gm.gemm_i8_host)(Ap[:, :k], Bp[:, :n], Cp[:, :n])
+    exp2 = expected(A, B, expected(A, B, C))
+    assert_same(Cp[:, :n], exp2, "second pipelined call")
+
+
 def test_non_default_stream(gm):
     A, B, C = gi.random_problem(903, 300, 260, 500, "i16")
     s = torch.cuda.Stream()
