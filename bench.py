@@ -37,7 +37,7 @@ L2_BYTES = 129 * 2 ** 20
 PROFILES = os.path.join(ROOT, "profiles")
 # per kernel of the library: its CUDA symbol, the sources it is built from, and its bound
 KERNEL_INFO = {
-    "split": ("split_kernel", ("split.cu",), "hbm"),
+    "split": ("split_tma_kernel", ("split.cu", "ptx.cuh", "tc_common.cuh"), "hbm"),
     "tc_i16": ("tc_gemm_kernel<2>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
     "tc_i8": ("tc_gemm_kernel<1>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
     "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh"), "hbm"),
