@@ -324,6 +324,11 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // Launched with programmatic stream serialization: the setup above may overlap the end of the
+  // previous kernel (the operand split); every global access comes after this wait.  The next
+  // kernel may be scheduled as this grid's CTAs retire.
+  pdl_wait();
+  pdl_launch_dependents();
 
   const int pair = static_cast<int>(cluster_id_x());
   const int npairs = static_cast<int>(cluster_count_x());
@@ -353,7 +358,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         // stages hold KPS consecutive K blocks of a segment (its last stage possibly fewer)
         for (int kb = kb0; kb < kb1; kb += KPS) {
           const int nsub = min(KPS, kb1 - kb);
-          if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
+          if (!spin_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
             report_status(P.status, tc::STATUS_TIMEOUT, 21);
             ok = false;
             break;
@@ -404,7 +409,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
             // chunk lengths are multiples of KPS, so chunks and stages share boundaries
             for (int kb = cb0; kb < cb1; kb += KPS) {
               const int nsub = min(KPS, cb1 - kb);
-              if (!bounded_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns)) {
+              if (!spin_wait(full0 + 8 * st.slot, st.phase, P.timeout_ns)) {
                 report_status(P.status, tc::STATUS_TIMEOUT, 23);
                 ok = false;
                 break;
@@ -493,16 +498,18 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
 
   auto kernel = tc_pair_kernel<NL, CS>;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(NUM_THREADS, 1, 1);
   cfg.dynamicSmemBytes = SMEM;
   cfg.stream = s;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 1;  // the occupancy query sees the cluster shape only
   // the shared-memory opt-in and the number of co-resident pairs, once per device
   static int max_pairs[64] = {};
   int dev = 0;
@@ -526,6 +533,7 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   const int npairs = static_cast<int>(useful < pairs_here ? useful : pairs_here);
   cfg.gridDim = dim3(2 * static_cast<unsigned>(npairs), 1, 1);
   *why = "tcgen05 pair GEMM launch";
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kernel, maps[0], maps[1], maps[2], maps[3], mapC, P);
 }
 

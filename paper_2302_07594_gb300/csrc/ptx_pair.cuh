@@ -69,6 +69,19 @@ __device__ __forceinline__ bool bounded_wait_cluster(uint32_t bar, uint32_t pari
   }
 }
 
+// Bounded wait for the two threads on the pipeline's critical loop (TMA producer, MMA issuer):
+// it polls without the suspend hint of bounded_wait, which measurably delays the wake-up after a
+// stage completes, and reads the clock every 256 polls.
+__device__ __forceinline__ bool spin_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    for (int i = 0; i < 256; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
+}
+
 // 2-D tiled TMA load into this CTA's shared memory whose completion (bytes) is counted on an
 // mbarrier that may sit in either CTA of the pair (`bar` is a shared::cluster address).
 __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* map, uint32_t bar, int32_t x, int32_t y) {

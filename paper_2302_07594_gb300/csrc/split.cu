@@ -177,6 +177,7 @@ template <typename T, int NL>
 __global__ void __launch_bounds__(THREADS)
 split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_tiles) {
   __shared__ __align__(16) __half sm[NL][TT * TT];
+  pdl_launch_dependents();
   if (static_cast<int>(blockIdx.x) < a_blocks) split_rows<T, NL>(a, a_blocks);
   else split_cols<T, NL>(b, a_blocks, b_tiles_j, b_tiles, sm);
 }
@@ -241,6 +242,9 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
   const int64_t items = P.a_items + P.b_items;
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
+  // a GEMM launched after this split with programmatic stream serialization may set itself up
+  // meanwhile; it waits for this grid's completion before it reads the planes
+  pdl_launch_dependents();
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
