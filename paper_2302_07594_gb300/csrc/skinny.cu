@@ -6,6 +6,9 @@
 // large and two small dimensions (Section 2, IM2COL lowering).  This kernel is
 // built around the stream of B:
 //
+//   * the CTA's slice of A is fetched by bulk copies (one per row) issued with the first B stages
+//     and split into limbs in place, so B starts streaming at once (with plain loads issued by the
+//     consumers, the first B stage waited about 3 us for them);
 //   * B is cut into column blocks of 512 (1 KB contiguous of every row, which
 //     DRAM streams markedly better than 512-byte runs) and the reduction
 //     dimension into ranges, one (column block, range) per CTA, about one CTA
@@ -64,12 +67,21 @@ struct SkParams {
   int64_t stages_per_cta;   // reduction range of one CTA, in stages
   int64_t total_stages;
   int atomic_out;
+  int a_bulk;               // A's slices can be bulk-copied: 16-byte aligned rows, k % 8 == 0
   uint64_t timeout_ns;
   uint32_t* status;
 };
 
+// Bulk copy global -> this CTA's shared memory, completion (bytes) counted on `bar`.  Both
+// addresses 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
 constexpr size_t sk_smem() {
-  return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * A_LIMB_BYTES + 8 * (2 * STAGES) + 16;
+  return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * A_LIMB_BYTES + 8 * (2 * STAGES + 1) + 16;
 }
 static_assert(sk_smem() <= 227 * 1024, "shared memory budget");
 
@@ -121,6 +133,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   uint64_t* bars = reinterpret_cast<uint64_t*>(a_lo + A_ROWS * A_STRIDE);
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t abar = empty0 + 8 * STAGES;  // the CTA's A slice has landed
 
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
@@ -136,6 +149,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, NCONS);
     }
+    mbar_init(abar, 1);
     fence_mbar_init();
   }
   __syncthreads();
@@ -145,6 +159,17 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&mapB);
+      if (P.a_bulk && nst > 0) {
+        // rows 0..m-1 of A, reduction indices k0 .. k0 + kv, land in the low-limb area (row r at
+        // r * A_STRIDE words), where the consumers split them in place
+        const int64_t k0 = st_begin * KS;
+        const int64_t kv = min(nst * KS, P.k - k0);
+        const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
+        const int rows = static_cast<int>(P.m < A_ROWS ? P.m : A_ROWS);
+        mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
+        for (int r = 0; r < rows; ++r)
+          bulk_load(smem_u32(a_lo + r * A_STRIDE), P.A + r * P.lda + k0, row_bytes, abar);
+      }
       int64_t issued = 0;
       for (int64_t i = 0; i < nst; ++i) {
         const int s = static_cast<int>(i % STAGES);
@@ -172,7 +197,27 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   // ------------------------------------------------------------ consumers
   // Split this CTA's slice of A once: rows 0..15 (zero beyond m), reduction indices
   // k0 .. k0 + KS*nst (zero beyond k), as packed fp16 pairs of the high and low limbs.
-  {
+  if (P.a_bulk) {
+    bool landed = true;
+    if (nst > 0) {
+      landed = __all_sync(0xFFFFFFFFu, bounded_wait(abar, 0, P.timeout_ns));
+      if (!landed && lane == 0) report_status(P.status, STATUS_TIMEOUT, 13);
+    }
+    const int64_t k0 = st_begin * KS;
+    const int64_t kv = nst > 0 ? min(nst * KS, P.k - k0) : 0;
+    const int pairs = landed ? static_cast<int>(nst * KS / 2) : 0;
+    for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
+      const int row = idx / pairs;
+      const int kp = idx - row * pairs;
+      const uint32_t x = (row < P.m && 2 * kp < kv) ? a_lo[row * A_STRIDE + kp] : 0u;
+      uint32_t hi, lo;
+      split_pair(x, hi, lo);
+      a_hi[row * A_STRIDE + kp] = hi;
+      a_lo[row * A_STRIDE + kp] = lo;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // every consumer warp arrives
+    if (!landed) return;
+  } else {
     const int64_t k0 = st_begin * KS;
     const int pairs = static_cast<int>(nst * KS / 2);
     for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
@@ -333,6 +378,7 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   P.stages_per_cta = per;
   P.total_stages = total_stages;
   P.atomic_out = ksplit > 1 ? 1 : 0;
+  P.a_bulk = reinterpret_cast<uintptr_t>(a.A) % 16 == 0 && (a.lda * 2) % 16 == 0 && a.k % 8 == 0;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
   constexpr size_t smem = sk_smem();

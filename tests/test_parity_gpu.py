@@ -220,6 +220,22 @@ def test_skinny_unaligned_B(gm):
     assert_same(dC.cpu().numpy(), exp, "skinny unaligned B")
 
 
+# the CTA's slice of A is bulk-copied when A's rows are 16-byte aligned and k % 8 == 0, and
+# loaded element by element otherwise; both with padded leading dimensions and ragged k ranges
+@pytest.mark.parametrize("m,k,lda", [(8, 4096, 4096), (5, 1000, 1008), (16, 2040, 2048), (3, 1000, 1001),
+                                     (8, 999, 1000), (13, 96, 104)])
+def test_skinny_a_slice_paths(gm, m, k, lda):
+    n = 700
+    A, B, C = gi.random_problem(805 + m + k + lda, m, n, k, "i16")
+    Ap = torch.full((m, lda), 31000, dtype=torch.int16)
+    Ap[:, :k] = torch.from_numpy(A)
+    dA, dB, dC = Ap.cuda(), torch.from_numpy(B).cuda(), torch.from_numpy(C).cuda()
+    gm.gemm_i16(dA[:, :k], dB, dC)
+    torch.cuda.synchronize()
+    assert gm.device_status() == gm.OK
+    assert_same(dC.cpu().numpy(), expected(A, B, C), f"skinny m={m} k={k} lda={lda}")
+
+
 def test_skinny_extremes(gm):
     for a, b in ((-32768, -32768), (-1, -1), (32767, -32768), (255, 255)):
         A = np.full((8, 2000), a, np.int16)
