@@ -215,6 +215,20 @@ struct TmaSplitParams {
   uint64_t timeout_ns;
 };
 
+// Four int8 values packed in a word -> two fp16 pairs, exactly: u = w ^ 0x80808080 holds v + 128
+// in each byte; a byte permute puts each byte under the fp16 bit pattern 0x64xx = 1024 + xx, and
+// one fp16 subtraction of 1152 = 0x6480 per pair leaves v (every integer up to 2048 is exact).
+__device__ __forceinline__ void i8x4_to_half2x2(uint32_t w, uint32_t& h01, uint32_t& h23) {
+  const uint32_t u = w ^ 0x80808080u;
+  const uint32_t a = __byte_perm(u, 0x64646464u, 0x5140);
+  const uint32_t b = __byte_perm(u, 0x64646464u, 0x7362);
+  const __half2 k = __half2half2(__ushort_as_half(0x6480));
+  const __half2 ha = __hsub2(*reinterpret_cast<const __half2*>(&a), k);
+  const __half2 hb = __hsub2(*reinterpret_cast<const __half2*>(&b), k);
+  h01 = *reinterpret_cast<const uint32_t*>(&ha);
+  h23 = *reinterpret_cast<const uint32_t*>(&hb);
+}
+
 __device__ __forceinline__ void tma_store_2d(const void* map, uint32_t src, int32_t x, int32_t y) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
                    reinterpret_cast<uint64_t>(map)),
@@ -326,10 +340,10 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             if (col + 8 * h >= P.a_pitch) continue;
-            int v[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = static_cast<int8_t>((wv[2 * h + i / 4] >> (8 * (i % 4))) & 0xFFu);
-            store8<NL>(P.a_p0 + row * P.a_pitch + col + 8 * h, P.a_p1 + row * P.a_pitch + col + 8 * h, v);
+            uint4 o;
+            i8x4_to_half2x2(wv[2 * h], o.x, o.y);
+            i8x4_to_half2x2(wv[2 * h + 1], o.z, o.w);
+            *reinterpret_cast<uint4*>(P.a_p0 + row * P.a_pitch + col + 8 * h) = o;
           }
         }
       }
@@ -348,33 +362,62 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
       }
       uint8_t* sbuf = stg + buf * STG;
       constexpr int PAIRS = JB * 8 / CONSUMERS;  // (column, 8-row group) pairs per thread
-      int vals[PAIRS][8];
+      if constexpr (sizeof(T) == 2) {
+        int vals[PAIRS][8];
 #pragma unroll
-      for (int u = 0; u < PAIRS; ++u) {
-        const int q = tid + CONSUMERS * u;
-        const int j = q % JB;
-        const int g = q / JB;
+        for (int u = 0; u < PAIRS; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int j = q % JB;
+          const int g = q / JB;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int p = 8 * g + i;
-          if constexpr (sizeof(T) == 2) {
+          for (int i = 0; i < 8; ++i) {
+            const int p = 8 * g + i;
             const int off = p * 128 + ((((j >> 3) ^ (p & 7))) << 4) + ((j & 7) << 1);
             vals[u][i] = *reinterpret_cast<const int16_t*>(rawt + off);
-          } else {
-            const int off = p * 128 + ((((j >> 4) ^ (p & 7))) << 4) + (j & 15);
-            vals[u][i] = *reinterpret_cast<const int8_t*>(rawt + off);
           }
         }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
 #pragma unroll
-      for (int u = 0; u < PAIRS; ++u) {
-        const int q = tid + CONSUMERS * u;
-        const int j = q % JB;
-        const int g = q / JB;
-        const int off = j * 128 + ((g ^ (j & 7)) << 4);
-        store8<NL>(reinterpret_cast<__half*>(sbuf + off), reinterpret_cast<__half*>(sbuf + 8192 + off), vals[u]);
+        for (int u = 0; u < PAIRS; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int j = q % JB;
+          const int g = q / JB;
+          const int off = j * 128 + ((g ^ (j & 7)) << 4);
+          store8<NL>(reinterpret_cast<__half*>(sbuf + off), reinterpret_cast<__half*>(sbuf + 8192 + off), vals[u]);
+        }
+      } else {
+        // int8: the 8 bytes of column j in rows 8g .. 8g+7, packed four to a word
+        uint32_t wds[PAIRS][2];
+#pragma unroll
+        for (int u = 0; u < PAIRS; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int j = q % JB;
+          const int g = q / JB;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint32_t w = 0;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int p = 8 * g + 4 * h + i;
+              const int off = p * 128 + ((((j >> 4) ^ (p & 7))) << 4) + (j & 15);
+              w |= static_cast<uint32_t>(rawt[off]) << (8 * i);
+            }
+            wds[u][h] = w;
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+#pragma unroll
+        for (int u = 0; u < PAIRS; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int j = q % JB;
+          const int g = q / JB;
+          uint4 o;
+          i8x4_to_half2x2(wds[u][0], o.x, o.y);
+          i8x4_to_half2x2(wds[u][1], o.z, o.w);
+          *reinterpret_cast<uint4*>(sbuf + j * 128 + ((g ^ (j & 7)) << 4)) = o;
+        }
       }
       fence_proxy_async_smem();
       mbar_arrive(sfull0 + 8 * buf);
