@@ -203,6 +203,7 @@ constexpr int B_P = 64;
 constexpr int STG = 16384;
 constexpr int NBAR = 2 * STAGES + 4;  // full, empty, staging full x2, staging free x2
 constexpr size_t SMEM = 1024 + STAGES * RAW + 2 * STG + 8 * NBAR;
+static_assert((RAW / 16) % CONSUMERS == 0, "whole raw chunks per consumer thread");
 }  // namespace tsplit
 
 struct TmaSplitParams {
@@ -314,14 +315,15 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
     if (it < P.a_items) {
       // ---- A: row = q / 16, 16-byte chunk c = q % 16 of the 256-byte raw row
       const int64_t rt = it / P.a_tiles_k, kt = it - rt * P.a_tiles_k;
-      uint4 w[2];
+      constexpr int ACH = RAW / 16 / CONSUMERS;  // 16-byte raw chunks per thread
+      uint4 w[ACH];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) w[u] = *reinterpret_cast<const uint4*>(rawt + (tid + 256 * u) * 16);
+      for (int u = 0; u < ACH; ++u) w[u] = *reinterpret_cast<const uint4*>(rawt + (tid + CONSUMERS * u) * 16);
       __syncwarp();
       if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int q = tid + 256 * u;
+      for (int u = 0; u < ACH; ++u) {
+        const int q = tid + CONSUMERS * u;
         const int64_t row = rt * A_ROWS + (q >> 4);
         if (row >= P.m) continue;
         const uint32_t wv[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
