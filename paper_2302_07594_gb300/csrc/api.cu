@@ -2,8 +2,11 @@
 //
 // Dispatch (all paths bit-exact, see the kernels' headers):
 //   int16, m <= skinny limit (16) : skinny.cu   (B streamed once, tensor-core limb products)
-//   int16, otherwise              : split.cu (A and B -> fp16 limb planes) + gemm_tc.cu (tcgen05)
-//   int8                          : split.cu (A and B -> fp16 planes) + gemm_tc.cu (tcgen05)
+//   int16, n <= 64, A TMA-readable: gemm_fused.cu (A split on chip; B's planes from split.cu)
+//   int16 / int8, otherwise       : split.cu (operands -> fp16 limb planes), then gemm_pair.cu
+//                                   (tcgen05 on SM pairs) when C takes 16-byte reductions, else
+//                                   gemm_tc.cu (one SM per tile)
+//   *_host with m >= 1024         : the same, pipelined over row panels on copy streams
 #include <cuda_runtime.h>
 
 #include <algorithm>
