@@ -567,7 +567,7 @@ int host_gemm_pipelined(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k,
   if (rc != GEMMI_OK) return rc;
   cudaStream_t s = g_stream;
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
-  const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 7) / 8), 128)));
+  const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 15) / 16), 128)));
   const int64_t panels = (m + mb - 1) / mb;
   const size_t b_raw = round_up(static_cast<size_t>(k) * n * sizeof(OP), kAlign);
   const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
