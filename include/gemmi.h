@@ -217,11 +217,14 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_TC_PAIR      : 1 (default): tensor-core GEMMs run on pairs of SMs (tcgen05
  *                            cta_group::2, clusters of two CTAs) whenever C is 16-byte aligned
  *                            with ldc * sizeof(element) a multiple of 16; 0: one SM per tile.
+ *   GEMMI_OPT_SMALL_MAX_MACS : int16 GEMMs with m <= 256 and m*n*k <= this value (default 2^25)
+ *                            run as one launch of the skinny-M kernel, 16 rows of A per grid
+ *                            row; 0 disables it (so does GEMMI_OPT_SKINNY_MAX_M = 0).
  * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
 enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
        GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6,
-       GEMMI_OPT_FUSED_MAX_N = 7, GEMMI_OPT_TC_PAIR = 8 };
+       GEMMI_OPT_FUSED_MAX_N = 7, GEMMI_OPT_TC_PAIR = 8, GEMMI_OPT_SMALL_MAX_MACS = 9 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 

@@ -25,6 +25,7 @@ LIB_PATH = os.path.join(_HERE, "libgemmi.so")
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EARCH = 0, 1, 2, 3, 4, 5
 OPT_SKINNY_MAX_M, OPT_WAIT_TIMEOUT_US, OPT_SKINNY_KSPLIT = 1, 2, 3
 OPT_TC_CHUNK_SCALE, OPT_TC_GROUP_M, OPT_TC_L2_HINTS, OPT_FUSED_MAX_N, OPT_TC_PAIR = 4, 5, 6, 7, 8
+OPT_SMALL_MAX_MACS = 9
 EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
             "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_detail",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",

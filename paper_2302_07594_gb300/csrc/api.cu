@@ -125,6 +125,7 @@ int64_t g_tc_group_m = 16;
 int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
+int64_t g_small_max_macs = int64_t{1} << 25;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -434,7 +435,10 @@ int gemm_i16_locked(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t l
   DeviceState* d = nullptr;
   int rc = device_state(&d);
   if (rc != GEMMI_OK) return rc;
-  if (m <= g_skinny_max_m) return run_skinny(*d, m, n, k, A, lda, B, ldb, C, ldc, s);
+  // small m, or a small problem of at most 256 rows: one launch of the skinny kernel (B split on
+  // chip, one grid row per 16 rows of A) beats the split + tensor-core pair of launches
+  const bool small = g_skinny_max_m > 0 && m <= 256 && m * n <= g_small_max_macs / std::max<int64_t>(k, 1);
+  if (m <= g_skinny_max_m || small) return run_skinny(*d, m, n, k, A, lda, B, ldb, C, ldc, s);
   return run_tc(*d, 2, m, n, k, A, lda, B, ldb, C, ldc, s);
 }
 
@@ -962,6 +966,10 @@ int gemmi_set_option(int option, int64_t value) {
       if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "SM-pair option must be 0 or 1");
       g_tc_pair = value;
       return GEMMI_OK;
+    case GEMMI_OPT_SMALL_MAX_MACS:
+      if (value < 0 || value > (int64_t{1} << 40)) return set_error(GEMMI_EINVAL, "small-problem limit must be in [0, 2^40]");
+      g_small_max_macs = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -978,6 +986,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_TC_L2_HINTS: return g_tc_l2_hints;
     case GEMMI_OPT_FUSED_MAX_N: return g_fused_max_n;
     case GEMMI_OPT_TC_PAIR: return g_tc_pair;
+    case GEMMI_OPT_SMALL_MAX_MACS: return g_small_max_macs;
     default: return -1;
   }
 }

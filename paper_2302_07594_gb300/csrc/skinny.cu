@@ -1,4 +1,6 @@
-// skinny.cu -- exact int16 GEMM C (int64) += A*B for a small number of rows m <= 16.
+// skinny.cu -- exact int16 GEMM C (int64) += A*B for a small number of rows m <= 16, and for
+// small problems (up to 256 rows) as groups of 16 rows along the grid's z dimension: one launch,
+// no separate operand split, where the tensor-core path pays two launches and their latency.
 //
 // With m <= 16 (a batch of a few samples through a fully-connected layer) the
 // GEMM of Section 4.1 is bound by streaming B (k x n) once from HBM: every B
@@ -139,6 +141,11 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   const int lane = threadIdx.x % 32;
   const int64_t j_base = static_cast<int64_t>(blockIdx.x) * JB;
   const int64_t st_begin = static_cast<int64_t>(blockIdx.y) * P.stages_per_cta;
+  // grid z: groups of 16 rows of A and C (one group when m <= 16)
+  const int64_t row0 = static_cast<int64_t>(blockIdx.z) * A_ROWS;
+  const int64_t mrows = P.m - row0 < A_ROWS ? P.m - row0 : A_ROWS;
+  const int16_t* Ag = P.A + row0 * P.lda;
+  int64_t* Cg = P.C + row0 * P.ldc;
   int64_t st_end = st_begin + P.stages_per_cta;
   if (st_end > P.total_stages) st_end = P.total_stages;
   const int64_t nst = st_end > st_begin ? st_end - st_begin : 0;
@@ -165,10 +172,10 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         const int64_t k0 = st_begin * KS;
         const int64_t kv = min(nst * KS, P.k - k0);
         const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
-        const int rows = static_cast<int>(P.m < A_ROWS ? P.m : A_ROWS);
+        const int rows = static_cast<int>(mrows);
         mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
         for (int r = 0; r < rows; ++r)
-          bulk_load(smem_u32(a_lo + r * A_STRIDE), P.A + r * P.lda + k0, row_bytes, abar);
+          bulk_load(smem_u32(a_lo + r * A_STRIDE), Ag + r * P.lda + k0, row_bytes, abar);
       }
       int64_t issued = 0;
       for (int64_t i = 0; i < nst; ++i) {
@@ -209,7 +216,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
       const int row = idx / pairs;
       const int kp = idx - row * pairs;
-      const uint32_t x = (row < P.m && 2 * kp < kv) ? a_lo[row * A_STRIDE + kp] : 0u;
+      const uint32_t x = (row < mrows && 2 * kp < kv) ? a_lo[row * A_STRIDE + kp] : 0u;
       uint32_t hi, lo;
       split_pair(x, hi, lo);
       a_hi[row * A_STRIDE + kp] = hi;
@@ -225,8 +232,8 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       const int kp = idx - row * pairs;
       const int64_t k = k0 + 2 * kp;
       uint32_t x = 0;
-      if (row < P.m) {
-        const int16_t* src = P.A + row * P.lda + k;
+      if (row < mrows) {
+        const int16_t* src = Ag + row * P.lda + k;
         const uint32_t v0 = k < P.k ? static_cast<uint16_t>(src[0]) : 0u;
         const uint32_t v1 = k + 1 < P.k ? static_cast<uint16_t>(src[1]) : 0u;
         x = v0 | (v1 << 16);
@@ -330,8 +337,8 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       for (int c = 0; c < 4; ++c) {
         const int64_t i = nt * 8 + 2 * t + (c & 1);
         const int64_t j = j_base + warp * (16 * MT) + mt * 16 + g + 8 * (c >> 1);
-        if (i < P.m && j < P.n) {
-          unsigned long long* dst = reinterpret_cast<unsigned long long*>(P.C + i * P.ldc + j);
+        if (i < mrows && j < P.n) {
+          unsigned long long* dst = reinterpret_cast<unsigned long long*>(Cg + i * P.ldc + j);
           const unsigned long long v = static_cast<unsigned long long>(acc[mt][nt][c]);
           if (P.atomic_out) atomicAdd(dst, v);
           else *dst = *dst + v;
@@ -348,9 +355,10 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   const int64_t nj = (a.n + JB - 1) / JB;
   const int64_t total_stages = (a.k + KS - 1) / KS;
   int64_t ksplit = a.ksplit;
+  const int64_t groups = (a.m + A_ROWS - 1) / A_ROWS;
   if (ksplit <= 0) {
     // about one CTA per SM: the reduction range is split across the CTAs of a column block
-    ksplit = a.num_sms / nj;
+    ksplit = a.num_sms / (nj * groups);
     if (ksplit < 1) ksplit = 1;
     // keep at least 4 stages (128 reduction indices) per CTA
     const int64_t cap = total_stages / 4 > 0 ? total_stages / 4 : 1;
@@ -363,7 +371,7 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   if (ksplit < 1) ksplit = 1;
   const int64_t per = (total_stages + ksplit - 1) / ksplit;
   ksplit = (total_stages + per - 1) / per;
-  if (nj > 0x7FFFFFFF || ksplit > 65535) {
+  if (nj > 0x7FFFFFFF || ksplit > 65535 || groups > 65535) {
     *why = "skinny GEMM grid too large";
     return cudaErrorInvalidValue;
   }
@@ -395,7 +403,7 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   // programmatic stream serialization: the kernel may be scheduled while the previous kernel in
   // the stream drains; it waits (griddepcontrol.wait) before its first global memory access
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit));
+  cfg.gridDim = dim3(static_cast<unsigned>(nj), static_cast<unsigned>(ksplit), static_cast<unsigned>(groups));
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;

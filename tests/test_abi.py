@@ -126,6 +126,16 @@ def test_pair_option(L):
             gm.set_option(gm.OPT_TC_PAIR, bad)
 
 
+def test_small_problem_option(L):
+    assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 25
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)
+    assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 0
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 25)
+    for bad in (-1, (1 << 40) + 1):
+        with pytest.raises(gm.GemmiError):
+            gm.set_option(gm.OPT_SMALL_MAX_MACS, bad)
+
+
 def test_header_constants_match_binding():
     text = open(HEADER).read()
     consts = dict((name, int(v)) for name, v in re.findall(r"GEMMI_((?:OPT|KERNEL)_[A-Z0-9_]+)\s*=\s*(\d+)", text))

@@ -236,6 +236,49 @@ def test_skinny_a_slice_paths(gm, m, k, lda):
     assert_same(dC.cpu().numpy(), expected(A, B, C), f"skinny m={m} k={k} lda={lda}")
 
 
+def _kernel_counts(gm, fn):
+    gm.kernel_timing(True)
+    try:
+        fn()
+        torch.cuda.synchronize()
+        return {name: gm.kernel_time(kid)[1] for name, kid in gm.KERNELS}
+    finally:
+        gm.kernel_timing(False)
+
+
+# small problems (m <= 256, m*n*k <= 2^25 by default) run the skinny kernel with one grid row per
+# 16 rows of A: the last group ragged, several column blocks and reduction splits
+@pytest.mark.parametrize("m,n,k", [(17, 64, 64), (24, 300, 1000), (100, 513, 576), (255, 256, 256), (256, 256, 256),
+                                   (200, 40, 4000)])
+def test_skinny_row_groups(gm, m, n, k):
+    A, B, C = gi.random_problem(830 + m + n + k, m, n, k, "i16")
+    dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+    counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
+    assert gm.device_status() == gm.OK
+    assert counts["skinny"] == 1 and counts["split"] == 0, counts
+    assert_same(dC.cpu().numpy(), expected(A, B, C), f"skinny row groups {m}x{n}x{k}")
+
+
+def test_small_problem_rule(gm):
+    # beyond 256 rows, or above the work limit, the tensor-core path runs
+    for (m, n, k) in ((257, 64, 64), (256, 512, 512)):
+        A, B, C = gi.random_problem(840 + m + n, m, n, k, "i16")
+        dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+        counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["fused_i16"] == 1, counts
+        assert_same(dC.cpu().numpy(), expected(A, B, C), f"{m}x{n}x{k}")
+    # with the limit at 0 a small problem takes the tensor-core path too
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)
+    try:
+        A, B, C = gi.random_problem(850, 100, 300, 200, "i16")
+        dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+        counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] == 1, counts
+        assert_same(dC.cpu().numpy(), expected(A, B, C), "limit 0")
+    finally:
+        gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 25)
+
+
 def test_skinny_extremes(gm):
     for a, b in ((-32768, -32768), (-1, -1), (32767, -32768), (255, 255)):
         A = np.full((8, 2000), a, np.int16)
