@@ -223,3 +223,11 @@ def test_pair_stream_k_tails(gm, case, chunk_scale):
     kind, m, n, k = case
     A, B, C = gi.random_problem(5800 + m + n + k, m, n, k, kind)
     assert_same(run(gm, A, B, C), expected(A, B, C), f"stream-K {case}, chunk scale {chunk_scale}")
+
+
+# long reductions over few tiles: every pair's stream-K share starts and ends inside a tile and
+# crosses exact-chunk boundaries at arbitrary offsets
+@pytest.mark.parametrize("kind,m,n,k", [("i16", 130, 130, 20000), ("i8", 300, 260, 30011), ("i16", 1, 2, 65537)])
+def test_pair_long_reduction_stream_k(gm, kind, m, n, k, chunk_scale):
+    A, B, C = gi.random_problem(5900 + k, m, n, k, kind)
+    assert_same(run(gm, A, B, C), expected(A, B, C), f"{kind} {m}x{n}x{k}, chunk scale {chunk_scale}")
