@@ -202,7 +202,7 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_SKINNY_MAX_M : int16 GEMMs with m <= this value take the
  *                            skinny-M kernel (default 16, maximum 16; 0 disables it).
  *   GEMMI_OPT_WAIT_TIMEOUT_US : bound on every device-side pipeline wait, in
- *                            microseconds (default 4,000,000).
+ *                            microseconds (default 4,000,000; 1,000 to 60,000,000).
  *   GEMMI_OPT_SKINNY_KSPLIT : number of CTAs sharing the reduction dimension
  *                            of one skinny column block (0 = automatic).
  *   GEMMI_OPT_TC_CHUNK_SCALE : length of the exact fp32 accumulation runs of the tensor-core

@@ -938,7 +938,9 @@ int gemmi_set_option(int option, int64_t value) {
       g_skinny_max_m = value;
       return GEMMI_OK;
     case GEMMI_OPT_WAIT_TIMEOUT_US:
-      if (value < 1 || value > 60000000) return set_error(GEMMI_EINVAL, "timeout must be in [1 us, 60 s]");
+      // at least 1 ms: a CTA that gives up waits this long once more for its own copies in flight,
+      // which land within microseconds, before it exits
+      if (value < 1000 || value > 60000000) return set_error(GEMMI_EINVAL, "timeout must be in [1 ms, 60 s]");
       g_timeout_us = value;
       return GEMMI_OK;
     case GEMMI_OPT_SKINNY_KSPLIT:

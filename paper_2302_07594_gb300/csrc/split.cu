@@ -279,6 +279,7 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
       if (P.a_items) tma_prefetch_desc(&rawA);
       if (P.b_items) tma_prefetch_desc(&rawB);
       tc::RingPos st;
+      int64_t issued = 0;
       for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
         if (!bounded_wait(empty0 + 8 * st.slot, st.phase ^ 1u, P.timeout_ns)) {
           report_status(P.status, tc::STATUS_TIMEOUT, 31);
@@ -295,8 +296,14 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
           const int64_t pt = b / P.b_tiles_j, jt = b - (b / P.b_tiles_j) * P.b_tiles_j;
           tma_load_2d(dst, &rawB, fb, static_cast<int32_t>(jt * JB), static_cast<int32_t>(pt * B_P));
         }
+        ++issued;
         st.advance(STAGES);
       }
+      // stay until the last copies have landed: if the consumers gave up, the CTA must not exit
+      // with copies still writing its shared memory
+      const int64_t first = issued > STAGES ? issued - STAGES : 0;
+      for (int64_t i = first; i < issued; ++i)
+        bounded_wait(full0 + 8 * static_cast<int>(i % STAGES), static_cast<uint32_t>((i / STAGES) & 1), P.timeout_ns);
     }
     return;
   }
