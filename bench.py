@@ -302,6 +302,37 @@ def time_workload_packed(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES,
     return graph_ms, eager_ms, kt, nsets
 
 
+def time_read_floor(torch, w, steps=256, rotate_bytes=4 * L2_BYTES):
+    """ms per call of torch.sum over the bytes of workload w's B matrices (read as float32, rotated
+    past L2), CUDA-graph replay: one library kernel that reads them once."""
+    nb = w.k * w.n * 2
+    nsets = int(max(1, math.ceil(rotate_bytes / nb)))
+    Bs = [torch.zeros((w.k, w.n), dtype=torch.int16, device="cuda") for _ in range(nsets)]
+    views = [b.view(torch.float32) for b in Bs]  # the same bytes through torch's tuned float reduction
+    for v in views[:3]:
+        v.sum()
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    ncap = 64
+    with torch.cuda.graph(graph, stream=side):
+        for i in range(ncap):
+            views[i % nsets].sum()
+    graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(1, steps // ncap)
+    e0.record()
+    for _ in range(reps):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / (reps * ncap)
+    del graph, views, Bs
+    torch.cuda.empty_cache()
+    return ms
+
+
 def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_sets=64):
     """Device-resident timing of one workload; rotates input sets so the working set exceeds L2.
 
@@ -495,6 +526,16 @@ def run_gemmi(args):
             if int8_peak:
                 ent["frac_of_int8_roofline_div4" if ow.kind == "i16" else "frac_of_int8_roofline"] = (
                     ent["TOPS"] / (int8_peak / 4 if ow.kind == "i16" else int8_peak))
+            if name.startswith("skinny"):
+                # context for the per-call floor: a plain library reduction over the same bytes
+                # (torch.sum, one kernel reading them once), timed the same way
+                try:
+                    fms = time_read_floor(torch, ow)
+                    ent["read_floor"] = {"what": "torch.sum over the bytes of the same rotating B matrices "
+                                                 "(viewed as float32), CUDA-graph replay",
+                                         "ms": fms, "GB_per_s": ow.k * ow.n * 2 / (fms * 1e-3) / 1e9}
+                except Exception as ex:  # pragma: no cover
+                    ent["read_floor"] = {"error": str(ex)}
             extra[name] = ent
         # the same calls with the weights split once (gemmi_pack_b_*): the operand split then covers
         # A only, and the narrow-n kernel has no split at all
