@@ -158,12 +158,38 @@ def _draw_rows(seed: int, m: int, cols: int, r0: int, mr: int, dist, dtype) -> n
     return v.astype(dtype).reshape(mr, cols)
 
 
+def pack_nibbles(v: np.ndarray, ld: int | None = None, pad: int = 0) -> np.ndarray:
+    """Store signed 4-bit values two to a byte (the int4 operand format).
+
+    v: integer array (rows, cols) with values in [-8, 7].  Element (r, c) goes to byte c//2 of row
+    r, in the low nibble when c is even and the high nibble when c is odd, as its two's-complement
+    bit pattern (v & 15).  Rows are `ld` bytes apart (default ceil(cols/2)); the bytes past the
+    packed width and the spare high nibble of an odd-width row hold `pad`'s bit patterns.
+    """
+    rows, cols = v.shape
+    width = (cols + 1) // 2
+    ld = width if ld is None else ld
+    if ld < width:
+        raise ValueError("row pitch below the packed width")
+    if v.size and (v.min() < -8 or v.max() > 7):
+        raise ValueError("int4 values must lie in [-8, 7]")
+    nib = (v.astype(np.int64) & 15).astype(np.uint8)
+    if cols % 2:
+        nib = np.concatenate([nib, np.full((rows, 1), pad & 15, np.uint8)], axis=1)
+    out = np.full((rows, ld), pad & 0xFF, np.uint8)
+    out[:, :width] = nib[:, 0::2] | (nib[:, 1::2] << np.uint8(4))
+    return out
+
+
 def random_problem(seed: int, m: int, n: int, k: int, kind: str = "i16",
                    a_range=None, b_range=None, c_range=None):
-    """Arbitrary-shape seeded problem for tests (row-major, contiguous)."""
+    """Arbitrary-shape seeded problem for tests (row-major, contiguous).
+
+    kind "i4" draws int4 values in [-8, 7], held one per int8 element (pack_nibbles stores them).
+    """
     op = np.int16 if kind == "i16" else np.int8
     cd = np.int64 if kind == "i16" else np.int32
-    full = (-32768, 32767) if kind == "i16" else (-128, 127)
+    full = {"i16": (-32768, 32767), "i8": (-128, 127), "i4": (-8, 7)}[kind]
     a_range = a_range or full
     b_range = b_range or full
     c_range = c_range or ((-(1 << 40), 1 << 40) if kind == "i16" else (-(1 << 30), 1 << 30))

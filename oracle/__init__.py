@@ -50,6 +50,8 @@ def _bind(lib):
         f = getattr(lib, name)
         f.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int]
         f.restype = ctypes.c_int
+    lib.gemm_oracle_i4.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int]
+    lib.gemm_oracle_i4.restype = ctypes.c_int
     lib.gemm_oracle_i16_srs.argtypes = [i64, i64, i64, vp, i64, vp, i64, vp, i64, ctypes.c_int, ctypes.c_int]
     lib.gemm_oracle_i16_srs.restype = ctypes.c_int
     lib.gemm_oracle_conv2d_i16.argtypes = [i64] * 9 + [vp, vp, vp, ctypes.c_int]
@@ -96,6 +98,27 @@ def gemm(A: np.ndarray, B: np.ndarray, C: np.ndarray, nthreads: int = 1, lib=Non
         raise ValueError(f"shape mismatch: A {A.shape}, B {B.shape}, C {C.shape}")
     rc = fn(m, n, k, _ptr(A), _ld(A, A.itemsize), _ptr(B), _ld(B, B.itemsize),
             _ptr(C), _ld(C, C.itemsize), int(nthreads))
+    if rc != 0:
+        raise ValueError(f"oracle rejected the arguments (rc={rc})")
+    return C
+
+
+def gemm_i4(Ap: np.ndarray, Bp: np.ndarray, C: np.ndarray, k: int, nthreads: int = 1, lib=None) -> np.ndarray:
+    """In place: C (int32) += A @ B modulo 2^32, A and B signed 4-bit values packed two to a byte.
+
+    Ap: uint8 (m, >= ceil(k/2)) holding A's rows, element (i, p) in byte p//2 (low nibble for even
+    p, high nibble for odd p, two's complement); Bp: uint8 (k, >= ceil(n/2)) holding B's rows the
+    same way along j.  Row pitches may exceed the packed width (padding is never read).
+    """
+    lib = lib or load()
+    if Ap.dtype != np.uint8 or Bp.dtype != np.uint8 or C.dtype != np.int32:
+        raise TypeError("gemm_i4 takes uint8 packed A and B and an int32 C")
+    m, n = C.shape
+    if Ap.shape[0] != m or Bp.shape[0] != k or Ap.shape[1] < (k + 1) // 2 or Bp.shape[1] < (n + 1) // 2:
+        raise ValueError(f"shape mismatch: packed A {Ap.shape}, packed B {Bp.shape}, C {C.shape}, k {k}")
+    lda = _ld(Ap, 1) if m else max(1, (k + 1) // 2)
+    ldb = _ld(Bp, 1) if k else max(1, (n + 1) // 2)
+    rc = lib.gemm_oracle_i4(m, n, k, _ptr(Ap), lda, _ptr(Bp), ldb, _ptr(C), _ld(C, 4), int(nthreads))
     if rc != 0:
         raise ValueError(f"oracle rejected the arguments (rc={rc})")
     return C

@@ -102,6 +102,50 @@ int gemm_oracle_i8(int64_t m, int64_t n, int64_t k,
 }
 
 /*
+ * Lower precision (Section 5.1, the datatype discussion: the INT16 micro-kernel is the paper's
+ * baseline and its design is to be carried to lower precision).  The int4 variant is the same
+ * update with signed 4-bit operands and an int32 C, modulo 2^32.  Two operands share a byte: the
+ * element with even index sits in the low nibble (bits 0-3), the one with odd index in the high
+ * nibble (bits 4-7), each in two's complement (nibble values 8..15 stand for -8..-1).  A packs
+ * along its rows (element (i, p) in byte A[i*lda + p/2]), B along its rows too (element (p, j) in
+ * byte B[p*ldb + j/2]); lda and ldb count BYTES and must be at least ceil(k/2) and ceil(n/2).  The
+ * unused high nibble of a row's last byte (odd k for A, odd n for B) is never read.
+ */
+static int64_t oracle_nibble(const uint8_t* row, int64_t idx) {
+  const unsigned byte = row[idx / 2];
+  const unsigned v = (idx % 2 == 0) ? (byte & 15u) : (byte >> 4);
+  return v >= 8 ? (int64_t)v - 16 : (int64_t)v;
+}
+
+int gemm_oracle_i4(int64_t m, int64_t n, int64_t k,
+                   const uint8_t* A, int64_t lda,
+                   const uint8_t* B, int64_t ldb,
+                   int32_t* C, int64_t ldc, int nthreads) {
+  if (m < 0 || n < 0 || k < 0) return 1;
+  if (m == 0 || n == 0) return 0;
+  if (ldc < n || C == NULL) return 1;
+  if (k == 0) return 0;
+  if (lda < (k + 1) / 2 || ldb < (n + 1) / 2) return 1;
+  if (A == NULL || B == NULL) return 1;
+#ifdef _OPENMP
+  if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads)
+#else
+  (void)nthreads;
+#endif
+  for (int64_t i = 0; i < m; ++i) {
+    int32_t* c = C + i * ldc;
+    for (int64_t j = 0; j < n; ++j) {
+      uint64_t s = (uint64_t)(int64_t)c[j];
+      for (int64_t p = 0; p < k; ++p)
+        s += (uint64_t)(oracle_nibble(A + i * lda, p) * oracle_nibble(B + p * ldb, j));
+      c[j] = (int32_t)(uint32_t)s; /* keep the low 32 bits: modulo 2^32 */
+    }
+  }
+  return 0;
+}
+
+/*
  * The paper's micro-kernel output (Section 5.2, the simplified AIE micro-kernel listing): the
  * wide accumulator is shifted, rounded and saturated to 16 bits ("srs") and added to the int16
  * C block with a plain 16-bit vector addition.  The paper is silent on the rounding of the shift

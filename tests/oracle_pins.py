@@ -375,8 +375,101 @@ def check_conv_im2col_lowering(lib):
 
 CONV_CHECKS = (check_conv_golden, check_conv_1x1_is_gemm, check_conv_delta_kernels, check_conv_im2col_lowering)
 
+# ---- the int4 variant: C32 += A*B with operands packed two to a byte  (gemm_oracle_i4)
+I4_GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "i4_cases.json")
+
+
+def _run_i4(lib, Ap, Bp, C, k):
+    X = C.copy()
+    oracle.gemm_i4(Ap, Bp, X, k, lib=lib)
+    return X
+
+
+def unpack_nibbles_bigint(rows, cols):
+    """Signed 4-bit values read back from packed bytes with Python integers, written independently
+    of both the oracle and the packer: bit 4*(c%2) of byte c//2, sign from bit 3."""
+    out = []
+    for r in rows:
+        vals = []
+        for c in range(cols):
+            nib = (int(r[c // 2]) >> (4 * (c % 2))) & 15
+            vals.append(nib - 16 if nib & 8 else nib)
+        out.append(vals)
+    return np.array(out, dtype=np.int64).reshape(len(rows), cols)
+
+
+def check_i4_golden(lib):
+    """Worked examples (tests/golden/i4_cases.json): nibble order, two's complement, odd k and n,
+    row padding, wrap-around modulo 2^32."""
+    bad = []
+    with open(I4_GOLDEN) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        m, n, k = c["m"], c["n"], c["k"]
+        Ap = np.array(c["A"], np.uint8).reshape(m, c["lda"])
+        Bp = np.array(c["B"], np.uint8).reshape(k, c["ldb"])
+        C = np.array(c["C_in"], np.int32).reshape(m, n)
+        E = np.array(c["C_out"], np.int32).reshape(m, n)
+        got = _run_i4(lib, Ap[:, :(k + 1) // 2] if c["lda"] > (k + 1) // 2 else Ap,
+                      Bp[:, :(n + 1) // 2] if c["ldb"] > (n + 1) // 2 else Bp, C, k)
+        if not np.array_equal(got, E):
+            bad.append(f"i4 golden {c['name']}: got {got.tolist()} want {E.tolist()}")
+    return bad
+
+
+def check_i4_bruteforce(lib, shapes=((1, 1, 1), (2, 3, 5), (5, 7, 9), (3, 8, 17), (8, 1, 33))):
+    """Tiny shapes against Python integers on the values unpacked independently from the bytes;
+    the spare nibble of odd rows and the padding bytes hold a non-zero pattern."""
+    bad = []
+    for idx, (m, n, k) in enumerate(shapes):
+        A, B, C = gi.random_problem(7400 + idx, m, n, k, "i4")
+        Ap = gi.pack_nibbles(A, ld=(k + 1) // 2 + 2, pad=0x9B)
+        Bp = gi.pack_nibbles(B, ld=(n + 1) // 2 + 1, pad=0x6E)
+        Av = unpack_nibbles_bigint(Ap, k)
+        Bv = unpack_nibbles_bigint(Bp, n)
+        if not (np.array_equal(Av, A) and np.array_equal(Bv, B)):
+            bad.append(f"i4 packer does not store the documented format ({m}x{n}x{k})")
+        exp = bigint_gemm(Av, Bv, C.astype(np.int64), 32).astype(np.int32)
+        got = _run_i4(lib, Ap[:, :(k + 1) // 2], Bp[:, :(n + 1) // 2], C, k)
+        if not np.array_equal(got, exp):
+            bad.append(f"i4 bruteforce {m}x{n}x{k}")
+    return bad
+
+
+def check_i4_matches_i8(lib, shapes=((33, 20, 71), (64, 65, 128), (7, 130, 301))):
+    """A special case that reduces to a pinned routine: the int4 GEMM of values in [-8, 7] equals the
+    int8 GEMM of the same values (and numpy's exact matmul), padded rows and all."""
+    bad = []
+    for idx, (m, n, k) in enumerate(shapes):
+        A, B, C = gi.random_problem(7500 + idx, m, n, k, "i4")
+        Ap = gi.pack_nibbles(A, ld=(k + 1) // 2 + 3, pad=0x7F)
+        Bp = gi.pack_nibbles(B, ld=(n + 1) // 2 + 5, pad=0x81)
+        got = _run_i4(lib, Ap[:, :(k + 1) // 2], Bp[:, :(n + 1) // 2], C, k)
+        if not np.array_equal(got, _run(lib, A, B, C)):
+            bad.append(f"i4 != i8 GEMM of the same values on {(m, n, k)}")
+        if not np.array_equal(got, numpy_gemm(A, B, C)):
+            bad.append(f"i4 != numpy matmul on {(m, n, k)}")
+    return bad
+
+
+def check_i4_closed_forms(lib):
+    """Constant operands: every entry of C gains k*a*b."""
+    bad = []
+    for k in (1, 2, 7, 300):
+        for a, b in ((-8, -8), (7, -8), (7, 7), (-1, 1)):
+            m, n = 3, 5
+            Ap = gi.pack_nibbles(np.full((m, k), a, np.int8))
+            Bp = gi.pack_nibbles(np.full((k, n), b, np.int8))
+            got = _run_i4(lib, Ap, Bp, np.zeros((m, n), np.int32), k)
+            if not (got == k * a * b).all():
+                bad.append(f"i4 constant a={a} b={b} k={k}: got {got[0, 0]} want {k * a * b}")
+    return bad
+
+
+I4_CHECKS = (check_i4_golden, check_i4_bruteforce, check_i4_matches_i8, check_i4_closed_forms)
+
 ALL_CHECKS = (check_golden, check_extreme_bruteforce, check_closed_forms, check_identity_permutation,
-              check_blocked, check_padding, check_linearity, check_transpose, check_numpy) + SRS_CHECKS + CONV_CHECKS
+              check_blocked, check_padding, check_linearity, check_transpose, check_numpy) + SRS_CHECKS + CONV_CHECKS + I4_CHECKS
 
 
 def pin_failures(lib, bruteforce_shapes=None):

@@ -70,6 +70,42 @@ def test_conv_im2col_lowering(lib):
     assert pins.check_conv_im2col_lowering(lib) == []
 
 
+def test_i4_golden(lib):
+    assert pins.check_i4_golden(lib) == []
+
+
+def test_i4_bruteforce_tiny_shapes(lib):
+    assert pins.check_i4_bruteforce(lib) == []
+
+
+def test_i4_matches_i8_and_numpy(lib):
+    assert pins.check_i4_matches_i8(lib) == []
+
+
+def test_i4_closed_forms(lib):
+    assert pins.check_i4_closed_forms(lib) == []
+
+
+def test_i4_packer_matches_golden_bytes():
+    """The shared packer stores the format the hand-worked cases spell out byte by byte."""
+    v = np.array([[1, 2, -1, -8, 3]], np.int8)
+    assert gi.pack_nibbles(v).tolist() == [[0x21, 0x8F, 0x03]]
+    assert gi.pack_nibbles(v, ld=4, pad=0x55).tolist() == [[0x21, 0x8F, 0x53, 0x55]]
+
+
+def test_i4_invalid_arguments_rejected(lib):
+    b = np.zeros((4, 4), np.uint8)
+    c = np.zeros((4, 4), np.int32)
+    f = lib.gemm_oracle_i4
+    p, q = b.ctypes.data, c.ctypes.data
+    assert f(2, 3, 3, p, 2, p, 2, q, 3, 1) == 0
+    assert f(2, 3, 3, p, 1, p, 2, q, 3, 1) == 1   # lda < ceil(k/2)
+    assert f(2, 3, 3, p, 2, p, 1, q, 3, 1) == 1   # ldb < ceil(n/2)
+    assert f(2, 3, 3, p, 2, p, 2, q, 2, 1) == 1   # ldc < n
+    assert f(2, 3, 3, 0, 2, p, 2, q, 3, 1) == 1   # null A
+    assert f(2, 3, 0, 0, 0, 0, 0, q, 3, 1) == 0   # k = 0: C unchanged, A and B unused
+
+
 def test_closed_forms(lib):
     assert pins.check_closed_forms(lib) == []
 
@@ -170,6 +206,16 @@ MUTANTS = {
                                            "const int64_t w = (wo + s - pad_w + W) % W;"),
     "conv_drops_last_channel": ("for (int64_t c = 0; c < Cin; ++c) {\n            const int64_t a = (int64_t)x[c];",
                                 "for (int64_t c = 0; c + 1 < Cin; ++c) {\n            const int64_t a = (int64_t)x[c];"),
+    # the int4 variant
+    "i4_nibble_order_swapped": ("(idx % 2 == 0) ? (byte & 15u) : (byte >> 4)", "(idx % 2 == 0) ? (byte >> 4) : (byte & 15u)"),
+    "i4_unsigned_nibbles": ("return v >= 8 ? (int64_t)v - 16 : (int64_t)v;", "return (int64_t)v;"),
+    "i4_sign_threshold_off_by_one": ("return v >= 8 ? (int64_t)v - 16 : (int64_t)v;", "return v > 8 ? (int64_t)v - 16 : (int64_t)v;"),
+    "i4_row_pitch_in_elements": ("oracle_nibble(A + i * lda, p)", "oracle_nibble(A + i * lda / 2, p)"),
+    "i4_ignores_ldb": ("oracle_nibble(B + p * ldb, j)", "oracle_nibble(B + p * ((n + 1) / 2), j)"),
+    "i4_drops_last_term": ("for (int64_t p = 0; p < k; ++p)\n        s += (uint64_t)(oracle_nibble",
+                           "for (int64_t p = 0; p + 1 < k; ++p)\n        s += (uint64_t)(oracle_nibble"),
+    "i4_wraps_at_16_bits": ("s += (uint64_t)(oracle_nibble(A + i * lda, p) * oracle_nibble(B + p * ldb, j));\n      c[j] = (int32_t)(uint32_t)s;",
+                            "s += (uint64_t)(oracle_nibble(A + i * lda, p) * oracle_nibble(B + p * ldb, j));\n      c[j] = (int32_t)(int16_t)s;"),
     "conv_channel_stride_is_cout": ("const int16_t* x = X + ((n * H + h) * W + w) * Cin;",
                                     "const int16_t* x = X + ((n * H + h) * W + w) * Cout;"),
 }
