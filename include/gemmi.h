@@ -82,6 +82,30 @@ int gemm_i8_ex(int64_t m, int64_t n, int64_t k,
                int32_t* C, int64_t ldc, void* stream);
 
 /*
+ * gemm_i4 -- C (int32) += A (int4) * B (int4), exactly, modulo 2^32.
+ * Section 4.1 (problem statement) at a precision below the INT16 / INT8 of Section 6.1; the
+ * paper's datatype discussion (Section 5.1) leaves the lower-precision micro-kernel to future work.
+ * Operands are PACKED, two signed 4-bit values to a byte: element (i, p) of A is in byte
+ * A[i*lda + p/2], element (p, j) of B in byte B[p*ldb + j/2]; the even index in the low nibble
+ * (bits 0-3), the odd one in the high nibble (bits 4-7), two's complement (nibbles 8..15 stand
+ * for -8..-1).  lda and ldb count BYTES: lda >= max(1, ceil(k/2)), ldb >= max(1, ceil(n/2));
+ * ldc counts int32 elements, ldc >= max(1, n).  The spare high nibble of a row's last byte (odd
+ * k for A, odd n for B) and the bytes of the row padding are never read.
+ * Same pointer ownership (DEVICE pointers owned by the caller), stream, workspace and error
+ * behaviour as gemm_i16.  A C whose base is not 16-byte aligned, or whose ldc is not a multiple
+ * of 4, is accumulated through a zeroed scratch array in the workspace and added in one more pass.
+ */
+int gemm_i4(int64_t m, int64_t n, int64_t k,
+            const uint8_t* A, int64_t lda,
+            const uint8_t* B, int64_t ldb,
+            int32_t* C, int64_t ldc);
+
+int gemm_i4_ex(int64_t m, int64_t n, int64_t k,
+               const uint8_t* A, int64_t lda,
+               const uint8_t* B, int64_t ldb,
+               int32_t* C, int64_t ldc, void* stream);
+
+/*
  * gemm_i16_host / gemm_i8_host -- the same GEMMs on HOST buffers.
  * A, B, C are host pointers (pinned memory gives the fastest copies).  The
  * library copies A, B and C to device buffers it owns, runs the GEMM on its
@@ -208,6 +232,8 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_TC_CHUNK_SCALE : length of the exact fp32 accumulation runs of the tensor-core
  *                            GEMM: 2 (default) keeps every partial limb sum within 2^24, the limit
  *                            of exact fp32 integer sums; 1 keeps it within 2^23 (twice the drains).
+ *                            gemm_i4: 2 drains every 2^18 reduction indices (sums within 2^24),
+ *                            1 every 256 (sums within 2^14).
  *   GEMMI_OPT_TC_GROUP_M   : tile raster band height in 128-row tiles (default 16).
  *   GEMMI_OPT_TC_L2_HINTS  : L2 eviction policy of the operand tile loads, bits 0-1 for A,
  *                            bits 2-3 for B: 0 normal, 1 evict_last, 2 evict_first (default 0).
@@ -252,10 +278,14 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_SRS     : the requantising pass of gemm_i16_srs
  *   GEMMI_KERNEL_TC_PAIR_I16 : the tcgen05 int16 GEMM kernel on SM pairs
  *   GEMMI_KERNEL_TC_PAIR_I8  : the tcgen05 int8 GEMM kernel on SM pairs
+ *   GEMMI_KERNEL_TC_PAIR_I4  : the tcgen05 int4 GEMM kernel on SM pairs (E4M3 operands)
+ *   GEMMI_KERNEL_ADD_I32     : gemm_i4's add of its scratch result into a C that the pair
+ *                              kernel cannot reduce into directly
+ * (gemm_i4's operand conversion counts as GEMMI_KERNEL_SPLIT.)
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
        GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_TC_PAIR_I16 = 6, GEMMI_KERNEL_TC_PAIR_I8 = 7,
-       GEMMI_KERNEL_COUNT = 8 };
+       GEMMI_KERNEL_TC_PAIR_I4 = 8, GEMMI_KERNEL_ADD_I32 = 9, GEMMI_KERNEL_COUNT = 10 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

@@ -31,13 +31,14 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
-            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex", "gemmi_conv2d_i16")
+            "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex", "gemmi_conv2d_i16",
+            "gemm_i4", "gemm_i4_ex")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
-KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8 = 6, 7
+KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8, KERNEL_TC_PAIR_I4, KERNEL_ADD_I32 = 6, 7, 8, 9
 KERNELS = (("split", KERNEL_SPLIT), ("tc_i16", KERNEL_TC_I16), ("tc_i8", KERNEL_TC_I8), ("skinny", KERNEL_SKINNY),
            ("fused_i16", KERNEL_FUSED_I16), ("srs", KERNEL_SRS), ("tc_pair_i16", KERNEL_TC_PAIR_I16),
-           ("tc_pair_i8", KERNEL_TC_PAIR_I8))
+           ("tc_pair_i8", KERNEL_TC_PAIR_I8), ("tc_pair_i4", KERNEL_TC_PAIR_I4), ("add_i32", KERNEL_ADD_I32))
 
 _lib = None
 
@@ -63,10 +64,10 @@ def lib():
         L = ctypes.CDLL(LIB_PATH)
         i64, vp = ctypes.c_int64, ctypes.c_void_p
         core = [i64, i64, i64, vp, i64, vp, i64, vp, i64]
-        for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host"):
+        for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host", "gemm_i4"):
             getattr(L, name).argtypes = core
             getattr(L, name).restype = ctypes.c_int
-        for name in ("gemm_i16_ex", "gemm_i8_ex", "gemm_i16_noalloc"):
+        for name in ("gemm_i16_ex", "gemm_i8_ex", "gemm_i16_noalloc", "gemm_i4_ex"):
             getattr(L, name).argtypes = core + [vp]
             getattr(L, name).restype = ctypes.c_int
         L.gemm_i16_srs.argtypes = core + [ctypes.c_int]
@@ -230,6 +231,36 @@ def gemm_i8(A, B, C, stream=None):
     """C += A @ B on the GPU: int8 A, int8 B, int32 C; exact modulo 2^32."""
     import torch
     return _torch_call("gemm_i8_ex", A, B, C, torch.int8, torch.int32, stream)
+
+
+def gemm_i4(A, B, C, k, stream=None):
+    """C += A @ B on the GPU for signed 4-bit A (m x k) and B (k x n) packed two to a byte; int32 C,
+    exact modulo 2^32.
+
+    A: uint8 CUDA tensor (m, >= ceil(k/2)), element (i, p) in byte p // 2 of row i (low nibble for
+    even p, high for odd p, two's complement); B: uint8 (k, >= ceil(n/2)) packed the same way
+    along its rows; C: int32 (m, n).  k is passed because an odd k leaves a spare nibble per row.
+    """
+    import torch
+    for t, nm, dt in ((A, "A", torch.uint8), (B, "B", torch.uint8), (C, "C", torch.int32)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda:
+            raise TypeError(f"{nm} must be a CUDA tensor")
+        if t.dtype != dt:
+            raise TypeError(f"{nm} must be {dt}, got {t.dtype}")
+    if not (A.device == B.device == C.device):
+        raise ValueError("A, B and C must be on the same device")
+    m, n = C.shape
+    k = int(k)
+    if A.dim() != 2 or B.dim() != 2 or A.shape[0] != m or B.shape[0] != k or A.shape[1] < (k + 1) // 2 \
+            or B.shape[1] < (n + 1) // 2:
+        raise ValueError(f"shape mismatch: packed A {tuple(A.shape)}, packed B {tuple(B.shape)}, C {tuple(C.shape)}, k {k}")
+    if stream is None:
+        stream = torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = lib().gemm_i4_ex(m, n, k, A.data_ptr(), _dev_ld(A, "A"), B.data_ptr(), _dev_ld(B, "B"),
+                              C.data_ptr(), _dev_ld(C, "C"), stream.cuda_stream)
+    _check(rc)
+    return C
 
 
 # ------------------------------------------------------------------ pre-packed weights

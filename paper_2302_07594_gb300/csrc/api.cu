@@ -528,6 +528,76 @@ int gemm_i8_locked(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda
   return run_tc(*d, 1, m, n, k, A, lda, B, ldb, C, ldc, s);
 }
 
+// The int4 path (int4.cu, gemm_pair.cu): the packed operands become K-major E4M3 planes in the
+// workspace (pitch k rounded up to 16 bytes), then the pair kernel runs on kind::f8f6f4.  A C that
+// cannot take 16-byte bulk reductions gets a zeroed scratch result that one more pass adds into it.
+int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+                   int32_t* C, int64_t ldc, cudaStream_t s) {
+  if (m < 0 || n < 0 || k < 0) return set_error(GEMMI_EINVAL, "negative matrix dimension");
+  const int64_t wa = (k + 1) / 2, wb = (n + 1) / 2;  // packed bytes per row of A and of B
+  if (ldc < std::max<int64_t>(1, n)) return set_error(GEMMI_EINVAL, "ldc < max(1, n)");
+  if (lda < std::max<int64_t>(1, wa)) return set_error(GEMMI_EINVAL, "lda < max(1, ceil(k/2)) bytes");
+  if (ldb < std::max<int64_t>(1, wb)) return set_error(GEMMI_EINVAL, "ldb < max(1, ceil(n/2)) bytes");
+  if (m == 0 || n == 0) return GEMMI_OK;
+  if (C == nullptr) return set_error(GEMMI_EINVAL, "C is null");
+  if (k == 0) return GEMMI_OK;
+  if (A == nullptr || B == nullptr) return set_error(GEMMI_EINVAL, "A or B is null");
+  if (m > (int64_t(1) << 40) || n > (int64_t(1) << 31) || k > (int64_t(1) << 31))
+    return set_error(GEMMI_EINVAL, "matrix dimension too large");
+  const size_t a_bytes = static_cast<size_t>((m - 1) * lda + wa);
+  const size_t b_bytes = static_cast<size_t>((k - 1) * ldb + wb);
+  const size_t c_bytes = static_cast<size_t>((m - 1) * ldc + n) * 4;
+  if (overlaps(C, c_bytes, A, a_bytes) || overlaps(C, c_bytes, B, b_bytes))
+    return set_error(GEMMI_EINVAL, "C overlaps A or B");
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 16));
+  const size_t a_plane = round_up(static_cast<size_t>(m) * pitch, kAlign);
+  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch, kAlign);
+  const bool direct = reinterpret_cast<uintptr_t>(C) % 16 == 0 && ldc % 4 == 0;
+  const int64_t ldt = static_cast<int64_t>(round_up(static_cast<size_t>(n), 4));
+  const size_t t_bytes = direct ? 0 : static_cast<size_t>(m) * ldt * 4;
+  if ((rc = ensure_buffer(&d->ws, &d->ws_bytes, a_plane + b_plane + t_bytes)) != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(*d, s)) != GEMMI_OK) return rc;
+  char* ws = static_cast<char*>(d->ws);
+  const LimbPlanes pa{{ws, nullptr}, m, pitch};
+  const LimbPlanes pb{{ws + a_plane, nullptr}, n, pitch};
+  int32_t* T = direct ? nullptr : reinterpret_cast<int32_t*>(ws + a_plane + b_plane);
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+  cudaError_t e = gemmi::convert_i4(A, lda, B, ldb, m, n, k, pa, pb, d->sm_count, s);
+  timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, "int4 operand conversion launch");
+  if (!direct && (e = cudaMemsetAsync(T, 0, t_bytes, s)) != cudaSuccess) return cuda_error(e, "cudaMemsetAsync");
+  gemmi::TcGemmArgs ta;
+  ta.m = m;
+  ta.n = n;
+  ta.k = k;
+  ta.a = pa;
+  ta.b = pb;
+  ta.C = direct ? static_cast<void*>(C) : static_cast<void*>(T);
+  ta.ldc = direct ? ldc : ldt;
+  ta.status = d->status;
+  ta.timeout_ns = timeout_ns();
+  ta.num_sms = d->sm_count;
+  ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
+  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
+  ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
+  const char* why = "tcgen05 int4 GEMM launch";
+  cudaEvent_t t1 = timer_begin(GEMMI_KERNEL_TC_PAIR_I4, s);
+  e = gemmi::tc_pair_gemm_i4(ta, s, &why);
+  timer_end(GEMMI_KERNEL_TC_PAIR_I4, t1, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  if (!direct) {
+    cudaEvent_t t2 = timer_begin(GEMMI_KERNEL_ADD_I32, s);
+    e = gemmi::add_into_i32(C, ldc, T, ldt, m, n, d->sm_count, s);
+    timer_end(GEMMI_KERNEL_ADD_I32, t2, s);
+    if (e != cudaSuccess) return cuda_error(e, "int4 scratch add launch");
+  }
+  return end_workspace_use(*d, s);
+}
+
 int read_status_locked(DeviceState& d, bool clear) {
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
@@ -763,6 +833,18 @@ int gemm_i8(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const
             int32_t* C, int64_t ldc) {
   std::lock_guard<std::mutex> lock(g_mutex);
   return gemm_i8_locked(m, n, k, A, lda, B, ldb, C, ldc, g_stream);
+}
+
+int gemm_i4_ex(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+               int32_t* C, int64_t ldc, void* stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i4_locked(m, n, k, A, lda, B, ldb, C, ldc, static_cast<cudaStream_t>(stream));
+}
+
+int gemm_i4(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+            int32_t* C, int64_t ldc) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  return gemm_i4_locked(m, n, k, A, lda, B, ldb, C, ldc, g_stream);
 }
 
 int gemm_i16_host(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb,

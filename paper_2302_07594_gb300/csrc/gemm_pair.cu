@@ -18,6 +18,9 @@
 //          SM A_low * [B_high | B_low] (weights 2^8 | 1) for one 128 x 128 output tile.
 //   int8:  a 256 x 256 output tile; each SM holds 128 rows of A and 128 rows (output columns)
 //          of B, and accumulates its 128 rows x all 256 columns.
+//   int4:  the int8 geometry on E4M3 planes (int4.cu) with tcgen05.mma kind::f8f6f4, K = 32 per
+//          instruction: a K block is 128 one-byte elements, the same 128 bytes per operand row,
+//          so tiles, stages and descriptors are those of the fp16 planes, at twice the MMA rate.
 // Per K block of 64 each SM loads 32 KB (its A tile and its B tile) for 512 tensor cycles: 64 B
 // per cycle from L2, where a single-SM 128 x 256 int8 tile needs 96.
 //
@@ -167,11 +170,10 @@ struct PairSched {
 // on the CTA's A limb: 2^16 | 2^8 in the even CTA, 2^8 | 1 in the odd one.  Both CTAs drain
 // with the odd CTA's weights (one code path, constant shifts) and the even CTA scales its tile's
 // sums by 2^8 when it adds them into C: shifting commutes with addition modulo 2^64.
-template <int NL, int CS>
+template <int NL, int KPC>
 __device__ __forceinline__ void epilogue(const PairParams& P, const CUtensorMap* cmap, uint32_t rank,
                                          uint32_t tmem_base, uint32_t sfull0, uint32_t sempty_leader0, uint8_t* stg,
                                          int pair, int npairs) {
-  constexpr int KPC = 8 * CS;
   const uint32_t tile_shift = (NL == 2 && rank == 0) ? 8u : 0u;
   using G = PairGeom<NL>;
   using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
@@ -278,13 +280,25 @@ __device__ __forceinline__ void epilogue(const PairParams& P, const CUtensorMap*
   if (lane == 0) bulk_wait_all();
 }
 
-template <int NL, int CS>
+// K blocks per exact chunk.  fp16 limbs: a K block is 64 indices of products of magnitude <= 2^14,
+// so 8 * CS blocks keep every fp32 partial sum within 2^(23 + CS - 1).  E4M3 int4 values: a K block
+// is 128 indices of products <= 2^6; CS = 2 gives 2048 blocks (2^18 indices, sums <= 2^24), CS = 1
+// two blocks (256 indices, sums <= 2^14).  Every length is a multiple of KPS.
+template <int CS, bool F8>
+__host__ __device__ constexpr int chunk_kblocks() {
+  return F8 ? (CS == 2 ? 2048 : 2) : 8 * CS;
+}
+
+template <int NL, int CS, bool F8>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
                const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1,
                const __grid_constant__ CUtensorMap mapC, PairParams P) {
   using G = PairGeom<NL>;
-  constexpr int KPC = 8 * CS;  // K blocks per exact chunk: 512 * CS reduction indices
+  static_assert(!F8 || NL == 1, "the E4M3 path has one plane per operand");
+  constexpr int KPC = chunk_kblocks<CS, F8>();
+  static_assert(KPC % KPS == 0, "chunks end on stage boundaries");
+  constexpr int BKE = F8 ? 2 * BK : BK;  // elements per K block: 128 bytes of a row either way
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -369,8 +383,8 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           for (int j = 0; j < KPS; ++j) {
             if (j >= nsub) break;
             const uint32_t base = smem_u32(smem + st.slot * SB + j * SBK);
-            load_pair(base, ma, fb, (kb + j) * BK, arow, P.hint_a, pol_a);
-            load_pair(base + TILE_A, mb, fb, (kb + j) * BK, brow, P.hint_b, pol_b);
+            load_pair(base, ma, fb, (kb + j) * BKE, arow, P.hint_a, pol_a);
+            load_pair(base + TILE_A, mb, fb, (kb + j) * BKE, brow, P.hint_b, pol_b);
           }
           ++issued;
           st.advance(STAGES);
@@ -386,7 +400,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     // ------------------------------------------------------------ MMA issue (even CTA, one thread)
     if (lane == 0) {
       if (leader) {
-        constexpr uint32_t idesc = idesc_f16_f32(UMMA_M, UMMA_N);
+        constexpr uint32_t idesc = F8 ? idesc_e4m3_f32(UMMA_M, UMMA_N) : idesc_f16_f32(UMMA_M, UMMA_N);
         tc::RingPos st;
         int chunk = 0;
         bool ok = true;
@@ -423,8 +437,11 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
                 const uint64_t bdesc = smem_desc_kmajor<SWIZZLE>(base + TILE_A);
 #pragma unroll
                 for (int kk = 0; kk < BK / UMMA_K; ++kk) {
-                  // advancing the start address by 32 bytes (16 fp16) steps K inside the swizzled row
-                  tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb + j == cb0 && kk == 0) ? 0u : 1u);
+                  // advancing the start address by 32 bytes (16 fp16 or 32 E4M3) steps K inside the
+                  // swizzled row
+                  const uint32_t acc = (kb + j == cb0 && kk == 0) ? 0u : 1u;
+                  if constexpr (F8) tc_mma_f8_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, acc);
+                  else tc_mma_f16_pair(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, acc);
                 }
               }
               tc_commit_pair(empty0 + 8 * st.slot, 0x3);  // stage free in both CTAs once read
@@ -442,7 +459,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..7)
     const uint32_t sempty_leader0 = map_to_rank(sempty0, 0);
-    epilogue<NL, CS>(P, &mapC, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs);
+    epilogue<NL, KPC>(P, &mapC, rank, tmem_base, sfull0, sempty_leader0, stg, pair, npairs);
   }
 
   // Pair handshake: neither CTA exits (or frees tensor memory) while its peer may still signal it.
@@ -460,17 +477,19 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 }
 
 // ---------------------------------------------------------------- host side
-template <int NL, int CS>
+template <int NL, int CS, bool F8>
 cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   using G = PairGeom<NL>;
+  constexpr int BKE = F8 ? 2 * BK : BK;
+  constexpr int OPSZ = F8 ? 1 : 2;  // bytes per plane element
   CUtensorMap maps[4];
   const LimbPlanes* ops[2] = {&a.a, &a.b};
   for (int o = 0; o < 2; ++o) {
     for (int l = 0; l < 2; ++l) {
       const void* base = ops[o]->plane[l < NL ? l : 0];
-      if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
-                                static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
-                                HALF, SWIZZLE, why))
+      if (!encode_tensor_map_2d(&maps[2 * o + l], F8 ? 2 : 1, base, static_cast<uint64_t>(a.k),
+                                static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * OPSZ,
+                                BKE, HALF, SWIZZLE, why))
         return cudaErrorInvalidValue;
     }
   }
@@ -488,7 +507,7 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   P.ldc = a.ldc;
   P.num_m_tiles = static_cast<int>((a.m + G::TM - 1) / G::TM);
   P.num_n_tiles = static_cast<int>((a.n + G::TN - 1) / G::TN);
-  P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
+  P.num_k_blocks = static_cast<int>((a.k + BKE - 1) / BKE);
   P.group_m = a.group_m > 0 ? a.group_m : 16;
   P.hint_a = a.hint_a;
   P.hint_b = a.hint_b;
@@ -496,7 +515,7 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   P.status = a.status;
   const int64_t tiles = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles;
 
-  auto kernel = tc_pair_kernel<NL, CS>;
+  auto kernel = tc_pair_kernel<NL, CS, F8>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -540,10 +559,13 @@ cudaError_t launch_pair(const TcGemmArgs& a, cudaStream_t s, const char** why) {
 }  // namespace
 
 cudaError_t tc_pair_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why) {
-  return args.chunk_scale == 2 ? launch_pair<2, 2>(args, s, why) : launch_pair<2, 1>(args, s, why);
+  return args.chunk_scale == 2 ? launch_pair<2, 2, false>(args, s, why) : launch_pair<2, 1, false>(args, s, why);
 }
 cudaError_t tc_pair_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) {
-  return args.chunk_scale == 2 ? launch_pair<1, 2>(args, s, why) : launch_pair<1, 1>(args, s, why);
+  return args.chunk_scale == 2 ? launch_pair<1, 2, false>(args, s, why) : launch_pair<1, 1, false>(args, s, why);
+}
+cudaError_t tc_pair_gemm_i4(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch_pair<1, 2, true>(args, s, why) : launch_pair<1, 1, true>(args, s, why);
 }
 
 }  // namespace gemmi

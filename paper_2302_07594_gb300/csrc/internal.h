@@ -52,6 +52,18 @@ cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why)
 // bulk reductions: C 16-byte aligned and ldc * sizeof(C element) a multiple of 16.
 cudaError_t tc_pair_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_pair_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
+// int4: args.a / args.b hold one E4M3 plane each (int4.cu), pitch in bytes; C is int32.
+cudaError_t tc_pair_gemm_i4(const TcGemmArgs& args, cudaStream_t s, const char** why);
+
+// ---- int4.cu: packed int4 operands -> K-major E4M3 planes (pitch in bytes, a multiple of 16).
+// A: m x k values, two per byte along the row (even index in the low nibble), row pitch lda bytes;
+// B: k x n values packed along its rows (pitch ldb bytes), written transposed (rows = n).
+// A null A (or B) skips that operand.
+cudaError_t convert_i4(const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
+                       LimbPlanes pa, LimbPlanes pb, int num_sms, cudaStream_t s);
+// C (m x n, pitch ldc) += T (pitch ldt), int32 modulo 2^32.
+cudaError_t add_into_i32(int32_t* C, int64_t ldc, const int32_t* T, int64_t ldt, int64_t m, int64_t n, int num_sms,
+                         cudaStream_t s);
 
 // ---- gemm_fused.cu: int16 GEMM, n <= 64 per tile column, A read raw (int16) and split on chip.
 struct FusedArgs {

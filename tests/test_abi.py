@@ -81,6 +81,23 @@ def test_empty_problems_are_noops(L):
     assert L.gemm_i16(3, 3, 0, None, 1, None, 3, ctypes.c_void_p(0x3000), 3) == gm.OK
 
 
+def test_i4_argument_checks(L):
+    """gemm_i4 counts lda and ldb in packed bytes: ceil(k/2) and ceil(n/2) are the minimums."""
+    a, b, c = ctypes.c_void_p(0x1000), ctypes.c_void_p(0x90000), ctypes.c_void_p(0x200000)
+    assert L.gemm_i4(4, 5, 7, a, 3, b, 3, c, 5) == gm.EINVAL       # lda < ceil(7/2) = 4
+    assert "lda" in gm.last_error()
+    assert L.gemm_i4(4, 5, 7, a, 4, b, 2, c, 5) == gm.EINVAL       # ldb < ceil(5/2) = 3
+    assert "ldb" in gm.last_error()
+    assert L.gemm_i4(4, 5, 7, a, 4, b, 3, c, 4) == gm.EINVAL       # ldc < n
+    assert L.gemm_i4(-1, 5, 7, a, 4, b, 3, c, 5) == gm.EINVAL
+    assert L.gemm_i4(4, 5, 7, None, 4, b, 3, c, 5) == gm.EINVAL
+    assert L.gemm_i4(4, 5, 7, a, 4, b, 3, ctypes.c_void_p(0x1002), 5) == gm.EINVAL  # C overlaps A
+    assert "overlap" in gm.last_error()
+    # empty problems and k == 0 are no-ops that touch no device
+    assert L.gemm_i4(0, 5, 7, None, 4, None, 3, None, 5) == gm.OK
+    assert L.gemm_i4(4, 5, 0, None, 1, None, 3, c, 5) == gm.OK
+
+
 def test_options(L):
     old = gm.get_option(gm.OPT_SKINNY_MAX_M)
     gm.set_option(gm.OPT_SKINNY_MAX_M, 4)
