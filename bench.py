@@ -45,7 +45,12 @@ KERNEL_INFO = {
     "srs": ("srs_add_kernel", ("requant.cu",), "hbm"),
     "tc_pair_i16": ("tc_pair_kernel<2>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "tensor"),
     "tc_pair_i8": ("tc_pair_kernel<1>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "tensor"),
+    "tc_pair_i4": ("tc_pair_kernel<1,e4m3>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"),
+                   "tensor"),
+    "add_i32": ("add_i32", ("int4.cu",), "hbm"),
+    "convert_i4": ("convert_rows_i4+convert_cols_i4", ("int4.cu",), "hbm"),
 }
+FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
 
 
 def parse_args():
@@ -58,7 +63,7 @@ def parse_args_list(argv):
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=("gemmi", "reference"), default="gemmi")
-    p.add_argument("--workload", default="i16_8192", choices=list(gi.WORKLOADS))
+    p.add_argument("--workload", default="i16_8192", choices=[n for n, w in gi.WORKLOADS.items() if w.kind != "i4"])
     p.add_argument("--no-extra", action="store_true", help="skip the per-workload table")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU budget of the oracle baseline")
@@ -147,9 +152,11 @@ def recorded_traffic(kernel: str, src_hash: str):
 
 
 def workload_bytes(w):
-    """Algorithmic HBM bytes of one call: read A, B and C once, write C once."""
-    op = 2 if w.kind == "i16" else 1
+    """Algorithmic HBM bytes of one call: read A, B and C once, write C once (int4 operands packed)."""
     cb = 8 if w.kind == "i16" else 4
+    if w.kind == "i4":
+        return w.m * ((w.k + 1) // 2) + w.k * ((w.n + 1) // 2) + 2 * w.m * w.n * cb
+    op = 2 if w.kind == "i16" else 1
     return w.m * w.k * op + w.k * w.n * op + 2 * w.m * w.n * cb
 
 
@@ -285,7 +292,11 @@ def time_workload_packed(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES,
     nsets = int(min(max_sets, max(1, math.ceil(rotate_bytes / per_set))))
     A, B, C = gi.make_inputs(w)
     sets, packs = [], []
-    pack = gm.pack_b_i16 if w.kind == "i16" else gm.pack_b_i8
+    if w.kind == "i4":
+        A, B = gi.pack_nibbles(A), gi.pack_nibbles(B)
+        pack = lambda b: gm.pack_b_i4(b, w.n)  # noqa: E731
+    else:
+        pack = gm.pack_b_i16 if w.kind == "i16" else gm.pack_b_i8
     for _ in range(nsets):
         dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
         pk = pack(dB)
@@ -293,7 +304,7 @@ def time_workload_packed(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES,
         packs.append(pk)
         sets.append((dA, pk, dC))
     torch.cuda.synchronize()
-    fn = gm.gemm_i16_packed if w.kind == "i16" else gm.gemm_i8_packed
+    fn = {"i16": gm.gemm_i16_packed, "i8": gm.gemm_i8_packed, "i4": gm.gemm_i4_packed}[w.kind]
     graph_ms, eager_ms, kt = _time_calls(gm, torch, sets, fn, steps, warmup)
     del sets
     for pk in packs:
@@ -343,8 +354,13 @@ def time_workload(gm, torch, w, steps, warmup, rotate_bytes=4 * L2_BYTES, max_se
     per_set = workload_bytes(w)
     nsets = int(min(max_sets, max(1, math.ceil(rotate_bytes / per_set))))
     A, B, C = gi.make_inputs(w)
+    if w.kind == "i4":
+        A, B = gi.pack_nibbles(A), gi.pack_nibbles(B)
     sets = [tuple(torch.from_numpy(x).cuda() for x in (A, B, C)) for _ in range(nsets)]
-    fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
+    if w.kind == "i4":
+        fn = lambda a, b, c: gm.gemm_i4(a, b, c, w.k)  # noqa: E731
+    else:
+        fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
     graph_ms, eager_ms, kt = _time_calls(gm, torch, sets, fn, steps, warmup)
     del sets
     torch.cuda.empty_cache()
@@ -520,10 +536,14 @@ def run_gemmi(args):
                                 for name in KERNEL_INFO if okt[name][1] > 0}
             if ow.kind == "i8":
                 ent["frac_of_fp16_tensor_peak"] = ent["TOPS"] / peaks["bf16_tflops"]
+            elif ow.kind == "i4":
+                ent["frac_of_fp8_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] * FP8_PER_BF16)
+                ent["fp8_peak_note"] = (f"bf16 burst {peaks['bf16_tflops']} TFLOP/s ({peaks['source']}) x "
+                                        f"{FP8_PER_BF16} (nominal fp8 / bf16 dense rate)")
             else:
                 ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
                 ent["frac_of_hbm"] = ent["GB_per_s"] / peaks["hbm_gbs"]
-            if int8_peak:
+            if int8_peak and ow.kind != "i4":
                 ent["frac_of_int8_roofline_div4" if ow.kind == "i16" else "frac_of_int8_roofline"] = (
                     ent["TOPS"] / (int8_peak / 4 if ow.kind == "i16" else int8_peak))
             if name.startswith("skinny"):
@@ -539,7 +559,7 @@ def run_gemmi(args):
             extra[name] = ent
         # the same calls with the weights split once (gemmi_pack_b_*): the operand split then covers
         # A only, and the narrow-n kernel has no split at all
-        for name in ("i16_8192", "i8_4096", "conv3x3_im2col"):
+        for name in ("i16_8192", "i8_4096", "conv3x3_im2col", "i4_8192"):
             ow = gi.WORKLOADS[name]
             try:
                 oms, eager_ms, okt, nsets = time_workload_packed(gm, torch, ow, steps=30 if ow.ops > 1e11 else 128,
@@ -552,9 +572,28 @@ def run_gemmi(args):
                    "kernel_ms": {KERNEL_INFO[k][0]: okt[k][0] / okt[k][1] for k in KERNEL_INFO if okt[k][1] > 0}}
             if ow.kind == "i8":
                 ent["frac_of_fp16_tensor_peak"] = ent["TOPS"] / peaks["bf16_tflops"]
+            elif ow.kind == "i4":
+                ent["frac_of_fp8_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] * FP8_PER_BF16)
             else:
                 ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
             extra[name + "_packed_b"] = ent
+        # the precision sweep at equal sizes: int8 at 8192^3 and int4 at 4096^3 beside the table's
+        # int16 / int4 8192^3 and int8 4096^3 (same value distributions as those workloads)
+        sweep = {}
+        for sw in (gi.Workload("i8_8192", "i8", 8192, 8192, 8192, 1008, ("uniform", -128, 127),
+                               ("uniform", -128, 127), ("zero",), "int8 GEMM 8192^3"),
+                   gi.Workload("i4_4096", "i4", 4096, 4096, 4096, 1009, ("uniform", -8, 7), ("uniform", -8, 7),
+                               ("zero",), "int4 GEMM 4096^3")):
+            try:
+                sms, seager, skt, sn = time_workload(gm, torch, sw, steps=30, warmup=5)
+            except Exception as ex:  # pragma: no cover
+                sweep[sw.name] = {"error": str(ex)}
+                continue
+            sweep[sw.name] = {"ms": sms, "timing": "CUDA-graph replay, per call", "eager_ms": seager,
+                              "TOPS": sw.ops / (sms * 1e-3) / 1e12, "input_sets_rotated": sn,
+                              "kernel_ms": {KERNEL_INFO[k][0]: skt[k][0] / skt[k][1] for k in KERNEL_INFO
+                                            if skt[k][1] > 0}}
+        extra["precision_sweep"] = sweep
         try:
             cms, ceager, ckt, cn = time_conv(gm, torch, steps=128, warmup=5)
             ops = 2 * CONV["N"] * CONV["H"] * CONV["W"] * CONV["Cout"] * CONV["R"] * CONV["S"] * CONV["Cin"]

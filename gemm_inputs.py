@@ -18,10 +18,12 @@ im2col activation matrix of the 3x3-convolution workload is 50% exact zeros:
 the top bit of r decides zero / non-zero and the non-zero branch takes
 r mod 4096, so P(value == 0) = 0.5 + 0.5/4096.
 
-The five workloads (matrix shapes, operand types and value distributions) are
+The workloads (matrix shapes, operand types and value distributions) are
 those of the GEMM problem of Section 4.1 of the paper at the sizes the
 benchmark studies; the paper itself uses INT16 operands (Section 6.1) and
 lowers convolutions to GEMM through IM2COL/IM2ROW (Sections 2, 4.2, 5.1).
+The int4 workload is the lower-precision point the paper leaves to future
+work (Section 5.1).
 Matrix X of workload w is drawn from stream 4*seed_w + {A: 0, B: 1, C: 2}.
 """
 from __future__ import annotations
@@ -74,7 +76,8 @@ def half_zero_uniform(seed: int, shape, hi: int, dtype) -> np.ndarray:
 class Workload:
     """One benchmark workload: C (m x n) += A (m x k) * B (k x n)."""
     name: str
-    kind: str          # "i16" (int16 operands, int64 C) or "i8" (int8 operands, int32 C)
+    kind: str          # "i16" (int16 operands, int64 C), "i8" (int8, int32 C) or "i4" (int4 values held
+                       # one per int8 element, stored packed two to a byte by pack_nibbles; int32 C)
     m: int
     n: int
     k: int
@@ -114,6 +117,8 @@ WORKLOADS = {
                          "int16 GEMM 8192^3, full-range operands, C int64 = 0"),
     "skinny_8x4096x4096": Workload("skinny_8x4096x4096", "i16", 8, 4096, 4096, 1005, FULL16, FULL16,
                                    ("zero",), "batch-8 fully-connected layer, m=8, n=k=4096"),
+    "i4_8192": Workload("i4_8192", "i4", 8192, 8192, 8192, 1007, ("uniform", -8, 7), ("uniform", -8, 7), ("zero",),
+                        "int4 GEMM 8192^3 (the lower-precision point), operands uniform in [-8, 7], C int32 = 0"),
 }
 
 

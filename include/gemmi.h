@@ -181,7 +181,9 @@ int gemmi_conv2d_i16(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout,
  * DEVICE pointer, only read) once into the library's internal limb planes,
  * held in device memory the handle owns (allocated by this call), on `stream`.
  * gemm_*_packed then computes C += A * B for any A (m x k) with that B,
- * converting only A per call; the result is bit-identical to gemm_i16/gemm_i8.
+ * converting only A per call; the result is bit-identical to gemm_i16/gemm_i8/gemm_i4.
+ * gemmi_pack_b_i4 takes B in gemm_i4's packed-nibble format (ldb in bytes,
+ * >= ceil(n/2)) and gemm_i4_packed an A in that format (lda >= ceil(k/2) bytes).
  * Packed GEMMs always take the tensor-core path (for m <= 16, gemm_i16 on the
  * raw B streams fewer bytes).  The handle belongs to the device that was
  * current when it was made; gemmi_packed_b_free() synchronises that device and
@@ -194,6 +196,9 @@ int gemmi_pack_b_i8(int64_t k, int64_t n, const int8_t* B, int64_t ldb, void* st
 int gemm_i16_packed(int64_t m, const int16_t* A, int64_t lda, const gemmi_packed_b* B, int64_t* C, int64_t ldc,
                     void* stream);
 int gemm_i8_packed(int64_t m, const int8_t* A, int64_t lda, const gemmi_packed_b* B, int32_t* C, int64_t ldc,
+                   void* stream);
+int gemmi_pack_b_i4(int64_t k, int64_t n, const uint8_t* B, int64_t ldb, void* stream, gemmi_packed_b** out);
+int gemm_i4_packed(int64_t m, const uint8_t* A, int64_t lda, const gemmi_packed_b* B, int32_t* C, int64_t ldc,
                    void* stream);
 int gemmi_packed_b_free(gemmi_packed_b* packed);
 /* k and n of a packed operand (0 for a null handle). */
@@ -281,11 +286,12 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_TC_PAIR_I4  : the tcgen05 int4 GEMM kernel on SM pairs (E4M3 operands)
  *   GEMMI_KERNEL_ADD_I32     : gemm_i4's add of its scratch result into a C that the pair
  *                              kernel cannot reduce into directly
- * (gemm_i4's operand conversion counts as GEMMI_KERNEL_SPLIT.)
+ *   GEMMI_KERNEL_CONVERT_I4  : gemm_i4's conversion of the packed operands to E4M3 planes
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
        GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_TC_PAIR_I16 = 6, GEMMI_KERNEL_TC_PAIR_I8 = 7,
-       GEMMI_KERNEL_TC_PAIR_I4 = 8, GEMMI_KERNEL_ADD_I32 = 9, GEMMI_KERNEL_COUNT = 10 };
+       GEMMI_KERNEL_TC_PAIR_I4 = 8, GEMMI_KERNEL_ADD_I32 = 9, GEMMI_KERNEL_CONVERT_I4 = 10,
+       GEMMI_KERNEL_COUNT = 11 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

@@ -32,13 +32,14 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
             "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex", "gemmi_conv2d_i16",
-            "gemm_i4", "gemm_i4_ex")
+            "gemm_i4", "gemm_i4_ex", "gemmi_pack_b_i4", "gemm_i4_packed")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
-KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8, KERNEL_TC_PAIR_I4, KERNEL_ADD_I32 = 6, 7, 8, 9
+KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8, KERNEL_TC_PAIR_I4, KERNEL_ADD_I32, KERNEL_CONVERT_I4 = 6, 7, 8, 9, 10
 KERNELS = (("split", KERNEL_SPLIT), ("tc_i16", KERNEL_TC_I16), ("tc_i8", KERNEL_TC_I8), ("skinny", KERNEL_SKINNY),
            ("fused_i16", KERNEL_FUSED_I16), ("srs", KERNEL_SRS), ("tc_pair_i16", KERNEL_TC_PAIR_I16),
-           ("tc_pair_i8", KERNEL_TC_PAIR_I8), ("tc_pair_i4", KERNEL_TC_PAIR_I4), ("add_i32", KERNEL_ADD_I32))
+           ("tc_pair_i8", KERNEL_TC_PAIR_I8), ("tc_pair_i4", KERNEL_TC_PAIR_I4), ("add_i32", KERNEL_ADD_I32),
+           ("convert_i4", KERNEL_CONVERT_I4))
 
 _lib = None
 
@@ -94,10 +95,10 @@ def lib():
         L.gemmi_kernel_time.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
         L.gemmi_kernel_time.restype = ctypes.c_int
         L.gemmi_version.restype = ctypes.c_char_p
-        for name in ("gemmi_pack_b_i16", "gemmi_pack_b_i8"):
+        for name in ("gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemmi_pack_b_i4"):
             getattr(L, name).argtypes = [i64, i64, vp, i64, vp, ctypes.POINTER(vp)]
             getattr(L, name).restype = ctypes.c_int
-        for name in ("gemm_i16_packed", "gemm_i8_packed"):
+        for name in ("gemm_i16_packed", "gemm_i8_packed", "gemm_i4_packed"):
             getattr(L, name).argtypes = [i64, vp, i64, vp, vp, i64, vp]
             getattr(L, name).restype = ctypes.c_int
         L.gemmi_packed_b_free.argtypes = [vp]
@@ -290,11 +291,14 @@ class PackedB:
             pass
 
 
-def _pack(fn_name, kind, B, dtype, stream):
+def _pack(fn_name, kind, B, dtype, stream, n=None):
     import torch
     if not isinstance(B, torch.Tensor) or not B.is_cuda or B.dtype != dtype:
         raise TypeError(f"B must be a CUDA {dtype} tensor")
-    k, n = B.shape
+    k, cols = B.shape
+    n = cols if n is None else int(n)
+    if cols < (n + 1) // 2:
+        raise ValueError(f"packed B {tuple(B.shape)} is too narrow for n = {n}")
     if stream is None:
         stream = torch.cuda.current_stream(B.device)
     out = ctypes.c_void_p(0)
@@ -316,6 +320,12 @@ def pack_b_i8(B, stream=None) -> PackedB:
     return _pack("gemmi_pack_b_i8", "i8", B, torch.int8, stream)
 
 
+def pack_b_i4(B, n, stream=None) -> PackedB:
+    """Pack an int4 B for gemm_i4_packed: B a uint8 (k, >= ceil(n/2)) tensor in gemm_i4's format."""
+    import torch
+    return _pack("gemmi_pack_b_i4", "i4", B, torch.uint8, stream, n=n)
+
+
 def _packed_call(fn_name, kind, A, Bp, C, op_dtype, c_dtype, stream):
     import torch
     if not isinstance(Bp, PackedB) or Bp.kind != kind:
@@ -324,6 +334,8 @@ def _packed_call(fn_name, kind, A, Bp, C, op_dtype, c_dtype, stream):
         if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dtype != dt:
             raise TypeError(f"{nm} must be a CUDA {dt} tensor")
     m, k = A.shape
+    if kind == "i4":  # A packed: k comes from the handle
+        k = Bp.k if A.shape[1] >= (Bp.k + 1) // 2 else -1
     if k != Bp.k or tuple(C.shape) != (m, Bp.n):
         raise ValueError(f"shape mismatch: A {tuple(A.shape)}, packed B {(Bp.k, Bp.n)}, C {tuple(C.shape)}")
     if stream is None:
@@ -345,6 +357,12 @@ def gemm_i8_packed(A, Bp, C, stream=None):
     """C += A @ B with B pre-packed by pack_b_i8 (bit-identical to gemm_i8)."""
     import torch
     return _packed_call("gemm_i8_packed", "i8", A, Bp, C, torch.int8, torch.int32, stream)
+
+
+def gemm_i4_packed(A, Bp, C, stream=None):
+    """C += A @ B with B pre-packed by pack_b_i4 and A packed as for gemm_i4 (bit-identical to gemm_i4)."""
+    import torch
+    return _packed_call("gemm_i4_packed", "i4", A, Bp, C, torch.uint8, torch.int32, stream)
 
 
 # ------------------------------------------------------------------ host-buffer entry points

@@ -531,8 +531,10 @@ int gemm_i8_locked(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda
 // The int4 path (int4.cu, gemm_pair.cu): the packed operands become K-major E4M3 planes in the
 // workspace (pitch k rounded up to 16 bytes), then the pair kernel runs on kind::f8f6f4.  A C that
 // cannot take 16-byte bulk reductions gets a zeroed scratch result that one more pass adds into it.
-int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
-                   int32_t* C, int64_t ldc, cudaStream_t s) {
+// Checks of gemm_i4's arguments (lda, ldb in packed bytes); -1 to proceed, or a status to return.
+// `b_bytes` > 0 replaces B's extent in the overlap check (the planes of a packed B).
+int check_args_i4(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B, int64_t ldb,
+                  const void* C, int64_t ldc, size_t b_bytes = 0) {
   if (m < 0 || n < 0 || k < 0) return set_error(GEMMI_EINVAL, "negative matrix dimension");
   const int64_t wa = (k + 1) / 2, wb = (n + 1) / 2;  // packed bytes per row of A and of B
   if (ldc < std::max<int64_t>(1, n)) return set_error(GEMMI_EINVAL, "ldc < max(1, n)");
@@ -545,28 +547,31 @@ int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t ld
   if (m > (int64_t(1) << 40) || n > (int64_t(1) << 31) || k > (int64_t(1) << 31))
     return set_error(GEMMI_EINVAL, "matrix dimension too large");
   const size_t a_bytes = static_cast<size_t>((m - 1) * lda + wa);
-  const size_t b_bytes = static_cast<size_t>((k - 1) * ldb + wb);
+  if (b_bytes == 0) b_bytes = static_cast<size_t>((k - 1) * ldb + wb);
   const size_t c_bytes = static_cast<size_t>((m - 1) * ldc + n) * 4;
   if (overlaps(C, c_bytes, A, a_bytes) || overlaps(C, c_bytes, B, b_bytes))
     return set_error(GEMMI_EINVAL, "C overlaps A or B");
-  DeviceState* d = nullptr;
-  int rc = device_state(&d);
-  if (rc != GEMMI_OK) return rc;
+  return -1;
+}
+
+int run_i4(DeviceState& d, int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B,
+           int64_t ldb, int32_t* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b = nullptr) {
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 16));
   const size_t a_plane = round_up(static_cast<size_t>(m) * pitch, kAlign);
-  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch, kAlign);
+  const size_t b_plane = packed_b ? 0 : round_up(static_cast<size_t>(n) * pitch, kAlign);
   const bool direct = reinterpret_cast<uintptr_t>(C) % 16 == 0 && ldc % 4 == 0;
   const int64_t ldt = static_cast<int64_t>(round_up(static_cast<size_t>(n), 4));
   const size_t t_bytes = direct ? 0 : static_cast<size_t>(m) * ldt * 4;
-  if ((rc = ensure_buffer(&d->ws, &d->ws_bytes, a_plane + b_plane + t_bytes)) != GEMMI_OK) return rc;
-  if ((rc = begin_workspace_use(*d, s)) != GEMMI_OK) return rc;
-  char* ws = static_cast<char*>(d->ws);
+  int rc = ensure_buffer(&d.ws, &d.ws_bytes, a_plane + b_plane + t_bytes);
+  if (rc != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+  char* ws = static_cast<char*>(d.ws);
   const LimbPlanes pa{{ws, nullptr}, m, pitch};
-  const LimbPlanes pb{{ws + a_plane, nullptr}, n, pitch};
+  const LimbPlanes pb = packed_b ? *packed_b : LimbPlanes{{ws + a_plane, nullptr}, n, pitch};
   int32_t* T = direct ? nullptr : reinterpret_cast<int32_t*>(ws + a_plane + b_plane);
-  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
-  cudaError_t e = gemmi::convert_i4(A, lda, B, ldb, m, n, k, pa, pb, d->sm_count, s);
-  timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_CONVERT_I4, s);
+  cudaError_t e = gemmi::convert_i4(A, lda, packed_b ? nullptr : B, ldb, m, n, k, pa, pb, d.sm_count, s);
+  timer_end(GEMMI_KERNEL_CONVERT_I4, t0, s);
   if (e != cudaSuccess) return cuda_error(e, "int4 operand conversion launch");
   if (!direct && (e = cudaMemsetAsync(T, 0, t_bytes, s)) != cudaSuccess) return cuda_error(e, "cudaMemsetAsync");
   gemmi::TcGemmArgs ta;
@@ -577,9 +582,9 @@ int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t ld
   ta.b = pb;
   ta.C = direct ? static_cast<void*>(C) : static_cast<void*>(T);
   ta.ldc = direct ? ldc : ldt;
-  ta.status = d->status;
+  ta.status = d.status;
   ta.timeout_ns = timeout_ns();
-  ta.num_sms = d->sm_count;
+  ta.num_sms = d.sm_count;
   ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
   ta.group_m = static_cast<int>(g_tc_group_m);
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
@@ -591,11 +596,21 @@ int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t ld
   if (e != cudaSuccess) return cuda_error(e, why);
   if (!direct) {
     cudaEvent_t t2 = timer_begin(GEMMI_KERNEL_ADD_I32, s);
-    e = gemmi::add_into_i32(C, ldc, T, ldt, m, n, d->sm_count, s);
+    e = gemmi::add_into_i32(C, ldc, T, ldt, m, n, d.sm_count, s);
     timer_end(GEMMI_KERNEL_ADD_I32, t2, s);
     if (e != cudaSuccess) return cuda_error(e, "int4 scratch add launch");
   }
-  return end_workspace_use(*d, s);
+  return end_workspace_use(d, s);
+}
+
+int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+                   int32_t* C, int64_t ldc, cudaStream_t s) {
+  const int pre = check_args_i4(m, n, k, A, lda, B, ldb, C, ldc);
+  if (pre >= 0) return pre;
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  return run_i4(*d, m, n, k, A, lda, B, ldb, C, ldc, s);
 }
 
 int read_status_locked(DeviceState& d, bool clear) {
@@ -860,7 +875,7 @@ int gemm_i8_host(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, 
 }  // extern "C"
 
 struct gemmi_packed_b {
-  int nl;        // 2: int16 limb planes, 1: int8 values as fp16
+  int nl;        // 2: int16 limb planes, 1: int8 values as fp16, 4: int4 values as E4M3 bytes
   int device;
   int64_t k, n, pitch;
   void* mem;     // the planes, owned by the handle
@@ -872,7 +887,7 @@ int pack_b(int nl, int64_t k, int64_t n, const void* B, int64_t ldb, void* strea
   if (out == nullptr) return set_error(GEMMI_EINVAL, "null output handle");
   *out = nullptr;
   if (k < 1 || n < 1) return set_error(GEMMI_EINVAL, "packed operand needs k >= 1 and n >= 1");
-  if (ldb < n) return set_error(GEMMI_EINVAL, "ldb < n");
+  if (ldb < (nl == 4 ? (n + 1) / 2 : n)) return set_error(GEMMI_EINVAL, nl == 4 ? "ldb < ceil(n/2) bytes" : "ldb < n");
   if (B == nullptr) return set_error(GEMMI_EINVAL, "B is null");
   if (k > (int64_t(1) << 31) || n > (int64_t(1) << 31)) return set_error(GEMMI_EINVAL, "matrix dimension too large");
   std::lock_guard<std::mutex> lock(g_mutex);
@@ -881,10 +896,11 @@ int pack_b(int nl, int64_t k, int64_t n, const void* B, int64_t ldb, void* strea
   if (rc != GEMMI_OK) return rc;
   int dev = 0;
   cudaGetDevice(&dev);
-  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
-  const size_t plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
+  const bool i4 = nl == 4;
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), i4 ? 16 : 8));
+  const size_t plane = round_up(static_cast<size_t>(n) * pitch * (i4 ? 1 : 2), kAlign);
   void* mem = nullptr;
-  if (cudaMalloc(&mem, plane * nl) != cudaSuccess) {
+  if (cudaMalloc(&mem, plane * (nl == 2 ? 2 : 1)) != cudaSuccess) {
     cudaGetLastError();
     return set_error(GEMMI_ENOMEM, "cannot allocate the packed operand");
   }
@@ -892,8 +908,10 @@ int pack_b(int nl, int64_t k, int64_t n, const void* B, int64_t ldb, void* strea
   LimbPlanes pb{{base, base + (nl == 2 ? plane : 0)}, n, pitch};
   LimbPlanes none{{nullptr, nullptr}, 0, pitch};
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e = nl == 2 ? gemmi::split_i16(nullptr, k, static_cast<const int16_t*>(B), ldb, 0, n, k, none, pb, s)
-                          : gemmi::convert_i8(nullptr, k, static_cast<const int8_t*>(B), ldb, 0, n, k, none, pb, s);
+  cudaError_t e =
+      nl == 2 ? gemmi::split_i16(nullptr, k, static_cast<const int16_t*>(B), ldb, 0, n, k, none, pb, s)
+      : i4    ? gemmi::convert_i4(nullptr, 1, static_cast<const uint8_t*>(B), ldb, 0, n, k, none, pb, d->sm_count, s)
+              : gemmi::convert_i8(nullptr, k, static_cast<const int8_t*>(B), ldb, 0, n, k, none, pb, s);
   if (e != cudaSuccess) {
     cudaFree(mem);
     return cuda_error(e, "packing launch");
@@ -905,7 +923,7 @@ int pack_b(int nl, int64_t k, int64_t n, const void* B, int64_t ldb, void* strea
 int gemm_packed(int nl, int64_t m, const void* A, int64_t lda, const gemmi_packed_b* Bp, void* C, int64_t ldc,
                 void* stream) {
   if (Bp == nullptr) return set_error(GEMMI_EINVAL, "null packed operand");
-  if (Bp->nl != nl) return set_error(GEMMI_EINVAL, "packed operand has the other element type");
+  if (Bp->nl != nl) return set_error(GEMMI_EINVAL, "packed operand has another element type");
   const int64_t n = Bp->n, k = Bp->k;
   const size_t op = nl == 2 ? 2 : 1, cs = nl == 2 ? 8 : 4;
   // the packed planes stand in for B in the overlap check (C must not overlap them either)
@@ -924,9 +942,38 @@ int gemm_packed(int nl, int64_t m, const void* A, int64_t lda, const gemmi_packe
   return run_tc(*d, nl, m, n, k, A, lda, nullptr, n, C, ldc, static_cast<cudaStream_t>(stream), &pb);
 }
 
+int gemm_i4_packed_impl(int64_t m, const uint8_t* A, int64_t lda, const gemmi_packed_b* Bp, int32_t* C, int64_t ldc,
+                        void* stream) {
+  if (Bp == nullptr) return set_error(GEMMI_EINVAL, "null packed operand");
+  if (Bp->nl != 4) return set_error(GEMMI_EINVAL, "packed operand has another element type");
+  const int64_t n = Bp->n, k = Bp->k;
+  const size_t plane = round_up(static_cast<size_t>(n) * Bp->pitch, kAlign);
+  // the packed plane stands in for B in the checks (C must not overlap it either)
+  const int pre = check_args_i4(m, n, k, A, lda, Bp->mem, (n + 1) / 2, C, ldc, plane);
+  if (pre >= 0) return pre;
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != Bp->device) return set_error(GEMMI_EINVAL, "packed operand belongs to another device");
+  const LimbPlanes pb{{Bp->mem, nullptr}, n, Bp->pitch};
+  return run_i4(*d, m, n, k, A, lda, nullptr, (n + 1) / 2, C, ldc, static_cast<cudaStream_t>(stream), &pb);
+}
+
 }  // namespace
 
 extern "C" {
+
+int gemmi_pack_b_i4(int64_t k, int64_t n, const uint8_t* B, int64_t ldb, void* stream, gemmi_packed_b** out) {
+  return pack_b(4, k, n, B, ldb, stream, out);
+}
+
+int gemm_i4_packed(int64_t m, const uint8_t* A, int64_t lda, const gemmi_packed_b* B, int32_t* C, int64_t ldc,
+                   void* stream) {
+  return gemm_i4_packed_impl(m, A, lda, B, C, ldc, stream);
+}
 
 int gemmi_pack_b_i16(int64_t k, int64_t n, const int16_t* B, int64_t ldb, void* stream, gemmi_packed_b** out) {
   return pack_b(2, k, n, B, ldb, stream, out);

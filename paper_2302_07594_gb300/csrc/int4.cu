@@ -16,134 +16,156 @@
 namespace gemmi {
 namespace {
 
-// The E4M3 encoding of an integer v in [-8, 8], from the format's definition: sign bit, 4-bit
-// exponent with bias 7, 3-bit fraction; |v| = 2^e * (1 + f/8) with e = floor(log2 |v|).
-__device__ __forceinline__ uint32_t e4m3_of_int(int v) {
-  if (v == 0) return 0u;
-  const uint32_t sign = v < 0 ? 0x80u : 0u;
-  const int a = v < 0 ? -v : v;
-  const int e = 31 - __clz(a);
-  const int f = ((a << 3) >> e) - 8;
-  return sign | (static_cast<uint32_t>(e + 7) << 3) | static_cast<uint32_t>(f);
+// E4M3 codes of the 4-bit values, from the format's definition (sign bit, 4-bit exponent with
+// bias 7, 3-bit fraction: |v| = 2^e * (1 + f/8)), four to a word, indexed by the low three bits of
+// the nibble: kPos for nibbles 0..7 (values 0..7), kNeg for nibbles 8..15 (values -8..-1).
+//   0 -> 0x00, 1 -> 0x38, 2 -> 0x40, 3 -> 0x44, 4 -> 0x48, 5 -> 0x4A, 6 -> 0x4C, 7 -> 0x4E,
+//  -8 -> 0xD0, -7 -> 0xCE, -6 -> 0xCC, -5 -> 0xCA, -4 -> 0xC8, -3 -> 0xC4, -2 -> 0xC0, -1 -> 0xB8.
+constexpr uint32_t kPos0 = 0x44403800u, kPos1 = 0x4E4C4A48u;
+constexpr uint32_t kNeg0 = 0xCACCCED0u, kNeg1 = 0xB8C0C4C8u;
+
+// Four nibbles, as 4-bit fields in bits 0-15 of `sel`, -> their four E4M3 bytes: two byte
+// permutes look up the non-negative and the negative code of each, a third keeps one per byte
+// by the nibble's top bit (byte selector i or i + 4).
+__device__ __forceinline__ uint32_t e4m3x4(uint32_t sel) {
+  const uint32_t idx = sel & 0x7777u;
+  const uint32_t pos = __byte_perm(kPos0, kPos1, idx);
+  const uint32_t neg = __byte_perm(kNeg0, kNeg1, idx);
+  return __byte_perm(pos, neg, 0x3210u | ((sel >> 1) & 0x4444u));
 }
 
-__device__ __forceinline__ int nibble_value(uint32_t nib) { return nib >= 8u ? static_cast<int>(nib) - 16 : static_cast<int>(nib); }
+// A word of eight packed nibbles (elements 8q .. 8q+7 of a row, in order) -> eight E4M3 bytes.
+__device__ __forceinline__ uint2 e4m3x8_row(uint32_t w) { return make_uint2(e4m3x4(w & 0xFFFFu), e4m3x4(w >> 16)); }
 
-// Shared table: packed byte -> its two E4M3 bytes (low nibble's code in the low byte).
-__device__ __forceinline__ void fill_pair_table(uint16_t* lut) {
-  for (int b = threadIdx.x; b < 256; b += blockDim.x)
-    lut[b] = static_cast<uint16_t>(e4m3_of_int(nibble_value(b & 15u)) | (e4m3_of_int(nibble_value(b >> 4)) << 8));
+// Four packed bytes of four consecutive rows (byte i from row p+i) -> the E4M3 bytes of the four
+// low nibbles (column 2c) and of the four high nibbles (column 2c+1), each in row order.
+__device__ __forceinline__ uint2 e4m3x4_cols(uint32_t w) {
+  const uint32_t lo = w & 0x0F0F0F0Fu, hi = (w >> 4) & 0x0F0F0F0Fu;
+  // gather the nibbles of bytes 0..3 into 4-bit fields 0..3
+  const uint32_t sl = __byte_perm(lo | (lo >> 4), 0u, 0x4420u);
+  const uint32_t sh = __byte_perm(hi | (hi >> 4), 0u, 0x4420u);
+  return make_uint2(e4m3x4(sl), e4m3x4(sh));
 }
 
-__device__ __forceinline__ uint32_t pairs_of4(const uint16_t* lut, uint32_t w, int half) {
-  // two packed bytes of w (half 0: bytes 0-1, 1: bytes 2-3) -> four E4M3 bytes
-  const uint32_t b0 = (w >> (16 * half)) & 0xFFu, b1 = (w >> (16 * half + 8)) & 0xFFu;
-  return static_cast<uint32_t>(lut[b0]) | (static_cast<uint32_t>(lut[b1]) << 16);
-}
+// One launch converts both operands.  Blocks [0, a_blocks) convert A: block b takes the 512
+// 16-byte units b*512 + tid and b*512 + 256 + tid of A's rows (unit u = row i, bytes 16c .. 16c+15
+// with u = i * upr + c), each into 32 plane bytes.  The other blocks transpose B: block
+// a_blocks + t takes tile t of 128 rows p x 64 packed bytes (128 columns j) into 128 plane rows
+// of 128 bytes.
+struct ConvertI4Params {
+  const uint8_t* A;
+  int64_t lda, m;
+  uint8_t* pa;
+  const uint8_t* B;
+  int64_t ldb, n;
+  uint8_t* pb;
+  int64_t k, pitch;
+  int64_t a_blocks, b_tiles_j;
+  int a_vec, b_vec;
+};
+constexpr int TP = 128, TJB = 64;
 
-// A (m rows of wb = ceil(k/2) packed bytes, row pitch lda bytes) -> plane rows of k E4M3 bytes.
-// Thread t converts packed bytes 16c .. 16c+15 of row i (t = i * cpr + c) into 32 plane bytes.
-template <bool VEC>
-__global__ void __launch_bounds__(256) convert_rows_i4(const uint8_t* __restrict__ A, int64_t lda, int64_t m,
-                                                       int64_t k, uint8_t* __restrict__ plane, int64_t pitch) {
-  __shared__ uint16_t lut[256];
-  fill_pair_table(lut);
-  __syncthreads();
-  const int64_t wb = (k + 1) / 2;
-  const int64_t cpr = (wb + 15) / 16;
-  const int64_t total = m * cpr;
-  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t i = t / cpr;
-    const int64_t c = t - i * cpr;
-    const uint8_t* src = A + i * lda + 16 * c;
-    uint8_t* dst = plane + i * pitch + 32 * c;
-    if (VEC && 16 * c + 16 <= wb && (k % 2 == 0 || 16 * c + 16 < wb)) {
-      const uint4 w = __ldg(reinterpret_cast<const uint4*>(src));
-      uint4 lo, hi;
-      lo.x = pairs_of4(lut, w.x, 0);
-      lo.y = pairs_of4(lut, w.x, 1);
-      lo.z = pairs_of4(lut, w.y, 0);
-      lo.w = pairs_of4(lut, w.y, 1);
-      hi.x = pairs_of4(lut, w.z, 0);
-      hi.y = pairs_of4(lut, w.z, 1);
-      hi.z = pairs_of4(lut, w.w, 0);
-      hi.w = pairs_of4(lut, w.w, 1);
-      reinterpret_cast<uint4*>(dst)[0] = lo;
-      reinterpret_cast<uint4*>(dst)[1] = hi;
-    } else {
-      // a row's tail (or an unaligned operand): byte by byte; the spare high nibble of an odd
-      // k's last byte becomes a zero (the GEMM never reads it)
-      const int64_t end = (16 * c + 16 < wb) ? 16 * c + 16 : wb;
-      for (int64_t b = 16 * c; b < end; ++b) {
-        const uint32_t byte = src[b - 16 * c];
-        dst[2 * (b - 16 * c)] = static_cast<uint8_t>(e4m3_of_int(nibble_value(byte & 15u)));
-        dst[2 * (b - 16 * c) + 1] =
-            2 * b + 1 < k ? static_cast<uint8_t>(e4m3_of_int(nibble_value(byte >> 4))) : static_cast<uint8_t>(0);
-      }
-    }
+__device__ __forceinline__ void convert_a_unit(const ConvertI4Params& P, int64_t u, uint4 w, bool have) {
+  const int64_t wb = (P.k + 1) / 2;
+  const int64_t upr = (wb + 15) / 16;
+  const int64_t i = u / upr;
+  const int64_t c = u - i * upr;
+  uint8_t* dst = P.pa + i * P.pitch + 32 * c;
+  if (have) {
+    const uint2 a = e4m3x8_row(w.x), b = e4m3x8_row(w.y), d = e4m3x8_row(w.z), e = e4m3x8_row(w.w);
+    reinterpret_cast<uint4*>(dst)[0] = make_uint4(a.x, a.y, b.x, b.y);
+    reinterpret_cast<uint4*>(dst)[1] = make_uint4(d.x, d.y, e.x, e.y);
+    return;
+  }
+  // a row's last unit when it is partial or holds an odd k's spare nibble, or an operand whose
+  // rows are not 16-byte aligned: byte by byte (the spare nibble becomes a zero, never read)
+  const uint8_t* src = P.A + i * P.lda + 16 * c;
+  const int64_t nb = (16 * c + 16 < wb) ? 16 : wb - 16 * c;
+  for (int64_t b = 0; b < nb; ++b) {
+    const uint32_t codes = e4m3x4(static_cast<uint32_t>(src[b]));
+    dst[2 * b] = static_cast<uint8_t>(codes & 0xFFu);
+    dst[2 * b + 1] = 2 * (16 * c + b) + 1 < P.k ? static_cast<uint8_t>((codes >> 8) & 0xFFu) : static_cast<uint8_t>(0);
   }
 }
 
-// B (k rows of wbn = ceil(n/2) packed bytes, pitch ldb) -> plane rows j (one per column of B) of k
-// E4M3 bytes.  A block transposes tiles of 64 rows p x 64 packed bytes (128 columns j), tile
-// t = pt * ntj + jt for t = blockIdx.x, blockIdx.x + gridDim.x, ...
-constexpr int TP = 64, TJB = 64;
-template <bool VEC>
-__global__ void __launch_bounds__(256) convert_cols_i4(const uint8_t* __restrict__ B, int64_t ldb, int64_t k,
-                                                       int64_t n, uint8_t* __restrict__ plane, int64_t pitch) {
-  __shared__ uint8_t lut8[16];
-  __shared__ __align__(16) uint8_t tile[TP][TJB + 16];
-  if (threadIdx.x < 16) lut8[threadIdx.x] = static_cast<uint8_t>(e4m3_of_int(nibble_value(threadIdx.x)));
-  const int64_t wbn = (n + 1) / 2;
-  const int64_t ntj = (wbn + TJB - 1) / TJB, ntp = (k + TP - 1) / TP;
-  for (int64_t t = blockIdx.x; t < ntj * ntp; t += gridDim.x) {
-    const int64_t jb0 = (t % ntj) * TJB;  // first packed byte (column j0 = 2 * jb0)
-    const int64_t p0 = (t / ntj) * TP;
-    __syncthreads();  // the previous tile has been read
-    {
-      const int r = threadIdx.x / 4, q = threadIdx.x % 4;  // row r of the tile, 16-byte segment q
-      const int64_t p = p0 + r;
-      const int64_t b = jb0 + 16 * q;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (p < k) {
-        const uint8_t* src = B + p * ldb + b;
-        if (VEC && b + 16 <= wbn) {
-          v = __ldg(reinterpret_cast<const uint4*>(src));
-        } else {
-          uint32_t w[4] = {0u, 0u, 0u, 0u};
+__global__ void __launch_bounds__(256) convert_i4_kernel(const ConvertI4Params P) {
+  __shared__ __align__(16) uint8_t tile[TP][TJB];
+  if (blockIdx.x < P.a_blocks) {
+    // ---- A: two units per thread, both loads issued before either is converted
+    const int64_t wb = (P.k + 1) / 2;
+    const int64_t upr = (wb + 15) / 16;
+    const int64_t units = P.m * upr;
+    int64_t u[2];
+    uint4 w[2];
+    bool full[2];
 #pragma unroll
-          for (int e = 0; e < 16; ++e)
-            if (b + e < wbn) w[e / 4] |= static_cast<uint32_t>(src[e]) << (8 * (e % 4));
-          v = make_uint4(w[0], w[1], w[2], w[3]);
-        }
+    for (int h = 0; h < 2; ++h) {
+      u[h] = static_cast<int64_t>(blockIdx.x) * 512 + 256 * h + threadIdx.x;
+      full[h] = false;
+      w[h] = make_uint4(0u, 0u, 0u, 0u);
+      if (u[h] < units && P.a_vec) {
+        const int64_t i = u[h] / upr, c = u[h] - (u[h] / upr) * upr;
+        // whole 16-byte units only, and not the one that holds an odd k's spare nibble
+        full[h] = 16 * c + 16 < wb || (16 * c + 16 == wb && P.k % 2 == 0);
+        if (full[h]) w[h] = __ldg(reinterpret_cast<const uint4*>(P.A + i * P.lda + 16 * c));
       }
-      *reinterpret_cast<uint4*>(&tile[r][16 * q]) = v;
     }
-    __syncthreads();
-    // thread t writes plane row j = 2 * jb0 + t / 2, bytes p0 + 32 * (t % 2) .. +31
-    const int jl = threadIdx.x / 2, h = threadIdx.x % 2;
-    const int64_t j = 2 * jb0 + jl;
-    if (j >= n) continue;
-    uint8_t* dst = plane + j * pitch + p0 + 32 * h;
-    const int shift = 4 * (jl & 1);
 #pragma unroll
-    for (int s = 0; s < 2; ++s) {
-      if (p0 + 32 * h + 16 * s >= pitch) break;  // pitch is a multiple of 16: whole 16-byte units
-      uint32_t w[4];
+    for (int h = 0; h < 2; ++h)
+      if (u[h] < units) convert_a_unit(P, u[h], w[h], full[h]);
+    return;
+  }
+  // ---- B: one tile of 128 rows p x 64 packed bytes
+  const int64_t t = static_cast<int64_t>(blockIdx.x) - P.a_blocks;
+  const int64_t wbn = (P.n + 1) / 2;
+  const int64_t jb0 = (t % P.b_tiles_j) * TJB;  // first packed byte of the tile (column 2 * jb0)
+  const int64_t p0 = (t / P.b_tiles_j) * TP;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        uint32_t word = 0;
+  for (int h = 0; h < 2; ++h) {
+    const int r = (threadIdx.x >> 2) + 64 * h, q = threadIdx.x & 3;  // tile row r, 16-byte segment q
+    const int64_t p = p0 + r;
+    const int64_t b = jb0 + 16 * q;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (p < P.k) {
+      const uint8_t* src = P.B + p * P.ldb + b;
+      if (P.b_vec && b + 16 <= wbn) {
+        v = __ldg(reinterpret_cast<const uint4*>(src));
+      } else {
+        uint32_t x[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-        for (int bb = 0; bb < 4; ++bb) {
-          const int r = 32 * h + 16 * s + 4 * e + bb;
-          const uint32_t nib = (tile[r][jl / 2] >> shift) & 15u;
-          word |= static_cast<uint32_t>(lut8[nib]) << (8 * bb);
-        }
-        w[e] = word;
+        for (int e = 0; e < 16; ++e)
+          if (b + e < wbn) x[e / 4] |= static_cast<uint32_t>(src[e]) << (8 * (e % 4));
+        v = make_uint4(x[0], x[1], x[2], x[3]);
       }
-      reinterpret_cast<uint4*>(dst)[s] = make_uint4(w[0], w[1], w[2], w[3]);
     }
+    *reinterpret_cast<uint4*>(&tile[r][16 * q]) = v;
+  }
+  __syncthreads();
+  // thread (jb, pq): packed byte column jb of tile rows 32pq .. 32pq+31 -> 32 plane bytes of
+  // column 2*(jb0+jb) (low nibbles) and 32 of column 2*(jb0+jb)+1 (high nibbles)
+  const int jb = threadIdx.x & 63, pq = threadIdx.x >> 6;
+  const int64_t j = 2 * (jb0 + jb);
+  const int64_t pstart = p0 + 32 * pq;
+  if (j >= P.n || pstart >= P.pitch) return;
+  uint32_t lo[8], hi[8];
+#pragma unroll
+  for (int g = 0; g < 8; ++g) {
+    const int r = 32 * pq + 4 * g;
+    const uint32_t word = static_cast<uint32_t>(tile[r][jb]) | (static_cast<uint32_t>(tile[r + 1][jb]) << 8) |
+                          (static_cast<uint32_t>(tile[r + 2][jb]) << 16) | (static_cast<uint32_t>(tile[r + 3][jb]) << 24);
+    const uint2 c = e4m3x4_cols(word);
+    lo[g] = c.x;
+    hi[g] = c.y;
+  }
+  // the plane rows end at pitch, a multiple of 16: whole 16-byte units
+  const bool second = pstart + 16 < P.pitch;
+  uint4* d0 = reinterpret_cast<uint4*>(P.pb + j * P.pitch + pstart);
+  d0[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+  if (second) d0[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+  if (j + 1 < P.n) {
+    uint4* d1 = reinterpret_cast<uint4*>(P.pb + (j + 1) * P.pitch + pstart);
+    d1[0] = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    if (second) d1[1] = make_uint4(hi[4], hi[5], hi[6], hi[7]);
   }
 }
 
@@ -168,26 +190,31 @@ unsigned grid_for(int64_t work, int num_sms) {
 
 cudaError_t convert_i4(const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
                        LimbPlanes pa, LimbPlanes pb, int num_sms, cudaStream_t s) {
+  (void)num_sms;
   if (k <= 0) return cudaSuccess;
-  if (A != nullptr && m > 0) {
-    const bool vec = reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 16 == 0;
-    const int64_t work = m * (((k + 1) / 2 + 15) / 16);
-    const unsigned g = grid_for(work, num_sms);
-    if (vec) convert_rows_i4<true><<<g, 256, 0, s>>>(A, lda, m, k, static_cast<uint8_t*>(pa.plane[0]), pa.pitch);
-    else convert_rows_i4<false><<<g, 256, 0, s>>>(A, lda, m, k, static_cast<uint8_t*>(pa.plane[0]), pa.pitch);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  if (B != nullptr && n > 0) {
-    const bool vec = reinterpret_cast<uintptr_t>(B) % 16 == 0 && ldb % 16 == 0;
-    const int64_t tiles = (((n + 1) / 2 + TJB - 1) / TJB) * ((k + TP - 1) / TP);
-    const int64_t cap = static_cast<int64_t>(num_sms > 0 ? num_sms : 148) * 8;
-    const unsigned g = static_cast<unsigned>(tiles < cap ? tiles : cap);
-    if (vec) convert_cols_i4<true><<<g, 256, 0, s>>>(B, ldb, k, n, static_cast<uint8_t*>(pb.plane[0]), pb.pitch);
-    else convert_cols_i4<false><<<g, 256, 0, s>>>(B, ldb, k, n, static_cast<uint8_t*>(pb.plane[0]), pb.pitch);
-    return cudaGetLastError();
-  }
-  return cudaSuccess;
+  ConvertI4Params P{};
+  P.A = A;
+  P.lda = lda;
+  P.m = A != nullptr ? m : 0;
+  P.pa = static_cast<uint8_t*>(pa.plane[0]);
+  P.B = B;
+  P.ldb = ldb;
+  P.n = B != nullptr ? n : 0;
+  P.pb = static_cast<uint8_t*>(pb.plane[0]);
+  P.k = k;
+  P.pitch = A != nullptr ? pa.pitch : pb.pitch;
+  if (A != nullptr && B != nullptr && pa.pitch != pb.pitch) return cudaErrorInvalidValue;
+  const int64_t a_units = P.m * (((k + 1) / 2 + 15) / 16);
+  P.a_blocks = (a_units + 511) / 512;
+  P.b_tiles_j = ((P.n + 1) / 2 + TJB - 1) / TJB;
+  const int64_t b_tiles = P.n > 0 ? P.b_tiles_j * ((k + TP - 1) / TP) : 0;
+  P.a_vec = A != nullptr && reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 16 == 0;
+  P.b_vec = B != nullptr && reinterpret_cast<uintptr_t>(B) % 16 == 0 && ldb % 16 == 0;
+  const int64_t blocks = P.a_blocks + b_tiles;
+  if (blocks == 0) return cudaSuccess;
+  if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  convert_i4_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(P);
+  return cudaGetLastError();
 }
 
 cudaError_t add_into_i32(int32_t* C, int64_t ldc, const int32_t* T, int64_t ldt, int64_t m, int64_t n, int num_sms,

@@ -76,7 +76,7 @@ def run(gm, A, B, C, lda=None, ldb=None, ldc=None, pad=0x9B, c_offset=0, expect_
     dCb = torch.from_numpy(Cbuf).cuda()
     counts = counts_of(gm, lambda: gm.gemm_i4(dA, dB, dCb[:, c_offset:c_offset + n], k))
     assert gm.device_status() == gm.OK
-    assert counts["tc_pair_i4"] == 1, counts
+    assert counts["tc_pair_i4"] == 1 and counts["convert_i4"] == 1 and counts["split"] == 0, counts
     if expect_direct is not None:
         assert counts["add_i32"] == (0 if expect_direct else 1), counts
     got = dCb.cpu().numpy()
@@ -200,3 +200,25 @@ def test_i4_empty_problems(gm):
                torch.zeros((0, 3), dtype=torch.uint8, device="cuda"), dC, 0)
     torch.cuda.synchronize()
     assert int(dC.abs().sum()) == 0
+
+
+@pytest.mark.parametrize("case", [(300, 200, 400, None), (77, 131, 257, 80), (1, 6, 3, None)])
+def test_i4_packed_weights(gm, case):
+    # B converted once to its E4M3 plane (gemmi_pack_b_i4), then used for two different A
+    m, n, k, ldb = case
+    A, B, C = gi.random_problem(8700 + m, m, n, k, "i4")
+    A2 = gi.uniform_int(8701 + m, (m, k), -8, 7, np.int8)
+    Bp = gi.pack_nibbles(B, ld=ldb, pad=0x5A)
+    packed = gm.pack_b_i4(torch.from_numpy(Bp).cuda()[:, :(n + 1) // 2], n)
+    try:
+        exp = C.copy()
+        for X in (A, A2):
+            Ap = gi.pack_nibbles(X)
+            dC = torch.from_numpy(exp.copy()).cuda()
+            counts = counts_of(gm, lambda: gm.gemm_i4_packed(torch.from_numpy(Ap).cuda(), packed, dC))
+            assert counts["tc_pair_i4"] == 1 and counts["convert_i4"] == 1, counts
+            assert gm.device_status() == gm.OK
+            oracle.gemm_i4(Ap, Bp[:, :(n + 1) // 2], exp, k, nthreads=8)
+            assert_same(dC.cpu().numpy(), exp, f"packed i4 {case}")
+    finally:
+        packed.close()

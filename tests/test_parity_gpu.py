@@ -37,6 +37,12 @@ def expected(A, B, C, threads=8):
 
 def run_gpu(gm, A, B, C, kind=None):
     kind = kind or ("i16" if A.dtype == np.int16 else "i8")
+    if kind == "i4":  # int4 values in int8 arrays, stored packed for the device
+        dA, dB, dC = (torch.from_numpy(x).cuda() for x in (gi.pack_nibbles(A), gi.pack_nibbles(B), C))
+        gm.gemm_i4(dA, dB, dC, A.shape[1])
+        torch.cuda.synchronize()
+        assert gm.device_status() == gm.OK
+        return dC.cpu().numpy()
     dA, dB, dC = (torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (A, B, C))
     (gm.gemm_i16 if kind == "i16" else gm.gemm_i8)(dA, dB, dC)
     torch.cuda.synchronize()
@@ -304,7 +310,12 @@ def test_workload(gm, name):
         assert_same(got, expected(A, B, C), name)
         return
     rows = _sample_rows(w.m)
-    assert_same(got[rows], expected(A[rows], B, C[rows]), f"{name} sampled rows {rows[:4]}...")
+    if w.kind == "i4":
+        exp = C[rows].copy()
+        oracle.gemm_i4(gi.pack_nibbles(A[rows]), gi.pack_nibbles(B), exp, w.k, nthreads=8)
+    else:
+        exp = expected(A[rows], B, C[rows])
+    assert_same(got[rows], exp, f"{name} sampled rows {rows[:4]}...")
     # every output through row and column sums (exact int64 arithmetic modulo 2^64)
     with np.errstate(over="ignore"):
         Bsum = B.astype(np.int64).sum(axis=1)
@@ -313,7 +324,7 @@ def test_workload(gm, name):
         col_exp = Asum @ B.astype(np.int64) + C.astype(np.int64).sum(axis=0)
         row_got = got.astype(np.int64).sum(axis=1)
         col_got = got.astype(np.int64).sum(axis=0)
-    if w.kind == "i8":  # int32 C: the sums compare modulo 2^32
+    if w.kind != "i16":  # int32 C: the sums compare modulo 2^32
         row_exp, row_got, col_exp, col_got = (x & 0xFFFFFFFF for x in (row_exp, row_got, col_exp, col_got))
     assert np.array_equal(row_got, row_exp), f"{name}: row sums differ"
     assert np.array_equal(col_got, col_exp), f"{name}: column sums differ"
