@@ -63,7 +63,7 @@ def parse_args_list(argv):
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=("gemmi", "reference"), default="gemmi")
-    p.add_argument("--workload", default="i16_8192", choices=[n for n, w in gi.WORKLOADS.items() if w.kind != "i4"])
+    p.add_argument("--workload", default="i16_8192", choices=list(gi.WORKLOADS))
     p.add_argument("--no-extra", action="store_true", help="skip the per-workload table")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU budget of the oracle baseline")
@@ -189,17 +189,25 @@ def oracle_rate(w, seconds: float, threads: int):
     import oracle
     oracle.build()
     _, B, _ = gi.make_inputs(w, rows=slice(0, 1))
+
+    def run(A, C):
+        if w.kind == "i4":
+            oracle.gemm_i4(gi.pack_nibbles(A), Bp, C, w.k, nthreads=threads)
+        else:
+            oracle.gemm(A, B, C, nthreads=threads)
+
+    Bp = gi.pack_nibbles(B) if w.kind == "i4" else None
     probe = max(1, min(w.m, threads))
     A, _, C = gi.make_inputs(w, rows=slice(0, probe))
     t0 = time.perf_counter()
-    oracle.gemm(A, B, C, nthreads=threads)
+    run(A, C)
     t_probe = time.perf_counter() - t0
     per_row = t_probe / probe
     rows = int(max(1, min(w.m, seconds / max(per_row, 1e-9))))
     rows = max(probe, (rows // threads) * threads) if rows >= threads else rows
     A, _, C = gi.make_inputs(w, rows=slice(0, rows))
     t0 = time.perf_counter()
-    oracle.gemm(A, B, C, nthreads=threads)
+    run(A, C)
     t = time.perf_counter() - t0
     ops = 2 * rows * w.n * w.k
     return ops / t / 1e12, t, rows
@@ -430,8 +438,13 @@ def run_gemmi(args):
     peaks = measured_peaks()
     w = gi.WORKLOADS[args.workload]
     A, B, C = gi.make_inputs(w)
+    if w.kind == "i4":  # the int4 operands travel packed, two values to a byte
+        A, B = gi.pack_nibbles(A), gi.pack_nibbles(B)
     dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
-    fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
+    if w.kind == "i4":
+        fn = lambda a, b, c: gm.gemm_i4(a, b, c, w.k)  # noqa: E731
+    else:
+        fn = gm.gemm_i16 if w.kind == "i16" else gm.gemm_i8
     for _ in range(args.warmup):
         fn(dA, dB, dC)
     torch.cuda.synchronize()
@@ -475,6 +488,14 @@ def run_gemmi(args):
                              "fp16 = bf16 rate) / 4 limb products per int16 multiply-add",
                 "frac_of_sustained": achieved / (peaks["bf16_tflops_sustained"] / 4.0),
                 "kernel_ms": per_launch_ms}
+    elif bound == "tensor" and w.kind == "i4":
+        achieved = w.ops / (per_launch_ms * 1e-3) / 1e12
+        peak = peaks["bf16_tflops"] * FP8_PER_BF16
+        roof = {"bound": "tensor", "kernel": sym, "achieved": achieved, "peak": peak, "unit": "TOPS",
+                "frac": achieved / peak,
+                "peak_note": f"fp8 dense tensor peak: {peaks['source']} bf16 burst {peaks['bf16_tflops']} TFLOP/s x "
+                             f"{FP8_PER_BF16} (nominal fp8 / bf16 rate); one E4M3 product per int4 multiply-add",
+                "kernel_ms": per_launch_ms}
     elif bound == "tensor":
         achieved = w.ops / (per_launch_ms * 1e-3) / 1e12
         peak = peaks["bf16_tflops"]
@@ -494,7 +515,7 @@ def run_gemmi(args):
     int8_peak = int8_tensor_peak(torch)
 
     # ---- end to end through the host-buffer C ABI (copies inside the timed region)
-    op_t = torch.int16 if w.kind == "i16" else torch.int8
+    op_t = {"i16": torch.int16, "i8": torch.int8, "i4": torch.uint8}[w.kind]
     c_t = torch.int64 if w.kind == "i16" else torch.int32
     hA = torch.empty(A.shape, dtype=op_t, pin_memory=True).numpy()
     hB = torch.empty(B.shape, dtype=op_t, pin_memory=True).numpy()
@@ -502,7 +523,10 @@ def run_gemmi(args):
     hA[...] = A
     hB[...] = B
     hC[...] = C
-    host_fn = gm.gemm_i16_host if w.kind == "i16" else gm.gemm_i8_host
+    if w.kind == "i4":
+        host_fn = lambda a, b, c: gm.gemm_i4_host(a, b, c, w.k)  # noqa: E731
+    else:
+        host_fn = gm.gemm_i16_host if w.kind == "i16" else gm.gemm_i8_host
     gm.set_stream(torch.cuda.current_stream())
     host_fn(hA, hB, hC)
     e2e_steps = max(3, min(args.steps, 20))
@@ -515,7 +539,7 @@ def run_gemmi(args):
     e2e_s = max_over_ranks(e2e_s, world)
     e2e = {"value": job_throughput(w.ops, e2e_s, world) / 1e12, "unit": "TOPS", "ms_per_step": e2e_s * 1e3,
            "h2d_bytes_per_step": int(A.nbytes + B.nbytes + C.nbytes), "d2h_bytes_per_step": int(C.nbytes),
-           "steps": e2e_steps, "api": "gemm_i16_host" if w.kind == "i16" else "gemm_i8_host"}
+           "steps": e2e_steps, "api": f"gemm_{w.kind}_host"}
     del hA, hB, hC
 
     # ---- per-workload table (each workload's own bound), rank 0 only
@@ -618,7 +642,7 @@ def run_gemmi(args):
 
     if rank == 0:
         line = {
-            "metric": "int16 GEMM TOPS (2mnk/s)" if w.kind == "i16" else "int8 GEMM TOPS (2mnk/s)",
+            "metric": {"i16": "int16", "i8": "int8", "i4": "int4"}[w.kind] + " GEMM TOPS (2mnk/s)",
             "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "int64" if w.kind == "i16" else "int32",

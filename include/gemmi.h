@@ -123,6 +123,13 @@ int gemm_i8_host(int64_t m, int64_t n, int64_t k,
                  const int8_t* B, int64_t ldb,
                  int32_t* C, int64_t ldc);
 
+/* gemm_i4 on HOST buffers (A and B in gemm_i4's packed format, lda and ldb in bytes); copies,
+ * result and errors as gemm_i16_host. */
+int gemm_i4_host(int64_t m, int64_t n, int64_t k,
+                 const uint8_t* A, int64_t lda,
+                 const uint8_t* B, int64_t ldb,
+                 int32_t* C, int64_t ldc);
+
 /*
  * gemm_i16_srs -- the output of the paper's AIE micro-kernel (Section 5.2, the
  * simplified micro-kernel listing): the wide accumulator is shifted, rounded and

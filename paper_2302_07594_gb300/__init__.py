@@ -32,7 +32,7 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
             "gemmi_packed_b_free", "gemmi_packed_b_k", "gemmi_packed_b_n", "gemm_i16_srs", "gemm_i16_srs_ex", "gemmi_conv2d_i16",
-            "gemm_i4", "gemm_i4_ex", "gemmi_pack_b_i4", "gemm_i4_packed")
+            "gemm_i4", "gemm_i4_ex", "gemmi_pack_b_i4", "gemm_i4_packed", "gemm_i4_host")
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
 KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8, KERNEL_TC_PAIR_I4, KERNEL_ADD_I32, KERNEL_CONVERT_I4 = 6, 7, 8, 9, 10
@@ -65,7 +65,7 @@ def lib():
         L = ctypes.CDLL(LIB_PATH)
         i64, vp = ctypes.c_int64, ctypes.c_void_p
         core = [i64, i64, i64, vp, i64, vp, i64, vp, i64]
-        for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host", "gemm_i4"):
+        for name in ("gemm_i16", "gemm_i8", "gemm_i16_host", "gemm_i8_host", "gemm_i4", "gemm_i4_host"):
             getattr(L, name).argtypes = core
             getattr(L, name).restype = ctypes.c_int
         for name in ("gemm_i16_ex", "gemm_i8_ex", "gemm_i16_noalloc", "gemm_i4_ex"):
@@ -404,6 +404,26 @@ def gemm_i16_host(A, B, C):
 def gemm_i8_host(A, B, C):
     import numpy as np
     return _host_call("gemm_i8_host", A, B, C, np.int8, np.int32)
+
+
+def gemm_i4_host(A, B, C, k):
+    """gemm_i4 on numpy (host) arrays: A uint8 (m, >= ceil(k/2)) and B uint8 (k, >= ceil(n/2)) packed
+    as for gemm_i4, C int32 (m, n)."""
+    import numpy as np
+    for x, nm, dt in ((A, "A", np.uint8), (B, "B", np.uint8), (C, "C", np.int32)):
+        if not isinstance(x, np.ndarray) or x.dtype != dt:
+            raise TypeError(f"{nm} must be a numpy {np.dtype(dt).name} array")
+    if not C.flags.writeable:
+        raise ValueError("C must be writeable")
+    m, n = C.shape
+    k = int(k)
+    if A.ndim != 2 or B.ndim != 2 or A.shape[0] != m or B.shape[0] != k or A.shape[1] < (k + 1) // 2 \
+            or B.shape[1] < (n + 1) // 2:
+        raise ValueError(f"shape mismatch: packed A {A.shape}, packed B {B.shape}, C {C.shape}, k {k}")
+    rc = lib().gemm_i4_host(m, n, k, A.ctypes.data, _host_ld(A, "A"), B.ctypes.data, _host_ld(B, "B"),
+                            C.ctypes.data, _host_ld(C, "C"))
+    _check(rc)
+    return C
 
 
 # ------------------------------------------------------------------ control

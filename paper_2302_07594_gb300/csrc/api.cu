@@ -783,6 +783,48 @@ int host_gemm(int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda, const O
   return GEMMI_OK;
 }
 
+// gemm_i4 on host buffers: packed A and B and C are copied into device buffers whose row pitches
+// (16 bytes for the operands, 4 elements for C) keep the conversion and the pair kernel on their
+// aligned paths, the GEMM runs, and C is copied back.
+int host_gemm_i4(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+                 int32_t* C, int64_t ldc) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  const int pre = check_args_i4(m, n, k, A, lda, B, ldb, C, ldc);
+  if (pre >= 0) return pre;
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const int64_t wa = (k + 1) / 2, wb = (n + 1) / 2;
+  const int64_t dlda = static_cast<int64_t>(round_up(static_cast<size_t>(wa), 16));
+  const int64_t dldb = static_cast<int64_t>(round_up(static_cast<size_t>(wb), 16));
+  const int64_t dldc = static_cast<int64_t>(round_up(static_cast<size_t>(n), 4));
+  const size_t a_bytes = round_up(static_cast<size_t>(m) * dlda, kAlign);
+  const size_t b_bytes = round_up(static_cast<size_t>(k) * dldb, kAlign);
+  const size_t c_bytes = round_up(static_cast<size_t>(m) * dldc * 4, kAlign);
+  if ((rc = ensure_buffer(&d->host_buf, &d->host_buf_bytes, a_bytes + b_bytes + c_bytes)) != GEMMI_OK) return rc;
+  char* base = static_cast<char*>(d->host_buf);
+  uint8_t* dA = reinterpret_cast<uint8_t*>(base);
+  uint8_t* dB = reinterpret_cast<uint8_t*>(base + a_bytes);
+  int32_t* dC = reinterpret_cast<int32_t*>(base + a_bytes + b_bytes);
+  cudaStream_t s = g_stream;
+  cudaError_t e = cudaMemcpy2DAsync(dA, dlda, A, lda, wa, m, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpy2DAsync(dB, dldb, B, ldb, wb, k, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2DAsync(dC, dldc * 4, C, ldc * 4, n * 4, m, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_error(e, "host-to-device copy");
+  rc = run_i4(*d, m, n, k, dA, dlda, dB, dldb, dC, dldc, s);
+  if (rc != GEMMI_OK) return rc;
+  e = cudaMemcpy2DAsync(C, ldc * 4, dC, dldc * 4, n * 4, m, cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_error(e, "device-to-host copy");
+  e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize");
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, d->status, sizeof(word), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
+  if (word != 0) return read_status_locked(*d, true);
+  return GEMMI_OK;
+}
+
 __global__ void wait_probe_kernel(uint32_t* status, uint64_t timeout_ns) {
   __shared__ uint64_t bar;
   if (threadIdx.x == 0) {
@@ -870,6 +912,11 @@ int gemm_i16_host(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda
 int gemm_i8_host(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb,
                  int32_t* C, int64_t ldc) {
   return host_gemm(m, n, k, A, lda, B, ldb, C, ldc, gemm_i8_locked);
+}
+
+int gemm_i4_host(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda, const uint8_t* B, int64_t ldb,
+                 int32_t* C, int64_t ldc) {
+  return host_gemm_i4(m, n, k, A, lda, B, ldb, C, ldc);
 }
 
 }  // extern "C"

@@ -65,11 +65,8 @@ struct ConvertI4Params {
 };
 constexpr int TP = 128, TJB = 64;
 
-__device__ __forceinline__ void convert_a_unit(const ConvertI4Params& P, int64_t u, uint4 w, bool have) {
+__device__ __forceinline__ void convert_a_unit(const ConvertI4Params& P, int64_t i, int64_t c, uint4 w, bool have) {
   const int64_t wb = (P.k + 1) / 2;
-  const int64_t upr = (wb + 15) / 16;
-  const int64_t i = u / upr;
-  const int64_t c = u - i * upr;
   uint8_t* dst = P.pa + i * P.pitch + 32 * c;
   if (have) {
     const uint2 a = e4m3x8_row(w.x), b = e4m3x8_row(w.y), d = e4m3x8_row(w.z), e = e4m3x8_row(w.w);
@@ -95,24 +92,34 @@ __global__ void __launch_bounds__(256) convert_i4_kernel(const ConvertI4Params P
     const int64_t wb = (P.k + 1) / 2;
     const int64_t upr = (wb + 15) / 16;
     const int64_t units = P.m * upr;
-    int64_t u[2];
+    int64_t row[2], col[2];
     uint4 w[2];
     bool full[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      u[h] = static_cast<int64_t>(blockIdx.x) * 512 + 256 * h + threadIdx.x;
+      const int64_t u = static_cast<int64_t>(blockIdx.x) * 512 + 256 * h + threadIdx.x;
       full[h] = false;
       w[h] = make_uint4(0u, 0u, 0u, 0u);
-      if (u[h] < units && P.a_vec) {
-        const int64_t i = u[h] / upr, c = u[h] - (u[h] / upr) * upr;
+      row[h] = -1;
+      if (u < units) {
+        // unit -> (row, unit in row): 32-bit division when the unit count allows (the usual case)
+        if (units <= 0xFFFFFFFFll) {
+          const uint32_t q = static_cast<uint32_t>(u) / static_cast<uint32_t>(upr);
+          row[h] = q;
+          col[h] = static_cast<int64_t>(static_cast<uint32_t>(u) - q * static_cast<uint32_t>(upr));
+        } else {
+          row[h] = u / upr;
+          col[h] = u - row[h] * upr;
+        }
         // whole 16-byte units only, and not the one that holds an odd k's spare nibble
-        full[h] = 16 * c + 16 < wb || (16 * c + 16 == wb && P.k % 2 == 0);
-        if (full[h]) w[h] = __ldg(reinterpret_cast<const uint4*>(P.A + i * P.lda + 16 * c));
+        const int64_t c = col[h];
+        full[h] = P.a_vec && (16 * c + 16 < wb || (16 * c + 16 == wb && P.k % 2 == 0));
+        if (full[h]) w[h] = __ldg(reinterpret_cast<const uint4*>(P.A + row[h] * P.lda + 16 * c));
       }
     }
 #pragma unroll
     for (int h = 0; h < 2; ++h)
-      if (u[h] < units) convert_a_unit(P, u[h], w[h], full[h]);
+      if (row[h] >= 0) convert_a_unit(P, row[h], col[h], w[h], full[h]);
     return;
   }
   // ---- B: one tile of 128 rows p x 64 packed bytes
@@ -151,8 +158,8 @@ __global__ void __launch_bounds__(256) convert_i4_kernel(const ConvertI4Params P
 #pragma unroll
   for (int g = 0; g < 8; ++g) {
     const int r = 32 * pq + 4 * g;
-    const uint32_t word = static_cast<uint32_t>(tile[r][jb]) | (static_cast<uint32_t>(tile[r + 1][jb]) << 8) |
-                          (static_cast<uint32_t>(tile[r + 2][jb]) << 16) | (static_cast<uint32_t>(tile[r + 3][jb]) << 24);
+    const uint32_t word = __byte_perm(__byte_perm(tile[r][jb], tile[r + 1][jb], 0x0040u),
+                                      __byte_perm(tile[r + 2][jb], tile[r + 3][jb], 0x0040u), 0x5410u);
     const uint2 c = e4m3x4_cols(word);
     lo[g] = c.x;
     hi[g] = c.y;

@@ -232,14 +232,4 @@ __host__ __device__ constexpr uint32_t idesc_f16_f32(uint32_t M, uint32_t N) {
          | ((M >> 4) << 24);  // M / 16
 }
 
-// Instruction descriptor of tcgen05.mma.kind::f8f6f4 with E4M3 A and B (format code 0 in both
-// fields, K-major) and an fp32 D, M x N.
-__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t M, uint32_t N) {
-  return (1u << 4)            // D format: f32
-         | (0u << 7)          // A format: E4M3
-         | (0u << 10)         // B format: E4M3
-         | ((N >> 3) << 17)   // N / 8
-         | ((M >> 4) << 24);  // M / 16
-}
-
 }  // namespace gemmi

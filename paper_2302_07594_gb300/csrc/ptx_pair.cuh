@@ -127,6 +127,16 @@ __device__ __forceinline__ void tc_mma_f16_pair(uint32_t d_tmem, uint64_t a_desc
       : "memory");
 }
 
+// Instruction descriptor of tcgen05.mma.kind::f8f6f4 with E4M3 A and B (format code 0 in both
+// fields, K-major) and an fp32 D, M x N.
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t M, uint32_t N) {
+  return (1u << 4)            // D format: f32
+         | (0u << 7)          // A format: E4M3
+         | (0u << 10)         // B format: E4M3
+         | ((N >> 3) << 17)   // N / 8
+         | ((M >> 4) << 24);  // M / 16
+}
+
 // The same pair MMA on 8-bit operands (kind::f8f6f4, formats in the instruction descriptor):
 // M = 256, N from the descriptor, K = 32 -- again 32 bytes of each operand row per instruction.
 __device__ __forceinline__ void tc_mma_f8_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,

@@ -222,3 +222,17 @@ def test_i4_packed_weights(gm, case):
             assert_same(dC.cpu().numpy(), exp, f"packed i4 {case}")
     finally:
         packed.close()
+
+
+@pytest.mark.parametrize("case", [(300, 201, 333, None, None), (129, 64, 1000, 520, 40)])
+def test_i4_host_buffers(gm, case):
+    # host arrays with padded byte pitches; the library stages them on the device with aligned pitches
+    m, n, k, lda, ldb = case
+    A, B, C = gi.random_problem(8800 + m, m, n, k, "i4")
+    Ap = gi.pack_nibbles(A, ld=lda, pad=0x3C)[:, :(k + 1) // 2]
+    Bp = gi.pack_nibbles(B, ld=ldb, pad=0xC3)[:, :(n + 1) // 2]
+    X = C.copy()
+    gm.gemm_i4_host(Ap, Bp, X, k)
+    exp = C.copy()
+    oracle.gemm_i4(np.ascontiguousarray(Ap), np.ascontiguousarray(Bp), exp, k, nthreads=8)
+    assert_same(X, exp, f"host i4 {case}")
