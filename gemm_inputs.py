@@ -23,7 +23,7 @@ those of the GEMM problem of Section 4.1 of the paper at the sizes the
 benchmark studies; the paper itself uses INT16 operands (Section 6.1) and
 lowers convolutions to GEMM through IM2COL/IM2ROW (Sections 2, 4.2, 5.1).
 The int4 workload is the lower-precision point the paper leaves to future
-work (Section 5.1).
+work (Section 6.1).
 Matrix X of workload w is drawn from stream 4*seed_w + {A: 0, B: 1, C: 2}.
 """
 from __future__ import annotations

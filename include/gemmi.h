@@ -83,8 +83,8 @@ int gemm_i8_ex(int64_t m, int64_t n, int64_t k,
 
 /*
  * gemm_i4 -- C (int32) += A (int4) * B (int4), exactly, modulo 2^32.
- * Section 4.1 (problem statement) at a precision below the INT16 / INT8 of Section 6.1; the
- * paper's datatype discussion (Section 5.1) leaves the lower-precision micro-kernel to future work.
+ * Section 4.1 (problem statement) at a precision below the INT16 / INT8 the paper measures; the
+ * paper's datatype discussion (Section 6.1) leaves the lower-precision micro-kernel to future work.
  * Operands are PACKED, two signed 4-bit values to a byte: element (i, p) of A is in byte
  * A[i*lda + p/2], element (p, j) of B in byte B[p*ldb + j/2]; the even index in the low nibble
  * (bits 0-3), the odd one in the high nibble (bits 4-7), two's complement (nibbles 8..15 stand

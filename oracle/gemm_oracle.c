@@ -102,7 +102,7 @@ int gemm_oracle_i8(int64_t m, int64_t n, int64_t k,
 }
 
 /*
- * Lower precision (Section 5.1, the datatype discussion: the INT16 micro-kernel is the paper's
+ * Lower precision (Section 6.1, the datatype discussion: the INT16 micro-kernel is the paper's
  * baseline and its design is to be carried to lower precision).  The int4 variant is the same
  * update with signed 4-bit operands and an int32 C, modulo 2^32.  Two operands share a byte: the
  * element with even index sits in the low nibble (bits 0-3), the one with odd index in the high

@@ -1,7 +1,7 @@
 // int4.cu -- operand conversion for the int4 GEMM, and the add of a scratch result into C.
 //
-// The int4 GEMM (the lower-precision point of Section 5.1: the paper carries its INT16 design to
-// narrower types) runs on the fp8 tensor-core path, tcgen05.mma kind::f8f6f4 with E4M3 operands:
+// The int4 GEMM (a lower-precision point: Section 6.1 leaves the adaptation of the paper's INT16
+// design to narrower types to future work) runs on the fp8 tensor-core path, tcgen05.mma kind::f8f6f4 with E4M3 operands:
 // every integer in [-8, 8] is an E4M3 value exactly (at most three significant bits), so the
 // products, at most 64 in magnitude, are exact and so are fp32 sums of up to 2^18 of them.
 //
