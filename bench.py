@@ -48,7 +48,7 @@ KERNEL_INFO = {
     "tc_pair_i4": ("tc_pair_kernel<1,e4m3>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"),
                    "tensor"),
     "add_i32": ("add_i32", ("int4.cu",), "hbm"),
-    "convert_i4": ("convert_rows_i4+convert_cols_i4", ("int4.cu",), "hbm"),
+    "convert_i4": ("convert_i4_kernel", ("int4.cu",), "hbm"),
 }
 FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
 
