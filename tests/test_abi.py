@@ -96,6 +96,13 @@ def test_i4_argument_checks(L):
     # empty problems and k == 0 are no-ops that touch no device
     assert L.gemm_i4(0, 5, 7, None, 4, None, 3, None, 5) == gm.OK
     assert L.gemm_i4(4, 5, 0, None, 1, None, 3, c, 5) == gm.OK
+    assert L.gemm_i4_host(4, 5, 7, a, 3, b, 3, c, 5) == gm.EINVAL  # the host entry point checks the same
+    # packing B: ldb counts bytes too
+    out = ctypes.c_void_p(0)
+    assert L.gemmi_pack_b_i4(7, 5, b, 2, None, ctypes.byref(out)) == gm.EINVAL   # ldb < ceil(5/2)
+    assert L.gemmi_pack_b_i4(0, 5, b, 3, None, ctypes.byref(out)) == gm.EINVAL
+    assert L.gemmi_pack_b_i4(7, 5, None, 3, None, ctypes.byref(out)) == gm.EINVAL
+    assert out.value is None
 
 
 def test_options(L):

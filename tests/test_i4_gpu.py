@@ -236,3 +236,67 @@ def test_i4_host_buffers(gm, case):
     exp = C.copy()
     oracle.gemm_i4(np.ascontiguousarray(Ap), np.ascontiguousarray(Bp), exp, k, nthreads=8)
     assert_same(X, exp, f"host i4 {case}")
+
+
+def test_i4_captured_in_a_cuda_graph_and_on_a_side_stream(gm):
+    """Captured calls replay exactly -- the aligned-C path and the scratch path (zeroing and the add
+    pass are captured too) -- and calls on a non-default stream order correctly."""
+    s = torch.cuda.Stream()
+    for n, ldc in ((264, 264), (37, 37)):
+        m, k = 300, 333
+        A, B, C = gi.random_problem(8900 + n, m, n, k, "i4")
+        Ap, Bp = gi.pack_nibbles(A), gi.pack_nibbles(B)
+        dA, dB = torch.from_numpy(Ap).cuda(), torch.from_numpy(Bp).cuda()
+        dC = torch.from_numpy(C).cuda()
+        with torch.cuda.stream(s):
+            gm.gemm_i4(dA, dB, torch.from_numpy(C).cuda(), k)  # warm-up outside the capture (workspace growth)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            gm.gemm_i4(dA, dB, dC, k)
+        dC.copy_(torch.from_numpy(C).cuda())
+        g.replay()
+        g.replay()
+        torch.cuda.synchronize()
+        exp = expected(Ap, Bp, C, k)
+        oracle.gemm_i4(Ap, Bp, exp, k)
+        assert_same(dC.cpu().numpy(), exp, f"graph x2 n={n}")
+        # the same call eagerly on a side stream
+        dC2 = torch.from_numpy(C).cuda()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            gm.gemm_i4(dA, dB, dC2, k)
+        s.synchronize()
+        assert_same(dC2.cpu().numpy(), expected(Ap, Bp, C, k), f"side stream n={n}")
+
+
+def test_i4_binding_rejects_bad_arguments(gm):
+    u8 = lambda *shape: torch.zeros(shape, dtype=torch.uint8, device="cuda")  # noqa: E731
+    c32 = torch.zeros((4, 6), dtype=torch.int32, device="cuda")
+    with pytest.raises(TypeError):
+        gm.gemm_i4(torch.zeros((4, 4), dtype=torch.int8, device="cuda"), u8(8, 3), c32, 8)
+    with pytest.raises(TypeError):
+        gm.gemm_i4(u8(4, 4), u8(8, 3), torch.zeros((4, 6), dtype=torch.int64, device="cuda"), 8)
+    with pytest.raises(ValueError):
+        gm.gemm_i4(u8(4, 3), u8(8, 3), c32, 8)      # A holds 6 values per row, k = 8
+    with pytest.raises(ValueError):
+        gm.gemm_i4(u8(4, 4), u8(8, 2), c32, 8)      # B holds 4 values per row, n = 6
+    with pytest.raises(ValueError):
+        gm.gemm_i4(u8(4, 4), u8(7, 3), c32, 8)      # B has 7 rows, k = 8
+    packed = gm.pack_b_i4(u8(8, 3), 6)
+    try:
+        with pytest.raises(TypeError):               # an int4 handle in the int8 call
+            gm.gemm_i8_packed(torch.zeros((4, 8), dtype=torch.int8, device="cuda"), packed, c32)
+        with pytest.raises(ValueError):              # A too narrow for the handle's k
+            gm.gemm_i4_packed(u8(4, 3), packed, c32)
+        # the C ABI itself refuses a handle of another element type
+        lib = gm.lib()
+        assert lib.gemm_i8_packed(4, torch.zeros((4, 8), dtype=torch.int8, device="cuda").data_ptr(), 8,
+                                  packed.handle, c32.data_ptr(), 6, None) == gm.EINVAL
+    finally:
+        packed.close()
+    i8 = gm.pack_b_i8(torch.zeros((8, 6), dtype=torch.int8, device="cuda"))
+    try:
+        assert gm.lib().gemm_i4_packed(4, u8(4, 4).data_ptr(), 4, i8.handle, c32.data_ptr(), 6, None) == gm.EINVAL
+    finally:
+        i8.close()
