@@ -639,6 +639,16 @@ def run_gemmi(args):
         v, t, rows = oracle_rate(w, args.cpu_seconds, cores)
         cpu = {"value": v, "unit": "TOPS", "cores": cores, "kind": "oracle",
                "sample": f"rows 0..{rows - 1} of {w.m} (full n={w.n}, k={w.k}), {t:.1f} s on {cores} threads"}
+        # the two small workloads whole, on one thread (the oracle's plain loop, for scale)
+        single = {}
+        for sname in ("i16_256", "skinny_8x4096x4096"):
+            sw = gi.WORKLOADS[sname]
+            sA, sB, sC = gi.make_inputs(sw)
+            t0 = time.perf_counter()
+            oracle.gemm(sA, sB, sC, nthreads=1)
+            st = time.perf_counter() - t0
+            single[sname] = {"ms": st * 1e3, "TOPS": sw.ops / st / 1e12, "threads": 1}
+        cpu["single_thread_whole_workloads"] = single
 
     if rank == 0:
         line = {
