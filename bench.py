@@ -528,11 +528,12 @@ def run_gemmi(args):
     else:
         host_fn = gm.gemm_i16_host if w.kind == "i16" else gm.gemm_i8_host
     gm.set_stream(torch.cuda.current_stream())
-    # warm-up calls as for the device-resident leg: the first host-path calls of a process pay
-    # one-time costs (the staging buffers' first use) that a short timed loop would average in
+    # warm-up calls as for the device-resident leg (the first host-path call of a process sets up
+    # its staging buffers and streams); the timed loop is long enough (up to 60 calls, about
+    # 0.3 s at 8192^3) that an occasional host-side stall of a few tens of ms weighs little
     for _ in range(max(3, min(args.warmup, 5))):
         host_fn(hA, hB, hC)
-    e2e_steps = max(3, min(args.steps, 20))
+    e2e_steps = max(3, min(args.steps, 60))
     if world > 1:
         dist.barrier()
     t0 = time.perf_counter()
