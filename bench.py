@@ -224,25 +224,38 @@ def run_reference(args):
     # one step = the oracle on a bounded row sample; the whole run is kept near 90 s of CPU time
     step_s = min(1.5, max(0.05, 90.0 / max(1, args.steps + args.warmup)))
     _, B, _ = gi.make_inputs(w, rows=slice(0, 1))
-    A1, _, C1 = gi.make_inputs(w, rows=slice(0, min(w.m, threads)))
+    if w.kind == "i4":  # the oracle takes the operands in their packed form
+        B = gi.pack_nibbles(B)
+
+    def run(A, X):
+        if w.kind == "i4":
+            oracle.gemm_i4(A, B, X, w.k, nthreads=threads)
+        else:
+            oracle.gemm(A, B, X, nthreads=threads)
+
+    def rows_of(r):
+        A, _, C = gi.make_inputs(w, rows=slice(0, r))
+        return (gi.pack_nibbles(A) if w.kind == "i4" else A), C
+
+    A1, C1 = rows_of(min(w.m, threads))
     t0 = time.perf_counter()
-    oracle.gemm(A1, B, C1, nthreads=threads)
+    run(A1, C1)
     per_row = (time.perf_counter() - t0) / A1.shape[0]
     rows = int(max(1, min(w.m, step_s / max(per_row, 1e-9))))
-    A, _, C = gi.make_inputs(w, rows=slice(0, rows))
+    A, C = rows_of(rows)
     for _ in range(args.warmup):
-        oracle.gemm(A, B, C.copy(), nthreads=threads)
+        run(A, C.copy())
     times = []
     for _ in range(args.steps):
         X = C.copy()
         t0 = time.perf_counter()
-        oracle.gemm(A, B, X, nthreads=threads)
+        run(A, X)
         times.append(time.perf_counter() - t0)
     t = sum(times) / len(times)
     ops = 2 * rows * w.n * w.k
     value = ops / t / 1e12
     sample = f"rows 0..{rows - 1} of {w.m} (full n={w.n}, k={w.k}) per step"
-    line = {"metric": "int16 GEMM TOPS (2mnk/s)" if w.kind == "i16" else "int8 GEMM TOPS (2mnk/s)",
+    line = {"metric": {"i16": "int16", "i8": "int8", "i4": "int4"}[w.kind] + " GEMM TOPS (2mnk/s)",
             "value": value, "unit": "TOPS", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "int64" if w.kind == "i16" else "int32", "data": "synthetic (seeded SplitMix64)",

@@ -65,3 +65,23 @@ def test_reference_arm_runs_on_rank_0_only(monkeypatch):
     monkeypatch.setenv("WORLD_SIZE", "2")
     args = bench.parse_args_list(["--impl", "reference", "--steps", "1", "--warmup", "0"])
     assert bench.run_reference(args) == 0
+
+
+@pytest.mark.parametrize("workload", ["i16_256", "i4_8192"])
+def test_reference_arm_prints_one_json_line(workload):
+    # the reference arm is the CPU oracle on bounded row samples: it runs here, without a GPU
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload", workload,
+                        "--steps", "2", "--warmup", "1"], capture_output=True, text=True, timeout=600,
+                       env={**os.environ, "RANK": "0", "WORLD_SIZE": "1"})
+    assert r.returncode == 0, r.stderr
+    lines = [ln for ln in r.stdout.splitlines() if ln.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["steps"] == 2 and d["warmup"] == 1
+    assert d["metric"].startswith({"i16_256": "int16", "i4_8192": "int4"}[workload])
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["config"]["workload"] == workload
