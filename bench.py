@@ -50,7 +50,8 @@ KERNEL_INFO = {
     "add_i32": ("add_i32", ("int4.cu",), "hbm"),
     "convert_i4": ("convert_i4_kernel", ("int4.cu",), "hbm"),
 }
-FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
+FP8_PER_BF16 = 2.0
+FULL16_RANGE = ("uniform", -32768, 32767)  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
 
 
 def parse_args():
@@ -618,10 +619,12 @@ def run_gemmi(args):
             else:
                 ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
             extra[name + "_packed_b"] = ent
-        # the precision sweep at equal sizes: int8 at 8192^3 and int4 at 4096^3 beside the table's
-        # int16 / int4 8192^3 and int8 4096^3 (same value distributions as those workloads)
+        # the precision sweep at equal sizes: int16 at 4096^3, int8 at 8192^3 and int4 at 4096^3
+        # beside the table's int16 / int4 8192^3 and int8 4096^3 (same value distributions)
         sweep = {}
-        for sw in (gi.Workload("i8_8192", "i8", 8192, 8192, 8192, 1008, ("uniform", -128, 127),
+        for sw in (gi.Workload("i16_4096", "i16", 4096, 4096, 4096, 1010, FULL16_RANGE, FULL16_RANGE, ("zero",),
+                               "int16 GEMM 4096^3"),
+                   gi.Workload("i8_8192", "i8", 8192, 8192, 8192, 1008, ("uniform", -128, 127),
                                ("uniform", -128, 127), ("zero",), "int8 GEMM 8192^3"),
                    gi.Workload("i4_4096", "i4", 4096, 4096, 4096, 1009, ("uniform", -8, 7), ("uniform", -8, 7),
                                ("zero",), "int4 GEMM 4096^3")):
