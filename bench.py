@@ -50,8 +50,8 @@ KERNEL_INFO = {
     "add_i32": ("add_i32", ("int4.cu",), "hbm"),
     "convert_i4": ("convert_i4_kernel", ("int4.cu",), "hbm"),
 }
-FP8_PER_BF16 = 2.0
-FULL16_RANGE = ("uniform", -32768, 32767)  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
+FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
+FULL16_RANGE = ("uniform", -32768, 32767)
 
 
 def parse_args():
