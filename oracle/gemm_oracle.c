@@ -20,7 +20,10 @@
  * and commutative, the final C is unique whatever order a fast implementation
  * sums in, so the comparison against a GPU result is bit-exact.  The int8
  * variant is the same update with int8 operands and an int32 C, taken modulo
- * 2^32 (computed in 64 bits, then truncated, which is the same thing).
+ * 2^32 (computed in 64 bits, then truncated, which is the same thing).  Further
+ * down: the int4 variant (operands packed two to a byte), the paper's
+ * micro-kernel output (shift, round, saturate to int16) and the convolution
+ * written out from its definition; each states its own layout.
  *
  * Storage is row-major with leading dimensions: A[i*lda+p], B[p*ldb+j],
  * C[i*ldc+j]; entries of C outside the m x n block are never read or written.
