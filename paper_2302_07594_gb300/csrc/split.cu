@@ -204,6 +204,8 @@ constexpr int STG = 16384;
 constexpr int NBAR = 2 * STAGES + 4;  // full, empty, staging full x2, staging free x2
 constexpr size_t SMEM = 1024 + STAGES * RAW + 2 * STG + 8 * NBAR;
 static_assert((RAW / 16) % CONSUMERS == 0, "whole raw chunks per consumer thread");
+constexpr int CTAS_PER_SM = 3;  // 65 KB of shared memory each: three fit in an SM's 228 KB
+static_assert(CTAS_PER_SM * SMEM <= 228 * 1024, "resident CTAs per SM");
 }  // namespace tsplit
 
 struct TmaSplitParams {
@@ -453,6 +455,23 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
   if (tid == 0) bulk_wait_all();
 }
 
+// Streaming multiprocessors of the current device (queried once per device).
+int device_sms() {
+  static int sms[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return 148;
+  if (sms[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
+      cudaGetLastError();
+      v = 148;
+    }
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
 template <typename T, int NL>
 bool launch_tma(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int64_t n, int64_t k, LimbPlanes pa,
                 LimbPlanes pb, cudaStream_t s, uint32_t* status, uint64_t timeout_ns, cudaError_t* err) {
@@ -509,7 +528,8 @@ bool launch_tma(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, int
     }
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
   }
-  const int64_t grid = items < 152 * 3 ? items : 152 * 3;
+  const int64_t resident = static_cast<int64_t>(device_sms()) * tsplit::CTAS_PER_SM;
+  const int64_t grid = items < resident ? items : resident;
   split_tma_kernel<T, NL><<<static_cast<unsigned>(grid), tsplit::THREADS, tsplit::SMEM, s>>>(maps[0], maps[1], maps[2],
                                                                                             maps[3], P);
   *err = cudaGetLastError();
@@ -530,11 +550,12 @@ cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, 
   // A null operand is skipped (packing only the weights, or only the activations).
   const int64_t a_rows = A != nullptr ? m : 0;
   int64_t a_blocks = (a_rows + WARPS - 1) / WARPS;
-  if (a_blocks > 152 * 8) a_blocks = 152 * 8;
+  const int64_t cap = static_cast<int64_t>(device_sms()) * 8;
+  if (a_blocks > cap) a_blocks = cap;
   const int64_t tiles_p = (pb.pitch + TT - 1) / TT;  // cover the zero padding up to the pitch too
   const int64_t tiles_j = B != nullptr ? (n + TT - 1) / TT : 0;
   const int64_t b_tiles = tiles_p * tiles_j;
-  int64_t b_blocks = b_tiles < 152 * 8 ? b_tiles : 152 * 8;
+  int64_t b_blocks = b_tiles < cap ? b_tiles : cap;
   if (a_blocks + b_blocks < 1) return cudaSuccess;
   split_kernel<T, NL><<<static_cast<unsigned>(a_blocks + b_blocks), THREADS, 0, s>>>(
       a, b, static_cast<int>(a_blocks), tiles_j, b_tiles);
