@@ -19,7 +19,7 @@ torch = pytest.importorskip("torch")
 EDGE = [1, 2, 3, 7, 8, 15, 16, 17, 31, 33, 63, 64, 65, 127, 128, 129, 255, 256, 257]
 
 
-def draw_cases(count=72, seed=20230215):
+def draw_cases(count=240, seed=20230215):
     rng = np.random.default_rng(seed)
 
     def dim(lo, hi):
