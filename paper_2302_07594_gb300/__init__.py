@@ -6,8 +6,11 @@ no CPU fallback: if the library is missing, every call raises.
 
     gemm_i16(A, B, C)       torch CUDA tensors: int16 A (m x k), B (k x n), int64 C (m x n)
     gemm_i8(A, B, C)        torch CUDA tensors: int8 A, B, int32 C
+    gemm_i4(A, B, C, k)     torch CUDA tensors: uint8 A, B holding int4 values two to a byte, int32 C
     gemm_i16_host(A, B, C)  numpy arrays (host memory): the library copies in and out
-    gemm_i8_host(A, B, C)
+    gemm_i8_host(A, B, C), gemm_i4_host(A, B, C, k)
+    pack_b_i16 / pack_b_i8 / pack_b_i4, gemm_*_packed   weights split once, reused by every call
+    gemm_i16_srs, conv2d_i16, gemm_i16_noalloc          the other entry points of include/gemmi.h
 
 Matrices are row-major with unit column stride; a row stride larger than the
 row length (padding) is passed as the leading dimension.  C is updated in
