@@ -783,6 +783,92 @@ int host_gemm(int64_t m, int64_t n, int64_t k, const OP* A, int64_t lda, const O
   return GEMMI_OK;
 }
 
+// gemm_i4 on host buffers with m >= 2 * kPanelMin, pipelined like host_gemm_pipelined: B is copied
+// and converted to its E4M3 plane once, then row panels of A and C pass through kPipeSlots device
+// slots, copies in and out on their own streams while each panel's GEMM runs on the caller's
+// stream.  Device pitches (16 bytes for packed operands, 4 elements for C) keep every kernel on
+// its aligned path.
+int host_gemm_i4_pipelined(DeviceState& d, int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda,
+                           const uint8_t* B, int64_t ldb, int32_t* C, int64_t ldc) {
+  int rc = ensure_pipeline(d);
+  if (rc != GEMMI_OK) return rc;
+  cudaStream_t s = g_stream;
+  const int64_t wa = (k + 1) / 2, wb = (n + 1) / 2;
+  const int64_t dlda = static_cast<int64_t>(round_up(static_cast<size_t>(wa), 16));
+  const int64_t dldb = static_cast<int64_t>(round_up(static_cast<size_t>(wb), 16));
+  const int64_t dldc = static_cast<int64_t>(round_up(static_cast<size_t>(n), 4));
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 16));
+  const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 15) / 16), 128)));
+  const int64_t panels = (m + mb - 1) / mb;
+  const size_t b_raw = round_up(static_cast<size_t>(k) * dldb, kAlign);
+  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch, kAlign);
+  const size_t a_slot = round_up(static_cast<size_t>(mb) * dlda, kAlign);
+  const size_t c_slot = round_up(static_cast<size_t>(mb) * dldc * 4, kAlign);
+  if ((rc = ensure_buffer(&d.host_buf, &d.host_buf_bytes, b_raw + b_plane + kPipeSlots * (a_slot + c_slot))) !=
+      GEMMI_OK)
+    return rc;
+  // one panel's A plane, sized now so no panel has to grow the workspace mid-pipeline
+  if ((rc = ensure_buffer(&d.ws, &d.ws_bytes, round_up(static_cast<size_t>(mb) * pitch, kAlign))) != GEMMI_OK)
+    return rc;
+  char* base = static_cast<char*>(d.host_buf);
+  uint8_t* dB = reinterpret_cast<uint8_t*>(base);
+  const LimbPlanes pb{{base + b_raw, nullptr}, n, pitch};
+  char* slots = base + b_raw + b_plane;
+  cudaEvent_t* ev = d.pipe_ev;  // 0 start, 1 B copied, 2-4 panel in, 5-7 panel done, 8-10 panel out, 11 end
+  auto settle = [&]() {
+    cudaStreamSynchronize(d.h2d);
+    cudaStreamSynchronize(s);
+    cudaStreamSynchronize(d.d2h);
+  };
+  auto fail = [&](cudaError_t e, const char* what) {
+    settle();
+    return cuda_error(e, what);
+  };
+  cudaError_t e = cudaEventRecord(ev[0], s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(d.h2d, ev[0], 0);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(d.d2h, ev[0], 0);
+  if (e == cudaSuccess) e = cudaMemcpy2DAsync(dB, dldb, B, ldb, wb, k, cudaMemcpyHostToDevice, d.h2d);
+  if (e == cudaSuccess) e = cudaEventRecord(ev[1], d.h2d);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[1], 0);
+  if (e != cudaSuccess) return fail(e, "host-to-device copy of B");
+  {
+    const LimbPlanes none{{nullptr, nullptr}, 0, pitch};
+    cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_CONVERT_I4, s);
+    e = gemmi::convert_i4(nullptr, 1, dB, dldb, 0, n, k, none, pb, d.sm_count, s);
+    timer_end(GEMMI_KERNEL_CONVERT_I4, t0, s);
+    if (e != cudaSuccess) return fail(e, "conversion of B");
+  }
+  for (int64_t p = 0; p < panels; ++p) {
+    const int r = static_cast<int>(p % kPipeSlots);
+    const int64_t r0 = p * mb, mi = std::min(mb, m - r0);
+    uint8_t* dA = reinterpret_cast<uint8_t*>(slots + r * (a_slot + c_slot));
+    int32_t* dC = reinterpret_cast<int32_t*>(slots + r * (a_slot + c_slot) + a_slot);
+    e = p >= kPipeSlots ? cudaStreamWaitEvent(d.h2d, ev[8 + r], 0) : cudaSuccess;  // slot's last copy out
+    if (e == cudaSuccess) e = cudaMemcpy2DAsync(dA, dlda, A + r0 * lda, lda, wa, mi, cudaMemcpyHostToDevice, d.h2d);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(dC, dldc * 4, C + r0 * ldc, ldc * 4, n * 4, mi, cudaMemcpyHostToDevice, d.h2d);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[2 + r], d.h2d);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[2 + r], 0);
+    if (e != cudaSuccess) return fail(e, "host-to-device copy of a panel");
+    rc = run_i4(d, mi, n, k, dA, dlda, nullptr, dldb, dC, dldc, s, &pb);
+    if (rc != GEMMI_OK) {
+      settle();
+      return rc;
+    }
+    e = cudaEventRecord(ev[5 + r], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(d.d2h, ev[5 + r], 0);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(C + r0 * ldc, ldc * 4, dC, dldc * 4, n * 4, mi, cudaMemcpyDeviceToHost, d.d2h);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[8 + r], d.d2h);
+    if (e != cudaSuccess) return fail(e, "device-to-host copy of a panel");
+  }
+  e = cudaEventRecord(ev[11], d.d2h);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[11], 0);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return fail(e, "cudaStreamSynchronize");
+  return GEMMI_OK;
+}
+
 // gemm_i4 on host buffers: packed A and B and C are copied into device buffers whose row pitches
 // (16 bytes for the operands, 4 elements for C) keep the conversion and the pair kernel on their
 // aligned paths, the GEMM runs, and C is copied back.
@@ -794,6 +880,15 @@ int host_gemm_i4(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t lda,
   DeviceState* d = nullptr;
   int rc = device_state(&d);
   if (rc != GEMMI_OK) return rc;
+  if (m >= 2 * kPanelMin) {
+    rc = host_gemm_i4_pipelined(*d, m, n, k, A, lda, B, ldb, C, ldc);
+    if (rc != GEMMI_OK) return rc;
+    uint32_t word = 0;
+    const cudaError_t e = cudaMemcpy(&word, d->status, sizeof(word), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
+    if (word != 0) return read_status_locked(*d, true);
+    return GEMMI_OK;
+  }
   const int64_t wa = (k + 1) / 2, wb = (n + 1) / 2;
   const int64_t dlda = static_cast<int64_t>(round_up(static_cast<size_t>(wa), 16));
   const int64_t dldb = static_cast<int64_t>(round_up(static_cast<size_t>(wb), 16));

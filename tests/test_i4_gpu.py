@@ -224,8 +224,10 @@ def test_i4_packed_weights(gm, case):
         packed.close()
 
 
-@pytest.mark.parametrize("case", [(300, 201, 333, None, None), (129, 64, 1000, 520, 40)])
+@pytest.mark.parametrize("case", [(300, 201, 333, None, None), (129, 64, 1000, 520, 40), (2100, 301, 777, 400, 160),
+                                  (1024, 64, 256, None, None)])
 def test_i4_host_buffers(gm, case):
+    # m >= 1024 takes the pipelined host path (row panels through device slots)
     # host arrays with padded byte pitches; the library stages them on the device with aligned pitches
     m, n, k, lda, ldb = case
     A, B, C = gi.random_problem(8800 + m, m, n, k, "i4")
