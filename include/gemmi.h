@@ -110,8 +110,10 @@ int gemm_i4_ex(int64_t m, int64_t n, int64_t k,
  * A, B, C are host pointers (pinned memory gives the fastest copies).  The
  * library copies A, B and C to device buffers it owns, runs the GEMM on its
  * current stream, copies C back and waits for the stream, so C holds the
- * result when the call returns.  Errors as above; a device-side timeout is
- * returned directly as GEMMI_ETIMEOUT.
+ * result when the call returns.  With m >= 1024 the copies are pipelined:
+ * B goes over once, then row panels of A and C pass through a ring of device
+ * slots on separate copy-in and copy-out streams while earlier panels compute.
+ * Errors as above; a device-side timeout is returned directly as GEMMI_ETIMEOUT.
  */
 int gemm_i16_host(int64_t m, int64_t n, int64_t k,
                   const int16_t* A, int64_t lda,
