@@ -103,6 +103,9 @@ def test_i4_argument_checks(L):
     assert L.gemmi_pack_b_i4(0, 5, b, 3, None, ctypes.byref(out)) == gm.EINVAL
     assert L.gemmi_pack_b_i4(7, 5, None, 3, None, ctypes.byref(out)) == gm.EINVAL
     assert out.value is None
+    # the packed entry point checks its handle and A before any device work
+    assert L.gemm_i4_packed(4, a, 4, None, c, 5, None) == gm.EINVAL
+    assert L.gemm_i4_packed(-1, a, 4, None, c, 5, None) == gm.EINVAL
 
 
 def test_options(L):

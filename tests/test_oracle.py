@@ -93,6 +93,16 @@ def test_i4_packer_matches_golden_bytes():
     assert gi.pack_nibbles(v, ld=4, pad=0x55).tolist() == [[0x21, 0x8F, 0x53, 0x55]]
 
 
+def test_i4_packer_rejects_bad_input():
+    with pytest.raises(ValueError):
+        gi.pack_nibbles(np.array([[8]], np.int8))           # outside [-8, 7]
+    with pytest.raises(ValueError):
+        gi.pack_nibbles(np.array([[-9, 0]], np.int8))
+    with pytest.raises(ValueError):
+        gi.pack_nibbles(np.zeros((2, 5), np.int8), ld=2)    # pitch below ceil(5/2) = 3 bytes
+    assert gi.pack_nibbles(np.zeros((0, 5), np.int8)).shape == (0, 3)
+
+
 def test_i4_invalid_arguments_rejected(lib):
     b = np.zeros((4, 4), np.uint8)
     c = np.zeros((4, 4), np.int32)
