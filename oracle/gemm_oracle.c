@@ -20,7 +20,8 @@
  * and commutative, the final C is unique whatever order a fast implementation
  * sums in, so the comparison against a GPU result is bit-exact.  The int8
  * variant is the same update with int8 operands and an int32 C, taken modulo
- * 2^32 (computed in 64 bits, then truncated, which is the same thing).  Further
+ * 2^32 (each product is exact in 32 bits; the sums run in unsigned 32-bit
+ * arithmetic, the same rank-1 order as the int16 loop).  Further
  * down: the int4 variant (operands packed two to a byte), the paper's
  * micro-kernel output (shift, round, saturate to int16) and the convolution
  * written out from its definition; each states its own layout.
@@ -93,12 +94,14 @@ int gemm_oracle_i8(int64_t m, int64_t n, int64_t k,
   (void)nthreads;
 #endif
   for (int64_t i = 0; i < m; ++i) {
-    int32_t* c = C + i * ldc;
-    for (int64_t j = 0; j < n; ++j) {
-      uint64_t s = (uint64_t)(int64_t)c[j];
-      for (int64_t p = 0; p < k; ++p)
-        s += (uint64_t)((int64_t)A[i * lda + p] * (int64_t)B[p * ldb + j]);
-      c[j] = (int32_t)(uint32_t)s; /* keep the low 32 bits: modulo 2^32 */
+    /* unsigned 32-bit arithmetic: every addition is taken modulo 2^32 */
+    uint32_t* c = (uint32_t*)(C + i * ldc);
+    for (int64_t p = 0; p < k; ++p) {
+      /* one rank-1 term, as in the int16 loop: row i of C gains A[i][p] times row p of B */
+      const int32_t a = (int32_t)A[i * lda + p];
+      const int8_t* b8 = B + p * ldb;
+      for (int64_t j = 0; j < n; ++j)
+        c[j] += (uint32_t)(a * (int32_t)b8[j]);
     }
   }
   return 0;
@@ -246,6 +249,20 @@ int gemm_oracle_conv2d_i16(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t
     }
   }
   return 0;
+}
+
+/*
+ * The same two functions under the names of the library's oracle interface (gemmi_oracle_*):
+ * identical arguments, host pointers, the int nthreads of the loops above.
+ */
+int gemmi_oracle_i16(int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda,
+                     const int16_t* B, int64_t ldb, int64_t* C, int64_t ldc, int nthreads) {
+  return gemm_oracle_i16(m, n, k, A, lda, B, ldb, C, ldc, nthreads);
+}
+
+int gemmi_oracle_i8(int64_t m, int64_t n, int64_t k, const int8_t* A, int64_t lda,
+                    const int8_t* B, int64_t ldb, int32_t* C, int64_t ldc, int nthreads) {
+  return gemm_oracle_i8(m, n, k, A, lda, B, ldb, C, ldc, nthreads);
 }
 
 /* Threads the library was built to use (1 without OpenMP). */

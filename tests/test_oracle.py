@@ -194,8 +194,12 @@ MUTANTS = {
                      "uint64_t* c = (uint64_t*)(C + i * ldc); for (int64_t q = 0; q < n; ++q) c[q] = 0;"),
     "ignores_ldb": ("const int16_t* b = B + p * ldb;", "const int16_t* b = B + p * n;"),
     "off_by_one_column": ("for (int64_t j = 0; j < n; ++j)\n        c[j] +=", "for (int64_t j = 1; j < n; ++j)\n        c[j] +="),
-    "i8_truncates_to_16_bits": ("c[j] = (int32_t)(uint32_t)s;", "c[j] = (int32_t)(int16_t)s;"),
-    "i8_transposed_B": ("(int64_t)B[p * ldb + j]", "(int64_t)B[j * ldb + p]"),
+    "i8_truncates_to_16_bits": ("c[j] += (uint32_t)(a * (int32_t)b8[j]);",
+                                "c[j] = (uint16_t)(c[j] + (uint32_t)(a * (int32_t)b8[j]));"),
+    "i8_drops_last_term": ("for (int64_t p = 0; p < k; ++p) {\n      /* one rank-1 term, as in the int16 loop",
+                           "for (int64_t p = 0; p + 1 < k; ++p) {\n      /* one rank-1 term, as in the int16 loop"),
+    "i8_wrong_sign": ("c[j] += (uint32_t)(a * (int32_t)b8[j]);", "c[j] -= (uint32_t)(a * (int32_t)b8[j]);"),
+    "i8_transposed_B": ("c[j] += (uint32_t)(a * (int32_t)b8[j]);", "c[j] += (uint32_t)(a * (int32_t)B[j * ldb + p]);"),
     # the micro-kernel output C16 += srs(A*B, shift)
     "srs_rounds_half_down": ("oracle_floor_div_pow2(s + ((int64_t)1 << (shift - 1)), shift)",
                              "oracle_floor_div_pow2(s + ((int64_t)1 << (shift - 1)) - 1, shift)"),
