@@ -2,9 +2,9 @@
 
 Expected values always come from the oracle (oracle/) run on the same seeded
 inputs (gemm_inputs.py); nothing here is produced by the CUDA path itself.
-The full-size workloads are checked on sampled rows (which the oracle
-computes one row block at a time) plus a row-sum/column-sum identity that
-covers every output:  sum_j C[i,j] = A[i,:] . (B 1),  sum_i C[i,j] = (1^T A) . B[:,j].
+The five full-size workloads are compared on every output element; the
+int4 workload on sampled rows plus a row-sum/column-sum identity that covers
+every output:  sum_j C[i,j] = A[i,:] . (B 1),  sum_i C[i,j] = (1^T A) . B[:,j].
 """
 import numpy as np
 import pytest
@@ -294,6 +294,13 @@ def test_skinny_extremes(gm):
 
 
 # ------------------------------------------------------------------ the five workloads
+# The five workloads of the exact-GEMM problem statement (paper Section 4.1) are compared with the
+# oracle on EVERY output element, at full size, on all host cores.  The int4 workload (a lower-
+# precision extension, Section 6.1) is compared on sampled rows only; every one of its outputs is
+# still covered by the row and column sums below.
+FULL_WORKLOADS = ("i16_256", "i8_4096", "conv3x3_im2col", "i16_8192", "skinny_8x4096x4096")
+
+
 def _sample_rows(m, count=24):
     rows = {0, 1, m - 1, m // 2, 127, 128, m - 129}
     rng = gi.uniform_int(4242 + m, (count,), 0, m - 1, np.int64)
@@ -301,22 +308,9 @@ def _sample_rows(m, count=24):
     return sorted(r for r in rows if 0 <= r < m)
 
 
-@pytest.mark.parametrize("name", list(gi.WORKLOADS))
-def test_workload(gm, name):
-    w = gi.WORKLOADS[name]
-    A, B, C = gi.make_inputs(w)
-    got = run_gpu(gm, A, B, C, w.kind)
-    if w.m * w.n * w.k <= 1 << 28:
-        assert_same(got, expected(A, B, C), name)
-        return
-    rows = _sample_rows(w.m)
-    if w.kind == "i4":
-        exp = C[rows].copy()
-        oracle.gemm_i4(gi.pack_nibbles(A[rows]), gi.pack_nibbles(B), exp, w.k, nthreads=8)
-    else:
-        exp = expected(A[rows], B, C[rows])
-    assert_same(got[rows], exp, f"{name} sampled rows {rows[:4]}...")
-    # every output through row and column sums (exact int64 arithmetic modulo 2^64)
+def _check_sums(name, kind, A, B, C, got):
+    """Every output through row and column sums (exact int64 arithmetic modulo 2^64): an extra
+    check beside the element-wise comparison."""
     with np.errstate(over="ignore"):
         Bsum = B.astype(np.int64).sum(axis=1)
         row_exp = A.astype(np.int64) @ Bsum + C.astype(np.int64).sum(axis=1)
@@ -324,10 +318,41 @@ def test_workload(gm, name):
         col_exp = Asum @ B.astype(np.int64) + C.astype(np.int64).sum(axis=0)
         row_got = got.astype(np.int64).sum(axis=1)
         col_got = got.astype(np.int64).sum(axis=0)
-    if w.kind != "i16":  # int32 C: the sums compare modulo 2^32
+    if kind != "i16":  # int32 C: the sums compare modulo 2^32
         row_exp, row_got, col_exp, col_got = (x & 0xFFFFFFFF for x in (row_exp, row_got, col_exp, col_got))
     assert np.array_equal(row_got, row_exp), f"{name}: row sums differ"
     assert np.array_equal(col_got, col_exp), f"{name}: column sums differ"
+
+
+def test_five_workloads_are_listed():
+    assert set(FULL_WORKLOADS) <= set(gi.WORKLOADS)
+
+
+@pytest.mark.parametrize("name", FULL_WORKLOADS)
+def test_workload_every_element(gm, name):
+    """Full-size workload, every element of C against the oracle (all host cores)."""
+    w = gi.WORKLOADS[name]
+    A, B, C = gi.make_inputs(w)
+    got = run_gpu(gm, A, B, C, w.kind)
+    assert_same(got, expected(A, B, C, threads=oracle.host_cores()), f"{name} (all {w.m}x{w.n} outputs)")
+    _check_sums(name, w.kind, A, B, C, got)
+
+
+@pytest.mark.parametrize("name", [n for n in gi.WORKLOADS if n not in FULL_WORKLOADS])
+def test_workload_sampled(gm, name):
+    """Workloads beyond the five (int4 8192^3): sampled rows through the oracle, all outputs
+    through row and column sums."""
+    w = gi.WORKLOADS[name]
+    A, B, C = gi.make_inputs(w)
+    got = run_gpu(gm, A, B, C, w.kind)
+    rows = _sample_rows(w.m)
+    if w.kind == "i4":
+        exp = C[rows].copy()
+        oracle.gemm_i4(gi.pack_nibbles(A[rows]), gi.pack_nibbles(B), exp, w.k, nthreads=oracle.host_cores())
+    else:
+        exp = expected(A[rows], B, C[rows], threads=oracle.host_cores())
+    assert_same(got[rows], exp, f"{name} sampled rows {rows[:4]}...")
+    _check_sums(name, w.kind, A, B, C, got)
 
 
 # ------------------------------------------------------------------ host-buffer API, streams, failure detection
