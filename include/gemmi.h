@@ -222,11 +222,21 @@ const char* gemmi_last_error(void);
 
 /*
  * Synchronises the current device and returns, then clears, its device status
- * word: GEMMI_OK, or GEMMI_ETIMEOUT if a kernel gave up a pipeline wait.
+ * words: GEMMI_OK, or GEMMI_ETIMEOUT if a kernel gave up a pipeline wait.  Two
+ * words are read: the library's own (written by every entry point except
+ * gemm_i16_noalloc) and, once gemm_i16_noalloc has run on the device, the word
+ * inside that entry point's fixed scratch array.  The first non-zero word
+ * decides the result; every non-zero word is cleared.
+ * gemmi_device_status_stream(stream) does the same after synchronising only
+ * `stream` (a cudaStream_t as void*; NULL = legacy default stream): it sees the
+ * failures of the kernels that stream ran, and of any other kernel that had
+ * finished by then.  Section 6.2 of the paper makes the accumulators wide so
+ * that nothing overflows; a wait that ran out is the one failure left to report.
  * gemmi_device_status_detail() returns the raw word of the last read
  * (low byte: status code; next byte: the wait site; upper half: block index).
  */
 int gemmi_device_status(void);
+int gemmi_device_status_stream(void* stream);
 uint32_t gemmi_device_status_detail(void);
 
 /* Frees the library-owned device workspace of the current device (synchronises it). */
@@ -317,14 +327,22 @@ int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
  * process exits.
  *
  * Same operation, layout, pointer ownership (DEVICE pointers owned by the
- * caller) and bit-exact result as gemm_i16, always on the tensor-core path,
- * asynchronous on `stream` (a cudaStream_t as void*; NULL = legacy default stream).
+ * caller) and bit-exact result as gemm_i16, always on the tensor-core path
+ * (the limb split, then the one-SM-per-tile tcgen05 kernel, whose 128x128 tiles
+ * cover problems of this size), asynchronous on `stream` (a cudaStream_t as
+ * void*; NULL = legacy default stream).
  * Limit: 4*(m+n)*roundup(k,8) + 256 <= GEMMI_NOALLOC_SCRATCH_BYTES (for m = n = k,
  * up to about 2000); larger problems return GEMMI_EINVAL with a message saying so.
  * The first call on a device looks up the array's device address (with that
  * device current) and caches it; make that first call before any stream capture.
  * Every call shares the one array: calls that overlap on the GPU (on different
  * streams, or from several threads) race on it and must be serialised by the caller.
+ * Every plane byte a call reads is written by that call first, so what an
+ * earlier call left in the array never reaches C.
+ * Device-side failures: both kernels bound their pipeline waits by
+ * GEMMI_OPT_WAIT_TIMEOUT_US and record a wait that ran out in a status word at
+ * the start of the array (sticky until read); gemmi_device_status() and
+ * gemmi_device_status_stream() read and clear it.
  * Returns GEMMI_OK, GEMMI_EINVAL, GEMMI_ECUDA or GEMMI_EARCH.
  */
 #define GEMMI_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
@@ -332,6 +350,16 @@ int gemm_i16_noalloc(int64_t m, int64_t n, int64_t k,
                      const int16_t* A, int64_t lda,
                      const int16_t* B, int64_t ldb,
                      int64_t* C, int64_t ldc, void* stream);
+
+/*
+ * Failure-detection self-test of gemm_i16_noalloc's status word (no paper
+ * counterpart, like the entry point itself): launches, on `stream`, the probe of
+ * gemmi_selftest_wait_timeout with the word inside the fixed scratch array as
+ * its status word (setting up the array's address on first use, as the entry
+ * point does).  Allocates nothing.  Returns GEMMI_OK once launched; a following
+ * gemmi_device_status_stream(stream) then returns GEMMI_ETIMEOUT.
+ */
+int gemmi_noalloc_selftest_wait_timeout(int64_t timeout_us, void* stream);
 
 /* Library version string. */
 const char* gemmi_version(void);

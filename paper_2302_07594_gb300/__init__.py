@@ -30,7 +30,8 @@ OPT_SKINNY_MAX_M, OPT_WAIT_TIMEOUT_US, OPT_SKINNY_KSPLIT = 1, 2, 3
 OPT_TC_CHUNK_SCALE, OPT_TC_GROUP_M, OPT_TC_L2_HINTS, OPT_FUSED_MAX_N, OPT_TC_PAIR = 4, 5, 6, 7, 8
 OPT_SMALL_MAX_MACS = 9
 EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
-            "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_detail",
+            "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_stream",
+            "gemmi_device_status_detail", "gemmi_noalloc_selftest_wait_timeout",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
@@ -84,6 +85,10 @@ def lib():
         L.gemmi_set_stream.restype = None
         L.gemmi_last_error.restype = ctypes.c_char_p
         L.gemmi_device_status.restype = ctypes.c_int
+        L.gemmi_device_status_stream.argtypes = [vp]
+        L.gemmi_device_status_stream.restype = ctypes.c_int
+        L.gemmi_noalloc_selftest_wait_timeout.argtypes = [i64, vp]
+        L.gemmi_noalloc_selftest_wait_timeout.restype = ctypes.c_int
         L.gemmi_device_status_detail.restype = ctypes.c_uint32
         L.gemmi_release_workspace.restype = ctypes.c_int
         L.gemmi_workspace_bytes.restype = ctypes.c_size_t
@@ -439,6 +444,13 @@ def set_stream(stream) -> None:
 def device_status() -> int:
     """Synchronises the device; returns and clears its status word (OK or ETIMEOUT)."""
     return int(lib().gemmi_device_status())
+
+
+def device_status_stream(stream=None) -> int:
+    """Synchronises one stream (a torch.cuda.Stream, a raw cudaStream_t or None for the legacy
+    default stream); returns and clears the device's status words (OK or ETIMEOUT)."""
+    handle = getattr(stream, "cuda_stream", stream)
+    return int(lib().gemmi_device_status_stream(ctypes.c_void_p(handle or 0)))
 
 
 def device_status_detail() -> int:

@@ -212,6 +212,17 @@ bool overlaps(const void* a, size_t abytes, const void* b, size_t bbytes) {
   return a0 < b0 + bbytes && b0 < a0 + abytes;
 }
 
+// Bytes spanned by `rows` rows (rows >= 1) of `cols` elements at pitch `ld` elements, or false on
+// 64-bit overflow (a huge leading dimension).
+bool span_bytes(int64_t rows, int64_t ld, int64_t cols, size_t esize, size_t* out) {
+  uint64_t a = 0, b = 0, c = 0;
+  if (__builtin_mul_overflow(static_cast<uint64_t>(rows - 1), static_cast<uint64_t>(ld), &a)) return false;
+  if (__builtin_add_overflow(a, static_cast<uint64_t>(cols), &b)) return false;
+  if (__builtin_mul_overflow(b, static_cast<uint64_t>(esize), &c)) return false;
+  *out = static_cast<size_t>(c);
+  return true;
+}
+
 // Checks shared by every entry point.  Returns -1 to proceed, or a status to return.
 int check_args(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B, int64_t ldb,
                const void* C, int64_t ldc, size_t op_size, size_t c_size) {
@@ -225,9 +236,10 @@ int check_args(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, cons
   if (A == nullptr || B == nullptr) return set_error(GEMMI_EINVAL, "A or B is null");
   if (m > (int64_t(1) << 40) || n > (int64_t(1) << 31) || k > (int64_t(1) << 31))
     return set_error(GEMMI_EINVAL, "matrix dimension too large");
-  const size_t a_bytes = static_cast<size_t>((m - 1) * lda + k) * op_size;
-  const size_t b_bytes = static_cast<size_t>((k - 1) * ldb + n) * op_size;
-  const size_t c_bytes = static_cast<size_t>((m - 1) * ldc + n) * c_size;
+  size_t a_bytes = 0, b_bytes = 0, c_bytes = 0;
+  if (!span_bytes(m, lda, k, op_size, &a_bytes) || !span_bytes(k, ldb, n, op_size, &b_bytes) ||
+      !span_bytes(m, ldc, n, c_size, &c_bytes))
+    return set_error(GEMMI_EINVAL, "leading dimension too large: the operand's extent overflows 64 bits");
   if (overlaps(C, c_bytes, A, a_bytes) || overlaps(C, c_bytes, B, b_bytes))
     return set_error(GEMMI_EINVAL, "C overlaps A or B");
   return -1;
@@ -546,9 +558,10 @@ int check_args_i4(int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, c
   if (A == nullptr || B == nullptr) return set_error(GEMMI_EINVAL, "A or B is null");
   if (m > (int64_t(1) << 40) || n > (int64_t(1) << 31) || k > (int64_t(1) << 31))
     return set_error(GEMMI_EINVAL, "matrix dimension too large");
-  const size_t a_bytes = static_cast<size_t>((m - 1) * lda + wa);
-  if (b_bytes == 0) b_bytes = static_cast<size_t>((k - 1) * ldb + wb);
-  const size_t c_bytes = static_cast<size_t>((m - 1) * ldc + n) * 4;
+  size_t a_bytes = 0, c_bytes = 0;
+  if (!span_bytes(m, lda, wa, 1, &a_bytes) || !span_bytes(m, ldc, n, 4, &c_bytes) ||
+      (b_bytes == 0 && !span_bytes(k, ldb, wb, 1, &b_bytes)))
+    return set_error(GEMMI_EINVAL, "leading dimension too large: the operand's extent overflows 64 bits");
   if (overlaps(C, c_bytes, A, a_bytes) || overlaps(C, c_bytes, B, b_bytes))
     return set_error(GEMMI_EINVAL, "C overlaps A or B");
   return -1;
@@ -613,23 +626,58 @@ int gemm_i4_locked(int64_t m, int64_t n, int64_t k, const uint8_t* A, int64_t ld
   return run_i4(*d, m, n, k, A, lda, B, ldb, C, ldc, s);
 }
 
-int read_status_locked(DeviceState& d, bool clear) {
-  cudaError_t e = cudaDeviceSynchronize();
-  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceSynchronize");
+// Reads the status words of the current device `dev` -- the library's own (when `d` is non-null)
+// and the allocation-free entry point's (when that entry point has run on the device) -- after
+// synchronising the device (s_only == false) or only stream `s`.  A non-zero word is cleared when
+// `clear`; the first non-zero word decides the return code.
+int read_status_words(int dev, DeviceState* d, bool clear, bool s_only, cudaStream_t s, bool with_noalloc = true) {
+  cudaError_t e = s_only ? cudaStreamSynchronize(s) : cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_error(e, s_only ? "cudaStreamSynchronize" : "cudaDeviceSynchronize");
+  uint32_t* words[2] = {d != nullptr ? d->status : nullptr, with_noalloc ? gemmi::noalloc_status_word(dev) : nullptr};
   uint32_t word = 0;
-  e = cudaMemcpy(&word, d.status, sizeof(word), cudaMemcpyDeviceToHost);
-  if (e != cudaSuccess) return cuda_error(e, "cudaMemcpy(status)");
-  d.last_detail = word;
-  if (clear && word != 0) {
-    e = cudaMemset(d.status, 0, sizeof(word));
-    if (e != cudaSuccess) return cuda_error(e, "cudaMemset(status)");
+  for (uint32_t* w : words) {
+    if (w == nullptr) continue;
+    uint32_t v = 0;
+    e = cudaMemcpyAsync(&v, w, sizeof(v), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_error(e, "reading a device status word");
+    if (clear && v != 0) {
+      e = cudaMemsetAsync(w, 0, sizeof(v), s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return cuda_error(e, "clearing a device status word");
+    }
+    if (word == 0) word = v;
   }
+  if (d != nullptr) d->last_detail = word;
+  g_dev[dev].last_detail = word;
   if (word == 0) return GEMMI_OK;
   const int code = static_cast<int>(word & 0xFFu);
   char buf[160];
   std::snprintf(buf, sizeof(buf), "device status 0x%08x: a pipeline wait (site %u, block %u) ran out of time",
                 word, (word >> 8) & 0xFFu, word >> 16);
   return set_error(code, buf);
+}
+
+// The library's own word only (the entry points that report their status themselves).
+int read_status_locked(DeviceState& d, bool clear) {
+  const int dev = static_cast<int>(&d - g_dev);
+  return read_status_words(dev, &d, clear, false, nullptr, false);
+}
+
+// gemmi_device_status / gemmi_device_status_stream.  A device on which only the allocation-free
+// entry point has run is read without setting up the library's own state (which allocates).
+int device_status_impl(bool s_only, cudaStream_t s) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return set_error(GEMMI_EINVAL, "device ordinal out of range");
+  if (!g_dev[dev].ready && gemmi::noalloc_status_word(dev) != nullptr)
+    return read_status_words(dev, nullptr, true, s_only, s);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  return read_status_words(dev, d, true, s_only, s);
 }
 
 int ensure_pipeline(DeviceState& d) {
@@ -1158,13 +1206,9 @@ void gemmi_set_stream(void* stream) {
 
 const char* gemmi_last_error(void) { return t_error.c_str(); }
 
-int gemmi_device_status(void) {
-  std::lock_guard<std::mutex> lock(g_mutex);
-  DeviceState* d = nullptr;
-  int rc = device_state(&d);
-  if (rc != GEMMI_OK) return rc;
-  return read_status_locked(*d, true);
-}
+int gemmi_device_status(void) { return device_status_impl(false, nullptr); }
+
+int gemmi_device_status_stream(void* stream) { return device_status_impl(true, static_cast<cudaStream_t>(stream)); }
 
 uint32_t gemmi_device_status_detail(void) {
   std::lock_guard<std::mutex> lock(g_mutex);

@@ -115,6 +115,10 @@ cudaError_t srs_add_i16(const int64_t* S, int64_t lds, int16_t* C, int64_t ldc, 
 cudaError_t im2col_i16(const int16_t* X, int16_t* Aout, int64_t lda, int64_t N, int64_t H, int64_t W, int64_t Cin,
                        int64_t R, int64_t S, int64_t ph, int64_t pw, cudaStream_t s);
 
+// ---- noalloc.cu: device address of the allocation-free entry point's status word on device `dev`
+// (inside its static scratch array), or null when that entry point has not run there.
+uint32_t* noalloc_status_word(int dev);
+
 // ---- selftest of the bounded wait.
 cudaError_t launch_wait_timeout_probe(uint32_t* status, uint64_t timeout_ns, cudaStream_t s);
 
