@@ -214,6 +214,14 @@ def oracle_rate(w, seconds: float, threads: int):
     return ops / t / 1e12, t, rows
 
 
+def config_of(w, world: int) -> dict:
+    """The `config` object of the JSON line; identical in both arms."""
+    return {"workload": w.name, "m": w.m, "n": w.n, "k": w.k, "note": w.note,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": f"inputs larger than L2 ({workload_bytes(w) / 2**20:.0f} MiB of A, B, C per step "
+                  f"vs {L2_BYTES / 2**20:.0f} MiB L2)"}
+
+
 def run_reference(args):
     world, rank, _ = dist_setup()
     if rank != 0:
@@ -261,7 +269,7 @@ def run_reference(args):
             "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "int64" if w.kind == "i16" else "int32", "data": "synthetic (seeded SplitMix64)",
             "impl": "reference",
-            "config": {"workload": w.name, "m": w.m, "n": w.n, "k": w.k, "note": w.note},
+            "config": config_of(w, world),
             "cpu_baseline": {"value": value, "unit": "TOPS", "cores": threads, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -438,6 +446,33 @@ def int8_tensor_peak(torch):
         return None
 
 
+# the five workloads of the problem statement, then the extensions, in the compact summary
+SUMMARY_ROWS = (("C1", "i16_256", "launch"), ("C2", "i8_4096", "tensor"), ("C3", "conv3x3_im2col", "hbm"),
+                ("C4", "i16_8192", "tensor"), ("C5", "skinny_8x4096x4096", "hbm"), ("int4", "i4_8192", "tensor"),
+                ("conv", "conv3x3_implicit", "hbm"), ("C4pk", "i16_8192_packed_b", "tensor"),
+                ("C2pk", "i8_4096_packed_b", "tensor"), ("C3pk", "conv3x3_im2col_packed_b", "hbm"))
+
+
+def summarize(extra: dict, peaks: dict) -> dict:
+    """One short entry per workload of the per-workload table: microseconds per call (CUDA-graph
+    replay), TOPS, GB/s of algorithmic bytes and the fraction of the roofline that bounds it."""
+    out = {}
+    for key, name, bound in SUMMARY_ROWS:
+        e = extra.get(name)
+        if not isinstance(e, dict) or "ms" not in e:
+            continue
+        ent = {"us": round(e["ms"] * 1e3, 1), "TOPS": round(e["TOPS"], 1), "bound": bound}
+        if "GB_per_s" in e:
+            ent["GBs"] = round(e["GB_per_s"])
+        for fk, tag in (("frac_of_fp16_tensor_peak", "fp16"), ("frac_of_fp8_tensor_peak", "fp8"),
+                        ("frac_of_limb_tensor_peak", "limb"), ("frac_of_hbm", "hbm")):
+            if fk in e:
+                ent[tag] = round(e[fk], 3)
+        out[key] = ent
+    out["peaks"] = {"hbm_GBs": peaks["hbm_gbs"], "bf16_TFs": peaks["bf16_tflops"], "src": peaks["source"]}
+    return out
+
+
 def run_gemmi(args):
     import torch
     import torch.distributed as dist
@@ -525,6 +560,26 @@ def run_gemmi(args):
     roof["traffic"] = traffic
     roof["source_hash"] = src_hash
     roof["peak_source"] = peaks["source"]
+
+    # ---- the same call back to back for about two seconds (not the timed region): the tensor-bound
+    # kernels reach the board's power cap within a fraction of a second and the SM clock settles
+    # below its maximum; this figure and its clock sit beside the short timed region's
+    sustained = None
+    if rank == 0:
+        n_sus = max(1, int(2000.0 / max(ms, 1e-3)))
+        sampler = ClockSampler(local)
+        sampler.start()
+        e0.record()
+        for _ in range(n_sus):
+            fn(dA, dB, dC)
+        e1.record()
+        torch.cuda.synchronize()
+        sclk = sampler.stop()
+        sms = e0.elapsed_time(e1) / n_sus
+        sustained = {"ms_per_step": sms, "value": w.ops / (sms * 1e-3) / 1e12, "unit": "TOPS", "steps": n_sus,
+                     "sm_mhz": sclk["sm_mhz"], "reasons": sclk["reasons"],
+                     "what": "the timed call back to back for about 2 s after the timed region"}
+        assert gm.device_status() == gm.OK
 
     int8_peak = int8_tensor_peak(torch)
 
@@ -677,10 +732,7 @@ def run_gemmi(args):
             "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "int64" if w.kind == "i16" else "int32",
             "data": "synthetic (seeded SplitMix64 inputs of the workload's shape and value distribution)",
-            "config": {"workload": w.name, "m": w.m, "n": w.n, "k": w.k, "note": w.note,
-                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                       "l2": f"inputs larger than L2 ({workload_bytes(w) / 2**20:.0f} MiB of A, B, C per step "
-                             f"vs {L2_BYTES / 2**20:.0f} MiB L2)"},
+            "config": config_of(w, world),
             "roofline": roof,
             "int8_roofline": None if int8_peak is None else {
                 "int8_tensor_tops": int8_peak, "how": "torch._int_mm (cuBLASLt) 8192^3 on this GPU",
@@ -692,7 +744,9 @@ def run_gemmi(args):
             "gpu_launches": int(launches),
             "clocks": clocks,
             "cpu_baseline": cpu,
+            "sustained": sustained,
             "workloads": extra,
+            "summary": summarize(extra, peaks),
         }
         print(json.dumps(line))
     if world > 1:

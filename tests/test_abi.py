@@ -74,6 +74,18 @@ def test_null_and_overlap_rejected(L):
     assert "overlap" in gm.last_error()
 
 
+def test_leading_dimension_overflow_rejected(L):
+    """An operand whose extent ((rows - 1) * ld + cols elements) overflows 64 bits is refused, not
+    wrapped around into a span that could slip past the overlap check."""
+    huge = 1 << 62
+    a, b, c = ctypes.c_void_p(0x1000), ctypes.c_void_p(0x2000), ctypes.c_void_p(0x3000)
+    assert L.gemm_i16(4, 4, 4, a, huge, b, 4, c, 4) == gm.EINVAL
+    assert "overflow" in gm.last_error()
+    assert L.gemm_i8(4, 4, 4, a, 4, b, huge, c, 4) == gm.EINVAL
+    assert L.gemm_i16_noalloc(4, 4, 4, a, 4, b, 4, c, huge, None) == gm.EINVAL
+    assert "overflow" in gm.last_error()
+
+
 def test_empty_problems_are_noops(L):
     assert L.gemm_i16(0, 4, 4, None, 4, None, 4, None, 4) == gm.OK
     assert L.gemm_i8(4, 0, 4, None, 4, None, 1, None, 1) == gm.OK
