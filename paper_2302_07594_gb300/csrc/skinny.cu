@@ -8,21 +8,27 @@
 // large and two small dimensions (Section 2, IM2COL lowering).  This kernel is
 // built around the stream of B:
 //
-//   * the CTA's slice of A is fetched by bulk copies (one per row) issued with the first B stages
-//     and split into limbs in place, so B starts streaming at once (with plain loads issued by the
-//     consumers, the first B stage waited about 3 us for them);
+//   * the CTA's slice of A is fetched by bulk copies (one per row) issued right after the first B
+//     stage and split into limbs in place, so B starts streaming at once (with plain loads issued
+//     by the consumers, the first B stage waited about 3 us for them);
 //   * B is cut into column blocks of 512 (1 KB contiguous of every row, which
 //     DRAM streams markedly better than 512-byte runs) and the reduction
 //     dimension into ranges, one (column block, range) per CTA, about one CTA
 //     per SM; a producer warp streams 32-row x 512-column stages of B (eight
-//     2-D TMA boxes, 128-byte swizzle) into a ring of shared-memory stages.  The CTA's slice of A (m <= 16 rows, at most 1024
-//     reduction indices) is split into fp16 limbs once, into shared memory, when
-//     the CTA starts, so the inner loop converts only B;
+//     2-D TMA boxes, 128-byte swizzle) into a ring of shared-memory stages: as many 32 KB
+//     stages (3 or 4) as fit beside the A limbs, which are sized for the CTA's own reduction
+//     range.  Under load a stage takes 2-3 us from request to landing, so the bytes in flight
+//     per SM, not the arithmetic, set the pace; the CTA's slice of A (m <= 16 rows, at most
+//     1024 reduction indices) is split into fp16 limbs once, into shared memory, when the CTA
+//     starts, so the inner loop converts only B;
 //   * sixteen consumer warps each own 32 columns of the block, two m16 tiles
 //     (four warps per scheduler, so the latencies of one warp's dependent
-//     ldmatrix / mma chains are covered by the others).  Per 16-row step a
-//     warp reads its B slab transposed with ldmatrix (the "A" operand of
-//     C^T = B^T A^T), splits every int16 into 8-bit limbs
+//     ldmatrix / mma chains are covered by the others).  A warp first reads its whole
+//     share of a stage (32 reduction indices x 32 columns) into registers, transposed with
+//     ldmatrix (the "A" operand of C^T = B^T A^T), and releases the stage at once, so the
+//     producer refills it while the warp computes (holding the stage through the arithmetic
+//     stretched every refill by about half a microsecond).  It then splits every int16 into
+//     8-bit limbs
 //         b = 256*hi + lo,  hi = b >> 8 in [-128,127],  lo = b & 255 in [0,255],
 //     exactly representable in fp16, and multiplies on the tensor cores with
 //     mma.sync m16n8k16 (fp16 in, fp32 accumulate) against the limbs of A;
@@ -30,9 +36,8 @@
 //     partial sum stays below 2^23 (a run of 128 reduction indices:
 //     128 * 255 * 255 < 2^23 and 128 * 2 * 128 * 255 < 2^23), then are drained
 //     into int64 registers as HH*2^16 + X*2^8 + LL;
-//   * each warp adds its partial sums into C: a plain read-modify-write when
-//     one CTA owns the whole reduction range of its columns, 64-bit atomic adds
-//     (exact and order-independent modulo 2^64) when the range is split.
+//   * each warp adds its partial sums into C: 64-bit atomic adds (exact and order-independent
+//     modulo 2^64) when the reduction range is split, a plain read-modify-write otherwise.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -46,13 +51,12 @@ constexpr int JB = 512;                 // columns of B per CTA (1 KB of every r
 constexpr int BOX_J = 64;               // columns per TMA box (128 bytes, the swizzle span)
 constexpr int NBOX = JB / BOX_J;        // 8 boxes per stage
 constexpr int KS = 32;                  // rows of B per stage (two 16-row mma steps)
-constexpr int STAGES = 4;
+constexpr int MIN_STAGES = 3;
+constexpr int MAX_STAGES = 4;           // more stages in flight measured slower (burstier arrival)
 constexpr int STAGE_BYTES = KS * JB * 2;         // 32 KB of B per stage
 constexpr int A_ROWS = 16;
 constexpr int KMAX_CTA = 1024;                   // reduction indices per CTA (bounds the A limbs in smem)
-constexpr int A_PAIRS = KMAX_CTA / 2;            // packed fp16 pairs per A row
-constexpr int A_STRIDE = A_PAIRS + 4;            // words per A limb row (+4 words: conflict-free fragment reads)
-constexpr int A_LIMB_BYTES = A_ROWS * A_STRIDE * 4;  // one limb (hi or lo) of the CTA's A slice
+constexpr size_t SMEM_MAX = 227 * 1024;
 constexpr int NCONS = 16;               // consumer warps
 constexpr int MT = JB / (16 * NCONS);   // m16 tiles (of 16 columns) per consumer warp
 static_assert(MT * 16 * NCONS == JB, "the consumer warps cover the column block");
@@ -70,6 +74,8 @@ struct SkParams {
   int64_t total_stages;
   int atomic_out;
   int a_bulk;               // A's slices can be bulk-copied: 16-byte aligned rows, k % 8 == 0
+  int stages;               // B stages in the ring, MIN_STAGES .. MAX_STAGES
+  int a_stride;             // 32-bit words per A limb row (a multiple of 32, plus 4)
   uint64_t timeout_ns;
   uint32_t* status;
 };
@@ -82,10 +88,13 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
                : "memory");
 }
 
-constexpr size_t sk_smem() {
-  return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * A_LIMB_BYTES + 8 * (2 * STAGES + 1) + 16;
+// Dynamic shared memory: alignment slack, the B ring, the two A limbs (16 rows of a_stride words
+// each), the barriers.
+constexpr size_t sk_smem(int stages, int a_stride) {
+  return 1024 + static_cast<size_t>(stages) * STAGE_BYTES + 2 * static_cast<size_t>(A_ROWS) * a_stride * 4 +
+         8 * (2 * stages + 1) + 16;
 }
-static_assert(sk_smem() <= 227 * 1024, "shared memory budget");
+static_assert(sk_smem(4, KMAX_CTA / 2 + 4) <= SMEM_MAX, "four stages fit beside the largest A slice");
 
 // int16 pair -> fp16 pairs of its high (signed) and low (unsigned) bytes, exactly.
 // 0x64xx as fp16 is 1024 + xx, so each byte is recovered by one subtraction.
@@ -130,12 +139,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint32_t* a_hi = reinterpret_cast<uint32_t*>(smem + STAGES * STAGE_BYTES);  // [16 rows][A_STRIDE] fp16 pairs
-  uint32_t* a_lo = a_hi + A_ROWS * A_STRIDE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(a_lo + A_ROWS * A_STRIDE);
+  const int stages = P.stages;
+  const int a_stride = P.a_stride;
+  uint32_t* a_hi = reinterpret_cast<uint32_t*>(smem + static_cast<size_t>(stages) * STAGE_BYTES);  // [16][a_stride]
+  uint32_t* a_lo = a_hi + A_ROWS * a_stride;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(a_lo + A_ROWS * a_stride);
   const uint32_t full0 = smem_u32(bars);
-  const uint32_t empty0 = full0 + 8 * STAGES;
-  const uint32_t abar = empty0 + 8 * STAGES;  // the CTA's A slice has landed
+  const uint32_t empty0 = full0 + 8 * stages;
+  const uint32_t abar = empty0 + 8 * stages;  // the CTA's A slice has landed
 
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
@@ -148,11 +159,11 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   int64_t* Cg = P.C + row0 * P.ldc;
   int64_t st_end = st_begin + P.stages_per_cta;
   if (st_end > P.total_stages) st_end = P.total_stages;
-  const int64_t nst = st_end > st_begin ? st_end - st_begin : 0;
+  const int nst = st_end > st_begin ? static_cast<int>(st_end - st_begin) : 0;
 
   pdl_launch_dependents();
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < stages; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, NCONS);
     }
@@ -166,42 +177,52 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&mapB);
-      if (P.a_bulk && nst > 0) {
-        // rows 0..m-1 of A, reduction indices k0 .. k0 + kv, land in the low-limb area (row r at
-        // r * A_STRIDE words), where the consumers split them in place
-        const int64_t k0 = st_begin * KS;
-        const int64_t kv = min(nst * KS, P.k - k0);
-        const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
-        const int rows = static_cast<int>(mrows);
-        mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
-        for (int r = 0; r < rows; ++r)
-          bulk_load(smem_u32(a_lo + r * A_STRIDE), Ag + r * P.lda + k0, row_bytes, abar);
-      }
-      int64_t issued = 0;
-      for (int64_t i = 0; i < nst; ++i) {
-        const int s = static_cast<int>(i % STAGES);
-        const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
+      int s = 0;
+      uint32_t par = 0;
+      int issued = 0;
+      for (int i = 0; i < nst; ++i) {
         if (!bounded_wait(empty0 + 8 * s, par ^ 1u, P.timeout_ns)) {
           report_status(P.status, STATUS_TIMEOUT, 11);
           break;
         }
         const uint32_t fb = full0 + 8 * s;
-        const uint32_t dst = smem_u32(smem + s * STAGE_BYTES);
+        const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * STAGE_BYTES);
         const int32_t krow = static_cast<int32_t>((st_begin + i) * KS);
         mbar_arrive_expect_tx(fb, STAGE_BYTES);
 #pragma unroll
         for (int b = 0; b < NBOX; ++b)
           tma_load_2d(dst + b * (KS * BOX_J * 2), &mapB, fb, static_cast<int32_t>(j_base + b * BOX_J), krow);
         ++issued;
+        if (i == 0 && P.a_bulk) {
+          // rows 0..m-1 of A, reduction indices k0 .. k0 + kv, land in the low-limb area (row r at
+          // r * a_stride words), where the consumers split them in place; they are needed when the
+          // first B stage is, so they go out right behind it (behind the first ring of stages the
+          // consumers waited for them: 1.35 us longer per call)
+          const int64_t k0 = st_begin * KS;
+          const int64_t kv = min(static_cast<int64_t>(nst) * KS, P.k - k0);
+          const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
+          const int rows = static_cast<int>(mrows);
+          mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
+          for (int r = 0; r < rows; ++r)
+            bulk_load(smem_u32(a_lo + r * a_stride), Ag + r * P.lda + k0, row_bytes, abar);
+        }
+        if (++s == stages) {
+          s = 0;
+          par ^= 1u;
+        }
       }
-      const int64_t first = issued > STAGES ? issued - STAGES : 0;
-      for (int64_t i = first; i < issued; ++i)
-        bounded_wait(full0 + 8 * static_cast<int>(i % STAGES), static_cast<uint32_t>((i / STAGES) & 1), P.timeout_ns);
+      // wait for the copies in flight before the CTA may exit
+      const int first = issued > stages ? issued - stages : 0;
+      for (int i = first; i < issued; ++i)
+        bounded_wait(full0 + 8 * (i % stages), static_cast<uint32_t>((i / stages) & 1), P.timeout_ns);
     }
     return;
   }
 
   // ------------------------------------------------------------ consumers
+  // A consumer warp that gives up a wait records it and skips the rest of its stages, but still
+  // reaches every named barrier of the other consumer warps (whose own waits are bounded too).
+  bool ok = true;
   // Split this CTA's slice of A once: rows 0..15 (zero beyond m), reduction indices
   // k0 .. k0 + KS*nst (zero beyond k), as packed fp16 pairs of the high and low limbs.
   if (P.a_bulk) {
@@ -211,22 +232,22 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       if (!landed && lane == 0) report_status(P.status, STATUS_TIMEOUT, 13);
     }
     const int64_t k0 = st_begin * KS;
-    const int64_t kv = nst > 0 ? min(nst * KS, P.k - k0) : 0;
-    const int pairs = landed ? static_cast<int>(nst * KS / 2) : 0;
+    const int64_t kv = nst > 0 ? min(static_cast<int64_t>(nst) * KS, P.k - k0) : 0;
+    const int pairs = landed ? nst * KS / 2 : 0;
     for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
       const int row = idx / pairs;
       const int kp = idx - row * pairs;
-      const uint32_t x = (row < mrows && 2 * kp < kv) ? a_lo[row * A_STRIDE + kp] : 0u;
+      const uint32_t x = (row < mrows && 2 * kp < kv) ? a_lo[row * a_stride + kp] : 0u;
       uint32_t hi, lo;
       split_pair(x, hi, lo);
-      a_hi[row * A_STRIDE + kp] = hi;
-      a_lo[row * A_STRIDE + kp] = lo;
+      a_hi[row * a_stride + kp] = hi;
+      a_lo[row * a_stride + kp] = lo;
     }
     asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // every consumer warp arrives
-    if (!landed) return;
+    ok = landed;
   } else {
     const int64_t k0 = st_begin * KS;
-    const int pairs = static_cast<int>(nst * KS / 2);
+    const int pairs = nst * KS / 2;
     for (int idx = threadIdx.x; idx < A_ROWS * pairs; idx += NCONS * 32) {
       const int row = idx / pairs;
       const int kp = idx - row * pairs;
@@ -240,8 +261,8 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       }
       uint32_t hi, lo;
       split_pair(x, hi, lo);
-      a_hi[row * A_STRIDE + kp] = hi;
-      a_lo[row * A_STRIDE + kp] = lo;
+      a_hi[row * a_stride + kp] = hi;
+      a_lo[row * a_stride + kp] = lo;
     }
     asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // consumer warps only
   }
@@ -273,45 +294,59 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   for (int mt = 0; mt < MT; ++mt)
     lane_off[mt] = box * (KS * BOX_J * 2) + lrow * 128 + (((chunk_base + mt * 2 + lchunk) ^ (lrow & 7)) << 4);
   const uint32_t a_hi_s = smem_u32(a_hi), a_lo_s = smem_u32(a_lo);
-  for (int64_t i = 0; i < nst; ++i) {
-    const int s = static_cast<int>(i % STAGES);
-    const uint32_t par = static_cast<uint32_t>((i / STAGES) & 1);
+  int s = 0;
+  uint32_t par = 0;
+  // this warp's share of a stage (32 reduction indices x 16*MT columns) in registers
+  auto load_stage = [&](uint32_t (&dst)[KS / 16][MT][4], int st) {
+    const uint32_t sbase = smem_u32(smem + static_cast<size_t>(st) * STAGE_BYTES);
+#pragma unroll
+    for (int ks = 0; ks < KS / 16; ++ks)
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) ldsm_x4_trans(sbase + ks * (16 * 128) + lane_off[mt], dst[ks][mt]);
+  };
+  auto compute_half = [&](const uint32_t (&bk)[MT][4], int i, int ks) {
+    // A fragments (the mma's B operand: 16 reduction indices x 8 rows of A), already split
+    uint32_t ahi[NT][2], alo[NT][2];
+    const int kp = i * (KS / 2) + ks * 8 + t;  // pair index of reduction index 2kp
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const uint32_t off = static_cast<uint32_t>(((nt * 8 + g) * a_stride + kp) * 4);
+      ahi[nt][0] = lds32(a_hi_s + off);
+      ahi[nt][1] = lds32(a_hi_s + off + 16);
+      alo[nt][0] = lds32(a_lo_s + off);
+      alo[nt][1] = lds32(a_lo_s + off + 16);
+    }
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      uint32_t bhi[4], blo[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) split_pair(bk[mt][q], bhi[q], blo[q]);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        mma16816(hh[mt][nt], bhi, ahi[nt][0], ahi[nt][1]);
+        mma16816(xx[mt][nt], bhi, alo[nt][0], alo[nt][1]);
+        mma16816(xx[mt][nt], blo, ahi[nt][0], ahi[nt][1]);
+        mma16816(ll[mt][nt], blo, alo[nt][0], alo[nt][1]);
+      }
+    }
+  };
+  uint32_t b[KS / 16][MT][4];
+  for (int i = 0; ok && i < nst; ++i) {
     const bool got = bounded_wait(full0 + 8 * s, par, P.timeout_ns);
     if (!__all_sync(0xFFFFFFFFu, got)) {
       if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 12);
-      return;
+      ok = false;
+      break;
     }
-    const uint32_t sbase = smem_u32(smem + s * STAGE_BYTES);
-#pragma unroll
-    for (int ks = 0; ks < KS / 16; ++ks) {
-      // A fragments (the mma's B operand: 16 reduction indices x 8 rows of A), already split
-      uint32_t ahi[NT][2], alo[NT][2];
-      const int kp = static_cast<int>(i) * (KS / 2) + ks * 8 + t;  // pair index of reduction index 2kp
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        const uint32_t off = static_cast<uint32_t>(((nt * 8 + g) * A_STRIDE + kp) * 4);
-        ahi[nt][0] = lds32(a_hi_s + off);
-        ahi[nt][1] = lds32(a_hi_s + off + 16);
-        alo[nt][0] = lds32(a_lo_s + off);
-        alo[nt][1] = lds32(a_lo_s + off + 16);
-      }
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
-        uint32_t b[4], bhi[4], blo[4];
-        ldsm_x4_trans(sbase + ks * (16 * 128) + lane_off[mt], b);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) split_pair(b[q], bhi[q], blo[q]);
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          mma16816(hh[mt][nt], bhi, ahi[nt][0], ahi[nt][1]);
-          mma16816(xx[mt][nt], bhi, alo[nt][0], alo[nt][1]);
-          mma16816(xx[mt][nt], blo, ahi[nt][0], ahi[nt][1]);
-          mma16816(ll[mt][nt], blo, alo[nt][0], alo[nt][1]);
-        }
-      }
-    }
+    load_stage(b, s);
     __syncwarp();
-    if (lane == 0) mbar_arrive(empty0 + 8 * s);
+    if (lane == 0) mbar_arrive(empty0 + 8 * s);  // the producer may refill it while this warp computes
+    if (++s == stages) {
+      s = 0;
+      par ^= 1u;
+    }
+    compute_half(b[0], i, 0);
+    compute_half(b[1], i, 1);
     if ((i + 1) % DRAIN_EVERY == 0 || i + 1 == nst) {
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt)
@@ -326,7 +361,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
           }
     }
   }
-  if (nst == 0) return;
+  if (nst == 0) return;  // the same for every warp of the CTA
   // C fragment (m16n8): c0 (row g, col 2t), c1 (g, 2t+1), c2 (g+8, 2t), c3 (g+8, 2t+1);
   // the mma's rows are columns j of C, its columns are rows i of C.
 #pragma unroll
@@ -389,14 +424,25 @@ cudaError_t launch(const SkinnyArgs& a, cudaStream_t s, const char** why) {
   P.a_bulk = reinterpret_cast<uintptr_t>(a.A) % 16 == 0 && (a.lda * 2) % 16 == 0 && a.k % 8 == 0;
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;
-  constexpr size_t smem = sk_smem();
-  // the shared-memory opt-in is set once per device for this kernel
+  // the A limbs hold the CTA's reduction range (pairs of indices); rows a multiple of 32 words
+  // plus 4 keep the fragment reads free of bank conflicts.  The rest of the shared memory goes to
+  // B stages.
+  const int64_t pairs = per * KS / 2;
+  P.a_stride = static_cast<int>((pairs + 31) / 32 * 32 + 4);
+  P.stages = MAX_STAGES;
+  while (P.stages > MIN_STAGES && sk_smem(P.stages, P.a_stride) > SMEM_MAX) --P.stages;
+  const size_t smem = sk_smem(P.stages, P.a_stride);
+  if (smem > SMEM_MAX) {
+    *why = "skinny GEMM shared-memory layout does not fit";
+    return cudaErrorInvalidValue;
+  }
+  // the shared-memory opt-in (the largest layout) is set once per device for this kernel
   static bool attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64 || !attr_done[dev]) {
     const cudaError_t attr = cudaFuncSetAttribute(skinny_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                  static_cast<int>(smem));
+                                                  static_cast<int>(SMEM_MAX));
     if (attr != cudaSuccess) return attr;
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
   }
