@@ -361,6 +361,17 @@ int gemm_i16_noalloc(int64_t m, int64_t n, int64_t k,
  */
 int gemmi_noalloc_selftest_wait_timeout(int64_t timeout_us, void* stream);
 
+/*
+ * Measurement aid (no counterpart in the paper): the read floor of the skinny-M
+ * path.  Reads the k x n int16 matrix B (a DEVICE pointer, 16-byte aligned,
+ * ldb % 8 == 0) exactly as the m <= 16 kernel streams its B -- the same grid,
+ * TMA boxes, four-stage ring and programmatic dependent launch -- and discards
+ * it.  Asynchronous on `stream`; a wait that runs out is reported by
+ * gemmi_device_status().  Returns GEMMI_OK, GEMMI_EINVAL, GEMMI_ECUDA or
+ * GEMMI_EARCH.
+ */
+int gemmi_stream_read_probe(int64_t k, int64_t n, const int16_t* B, int64_t ldb, void* stream);
+
 /* Library version string. */
 const char* gemmi_version(void);
 

@@ -31,7 +31,7 @@ OPT_TC_CHUNK_SCALE, OPT_TC_GROUP_M, OPT_TC_L2_HINTS, OPT_FUSED_MAX_N, OPT_TC_PAI
 OPT_SMALL_MAX_MACS = 9
 EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
             "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_stream",
-            "gemmi_device_status_detail", "gemmi_noalloc_selftest_wait_timeout",
+            "gemmi_device_status_detail", "gemmi_noalloc_selftest_wait_timeout", "gemmi_stream_read_probe",
             "gemmi_release_workspace", "gemmi_workspace_bytes", "gemmi_set_option", "gemmi_get_option",
             "gemmi_selftest_wait_timeout", "gemmi_kernel_timing", "gemmi_kernel_time", "gemmi_version",
             "gemm_i16_noalloc", "gemmi_pack_b_i16", "gemmi_pack_b_i8", "gemm_i16_packed", "gemm_i8_packed",
@@ -89,6 +89,8 @@ def lib():
         L.gemmi_device_status_stream.restype = ctypes.c_int
         L.gemmi_noalloc_selftest_wait_timeout.argtypes = [i64, vp]
         L.gemmi_noalloc_selftest_wait_timeout.restype = ctypes.c_int
+        L.gemmi_stream_read_probe.argtypes = [i64, i64, vp, i64, vp]
+        L.gemmi_stream_read_probe.restype = ctypes.c_int
         L.gemmi_device_status_detail.restype = ctypes.c_uint32
         L.gemmi_release_workspace.restype = ctypes.c_int
         L.gemmi_workspace_bytes.restype = ctypes.c_size_t
@@ -444,6 +446,18 @@ def set_stream(stream) -> None:
 def device_status() -> int:
     """Synchronises the device; returns and clears its status word (OK or ETIMEOUT)."""
     return int(lib().gemmi_device_status())
+
+
+def stream_read_probe(B, stream=None) -> None:
+    """Reads the int16 device matrix B the way the skinny-M kernel streams it and discards it
+    (gemmi_stream_read_probe): the read floor of that kernel, for measurements."""
+    import torch
+    if B.dtype != torch.int16 or B.dim() != 2 or B.stride(1) != 1 or not B.is_cuda:
+        raise TypeError("the read probe takes a 2-D row-major int16 CUDA tensor")
+    handle = getattr(stream, "cuda_stream", stream)
+    if handle is None:
+        handle = torch.cuda.current_stream().cuda_stream
+    _check(lib().gemmi_stream_read_probe(B.shape[0], B.shape[1], B.data_ptr(), B.stride(0), ctypes.c_void_p(handle)))
 
 
 def device_status_stream(stream=None) -> int:

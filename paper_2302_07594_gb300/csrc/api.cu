@@ -1340,6 +1340,25 @@ int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches) {
   return GEMMI_OK;
 }
 
+int gemmi_stream_read_probe(int64_t k, int64_t n, const int16_t* B, int64_t ldb, void* stream) {
+  if (k < 0 || n < 0) return set_error(GEMMI_EINVAL, "negative matrix dimension");
+  if (ldb < std::max<int64_t>(1, n)) return set_error(GEMMI_EINVAL, "ldb < max(1, n)");
+  if (k == 0 || n == 0) return GEMMI_OK;
+  if (B == nullptr) return set_error(GEMMI_EINVAL, "B is null");
+  if (reinterpret_cast<uintptr_t>(B) % 16 != 0 || ldb % 8 != 0)
+    return set_error(GEMMI_EINVAL, "the read probe needs a 16-byte aligned B with ldb % 8 == 0");
+  if (k > (int64_t(1) << 31) || n > (int64_t(1) << 31)) return set_error(GEMMI_EINVAL, "matrix dimension too large");
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState* d = nullptr;
+  int rc = device_state(&d);
+  if (rc != GEMMI_OK) return rc;
+  const char* why = "read probe launch";
+  const cudaError_t e = gemmi::stream_read_probe(B, k, n, ldb, d->sm_count, d->status, timeout_ns(),
+                                                 static_cast<cudaStream_t>(stream), &why);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return GEMMI_OK;
+}
+
 const char* gemmi_version(void) { return "gemmi 0.1 (sm_103a)"; }
 
 }  // extern "C"

@@ -104,6 +104,11 @@ struct SkinnyArgs {
 };
 cudaError_t skinny_gemm_i16(const SkinnyArgs& args, cudaStream_t s, const char** why);
 
+// ---- probe.cu: reads a k x n int16 matrix (16-byte aligned, ldb % 8 == 0) the way skinny.cu
+// streams B, and discards it (the skinny GEMM's read floor).
+cudaError_t stream_read_probe(const int16_t* B, int64_t k, int64_t n, int64_t ldb, int num_sms, uint32_t* status,
+                              uint64_t timeout_ns, cudaStream_t s, const char** why);
+
 // ---- error text of the calling thread, as returned by gemmi_last_error().
 void record_error(const char* msg);
 

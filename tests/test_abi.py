@@ -86,6 +86,15 @@ def test_leading_dimension_overflow_rejected(L):
     assert "overflow" in gm.last_error()
 
 
+def test_read_probe_argument_checks(L):
+    L.gemmi_stream_read_probe.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64,
+                                          ctypes.c_void_p]
+    assert L.gemmi_stream_read_probe(64, 64, ctypes.c_void_p(0x1008), 64, None) == gm.EINVAL  # not 16-byte aligned
+    assert L.gemmi_stream_read_probe(64, 64, ctypes.c_void_p(0x1000), 60, None) == gm.EINVAL  # ldb < n
+    assert L.gemmi_stream_read_probe(64, 60, ctypes.c_void_p(0x1000), 60, None) == gm.EINVAL  # ldb % 8 != 0
+    assert L.gemmi_stream_read_probe(0, 64, None, 64, None) == gm.OK
+
+
 def test_empty_problems_are_noops(L):
     assert L.gemm_i16(0, 4, 4, None, 4, None, 4, None, 4) == gm.OK
     assert L.gemm_i8(4, 0, 4, None, 4, None, 1, None, 1) == gm.OK

@@ -355,6 +355,16 @@ def test_workload_sampled(gm, name):
     _check_sums(name, w.kind, A, B, C, got)
 
 
+def test_read_probe_runs_clean(gm):
+    """The skinny kernel's read floor probe (gemmi_stream_read_probe) streams a full-size B and a
+    ragged one without a device-side failure."""
+    for k, n in ((4096, 4096), (1000, 1000)):
+        B = torch.zeros((k, n), dtype=torch.int16, device="cuda")
+        gm.stream_read_probe(B)
+        torch.cuda.synchronize()
+        assert gm.device_status() == gm.OK
+
+
 # ------------------------------------------------------------------ host-buffer API, streams, failure detection
 def test_host_api_i16_and_i8(gm):
     A, B, C = gi.random_problem(900, 150, 170, 400, "i16")
