@@ -49,6 +49,7 @@ KERNEL_INFO = {
                    "tensor"),
     "add_i32": ("add_i32", ("int4.cu",), "hbm"),
     "convert_i4": ("convert_i4_kernel", ("int4.cu",), "hbm"),
+    "tc_karatsuba": ("tc_gemm_kernel<3>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
 }
 FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
 FULL16_RANGE = ("uniform", -32768, 32767)
@@ -451,7 +452,8 @@ def int8_tensor_peak(torch):
 SUMMARY_ROWS = (("C1", "i16_256", "launch"), ("C2", "i8_4096", "tensor"), ("C3", "conv3x3_im2col", "hbm"),
                 ("C4", "i16_8192", "tensor"), ("C5", "skinny_8x4096x4096", "hbm"), ("int4", "i4_8192", "tensor"),
                 ("conv", "conv3x3_implicit", "hbm"), ("C4pk", "i16_8192_packed_b", "tensor"),
-                ("C2pk", "i8_4096_packed_b", "tensor"), ("C3pk", "conv3x3_im2col_packed_b", "hbm"))
+                ("C2pk", "i8_4096_packed_b", "tensor"), ("C3pk", "conv3x3_im2col_packed_b", "hbm"),
+                ("C4ka", "i16_8192_karatsuba", "tensor"))
 
 
 def summarize(extra: dict, peaks: dict) -> dict:
@@ -679,6 +681,24 @@ def run_gemmi(args):
             else:
                 ent["frac_of_limb_tensor_peak"] = ent["TOPS"] / (peaks["bf16_tflops"] / 4)
             extra[name + "_packed_b"] = ent
+        # Karatsuba's three limb products (GEMMI_OPT_KARATSUBA) against the four-product default, at
+        # int16 8192^3: the call and its kernels (the sum planes are timed with the split)
+        try:
+            ow = gi.WORKLOADS["i16_8192"]
+            gm.set_option(gm.OPT_KARATSUBA, 1)
+            try:
+                oms, eager_ms, okt, nsets = time_workload(gm, torch, ow, steps=20, warmup=3)
+            finally:
+                gm.set_option(gm.OPT_KARATSUBA, 0)
+            kms = {KERNEL_INFO[k][0]: okt[k][0] / okt[k][1] for k in KERNEL_INFO if okt[k][1] > 0}
+            kk = kms.get(KERNEL_INFO["tc_karatsuba"][0])
+            extra["i16_8192_karatsuba"] = {
+                "ms": oms, "timing": "CUDA-graph replay, per call", "eager_ms": eager_ms,
+                "TOPS": ow.ops / (oms * 1e-3) / 1e12, "kernel_ms": kms,
+                "kernel_TOPS": (ow.ops / (kk * 1e-3) / 1e12) if kk else None,
+                "what": "int16 8192^3 with three limb products (HH, LL, (h_a+l_a)(h_b+l_b)) on one SM per tile"}
+        except Exception as ex:  # pragma: no cover
+            extra["i16_8192_karatsuba"] = {"error": str(ex)}
         # the precision sweep at equal sizes: int16 at 4096^3, int8 at 8192^3 and int4 at 4096^3
         # beside the table's int16 / int4 8192^3 and int8 4096^3 (same value distributions)
         sweep = {}

@@ -126,6 +126,7 @@ int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
 int64_t g_small_max_macs = int64_t{1} << 25;
+int64_t g_karatsuba = 0;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -256,11 +257,53 @@ Layout plane_layout(int64_t m, int64_t n, int64_t pitch, int nl) {
   const size_t a_plane = round_up(static_cast<size_t>(m) * pitch * 2, kAlign);
   const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
   L.a0 = 0;
-  L.a1 = nl == 2 ? a_plane : 0;
+  L.a1 = nl >= 2 ? a_plane : 0;
   L.b0 = a_plane * nl;
-  L.b1 = nl == 2 ? L.b0 + b_plane : L.b0;
+  L.b1 = nl >= 2 ? L.b0 + b_plane : L.b0;
   L.total = a_plane * nl + b_plane * nl;
   return L;
+}
+
+// The Karatsuba variant (GEMMI_OPT_KARATSUBA): h, l and s = h + l planes of both operands in the
+// workspace, then the three-product kernel on one SM per tile.
+int run_karatsuba(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A, int64_t lda, const int16_t* B,
+                  int64_t ldb, int64_t* C, int64_t ldc, cudaStream_t s) {
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const size_t a_plane = round_up(static_cast<size_t>(m) * pitch * 2, kAlign);
+  const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
+  int rc = ensure_buffer(&d.ws, &d.ws_bytes, 3 * (a_plane + b_plane));
+  if (rc != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+  char* ws = static_cast<char*>(d.ws);
+  LimbPlanes pa{{ws, ws + a_plane, ws + 2 * a_plane}, m, pitch};
+  char* wb = ws + 3 * a_plane;
+  LimbPlanes pb{{wb, wb + b_plane, wb + 2 * b_plane}, n, pitch};
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+  cudaError_t e = gemmi::split_i16(A, lda, B, ldb, m, n, k, pa, pb, s, d.status, timeout_ns());
+  if (e == cudaSuccess) e = gemmi::limb_sum_planes(pa, pb, d.sm_count, s);
+  timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, "limb split launch");
+  gemmi::TcGemmArgs ta;
+  ta.m = m;
+  ta.n = n;
+  ta.k = k;
+  ta.a = pa;
+  ta.b = pb;
+  ta.C = C;
+  ta.ldc = ldc;
+  ta.status = d.status;
+  ta.timeout_ns = timeout_ns();
+  ta.num_sms = d.sm_count;
+  ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
+  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
+  ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
+  const char* why = "tcgen05 Karatsuba GEMM launch";
+  cudaEvent_t t1 = timer_begin(GEMMI_KERNEL_TC_KARATSUBA, s);
+  e = gemmi::tc_gemm_i16_karatsuba(ta, s, &why);
+  timer_end(GEMMI_KERNEL_TC_KARATSUBA, t1, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return end_workspace_use(d, s);
 }
 
 // The tensor-core path: split A (and B, unless `packed_b` already holds its planes) into the
@@ -337,6 +380,9 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   if (fused_applies(nl, n, A, lda, C))
     return run_fused(d, m, n, k, static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb,
                      static_cast<int64_t*>(C), ldc, s, packed_b);
+  if (nl == 2 && g_karatsuba != 0 && packed_b == nullptr)
+    return run_karatsuba(d, m, n, k, static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb,
+                         static_cast<int64_t*>(C), ldc, s);
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
   const Layout L = plane_layout(m, packed_b ? 0 : n, pitch, nl);
   int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
@@ -1287,6 +1333,10 @@ int gemmi_set_option(int option, int64_t value) {
       if (value < 0 || value > (int64_t{1} << 40)) return set_error(GEMMI_EINVAL, "small-problem limit must be in [0, 2^40]");
       g_small_max_macs = value;
       return GEMMI_OK;
+    case GEMMI_OPT_KARATSUBA:
+      if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "Karatsuba option must be 0 or 1");
+      g_karatsuba = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -1304,6 +1354,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_FUSED_MAX_N: return g_fused_max_n;
     case GEMMI_OPT_TC_PAIR: return g_tc_pair;
     case GEMMI_OPT_SMALL_MAX_MACS: return g_small_max_macs;
+    case GEMMI_OPT_KARATSUBA: return g_karatsuba;
     default: return -1;
   }
 }

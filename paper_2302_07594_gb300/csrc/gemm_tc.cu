@@ -96,7 +96,8 @@ struct TcParams {
 template <int NL, int CS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
-               const __grid_constant__ CUtensorMap mapB0, const __grid_constant__ CUtensorMap mapB1, TcParams P) {
+               const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB0,
+               const __grid_constant__ CUtensorMap mapB1, const __grid_constant__ CUtensorMap mapB2, TcParams P) {
   using S = Scheme<NL>;
   using G = Geom<NL>;
   constexpr int STAGES = G::STAGES;
@@ -109,8 +110,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   constexpr int SLOT_COLS = S::SLOT_COLS;
   constexpr int UMMA_N = S::UMMA_N;
   // C element type and the unsigned type of the running sum (wrap-around is modular, never UB)
-  using CT = typename std::conditional<NL == 2, int64_t, int32_t>::type;
-  using UT = typename std::conditional<NL == 2, uint64_t, uint32_t>::type;
+  using CT = typename std::conditional<NL >= 2, int64_t, int32_t>::type;
+  using UT = typename std::conditional<NL >= 2, uint64_t, uint32_t>::type;
+  const CUtensorMap* const amap[3] = {&mapA0, &mapA1, &mapA2};
+  const CUtensorMap* const bmap[3] = {&mapB0, &mapB1, &mapB2};
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -154,11 +157,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   if (warp == PRODUCER_WARP) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      tma_prefetch_desc(&mapA0);
-      tma_prefetch_desc(&mapB0);
-      if (NL == 2) {
-        tma_prefetch_desc(&mapA1);
-        tma_prefetch_desc(&mapB1);
+#pragma unroll
+      for (int l = 0; l < NL; ++l) {
+        tma_prefetch_desc(amap[l]);
+        tma_prefetch_desc(bmap[l]);
       }
       const uint64_t pol_a = l2_policy(P.hint_a);
       const uint64_t pol_b = l2_policy(P.hint_b);
@@ -180,10 +182,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           const uint32_t fb = full0 + 8 * stage;
           mbar_arrive_expect_tx(fb, SB);
           const uint32_t base = smem_u32(smem + stage * SB);
-          tma_load_2d_hint(base, &mapA0, fb, kb * BK, mt * BM, P.hint_a, pol_a);
-          if (NL == 2) tma_load_2d_hint(base + TILE_A, &mapA1, fb, kb * BK, mt * BM, P.hint_a, pol_a);
-          tma_load_2d_hint(base + NL * TILE_A, &mapB0, fb, kb * BK, nt * BN, P.hint_b, pol_b);
-          if (NL == 2) tma_load_2d_hint(base + NL * TILE_A + TILE_B, &mapB1, fb, kb * BK, nt * BN, P.hint_b, pol_b);
+#pragma unroll
+          for (int l = 0; l < NL; ++l)
+            tma_load_2d_hint(base + l * TILE_A, amap[l], fb, kb * BK, mt * BM, P.hint_a, pol_a);
+#pragma unroll
+          for (int l = 0; l < NL; ++l)
+            tma_load_2d_hint(base + NL * TILE_A + l * TILE_B, bmap[l], fb, kb * BK, nt * BN, P.hint_b, pol_b);
           ++issued;
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -296,7 +300,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const bool full_cols = col0 + COLS <= P.n;
       // running sum starts from C itself, so the tile ends with a plain store
       if (row_ok && full_cols && P.c_vec) {
-        if constexpr (NL == 2) {
+        if constexpr (NL >= 2) {
 #pragma unroll
           for (int c = 0; c < COLS; c += 2) {
             const longlong2 v = *reinterpret_cast<const longlong2*>(crow + c);
@@ -357,7 +361,24 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           tc_fence_after();
           // this warp's columns of the accumulator: all 128 (int8, one accumulator per half)
           // or its 64-column half (int16)
-          if constexpr (NL == 2) {
+          if constexpr (NL == 3) {
+            // Karatsuba: this warp's 64 columns of the 128-column accumulator, times its weight
+            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                                   static_cast<uint32_t>(s * SLOT_COLS + half * COLS);
+            const UT w = S::weight(a);
+#pragma unroll
+            for (int c = 0; c < COLS; c += 32) {
+              uint32_t r0[16], r1[16];
+              tc_ld_32x32b_x16(taddr + c, r0);
+              tc_ld_32x32b_x16(taddr + c + 16, r1);
+              tc_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                acc[c + i] += w * static_cast<UT>(static_cast<CT>(f32_to_i32(r0[i])));
+                acc[c + 16 + i] += w * static_cast<UT>(static_cast<CT>(f32_to_i32(r1[i])));
+              }
+            }
+          } else if constexpr (NL == 2) {
             // this warp's 64 output columns: the B-high part (accumulator columns 0-127) and the
             // B-low part (columns 128-255) of each, 16 columns at a time
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
@@ -399,7 +420,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       }
       if (!ok) break;
       if (row_ok && full_cols && P.c_vec) {
-        if constexpr (NL == 2) {
+        if constexpr (NL >= 2) {
 #pragma unroll
           for (int c = 0; c < COLS; c += 2)
             *reinterpret_cast<longlong2*>(crow + c) =
@@ -435,12 +456,12 @@ std::once_flag g_encode_once;
 template <int NL, int CS>
 cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   using G = Geom<NL>;
-  CUtensorMap maps[4];
+  CUtensorMap maps[6];
   const LimbPlanes* ops[2] = {&a.a, &a.b};
   for (int o = 0; o < 2; ++o) {
-    for (int l = 0; l < 2; ++l) {
+    for (int l = 0; l < 3; ++l) {
       const void* base = ops[o]->plane[l < NL ? l : 0];
-      if (!encode_tensor_map_2d(&maps[2 * o + l], 1, base, static_cast<uint64_t>(a.k),
+      if (!encode_tensor_map_2d(&maps[3 * o + l], 1, base, static_cast<uint64_t>(a.k),
                                 static_cast<uint64_t>(ops[o]->rows), static_cast<uint64_t>(ops[o]->pitch) * 2, BK,
                                 o == 0 ? BM : G::BN, G::SWIZZLE, why))
         return cudaErrorInvalidValue;
@@ -455,7 +476,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
   P.num_m_tiles = static_cast<int>((a.m + BM - 1) / BM);
   P.num_n_tiles = static_cast<int>((a.n + G::BN - 1) / G::BN);
   P.num_k_blocks = static_cast<int>((a.k + BK - 1) / BK);
-  const size_t esz = NL == 2 ? 8 : 4;
+  const size_t esz = NL >= 2 ? 8 : 4;
   P.c_vec = (reinterpret_cast<uintptr_t>(a.C) % 16 == 0) && ((a.ldc * esz) % 16 == 0);
   P.group_m = a.group_m > 0 ? a.group_m : 16;
   P.hint_a = a.hint_a;
@@ -475,7 +496,7 @@ cudaError_t launch(const TcGemmArgs& a, cudaStream_t s, const char** why) {
     if (attr != cudaSuccess) return attr;
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
   }
-  tc_gemm_kernel<NL, CS><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], P);
+  tc_gemm_kernel<NL, CS><<<grid, NUM_THREADS, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], P);
   return cudaGetLastError();
 }
 
@@ -524,6 +545,9 @@ cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why
 }
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why) {
   return args.chunk_scale == 2 ? launch<1, 2>(args, s, why) : launch<1, 1>(args, s, why);
+}
+cudaError_t tc_gemm_i16_karatsuba(const TcGemmArgs& args, cudaStream_t s, const char** why) {
+  return args.chunk_scale == 2 ? launch<3, 2>(args, s, why) : launch<3, 1>(args, s, why);
 }
 
 }  // namespace gemmi

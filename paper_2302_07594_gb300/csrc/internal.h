@@ -8,9 +8,10 @@
 namespace gemmi {
 
 // Limb planes of one operand: NL fp16 planes of `rows` x `pitch` elements (K-major:
-// element (r, p) of plane l at planes[l][r * pitch + p]).  pitch is a multiple of 8.
+// element (r, p) of plane l at planes[l][r * pitch + p]).  pitch is a multiple of 8.  The third
+// plane (s = h + l) is used by the Karatsuba variant only.
 struct LimbPlanes {
-  void* plane[2];
+  void* plane[3];
   int64_t rows;
   int64_t pitch;
 };
@@ -29,6 +30,10 @@ cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t l
 cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
                        LimbPlanes pa, LimbPlanes pb, cudaStream_t s, uint32_t* status = nullptr,
                        uint64_t timeout_ns = 4000000000ull);
+// The Karatsuba variant's third plane of each operand: plane[2] = plane[0] + plane[1] (h + l,
+// exact in fp16), for the `rows` x `pitch` planes of pa and pb (an operand with null plane[2] is
+// skipped).
+cudaError_t limb_sum_planes(LimbPlanes pa, LimbPlanes pb, int num_sms, cudaStream_t s);
 
 // ---- gemm_tc.cu: tcgen05 GEMM on limb planes, C (int64 for NL=2, int32 for NL=1) += combine(limb products).
 struct TcGemmArgs {
@@ -47,6 +52,8 @@ struct TcGemmArgs {
 };
 cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
+// int16 by Karatsuba's three products: args.a / args.b hold three planes each (h, l, h + l).
+cudaError_t tc_gemm_i16_karatsuba(const TcGemmArgs& args, cudaStream_t s, const char** why);
 
 // ---- gemm_pair.cu: the same GEMM on SM pairs (tcgen05 cta_group::2).  The kernel adds into C with
 // bulk reductions: C 16-byte aligned and ldc * sizeof(C element) a multiple of 16.

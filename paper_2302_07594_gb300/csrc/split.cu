@@ -562,6 +562,26 @@ cudaError_t launch(const T* A, int64_t lda, const T* B, int64_t ldb, int64_t m, 
   return cudaGetLastError();
 }
 
+// The Karatsuba variant's third plane: s = h + l, eight fp16 values per 16-byte access.  Both
+// limbs are integers of magnitude <= 128 and their sum (|s| <= 255) is exact in fp16.
+__global__ void __launch_bounds__(256) limb_sum_kernel(const uint4* __restrict__ h, const uint4* __restrict__ l,
+                                                       uint4* __restrict__ out, int64_t n_vec) {
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n_vec;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const uint4 a = __ldg(h + i), b = __ldg(l + i);
+    uint4 r;
+    const uint32_t* pa = &a.x;
+    const uint32_t* pb = &b.x;
+    uint32_t* pr = &r.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const __half2 sum = __hadd2(*reinterpret_cast<const __half2*>(pa + q), *reinterpret_cast<const __half2*>(pb + q));
+      pr[q] = *reinterpret_cast<const uint32_t*>(&sum);
+    }
+    out[i] = r;
+  }
+}
+
 }  // namespace
 
 cudaError_t split_i16(const int16_t* A, int64_t lda, const int16_t* B, int64_t ldb, int64_t m, int64_t n, int64_t k,
@@ -574,4 +594,22 @@ cudaError_t convert_i8(const int8_t* A, int64_t lda, const int8_t* B, int64_t ld
   return launch<int8_t, 1>(A, lda, B, ldb, m, n, k, pa, pb, s, status, timeout_ns);
 }
 
+}  // namespace gemmi
+
+namespace gemmi {
+cudaError_t limb_sum_planes(LimbPlanes pa, LimbPlanes pb, int num_sms, cudaStream_t s) {
+  const LimbPlanes* ops[2] = {&pa, &pb};
+  for (const LimbPlanes* p : ops) {
+    if (p->plane[2] == nullptr || p->rows == 0) continue;
+    // rows x pitch fp16 values, pitch a multiple of 8: whole 16-byte vectors
+    const int64_t n_vec = p->rows * p->pitch / 8;
+    const int64_t blocks = (n_vec + 255) / 256;
+    const int grid = static_cast<int>(blocks < 8 * static_cast<int64_t>(num_sms) ? blocks : 8 * static_cast<int64_t>(num_sms));
+    limb_sum_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4*>(p->plane[0]), static_cast<const uint4*>(p->plane[1]),
+                                         static_cast<uint4*>(p->plane[2]), n_vec);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
 }  // namespace gemmi

@@ -84,6 +84,46 @@ struct Scheme<1> {
   }
 };
 
+// int16 by Karatsuba's three products (an option, GEMMI_OPT_KARATSUBA): besides the limbs h and l
+// every operand has a third plane s = h + l (|s| <= 255, exact in fp16), and
+//     a*b = 2^16 h_a h_b + 2^8 (s_a s_b - h_a h_b - l_a l_b) + l_a l_b
+//         = (2^16 - 2^8) HH + 2^8 SS + (1 - 2^8) LL,
+// three products of N = 128 per K block (HH = h_a h_b, LL = l_a l_b, SS = s_a s_b) instead of the
+// four limb products (two of N = 256).  Issuer 0 owns HH and LL, issuer 1 owns SS.  HH and LL
+// products are at most 2^14 in magnitude (chunks of 512 * CS indices, staggered by half a chunk),
+// SS products up to 255^2 < 2^16: its chunks are 128 * CS indices (sums within 2^23 for CS = 1,
+// 2^24 for CS = 2).  Three accumulators live in four 128-column slots: one spare, into which the
+// owner moves an accumulator at its chunk end while the old slot is drained.
+template <>
+struct Scheme<3> {
+  static constexpr int BN = 128;
+  static constexpr int UMMA_N = 128;
+  static constexpr int NACC = 3;
+  static constexpr int NPROD = 3;         // product p: plane p of A times plane p of B
+  static constexpr int NSLOT = 4;
+  static constexpr int SLOT_COLS = 128;
+  static constexpr int EMPTY_COUNT = 2;   // both issuers read every stage
+  static constexpr int COLS = 64;         // C columns per epilogue thread (two warps per lane quadrant)
+  static constexpr int DRAIN_WARPS = 8;   // every epilogue warp drains every accumulator (its 64 columns)
+  __device__ static constexpr bool drains(int, int) { return true; }
+  __device__ static constexpr int a_limb(int p) { return p; }
+  __device__ static constexpr int b_limb(int p) { return p; }
+  __device__ static constexpr int b_row0(int) { return 0; }
+  __device__ static constexpr int acc(int p, int) { return p; }
+  __device__ static constexpr int issuer(int p, int) { return p == 2 ? 1 : 0; }
+  __device__ static constexpr int owner(int a) { return a == 2 ? 1 : 0; }
+  // weight of accumulator a (0: HH, 1: LL, 2: SS), modulo 2^64
+  __device__ static constexpr uint64_t weight(int a) {
+    return a == 0 ? uint64_t{65280} : a == 1 ? ~uint64_t{254} : uint64_t{256};  // 2^16 - 2^8, 1 - 2^8, 2^8
+  }
+  template <int CS>
+  __device__ static bool chunk_ends(int a, int kb, int nkb) {
+    if (kb == nkb - 1) return true;
+    if (a == 2) return (((kb + 1) * 64) % (128 * CS)) == 0;
+    return (((kb + 1) * 64 + a * 256 * CS) % (512 * CS)) == 0;
+  }
+};
+
 // Assignment of accumulators to the four TMEM slots, replayed identically by every role.
 // Spare slots form a FIFO: a chunk end moves the accumulator into the oldest spare and queues
 // its old slot.  rotate() returns the parity to wait on (the slot's empty barrier) before the
