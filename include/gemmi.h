@@ -258,7 +258,8 @@ size_t gemmi_workspace_bytes(void);
  *                            of exact fp32 integer sums; 1 keeps it within 2^23 (twice the drains).
  *                            gemm_i4: 2 drains every 2^18 reduction indices (sums within 2^24),
  *                            1 every 256 (sums within 2^14).
- *   GEMMI_OPT_TC_GROUP_M   : tile raster band height in 128-row tiles (default 16).
+ *   GEMMI_OPT_TC_GROUP_M   : tile raster band height in tile rows; 0 (default) = automatic: 8 for
+ *                            the int16 and int8 kernels, 16 for int4.
  *   GEMMI_OPT_TC_L2_HINTS  : L2 eviction policy of the operand tile loads, bits 0-1 for A,
  *                            bits 2-3 for B: 0 normal, 1 evict_last, 2 evict_first (default 0).
  *   GEMMI_OPT_FUSED_MAX_N  : int16 GEMMs with n <= this value (and an A whose base is 16-byte

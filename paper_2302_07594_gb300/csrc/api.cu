@@ -121,7 +121,7 @@ int64_t g_skinny_max_m = 16;
 int64_t g_timeout_us = 4000000;
 int64_t g_skinny_ksplit = 0;
 int64_t g_tc_chunk_scale = 2;
-int64_t g_tc_group_m = 16;
+int64_t g_tc_group_m = 0;  // 0: automatic (raster_band())
 int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
@@ -129,6 +129,15 @@ int64_t g_small_max_macs = int64_t{1} << 25;
 int64_t g_karatsuba = 0;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Height of the tile raster's bands (in tile rows).  Automatic: 8 for the kernels on fp16 limb
+// planes -- about sqrt(76) for the 76 SM pairs' concurrent 128 x 128 tiles, the fewest distinct A
+// and B panels per wave; at int16 8192^3 it measured 1.2 % faster than 16, at burst clocks and
+// under the power cap alike (less DRAM traffic) -- and 16 for int4, where 16 measured 0.5 % faster.
+int raster_band(bool int4) {
+  if (g_tc_group_m > 0) return static_cast<int>(g_tc_group_m);
+  return int4 ? 16 : 8;
+}
 
 // Current device's state, initialised on first use (caller holds g_mutex).
 int device_state(DeviceState** out) {
@@ -295,7 +304,7 @@ int run_karatsuba(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t
   ta.timeout_ns = timeout_ns();
   ta.num_sms = d.sm_count;
   ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
-  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.group_m = raster_band(false);
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
   ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
   const char* why = "tcgen05 Karatsuba GEMM launch";
@@ -356,7 +365,7 @@ int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A,
   fa.timeout_ns = timeout_ns();
   fa.num_sms = d.sm_count;
   fa.chunk_scale = static_cast<int>(g_tc_chunk_scale);
-  fa.group_m = static_cast<int>(g_tc_group_m);
+  fa.group_m = raster_band(false);
   if (conv != nullptr) {
     fa.conv = 1;
     fa.conv_pixels = conv->N * conv->H * conv->W;
@@ -415,7 +424,7 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   ta.timeout_ns = timeout_ns();
   ta.num_sms = d.sm_count;
   ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
-  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.group_m = raster_band(false);
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
   ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
   const char* why = "tcgen05 GEMM launch";
@@ -645,7 +654,7 @@ int run_i4(DeviceState& d, int64_t m, int64_t n, int64_t k, const uint8_t* A, in
   ta.timeout_ns = timeout_ns();
   ta.num_sms = d.sm_count;
   ta.chunk_scale = static_cast<int>(g_tc_chunk_scale);
-  ta.group_m = static_cast<int>(g_tc_group_m);
+  ta.group_m = raster_band(true);
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
   ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
   const char* why = "tcgen05 int4 GEMM launch";
@@ -1313,7 +1322,7 @@ int gemmi_set_option(int option, int64_t value) {
       g_tc_chunk_scale = value;
       return GEMMI_OK;
     case GEMMI_OPT_TC_GROUP_M:
-      if (value < 1 || value > 1024) return set_error(GEMMI_EINVAL, "raster band must be in [1, 1024]");
+      if (value < 0 || value > 1024) return set_error(GEMMI_EINVAL, "raster band must be in [0, 1024]");
       g_tc_group_m = value;
       return GEMMI_OK;
     case GEMMI_OPT_TC_L2_HINTS:
