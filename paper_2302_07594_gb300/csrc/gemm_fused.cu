@@ -59,6 +59,8 @@
 #include <cuda.h>
 #include <cuda_fp16.h>
 
+#include <type_traits>
+
 #include "internal.h"
 #include "ptx.cuh"
 #include "tc_common.cuh"
@@ -308,6 +310,11 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // Launched with programmatic stream serialization: the setup above may overlap the end of the
+  // previous kernel (B's limb split, or the previous GEMM); every global access comes after this
+  // wait.  The next kernel may be scheduled as this grid's CTAs retire.
+  pdl_wait();
+  pdl_launch_dependents();
 
   const int nkb = P.num_k_blocks;
   const int64_t total_units = static_cast<int64_t>(P.num_m_tiles) * P.num_n_tiles * nkb;
@@ -455,8 +462,12 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
     }
     } else {
     // ------------------------------------------------------------ MMA issuers (issuer me owns accumulator me)
-    const int me = warp - MMA_WARP0;
-    if (lane == 0) {
+    // `me` is a compile-time constant in each issuer's copy of the loop: indexed at run time, the
+    // slot ring's arrays lived in local memory, and every unit's few book-keeping steps waited on
+    // it behind the converters' shared-memory traffic (about 0.25 us per unit, with the tensor
+    // pipe idle meanwhile)
+    auto issuer = [&](auto me_c) {
+      constexpr int me = decltype(me_c)::value;
       constexpr uint32_t idesc = idesc_f16_f32(BM, UMMA_N);
       SlotRing<NACC, NSLOT> ring;
       ring.init();
@@ -511,6 +522,10 @@ fused_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ C
       }
       tc_commit(final_bar);
       bounded_wait(final_bar, 0, P.timeout_ns);
+    };
+    if (lane == 0) {
+      if (warp == MMA_WARP0) issuer(std::integral_constant<int, 0>{});
+      else issuer(std::integral_constant<int, 1>{});
     }
     }
   } else {
@@ -691,8 +706,17 @@ cudaError_t launch(const FusedArgs& a, cudaStream_t s, const char** why) {
       return cudaErrorInvalidConfiguration;
     }
   }
-  fused_kernel<CS><<<grid, NUM_THREADS, SMEM, s>>>(mapA, mapBH, mapBL, P);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, fused_kernel<CS>, mapA, mapBH, mapBL, P);
 }
 
 }  // namespace
