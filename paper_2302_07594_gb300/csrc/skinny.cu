@@ -177,6 +177,21 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&mapB);
+      // rows 0..m-1 of A, reduction indices k0 .. k0 + kv, land in the low-limb area (row r at
+      // r * a_stride words), where the consumers split them in place.  They are needed with the
+      // first B stage: for up to 8 rows they go out right behind it (9.08 against 9.47 us for
+      // 8 x 4096 x 4096 with A first), for 16-row groups first (7.9 against 8.2 us for the 256^3
+      // problem); behind the first ring of B stages the consumers waited for them (1.35 us longer).
+      auto load_a = [&]() {
+        const int64_t k0 = st_begin * KS;
+        const int64_t kv = min(static_cast<int64_t>(nst) * KS, P.k - k0);
+        const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
+        const int rows = static_cast<int>(mrows);
+        mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
+        for (int r = 0; r < rows; ++r)
+          bulk_load(smem_u32(a_lo + r * a_stride), Ag + r * P.lda + k0, row_bytes, abar);
+      };
+      if (NT == 2 && P.a_bulk && nst > 0) load_a();
       int s = 0;
       uint32_t par = 0;
       int issued = 0;
@@ -193,19 +208,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         for (int b = 0; b < NBOX; ++b)
           tma_load_2d(dst + b * (KS * BOX_J * 2), &mapB, fb, static_cast<int32_t>(j_base + b * BOX_J), krow);
         ++issued;
-        if (i == 0 && P.a_bulk) {
-          // rows 0..m-1 of A, reduction indices k0 .. k0 + kv, land in the low-limb area (row r at
-          // r * a_stride words), where the consumers split them in place; they are needed when the
-          // first B stage is, so they go out right behind it (behind the first ring of stages the
-          // consumers waited for them: 1.35 us longer per call)
-          const int64_t k0 = st_begin * KS;
-          const int64_t kv = min(static_cast<int64_t>(nst) * KS, P.k - k0);
-          const uint32_t row_bytes = static_cast<uint32_t>(kv * 2);
-          const int rows = static_cast<int>(mrows);
-          mbar_arrive_expect_tx(abar, static_cast<uint32_t>(rows) * row_bytes);
-          for (int r = 0; r < rows; ++r)
-            bulk_load(smem_u32(a_lo + r * a_stride), Ag + r * P.lda + k0, row_bytes, abar);
-        }
+        if (NT == 1 && i == 0 && P.a_bulk) load_a();
         if (++s == stages) {
           s = 0;
           par ^= 1u;
@@ -338,15 +341,30 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       ok = false;
       break;
     }
-    load_stage(b, s);
-    __syncwarp();
-    if (lane == 0) mbar_arrive(empty0 + 8 * s);  // the producer may refill it while this warp computes
+    if constexpr (NT == 1) {
+      load_stage(b, s);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * s);  // the producer may refill it while this warp computes
+      compute_half(b[0], i, 0);
+      compute_half(b[1], i, 1);
+    } else {
+      // two groups of 8 rows hold twice the accumulators: a whole stage's fragments at once would
+      // spill, so each half stage is loaded just before its products and the stage is handed back
+      // after both (loading both first measured 7.8 -> 8.7 us for the 256^3 problem)
+      const uint32_t sbase = smem_u32(smem + static_cast<size_t>(s) * STAGE_BYTES);
+#pragma unroll
+      for (int ks = 0; ks < KS / 16; ++ks) {
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) ldsm_x4_trans(sbase + ks * (16 * 128) + lane_off[mt], b[ks][mt]);
+        compute_half(b[ks], i, ks);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * s);
+    }
     if (++s == stages) {
       s = 0;
       par ^= 1u;
     }
-    compute_half(b[0], i, 0);
-    compute_half(b[1], i, 1);
     if ((i + 1) % DRAIN_EVERY == 0 || i + 1 == nst) {
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt)
