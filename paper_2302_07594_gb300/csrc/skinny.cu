@@ -33,8 +33,8 @@
 //     exactly representable in fp16, and multiplies on the tensor cores with
 //     mma.sync m16n8k16 (fp16 in, fp32 accumulate) against the limbs of A;
 //   * three fp32 accumulator sets HH, X, LL hold exact integer sums while every
-//     partial sum stays below 2^23 (a run of 128 reduction indices:
-//     128 * 255 * 255 < 2^23 and 128 * 2 * 128 * 255 < 2^23), then are drained
+//     partial sum stays within 2^24 (a run of 256 reduction indices:
+//     256 * 255 * 255 < 2^24 and 256 * 2 * 128 * 255 = 16,711,680 < 2^24), then are drained
 //     into int64 registers as HH*2^16 + X*2^8 + LL;
 //   * each warp adds its partial sums into C: 64-bit atomic adds (exact and order-independent
 //     modulo 2^64) when the reduction range is split, a plain read-modify-write otherwise.
@@ -61,7 +61,7 @@ constexpr int NCONS = 16;               // consumer warps
 constexpr int MT = JB / (16 * NCONS);   // m16 tiles (of 16 columns) per consumer warp
 static_assert(MT * 16 * NCONS == JB, "the consumer warps cover the column block");
 constexpr int THREADS = (NCONS + 1) * 32;
-constexpr int DRAIN_EVERY = 4;          // stages per drain: 4 x 32 = 128 reduction indices
+constexpr int DRAIN_EVERY = 8;          // stages per drain: 8 x 32 = 256 reduction indices
 constexpr uint32_t STATUS_TIMEOUT = 4;
 
 struct SkParams {

@@ -293,6 +293,23 @@ def test_skinny_extremes(gm):
         assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"skinny constant {(a, b)}")
 
 
+@pytest.mark.parametrize("m", [8, 16])
+def test_skinny_full_chunks_at_the_fp32_limit(gm, m):
+    """One CTA per column block (ksplit 1), so every drain covers a full run of 256 reduction
+    indices.  -32513 = 256 * (-128) + 255 makes both cross-term products -128 * 255 on every index:
+    the cross sums reach -256 * 65280 = -16,711,680, within 2^24 = 16,777,216; 255 * 255 products
+    drive the low sums, -32768 the high ones."""
+    gm.set_option(gm.OPT_SKINNY_KSPLIT, 1)
+    try:
+        for a, b in ((-32513, -32513), (255, 255), (-32768, -32768), (-32513, 255), (32767, -32513)):
+            A = np.full((m, 1024), a, np.int16)
+            B = np.full((1024, 600), b, np.int16)
+            C = gi.uniform_int(17, (m, 600), -(1 << 40), 1 << 40, np.int64)
+            assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"skinny full chunks {(a, b)} m={m}")
+    finally:
+        gm.set_option(gm.OPT_SKINNY_KSPLIT, 0)
+
+
 # ------------------------------------------------------------------ the five workloads
 # The five workloads of the exact-GEMM problem statement (paper Section 4.1) are compared with the
 # oracle on EVERY output element, at full size, on all host cores.  The int4 workload (a lower-
