@@ -188,9 +188,11 @@ split_kernel(Part<T> a, Part<T> b, int a_blocks, int64_t b_tiles_j, int64_t b_ti
 // keeps about 100 KB of loads in flight; eight consumer warps convert them.
 //   A item: 32 rows x 256 bytes of raw A -> fp16 planes with coalesced 16-byte stores.
 //   B item: 64 reduction indices x 128 bytes of raw B (64 int16 or 128 int8 columns), loaded
-//           with the 128-byte swizzle, so the transposing gather of one column j from 8
-//           consecutive rows touches 8 different bank groups; the fp16 result goes to a staging
-//           tile in the same swizzled layout (row j = 64 reduction indices) and out by a TMA store.
+//           with the 128-byte swizzle.  A warp converts 8 rows x 32 columns at a time: each lane
+//           reads the 2 columns of one row that an 8 x 8 matrix fragment holds (32-bit loads, no
+//           bank conflicts), converts them to an fp16 pair, and stmatrix.trans writes the four
+//           8 x 8 blocks transposed into a staging tile in the same swizzled layout (row j = 64
+//           reduction indices), which goes out by a TMA store.
 // Every wait is bounded; there is no hardware barrier after the start, so a timeout in one warp
 // can only make the others time out too.
 namespace tsplit {
@@ -230,6 +232,52 @@ __device__ __forceinline__ void i8x4_to_half2x2(uint32_t w, uint32_t& h01, uint3
   const __half2 hb = __hsub2(*reinterpret_cast<const __half2*>(&b), k);
   h01 = *reinterpret_cast<const uint32_t*>(&ha);
   h23 = *reinterpret_cast<const uint32_t*>(&hb);
+}
+
+// Centred limbs of both int16 halves of x as fp16 pairs, exactly (the same h, l as limbs16):
+//   l + 128 = lo_byte ^ 0x80,   h + 128 = (hi_byte ^ 0x80) + (lo_byte >> 7),
+// each placed under the fp16 bit pattern 0x6400 (1024 + v, v <= 256) and recovered by one fp16
+// subtraction of 1152 = 0x6480.
+__device__ __forceinline__ void limbs16x2(uint32_t x, uint32_t& hi, uint32_t& lo) {
+  const uint32_t l_bits = (x & 0x00FF00FFu) ^ 0x64806480u;
+  const uint32_t h_bits = (((x >> 8) & 0x00FF00FFu) ^ 0x64806480u) + ((x >> 7) & 0x00010001u);
+  const __half2 k = __half2half2(__ushort_as_half(0x6480));
+  const __half2 l = __hsub2(*reinterpret_cast<const __half2*>(&l_bits), k);
+  const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&h_bits), k);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Bytes s and s + 1 (s = 0 or 2) of a word of four int8 values -> one fp16 pair, exactly.
+__device__ __forceinline__ uint32_t i8x2_to_half2(uint32_t w, uint32_t s) {
+  const uint32_t b = __byte_perm(w ^ 0x80808080u, 0x64646464u, 0x4040u + s + (s << 8) + 0x0100u);
+  const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&b), __half2half2(__ushort_as_half(0x6480)));
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
+}
+
+// Four 8 x 8 b16 matrices, stored transposed: lane l holds (row l / 4, columns 2(l % 4), +1) of
+// matrix i in r[i]; lane 8i + t gives the address of the 16-byte row t of stored matrix i, which
+// receives column t of matrix i.
+__device__ __forceinline__ void stsm_x4_trans(uint32_t addr, const uint32_t (&r)[4]) {
+  asm volatile("stmatrix.sync.aligned.m8n8.x4.trans.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(r[0]),
+               "r"(r[1]), "r"(r[2]), "r"(r[3])
+               : "memory");
+}
+
+// q = a / b, r = a - q * b, in 32-bit arithmetic when both fit (a 64-bit division is a long
+// software routine, and it sat on every item of the split kernel).
+__device__ __forceinline__ void divmod(int64_t a, int64_t b, int64_t& q, int64_t& r) {
+  if (((static_cast<uint64_t>(a) | static_cast<uint64_t>(b)) >> 31) == 0)
+    q = static_cast<int64_t>(static_cast<uint32_t>(a) / static_cast<uint32_t>(b));
+  else
+    q = a / b;
+  r = a - q * b;
 }
 
 __device__ __forceinline__ void tma_store_2d(const void* map, uint32_t src, int32_t x, int32_t y) {
@@ -291,11 +339,12 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
         mbar_arrive_expect_tx(fb, RAW);
         const uint32_t dst = smem_u32(smem + st.slot * RAW);
         if (it < P.a_items) {
-          const int64_t rt = it / P.a_tiles_k, kt = it - (it / P.a_tiles_k) * P.a_tiles_k;
+          int64_t rt, kt;
+          divmod(it, P.a_tiles_k, rt, kt);
           tma_load_2d(dst, &rawA, fb, static_cast<int32_t>(kt * A_COLS), static_cast<int32_t>(rt * A_ROWS));
         } else {
-          const int64_t b = it - P.a_items;
-          const int64_t pt = b / P.b_tiles_j, jt = b - (b / P.b_tiles_j) * P.b_tiles_j;
+          int64_t pt, jt;
+          divmod(it - P.a_items, P.b_tiles_j, pt, jt);
           tma_load_2d(dst, &rawB, fb, static_cast<int32_t>(jt * JB), static_cast<int32_t>(pt * B_P));
         }
         ++issued;
@@ -322,46 +371,58 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
     }
     const uint8_t* rawt = smem + st.slot * RAW;
     if (it < P.a_items) {
-      // ---- A: row = q / 16, 16-byte chunk c = q % 16 of the 256-byte raw row
-      const int64_t rt = it / P.a_tiles_k, kt = it - rt * P.a_tiles_k;
-      constexpr int ACH = RAW / 16 / CONSUMERS;  // 16-byte raw chunks per thread
-      uint4 w[ACH];
+      int64_t rt, kt;
+      divmod(it, P.a_tiles_k, rt, kt);
+      if constexpr (sizeof(T) == 2) {
+        // ---- A (int16): row = q / 16, 16-byte chunk c = q % 16 of the 256-byte raw row; the 16
+        //      lanes of a row store 256 contiguous bytes of each plane row
+        constexpr int ACH = RAW / 16 / CONSUMERS;  // 16-byte raw chunks per thread
+        uint4 w[ACH];
 #pragma unroll
-      for (int u = 0; u < ACH; ++u) w[u] = *reinterpret_cast<const uint4*>(rawt + (tid + CONSUMERS * u) * 16);
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+        for (int u = 0; u < ACH; ++u) w[u] = *reinterpret_cast<const uint4*>(rawt + (tid + CONSUMERS * u) * 16);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
 #pragma unroll
-      for (int u = 0; u < ACH; ++u) {
-        const int q = tid + CONSUMERS * u;
-        const int64_t row = rt * A_ROWS + (q >> 4);
-        if (row >= P.m) continue;
-        const uint32_t wv[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
-        if constexpr (sizeof(T) == 2) {
+        for (int u = 0; u < ACH; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int64_t row = rt * A_ROWS + (q >> 4);
           const int64_t col = kt * A_COLS + (q & 15) * 8;
-          if (col >= P.a_pitch) continue;
-          int v[8];
+          if (row >= P.m || col >= P.a_pitch) continue;
+          uint4 h, l;
+          limbs16x2(w[u].x, h.x, l.x);
+          limbs16x2(w[u].y, h.y, l.y);
+          limbs16x2(w[u].z, h.z, l.z);
+          limbs16x2(w[u].w, h.w, l.w);
+          *reinterpret_cast<uint4*>(P.a_p0 + row * P.a_pitch + col) = h;
+          *reinterpret_cast<uint4*>(P.a_p1 + row * P.a_pitch + col) = l;
+        }
+      } else {
+        // ---- A (int8): 8-byte pieces; lane c of a warp takes piece c of one 256-byte raw row, so
+        //      each 16-byte store instruction writes 512 contiguous bytes of the plane row (with
+        //      16-byte pieces every store left half of each 32-byte sector to the next one)
+        constexpr int PIECES = RAW / 8 / CONSUMERS;
+        uint2 w[PIECES];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            v[2 * i] = static_cast<int16_t>(wv[i] & 0xFFFFu);
-            v[2 * i + 1] = static_cast<int16_t>(wv[i] >> 16);
-          }
-          store8<NL>(P.a_p0 + row * P.a_pitch + col, P.a_p1 + row * P.a_pitch + col, v);
-        } else {
-          const int64_t col = kt * A_COLS + (q & 15) * 16;
+        for (int u = 0; u < PIECES; ++u) w[u] = *reinterpret_cast<const uint2*>(rawt + (tid + CONSUMERS * u) * 8);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            if (col + 8 * h >= P.a_pitch) continue;
-            uint4 o;
-            i8x4_to_half2x2(wv[2 * h], o.x, o.y);
-            i8x4_to_half2x2(wv[2 * h + 1], o.z, o.w);
-            *reinterpret_cast<uint4*>(P.a_p0 + row * P.a_pitch + col + 8 * h) = o;
-          }
+        for (int u = 0; u < PIECES; ++u) {
+          const int q = tid + CONSUMERS * u;
+          const int64_t row = rt * A_ROWS + (q >> 5);
+          const int64_t col = kt * A_COLS + (q & 31) * 8;
+          if (row >= P.m || col >= P.a_pitch) continue;
+          uint4 o;
+          i8x4_to_half2x2(w[u].x, o.x, o.y);
+          i8x4_to_half2x2(w[u].y, o.z, o.w);
+          *reinterpret_cast<uint4*>(P.a_p0 + row * P.a_pitch + col) = o;
         }
       }
     } else {
-      // ---- B: gather column j of rows 8g .. 8g+7, convert, write 16 bytes per plane to staging
-      const int64_t b = it - P.a_items;
-      const int64_t pt = b / P.b_tiles_j, jt = b - pt * P.b_tiles_j;
+      // ---- B: 8 x 32 blocks (rows 8g .., columns 32jq ..) converted in fragments and written
+      //      transposed to the staging tile by stmatrix
+      int64_t pt, jt;
+      divmod(it - P.a_items, P.b_tiles_j, pt, jt);
       const int buf = nb & 1;
       const uint32_t use = static_cast<uint32_t>(nb >> 1);
       if (use > 0) {
@@ -372,62 +433,45 @@ split_tma_kernel(const __grid_constant__ CUtensorMap rawA, const __grid_constant
         }
       }
       uint8_t* sbuf = stg + buf * STG;
-      constexpr int PAIRS = JB * 8 / CONSUMERS;  // (column, 8-row group) pairs per thread
-      if constexpr (sizeof(T) == 2) {
-        int vals[PAIRS][8];
+      // warp w takes the units (p-block g, 32-column group jq) w, w + 8, ...; lane (r, q) =
+      // (l / 4, l % 4) reads columns 32jq + 8i + 2q, +1 (i = 0..3) of row 8g + r, the fragment
+      // of the 8 x 8 block i.  Eight rows meet eight different 16-byte chunk positions under the
+      // swizzle, so the 32 lanes' loads hit 32 banks (int8: lanes 2s and 2s + 1 share a word).
+      constexpr int JQ = JB / 32;                 // 32-column groups per raw tile: 2 (int16) / 4 (int8)
+      constexpr int UNITS = 8 * JQ / (CONSUMERS / 32);  // per warp
+      const int r = lane >> 2, q = lane & 3;
+      uint32_t raw[UNITS][4];
 #pragma unroll
-        for (int u = 0; u < PAIRS; ++u) {
-          const int q = tid + CONSUMERS * u;
-          const int j = q % JB;
-          const int g = q / JB;
+      for (int u = 0; u < UNITS; ++u) {
+        const int un = warp + (CONSUMERS / 32) * u;
+        const int g = un / JQ, jq = un % JQ;
+        const int p = 8 * g + r;
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int p = 8 * g + i;
-            const int off = p * 128 + ((((j >> 3) ^ (p & 7))) << 4) + ((j & 7) << 1);
-            vals[u][i] = *reinterpret_cast<const int16_t*>(rawt + off);
-          }
+        for (int i = 0; i < 4; ++i) {
+          const int x = static_cast<int>(sizeof(T)) * (32 * jq + 8 * i + 2 * q);  // byte offset in row p
+          raw[u][i] = lds32(smem_u32(rawt) + p * 128 + (((x >> 4) ^ (p & 7)) << 4) + (x & 12));
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
+      // lane 8i + t addresses staging row j = 32jq + 8i + t (block i's column t), chunk g
+      const int mi = lane >> 3, t = lane & 7;
 #pragma unroll
-        for (int u = 0; u < PAIRS; ++u) {
-          const int q = tid + CONSUMERS * u;
-          const int j = q % JB;
-          const int g = q / JB;
-          const int off = j * 128 + ((g ^ (j & 7)) << 4);
-          store8<NL>(reinterpret_cast<__half*>(sbuf + off), reinterpret_cast<__half*>(sbuf + 8192 + off), vals[u]);
-        }
-      } else {
-        // int8: the 8 bytes of column j in rows 8g .. 8g+7, packed four to a word
-        uint32_t wds[PAIRS][2];
+      for (int u = 0; u < UNITS; ++u) {
+        const int un = warp + (CONSUMERS / 32) * u;
+        const int g = un / JQ, jq = un % JQ;
+        const uint32_t row_addr = smem_u32(sbuf) + (32 * jq + 8 * mi + t) * 128 + ((g ^ t) << 4);
+        if constexpr (sizeof(T) == 2) {
+          uint32_t h[4], l[4];
 #pragma unroll
-        for (int u = 0; u < PAIRS; ++u) {
-          const int q = tid + CONSUMERS * u;
-          const int j = q % JB;
-          const int g = q / JB;
+          for (int i = 0; i < 4; ++i) limbs16x2(raw[u][i], h[i], l[i]);
+          stsm_x4_trans(row_addr, h);
+          stsm_x4_trans(row_addr + 8192, l);
+        } else {
+          uint32_t h[4];
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            uint32_t w = 0;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int p = 8 * g + 4 * h + i;
-              const int off = p * 128 + ((((j >> 4) ^ (p & 7))) << 4) + (j & 15);
-              w |= static_cast<uint32_t>(rawt[off]) << (8 * i);
-            }
-            wds[u][h] = w;
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty0 + 8 * st.slot);
-#pragma unroll
-        for (int u = 0; u < PAIRS; ++u) {
-          const int q = tid + CONSUMERS * u;
-          const int j = q % JB;
-          const int g = q / JB;
-          uint4 o;
-          i8x4_to_half2x2(wds[u][0], o.x, o.y);
-          i8x4_to_half2x2(wds[u][1], o.z, o.w);
-          *reinterpret_cast<uint4*>(sbuf + j * 128 + ((g ^ (j & 7)) << 4)) = o;
+          for (int i = 0; i < 4; ++i) h[i] = i8x2_to_half2(raw[u][i], static_cast<uint32_t>((2 * q) & 2));
+          stsm_x4_trans(row_addr, h);
         }
       }
       fence_proxy_async_smem();
