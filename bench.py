@@ -612,14 +612,23 @@ def run_gemmi(args):
     e2e_steps = max(3, min(args.steps, 60))
     if world > 1:
         dist.barrier()
+    # each call returns after its results are in host memory, so the calls are timed one by one as
+    # well: the mean over all of them is the figure, the median shows it without the occasional
+    # host-side stalls of tens of milliseconds that plain pinned copies of the same size see too
+    per_call = []
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
+        tc = time.perf_counter()
         host_fn(hA, hB, hC)
+        per_call.append(time.perf_counter() - tc)
     e2e_s = (time.perf_counter() - t0) / e2e_steps
     e2e_s = max_over_ranks(e2e_s, world)
+    med_s = max_over_ranks(statistics.median(per_call), world)
     e2e = {"value": job_throughput(w.ops, e2e_s, world) / 1e12, "unit": "TOPS", "ms_per_step": e2e_s * 1e3,
            "h2d_bytes_per_step": int(A.nbytes + B.nbytes + C.nbytes), "d2h_bytes_per_step": int(C.nbytes),
-           "steps": e2e_steps, "warmup": max(3, min(args.warmup, 5)), "api": f"gemm_{w.kind}_host"}
+           "steps": e2e_steps, "warmup": max(3, min(args.warmup, 5)), "api": f"gemm_{w.kind}_host",
+           "median_ms_per_call": med_s * 1e3, "median_value": job_throughput(w.ops, med_s, world) / 1e12,
+           "calls_over_1.5x_median": sum(1 for x in per_call if x > 1.5 * statistics.median(per_call))}
     del hA, hB, hC
 
     # ---- per-workload table (each workload's own bound), rank 0 only
