@@ -268,7 +268,7 @@ size_t gemmi_workspace_bytes(void);
  *   GEMMI_OPT_TC_PAIR      : 1 (default): tensor-core GEMMs run on pairs of SMs (tcgen05
  *                            cta_group::2, clusters of two CTAs) whenever C is 16-byte aligned
  *                            with ldc * sizeof(element) a multiple of 16; 0: one SM per tile.
- *   GEMMI_OPT_SMALL_MAX_MACS : int16 GEMMs with m <= 256 and m*n*k <= this value (default 2^25)
+ *   GEMMI_OPT_SMALL_MAX_MACS : int16 GEMMs with m <= 256 and m*n*k <= this value (default 2^28)
  *                            run as one launch of the skinny-M kernel, 16 rows of A per grid
  *                            row; 0 disables it (so does GEMMI_OPT_SKINNY_MAX_M = 0).
  *   GEMMI_OPT_KARATSUBA    : 1: int16 GEMMs on the tensor-core path (not skinny, not narrow-n,

@@ -125,7 +125,10 @@ int64_t g_tc_group_m = 0;  // 0: automatic (raster_band())
 int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
-int64_t g_small_max_macs = int64_t{1} << 25;
+// up to 2^28 multiply-adds the one-launch skinny path measured faster than split + tensor-core GEMM
+// for every m <= 256 tried (4.9 against 11.0 us at 256^3, 12.1 against 14.0 us at 256 x 1024^2);
+// at 2^29 they tie (256 x 2048 x 1024) and beyond the tensor cores win
+int64_t g_small_max_macs = int64_t{1} << 28;
 int64_t g_karatsuba = 0;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }

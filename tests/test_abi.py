@@ -175,10 +175,10 @@ def test_pair_option(L):
 
 
 def test_small_problem_option(L):
-    assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 25
+    assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 28
     gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)
     assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 0
-    gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 25)
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 28)
     for bad in (-1, (1 << 40) + 1):
         with pytest.raises(gm.GemmiError):
             gm.set_option(gm.OPT_SMALL_MAX_MACS, bad)

@@ -24,10 +24,11 @@ def gm():
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     gm.lib()
     gm.set_option(gm.OPT_FUSED_MAX_N, 64)
+    old_small = gm.get_option(gm.OPT_SMALL_MAX_MACS)
     gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)  # small shapes here test this kernel, not the skinny one
     yield gm
     gm.set_option(gm.OPT_FUSED_MAX_N, 64)
-    gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 25)
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, old_small)
 
 
 @pytest.fixture(params=[1, 2], ids=["chunks_2^23", "chunks_2^24"])

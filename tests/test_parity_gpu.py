@@ -78,8 +78,19 @@ def test_i8_shapes(gm, shape):
     assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"i8 {shape}")
 
 
+@pytest.fixture(params=["dispatch", "tensor_cores"])
+def path(request, gm):
+    """The library's own choice of kernel, and the tensor-core path forced for shapes that the
+    small-problem rule would give to the skinny kernel."""
+    old = gm.get_option(gm.OPT_SMALL_MAX_MACS)
+    if request.param == "tensor_cores":
+        gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)
+    yield request.param
+    gm.set_option(gm.OPT_SMALL_MAX_MACS, old)
+
+
 @pytest.mark.parametrize("k", [511, 512, 513, 1023, 1024, 1025, 4096])
-def test_i16_chunk_boundaries(gm, k):
+def test_i16_chunk_boundaries(gm, k, path):
     A, B, C = gi.random_problem(300 + k, 160, 136, k, "i16")
     assert_same(run_gpu(gm, A, B, C), expected(A, B, C), f"k={k}")
 
@@ -103,7 +114,7 @@ def chunk_scale(request, gm):
 
 @pytest.mark.parametrize("ab", EXTREMES)
 @pytest.mark.parametrize("m", [8, 200])
-def test_i16_constant_extremes(gm, ab, m, chunk_scale):
+def test_i16_constant_extremes(gm, ab, m, chunk_scale, path):
     a, b = ab
     n, k = 136, 2600
     A = np.full((m, k), a, np.int16)
@@ -113,7 +124,7 @@ def test_i16_constant_extremes(gm, ab, m, chunk_scale):
 
 
 @pytest.mark.parametrize("m", [8, 160])
-def test_i16_near_fp32_exactness_limit(gm, m, chunk_scale):
+def test_i16_near_fp32_exactness_limit(gm, m, chunk_scale, path):
     """Limb sums pushed toward the largest magnitudes a chunk allows, with odd low bits.
 
     32640 = 256*128 - 128 has limbs (h, l) = (128, -128): every limb product is
@@ -252,7 +263,7 @@ def _kernel_counts(gm, fn):
         gm.kernel_timing(False)
 
 
-# small problems (m <= 256, m*n*k <= 2^25 by default) run the skinny kernel with one grid row per
+# small problems (m <= 256, m*n*k <= 2^28 by default) run the skinny kernel with one grid row per
 # 16 rows of A: the last group ragged, several column blocks and reduction splits
 @pytest.mark.parametrize("m,n,k", [(17, 64, 64), (24, 300, 1000), (100, 513, 576), (255, 256, 256), (256, 256, 256),
                                    (200, 40, 4000)])
@@ -267,13 +278,14 @@ def test_skinny_row_groups(gm, m, n, k):
 
 def test_small_problem_rule(gm):
     # beyond 256 rows, or above the work limit, the tensor-core path runs
-    for (m, n, k) in ((257, 64, 64), (256, 512, 512)):
+    for (m, n, k) in ((257, 64, 64), (256, 1024, 2048)):
         A, B, C = gi.random_problem(840 + m + n, m, n, k, "i16")
         dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
         counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
         assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["fused_i16"] == 1, counts
         assert_same(dC.cpu().numpy(), expected(A, B, C), f"{m}x{n}x{k}")
     # with the limit at 0 a small problem takes the tensor-core path too
+    old = gm.get_option(gm.OPT_SMALL_MAX_MACS)
     gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)
     try:
         A, B, C = gi.random_problem(850, 100, 300, 200, "i16")
@@ -282,7 +294,7 @@ def test_small_problem_rule(gm):
         assert counts["skinny"] == 0 and counts["tc_pair_i16"] == 1, counts
         assert_same(dC.cpu().numpy(), expected(A, B, C), "limit 0")
     finally:
-        gm.set_option(gm.OPT_SMALL_MAX_MACS, 1 << 25)
+        gm.set_option(gm.OPT_SMALL_MAX_MACS, old)
 
 
 def test_skinny_extremes(gm):
