@@ -276,6 +276,22 @@ def test_skinny_row_groups(gm, m, n, k):
     assert_same(dC.cpu().numpy(), expected(A, B, C), f"skinny row groups {m}x{n}x{k}")
 
 
+@pytest.mark.parametrize("m,n,k,skinny", [(256, 1024, 1024, True), (255, 1000, 1050, True), (256, 1024, 1025, False)])
+def test_small_problem_limit(gm, m, n, k, skinny):
+    # at the default limit of 2^28 multiply-adds: 256 x 1024 x 1024 is the largest 256-row problem
+    # the skinny kernel takes (16 row groups x 2 column blocks x 4 reduction ranges of 8 stages)
+    assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 28
+    A, B, C = gi.random_problem(860 + m + n + k, m, n, k, "i16")
+    dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
+    counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
+    assert gm.device_status() == gm.OK
+    if skinny:
+        assert counts["skinny"] == 1 and counts["split"] == 0, counts
+    else:
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] == 1, counts
+    assert_same(dC.cpu().numpy(), expected(A, B, C, threads=16), f"{m}x{n}x{k}")
+
+
 def test_small_problem_rule(gm):
     # beyond 256 rows, or above the work limit, the tensor-core path runs
     for (m, n, k) in ((257, 64, 64), (256, 1024, 2048)):
