@@ -454,7 +454,7 @@ SUMMARY_ROWS = (("C1", "i16_256", "launch"), ("C2", "i8_4096", "tensor"), ("C3",
                 ("C4", "i16_8192", "tensor"), ("C5", "skinny_8x4096x4096", "hbm"), ("int4", "i4_8192", "tensor"),
                 ("conv", "conv3x3_implicit", "hbm"), ("C4pk", "i16_8192_packed_b", "tensor"),
                 ("C2pk", "i8_4096_packed_b", "tensor"), ("C3pk", "conv3x3_im2col_packed_b", "hbm"),
-                ("C4ka", "i16_8192_karatsuba", "tensor"))
+                ("C4ka", "i16_8192_karatsuba", "tensor"), ("C4srs", "i16_8192_srs", "tensor"))
 
 
 def summarize(extra: dict, peaks: dict) -> dict:
@@ -469,7 +469,8 @@ def summarize(extra: dict, peaks: dict) -> dict:
         if "GB_per_s" in e:
             ent["GBs"] = round(e["GB_per_s"])
         for fk, tag in (("frac_of_fp16_tensor_peak", "fp16"), ("frac_of_fp8_tensor_peak", "fp8"),
-                        ("frac_of_limb_tensor_peak", "limb"), ("frac_of_hbm", "hbm")):
+                        ("frac_of_limb_tensor_peak", "limb"), ("frac_of_hbm", "hbm"),
+                        ("srs_frac_of_hbm", "srs_hbm")):
             if fk in e:
                 ent[tag] = round(e[fk], 3)
         fl = e.get("read_floor")
@@ -709,6 +710,29 @@ def run_gemmi(args):
                 "what": "int16 8192^3 with three limb products (HH, LL, (h_a+l_a)(h_b+l_b)) on one SM per tile"}
         except Exception as ex:  # pragma: no cover
             extra["i16_8192_karatsuba"] = {"error": str(ex)}
+        # the requantising output (NEXT-3): int16 C += srs(A*B, 16) on the int16 8192^3 operands; the
+        # exact sums go to an int64 scratch, then one pass shifts, rounds, saturates and adds
+        try:
+            ow = gi.WORKLOADS["i16_8192"]
+            A16, B16, _ = gi.make_inputs(ow)
+            sset = [(torch.from_numpy(A16).cuda(), torch.from_numpy(B16).cuda(),
+                     torch.zeros((ow.m, ow.n), dtype=torch.int16, device="cuda"))]
+            oms, eager_ms, okt = _time_calls(gm, torch, sset, lambda a, b, c: gm.gemm_i16_srs(a, b, c, 16), 20, 3)
+            del sset
+            torch.cuda.empty_cache()
+            kms = {KERNEL_INFO[k][0]: okt[k][0] / okt[k][1] for k in KERNEL_INFO if okt[k][1] > 0}
+            srs_ms = kms.get(KERNEL_INFO["srs"][0])
+            srs_bytes = 12 * ow.m * ow.n  # the int64 sums read, the int16 C read and written
+            ent = {"ms": oms, "timing": "CUDA-graph replay, per call", "eager_ms": eager_ms,
+                   "TOPS": ow.ops / (oms * 1e-3) / 1e12, "kernel_ms": kms,
+                   "what": "gemm_i16_srs, shift 16, on the int16 8192^3 operands: exact sums into an int64 "
+                           "scratch (zeroed, then the GEMM), then one shift-round-saturate-add pass into int16 C"}
+            if srs_ms:
+                ent["srs_GB_per_s"] = srs_bytes / (srs_ms * 1e-3) / 1e9
+                ent["srs_frac_of_hbm"] = ent["srs_GB_per_s"] / peaks["hbm_gbs"]
+            extra["i16_8192_srs"] = ent
+        except Exception as ex:  # pragma: no cover
+            extra["i16_8192_srs"] = {"error": str(ex)}
         # the precision sweep at equal sizes: int16 at 4096^3, int8 at 8192^3 and int4 at 4096^3
         # beside the table's int16 / int4 8192^3 and int8 4096^3 (same value distributions)
         sweep = {}
