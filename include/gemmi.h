@@ -277,12 +277,18 @@ size_t gemmi_workspace_bytes(void);
  *                            tile, with a third plane per operand in the workspace; 0 (default):
  *                            four products.  The tensor work shrinks by a quarter; the measured
  *                            time is longer (shared-memory stages, drains).
+ *   GEMMI_OPT_SPLIT_AHEAD  : 1 (default): an int16 GEMM on SM pairs whose A is 16-byte aligned
+ *                            with lda % 8 == 0 and k % 8 == 0 splits only the row panels of A
+ *                            that the first wave of tiles reads (and B) before the GEMM
+ *                            kernel; two warps of every CTA of that kernel split the remaining
+ *                            panels while the tensor cores work, and a tile's loads wait until
+ *                            its panel is complete; 0: the whole split runs before the GEMM.
  * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
 enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
        GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6,
        GEMMI_OPT_FUSED_MAX_N = 7, GEMMI_OPT_TC_PAIR = 8, GEMMI_OPT_SMALL_MAX_MACS = 9,
-       GEMMI_OPT_KARATSUBA = 10 };
+       GEMMI_OPT_KARATSUBA = 10, GEMMI_OPT_SPLIT_AHEAD = 11 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 
@@ -316,11 +322,14 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_CONVERT_I4  : gemm_i4's conversion of the packed operands to E4M3 planes
  *   GEMMI_KERNEL_TC_KARATSUBA : the three-product int16 kernel (GEMMI_OPT_KARATSUBA; its limb-sum
  *                              planes are timed with GEMMI_KERNEL_SPLIT)
+ *   GEMMI_KERNEL_TC_PAIR_I16_AHEAD : the int16 GEMM kernel on SM pairs when its own warps split
+ *                              the later row panels of A (GEMMI_OPT_SPLIT_AHEAD); such a call
+ *                              counts here instead of GEMMI_KERNEL_TC_PAIR_I16
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
        GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_TC_PAIR_I16 = 6, GEMMI_KERNEL_TC_PAIR_I8 = 7,
        GEMMI_KERNEL_TC_PAIR_I4 = 8, GEMMI_KERNEL_ADD_I32 = 9, GEMMI_KERNEL_CONVERT_I4 = 10,
-       GEMMI_KERNEL_TC_KARATSUBA = 11, GEMMI_KERNEL_COUNT = 12 };
+       GEMMI_KERNEL_TC_KARATSUBA = 11, GEMMI_KERNEL_TC_PAIR_I16_AHEAD = 12, GEMMI_KERNEL_COUNT = 13 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

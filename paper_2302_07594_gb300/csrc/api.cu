@@ -125,6 +125,7 @@ int64_t g_tc_group_m = 0;  // 0: automatic (raster_band())
 int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
+int64_t g_split_ahead = 1;  // overlapped A split in the int16 pair kernel
 // up to 2^28 multiply-adds the one-launch skinny path measured faster than split + tensor-core GEMM
 // for every m <= 256 tried (4.9 against 11.0 us at 256^3, 12.1 against 14.0 us at 256 x 1024^2);
 // at 2^29 they tie (256 x 2048 x 1024) and beyond the tensor cores win
@@ -396,19 +397,40 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
     return run_karatsuba(d, m, n, k, static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb,
                          static_cast<int64_t*>(C), ldc, s);
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  // SM pairs (cta_group::2) unless switched off or C cannot take 16-byte bulk reductions
+  const int64_t esz = nl == 2 ? 8 : 4;
+  const bool pair = g_tc_pair != 0 && reinterpret_cast<uintptr_t>(C) % 16 == 0 && (ldc * esz) % 16 == 0;
+  // Overlapped A split (int16 on SM pairs): the split launch converts B and only the row panels
+  // of A that the first wave of tiles reads; the pair kernel's splitter warps convert the rest.
+  const int64_t m_panels = (m + 127) / 128;
+  int ahead_first = 0;
+  if (nl == 2 && pair && g_split_ahead != 0 && reinterpret_cast<uintptr_t>(A) % 16 == 0 && lda % 8 == 0 &&
+      k % 8 == 0 && m_panels < (int64_t{1} << 24)) {
+    ahead_first = gemmi::pair_first_wave_panels(m, n, raster_band(false), d.sm_count);
+    if (ahead_first >= m_panels) ahead_first = 0;
+  }
+  const bool ahead = ahead_first > 0;
   const Layout L = plane_layout(m, packed_b ? 0 : n, pitch, nl);
-  int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
+  const size_t ahead_off = round_up(L.total, kAlign);
+  const size_t ahead_bytes = ahead ? static_cast<size_t>(2 + m_panels) * 4 : 0;
+  int rc = ensure_buffer(&d.ws, &d.ws_bytes, ahead_off + ahead_bytes);
   if (rc != GEMMI_OK) return rc;
   if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
   char* ws = static_cast<char*>(d.ws);
   LimbPlanes pa{{ws + L.a0, ws + L.a1}, m, pitch};
   LimbPlanes pb = packed_b ? *packed_b : LimbPlanes{{ws + L.b0, ws + L.b1}, n, pitch};
   if (packed_b) B = nullptr;  // nothing to convert for B
+  uint32_t* ahead_words = ahead ? reinterpret_cast<uint32_t*>(ws + ahead_off) : nullptr;
   cudaError_t e;
+  if (ahead) {
+    e = cudaMemsetAsync(ahead_words, 0, ahead_bytes, s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(split counters)");
+  }
   cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
   if (nl == 2) {
-    e = gemmi::split_i16(static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb, m, n, k, pa, pb, s,
-                         d.status, timeout_ns());
+    const int64_t m_split = ahead ? std::min<int64_t>(m, static_cast<int64_t>(ahead_first) * 128) : m;
+    e = gemmi::split_i16(static_cast<const int16_t*>(A), lda, static_cast<const int16_t*>(B), ldb, m_split, n, k, pa,
+                         pb, s, d.status, timeout_ns());
   } else {
     e = gemmi::convert_i8(static_cast<const int8_t*>(A), lda, static_cast<const int8_t*>(B), ldb, m, n, k, pa, pb, s,
                           d.status, timeout_ns());
@@ -430,11 +452,15 @@ int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* 
   ta.group_m = raster_band(false);
   ta.hint_a = static_cast<int>(g_tc_l2_hints & 3);
   ta.hint_b = static_cast<int>((g_tc_l2_hints >> 2) & 3);
+  if (ahead) {
+    ta.a_raw = static_cast<const int16_t*>(A);
+    ta.lda = lda;
+    ta.ahead = ahead_words;
+    ta.ahead_first = ahead_first;
+  }
   const char* why = "tcgen05 GEMM launch";
-  // SM pairs (cta_group::2) unless switched off or C cannot take 16-byte bulk reductions
-  const int64_t esz = nl == 2 ? 8 : 4;
-  const bool pair = g_tc_pair != 0 && reinterpret_cast<uintptr_t>(C) % 16 == 0 && (ldc * esz) % 16 == 0;
-  const int kind = pair ? (nl == 2 ? GEMMI_KERNEL_TC_PAIR_I16 : GEMMI_KERNEL_TC_PAIR_I8)
+  const int kind = pair ? (nl == 2 ? (ahead ? GEMMI_KERNEL_TC_PAIR_I16_AHEAD : GEMMI_KERNEL_TC_PAIR_I16)
+                               : GEMMI_KERNEL_TC_PAIR_I8)
                         : (nl == 2 ? GEMMI_KERNEL_TC_I16 : GEMMI_KERNEL_TC_I8);
   cudaEvent_t t1 = timer_begin(kind, s);
   if (pair) e = nl == 2 ? gemmi::tc_pair_gemm_i16(ta, s, &why) : gemmi::tc_pair_gemm_i8(ta, s, &why);
@@ -1349,6 +1375,10 @@ int gemmi_set_option(int option, int64_t value) {
       if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "Karatsuba option must be 0 or 1");
       g_karatsuba = value;
       return GEMMI_OK;
+    case GEMMI_OPT_SPLIT_AHEAD:
+      if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "overlapped-split option must be 0 or 1");
+      g_split_ahead = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -1367,6 +1397,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_TC_PAIR: return g_tc_pair;
     case GEMMI_OPT_SMALL_MAX_MACS: return g_small_max_macs;
     case GEMMI_OPT_KARATSUBA: return g_karatsuba;
+    case GEMMI_OPT_SPLIT_AHEAD: return g_split_ahead;
     default: return -1;
   }
 }

@@ -49,6 +49,16 @@ struct TcGemmArgs {
   int group_m;   // tile raster band height (row tiles), 0 = default
   int hint_a;    // L2 policy for A / B tile loads: 0 normal, 1 evict_last, 2 evict_first
   int hint_b;
+  // Overlapped A split (tc_pair_gemm_i16 only).  When a_raw is not null, the caller has split
+  // only A's row panels (128 rows each) below ahead_first into args.a; two extra warps per CTA
+  // split the remaining panels from a_raw (16-byte aligned, lda % 8 == 0, k % 8 == 0, planes of
+  // pitch k) while the tensor cores work on the earlier ones, and each tile's loads wait until
+  // its panel is complete.  ahead: 2 + (number of row panels) words, zeroed by the caller before
+  // the launch.
+  const int16_t* a_raw = nullptr;
+  int64_t lda = 0;
+  uint32_t* ahead = nullptr;
+  int ahead_first = 0;
 };
 cudaError_t tc_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
 cudaError_t tc_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
@@ -58,6 +68,10 @@ cudaError_t tc_gemm_i16_karatsuba(const TcGemmArgs& args, cudaStream_t s, const 
 // ---- gemm_pair.cu: the same GEMM on SM pairs (tcgen05 cta_group::2).  The kernel adds into C with
 // bulk reductions: C 16-byte aligned and ldc * sizeof(C element) a multiple of 16.
 cudaError_t tc_pair_gemm_i16(const TcGemmArgs& args, cudaStream_t s, const char** why);
+// Row panels of A (128 rows each) that the first wave of pair-kernel tiles reads, for an int16
+// GEMM of m x n outputs with raster band group_m (0 = the default) on num_sms SMs: the panels the
+// caller splits before an overlapped-split launch.
+int pair_first_wave_panels(int64_t m, int64_t n, int group_m, int num_sms);
 cudaError_t tc_pair_gemm_i8(const TcGemmArgs& args, cudaStream_t s, const char** why);
 // int4: args.a / args.b hold one E4M3 plane each (int4.cu), pitch in bytes; C is int32.
 cudaError_t tc_pair_gemm_i4(const TcGemmArgs& args, cudaStream_t s, const char** why);

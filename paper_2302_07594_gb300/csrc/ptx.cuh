@@ -106,6 +106,41 @@ __device__ __forceinline__ void report_status(uint32_t* status, uint32_t code, u
   atomicCAS(status, 0u, word);
 }
 
+// ---------------------------------------------------------------- flags in global memory
+// A counter that one CTA advances after writing data which another CTA then reads through TMA.
+// Writer: plain stores, fence_proxy_async_global() and __threadfence() by every writing thread,
+// then one release increment.  Reader: acquire load, then fence_proxy_async_global() before the
+// TMA loads (the async proxy reads what the generic proxy wrote).
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Waits until *p >= target.  False if that did not happen within timeout_ns nanoseconds.
+__device__ __forceinline__ bool bounded_wait_counter(const uint32_t* p, uint32_t target, uint64_t timeout_ns) {
+  if (ld_acquire_gpu(p) >= target) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    __nanosleep(200);
+    if (ld_acquire_gpu(p) >= target) return true;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
+}
+// 16-byte load of read-only data (not kept in L1).
+__device__ __forceinline__ uint4 ld_nc_v4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
 // ---------------------------------------------------------------- programmatic dependent launch
 // Lets the next kernel in the stream (launched with programmatic stream serialization) start its
 // prologue on SMs as this grid's CTAs retire.  A no-op without such a dependent.

@@ -234,19 +234,7 @@ __device__ __forceinline__ void i8x4_to_half2x2(uint32_t w, uint32_t& h01, uint3
   h23 = *reinterpret_cast<const uint32_t*>(&hb);
 }
 
-// Centred limbs of both int16 halves of x as fp16 pairs, exactly (the same h, l as limbs16):
-//   l + 128 = lo_byte ^ 0x80,   h + 128 = (hi_byte ^ 0x80) + (lo_byte >> 7),
-// each placed under the fp16 bit pattern 0x6400 (1024 + v, v <= 256) and recovered by one fp16
-// subtraction of 1152 = 0x6480.
-__device__ __forceinline__ void limbs16x2(uint32_t x, uint32_t& hi, uint32_t& lo) {
-  const uint32_t l_bits = (x & 0x00FF00FFu) ^ 0x64806480u;
-  const uint32_t h_bits = (((x >> 8) & 0x00FF00FFu) ^ 0x64806480u) + ((x >> 7) & 0x00010001u);
-  const __half2 k = __half2half2(__ushort_as_half(0x6480));
-  const __half2 l = __hsub2(*reinterpret_cast<const __half2*>(&l_bits), k);
-  const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&h_bits), k);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-}
+using tc::limbs16x2;
 
 // Bytes s and s + 1 (s = 0 or 2) of a word of four int8 values -> one fp16 pair, exactly.
 __device__ __forceinline__ uint32_t i8x2_to_half2(uint32_t w, uint32_t s) {

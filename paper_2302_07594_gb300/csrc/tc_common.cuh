@@ -4,6 +4,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda_fp16.h>
 
 #include "ptx.cuh"
 
@@ -180,6 +181,21 @@ struct SlotRing<NACC, NACC> {
   }
 };
 
+// Centred limbs of both int16 halves of x as fp16 pairs, exactly: h = floor((a + 128) / 256) and
+// l = a - 256 h, computed with byte logic as
+//   l + 128 = lo_byte ^ 0x80,   h + 128 = (hi_byte ^ 0x80) + (lo_byte >> 7),
+// each placed under the fp16 bit pattern 0x6400 (1024 + v, v <= 256) and recovered by one fp16
+// subtraction of 1152 = 0x6480.
+__device__ __forceinline__ void limbs16x2(uint32_t x, uint32_t& hi, uint32_t& lo) {
+  const uint32_t l_bits = (x & 0x00FF00FFu) ^ 0x64806480u;
+  const uint32_t h_bits = (((x >> 8) & 0x00FF00FFu) ^ 0x64806480u) + ((x >> 7) & 0x00010001u);
+  const __half2 k = __half2half2(__ushort_as_half(0x6480));
+  const __half2 l = __hsub2(*reinterpret_cast<const __half2*>(&l_bits), k);
+  const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&h_bits), k);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+}
+
 // Position in a ring of n slots: the slot and the parity of its current use.  Pipeline loops
 // advance it by one per K block instead of dividing a running counter (64-bit division is a
 // long software routine on the GPU, and it sat on every producer's critical path).
@@ -194,11 +210,11 @@ struct RingPos {
   }
 };
 
-__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
+__host__ __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& mt, int& nt) {
   const int per_group = group_m * num_n;
   const int group = t / per_group;
   const int first_m = group * group_m;
-  const int rows_here = min(group_m, num_m - first_m);
+  const int rows_here = group_m < num_m - first_m ? group_m : num_m - first_m;
   const int in_group = t - group * per_group;
   mt = first_m + in_group % rows_here;
   nt = in_group / rows_here;

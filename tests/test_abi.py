@@ -174,6 +174,16 @@ def test_pair_option(L):
             gm.set_option(gm.OPT_TC_PAIR, bad)
 
 
+def test_split_ahead_option(L):
+    assert gm.get_option(gm.OPT_SPLIT_AHEAD) == 1
+    gm.set_option(gm.OPT_SPLIT_AHEAD, 0)
+    assert gm.get_option(gm.OPT_SPLIT_AHEAD) == 0
+    gm.set_option(gm.OPT_SPLIT_AHEAD, 1)
+    for bad in (-1, 2):
+        with pytest.raises(gm.GemmiError):
+            gm.set_option(gm.OPT_SPLIT_AHEAD, bad)
+
+
 def test_small_problem_option(L):
     assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 28
     gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)

@@ -80,7 +80,7 @@ def test_conv_implicit(gm, shape):
     N, H, W, Ci, Co, R, S, ph, pw = shape
     X, Wt, Y = make(900 + sum(shape), *shape)
     got, counts = run(gm, X, Wt, Y, R, S, ph, pw)
-    assert counts["fused_i16"] == 1 and counts["tc_i16"] + counts["tc_pair_i16"] == 0, counts
+    assert counts["fused_i16"] == 1 and counts["tc_i16"] + counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 0, counts
     assert_same(got, expected(X, Wt, Y, R, S, ph, pw), f"implicit {shape}")
 
 

@@ -74,7 +74,7 @@ def run(gm, A, B, C, expect_fused=True):
     counts = launches(gm, lambda: gm.gemm_i16(dA, dB, dC))
     assert gm.device_status() == gm.OK
     assert (counts["fused_i16"] == 1) == expect_fused, counts
-    assert counts["tc_i16"] + counts["tc_pair_i16"] == (0 if expect_fused else 1), counts
+    assert counts["tc_i16"] + counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == (0 if expect_fused else 1), counts
     return dC.cpu().numpy()
 
 
@@ -157,7 +157,7 @@ def test_fused_dispatch_rules(gm):
     dA = torch.from_numpy(Apad).cuda()[:, :96]
     dB, dC = torch.from_numpy(B).cuda(), torch.from_numpy(C).cuda()
     counts = launches(gm, lambda: gm.gemm_i16(dA, dB, dC))
-    assert counts["fused_i16"] == 0 and counts["tc_i16"] + counts["tc_pair_i16"] == 1, counts
+    assert counts["fused_i16"] == 0 and counts["tc_i16"] + counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 1, counts
     assert_same(dC.cpu().numpy(), expected(A, B, C), "lda=99")
     # lda a multiple of 8 with padding: fused
     Apad = np.zeros((200, 104), np.int16)

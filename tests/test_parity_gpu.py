@@ -288,7 +288,7 @@ def test_small_problem_limit(gm, m, n, k, skinny):
     if skinny:
         assert counts["skinny"] == 1 and counts["split"] == 0, counts
     else:
-        assert counts["skinny"] == 0 and counts["tc_pair_i16"] == 1, counts
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 1, counts
     assert_same(dC.cpu().numpy(), expected(A, B, C, threads=16), f"{m}x{n}x{k}")
 
 
@@ -298,7 +298,7 @@ def test_small_problem_rule(gm):
         A, B, C = gi.random_problem(840 + m + n, m, n, k, "i16")
         dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
         counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
-        assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["fused_i16"] == 1, counts
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] + counts["fused_i16"] == 1, counts
         assert_same(dC.cpu().numpy(), expected(A, B, C), f"{m}x{n}x{k}")
     # with the limit at 0 a small problem takes the tensor-core path too
     old = gm.get_option(gm.OPT_SMALL_MAX_MACS)
@@ -307,7 +307,7 @@ def test_small_problem_rule(gm):
         A, B, C = gi.random_problem(850, 100, 300, 200, "i16")
         dA, dB, dC = (torch.from_numpy(x).cuda() for x in (A, B, C))
         counts = _kernel_counts(gm, lambda: gm.gemm_i16(dA, dB, dC))
-        assert counts["skinny"] == 0 and counts["tc_pair_i16"] == 1, counts
+        assert counts["skinny"] == 0 and counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 1, counts
         assert_same(dC.cpu().numpy(), expected(A, B, C), "limit 0")
     finally:
         gm.set_option(gm.OPT_SMALL_MAX_MACS, old)
