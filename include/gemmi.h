@@ -172,8 +172,10 @@ int gemm_i16_srs_ex(int64_t m, int64_t n, int64_t k,
  * (N x Ho x Wo x Cout), dense, updated in place.  All device pointers, owned by
  * the caller; Y may not overlap X or Wt.  When Ho == H, Wo == W (a "same"
  * convolution), Cin % 64 == 0, Cout <= 256 and X is 16-byte aligned, the GEMM
- * reads X directly (no lowered matrix is formed); other shapes lower X into
- * library-owned memory first (released by gemmi_release_workspace).
+ * reads X directly (no lowered matrix is formed); with Cin == 64 and the further
+ * conditions of GEMMI_OPT_CONV_ROWS a direct kernel splits every input pixel once
+ * for all taps instead.  Other shapes lower X into library-owned memory first
+ * (released by gemmi_release_workspace).  Every path gives the same result.
  * Errors: GEMMI_EINVAL for negative sizes or paddings, R or S below 1, a filter
  * larger than the padded input, null pointers with non-zero sizes, overlapping Y;
  * otherwise as gemm_i16.  Empty outputs return GEMMI_OK.
@@ -283,12 +285,18 @@ size_t gemmi_workspace_bytes(void);
  *                            kernel; two warps of every CTA of that kernel split the remaining
  *                            panels while the tensor cores work, and a tile's loads wait until
  *                            its panel is complete; 0: the whole split runs before the GEMM.
+ *   GEMMI_OPT_CONV_ROWS    : 1 (default): gemmi_conv2d_i16 runs "same" convolutions with 64 input
+ *                            channels, odd R and S, R*S*64 within one exact chunk (512 * chunk
+ *                            scale), an even Cout, W + S - 1 <= 128 and 16-byte aligned X and Y
+ *                            on the direct kernel, which splits every input pixel once per tile of
+ *                            output rows (the taps are shifted windows of the split rows); 0:
+ *                            such convolutions take the lowered GEMM read tap by tap.
  * Results do not depend on any option; only speed does.  Returns GEMMI_OK or GEMMI_EINVAL.
  */
 enum { GEMMI_OPT_SKINNY_MAX_M = 1, GEMMI_OPT_WAIT_TIMEOUT_US = 2, GEMMI_OPT_SKINNY_KSPLIT = 3,
        GEMMI_OPT_TC_CHUNK_SCALE = 4, GEMMI_OPT_TC_GROUP_M = 5, GEMMI_OPT_TC_L2_HINTS = 6,
        GEMMI_OPT_FUSED_MAX_N = 7, GEMMI_OPT_TC_PAIR = 8, GEMMI_OPT_SMALL_MAX_MACS = 9,
-       GEMMI_OPT_KARATSUBA = 10, GEMMI_OPT_SPLIT_AHEAD = 11 };
+       GEMMI_OPT_KARATSUBA = 10, GEMMI_OPT_SPLIT_AHEAD = 11, GEMMI_OPT_CONV_ROWS = 12 };
 int gemmi_set_option(int option, int64_t value);
 int64_t gemmi_get_option(int option);
 
@@ -325,11 +333,14 @@ int gemmi_selftest_wait_timeout(int64_t timeout_us);
  *   GEMMI_KERNEL_TC_PAIR_I16_AHEAD : the int16 GEMM kernel on SM pairs when its own warps split
  *                              the later row panels of A (GEMMI_OPT_SPLIT_AHEAD); such a call
  *                              counts here instead of GEMMI_KERNEL_TC_PAIR_I16
+ *   GEMMI_KERNEL_CONV_ROWS   : gemmi_conv2d_i16's direct convolution kernel (GEMMI_OPT_CONV_ROWS;
+ *                              the split of its weights is timed with GEMMI_KERNEL_SPLIT)
  */
 enum { GEMMI_KERNEL_SPLIT = 0, GEMMI_KERNEL_TC_I16 = 1, GEMMI_KERNEL_TC_I8 = 2, GEMMI_KERNEL_SKINNY = 3,
        GEMMI_KERNEL_FUSED_I16 = 4, GEMMI_KERNEL_SRS = 5, GEMMI_KERNEL_TC_PAIR_I16 = 6, GEMMI_KERNEL_TC_PAIR_I8 = 7,
        GEMMI_KERNEL_TC_PAIR_I4 = 8, GEMMI_KERNEL_ADD_I32 = 9, GEMMI_KERNEL_CONVERT_I4 = 10,
-       GEMMI_KERNEL_TC_KARATSUBA = 11, GEMMI_KERNEL_TC_PAIR_I16_AHEAD = 12, GEMMI_KERNEL_COUNT = 13 };
+       GEMMI_KERNEL_TC_KARATSUBA = 11, GEMMI_KERNEL_TC_PAIR_I16_AHEAD = 12, GEMMI_KERNEL_CONV_ROWS = 13,
+       GEMMI_KERNEL_COUNT = 14 };
 int gemmi_kernel_timing(int enable);
 int gemmi_kernel_time(int kernel, double* total_ms, int64_t* launches);
 

@@ -28,7 +28,7 @@ LIB_PATH = os.path.join(_HERE, "libgemmi.so")
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EARCH = 0, 1, 2, 3, 4, 5
 OPT_SKINNY_MAX_M, OPT_WAIT_TIMEOUT_US, OPT_SKINNY_KSPLIT = 1, 2, 3
 OPT_TC_CHUNK_SCALE, OPT_TC_GROUP_M, OPT_TC_L2_HINTS, OPT_FUSED_MAX_N, OPT_TC_PAIR = 4, 5, 6, 7, 8
-OPT_SMALL_MAX_MACS, OPT_KARATSUBA, OPT_SPLIT_AHEAD = 9, 10, 11
+OPT_SMALL_MAX_MACS, OPT_KARATSUBA, OPT_SPLIT_AHEAD, OPT_CONV_ROWS = 9, 10, 11, 12
 EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host", "gemm_i8_host",
             "gemmi_set_stream", "gemmi_last_error", "gemmi_device_status", "gemmi_device_status_stream",
             "gemmi_device_status_detail", "gemmi_noalloc_selftest_wait_timeout", "gemmi_stream_read_probe",
@@ -40,12 +40,12 @@ EXPORTED = ("gemm_i16", "gemm_i16_ex", "gemm_i8", "gemm_i8_ex", "gemm_i16_host",
 NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 KERNEL_SPLIT, KERNEL_TC_I16, KERNEL_TC_I8, KERNEL_SKINNY, KERNEL_FUSED_I16, KERNEL_SRS = 0, 1, 2, 3, 4, 5
 KERNEL_TC_PAIR_I16, KERNEL_TC_PAIR_I8, KERNEL_TC_PAIR_I4, KERNEL_ADD_I32, KERNEL_CONVERT_I4 = 6, 7, 8, 9, 10
-KERNEL_TC_KARATSUBA, KERNEL_TC_PAIR_I16_AHEAD = 11, 12
+KERNEL_TC_KARATSUBA, KERNEL_TC_PAIR_I16_AHEAD, KERNEL_CONV_ROWS = 11, 12, 13
 KERNELS = (("split", KERNEL_SPLIT), ("tc_i16", KERNEL_TC_I16), ("tc_i8", KERNEL_TC_I8), ("skinny", KERNEL_SKINNY),
            ("fused_i16", KERNEL_FUSED_I16), ("srs", KERNEL_SRS), ("tc_pair_i16", KERNEL_TC_PAIR_I16),
            ("tc_pair_i8", KERNEL_TC_PAIR_I8), ("tc_pair_i4", KERNEL_TC_PAIR_I4), ("add_i32", KERNEL_ADD_I32),
            ("convert_i4", KERNEL_CONVERT_I4), ("tc_karatsuba", KERNEL_TC_KARATSUBA),
-           ("tc_pair_i16_ahead", KERNEL_TC_PAIR_I16_AHEAD))
+           ("tc_pair_i16_ahead", KERNEL_TC_PAIR_I16_AHEAD), ("conv_rows", KERNEL_CONV_ROWS))
 
 _lib = None
 

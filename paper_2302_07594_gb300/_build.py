@@ -13,7 +13,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT = os.path.join(PKG, "libgemmi.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
 SOURCES = ("api.cu", "split.cu", "gemm_tc.cu", "gemm_fused.cu", "skinny.cu", "noalloc.cu", "requant.cu", "im2col.cu",
-           "gemm_pair.cu", "int4.cu", "probe.cu")
+           "gemm_pair.cu", "int4.cu", "probe.cu", "conv_rows.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -126,6 +126,7 @@ int64_t g_tc_l2_hints = 0;
 int64_t g_fused_max_n = 64;
 int64_t g_tc_pair = 1;
 int64_t g_split_ahead = 1;  // overlapped A split in the int16 pair kernel
+int64_t g_conv_rows = 1;    // direct kernel for "same" convolutions with 64 input channels
 // up to 2^28 multiply-adds the one-launch skinny path measured faster than split + tensor-core GEMM
 // for every m <= 256 tried (4.9 against 11.0 us at 256^3, 12.1 against 14.0 us at 256 x 1024^2);
 // at 2^29 they tie (256 x 2048 x 1024) and beyond the tensor cores win
@@ -388,6 +389,45 @@ int run_fused(DeviceState& d, int64_t m, int64_t n, int64_t k, const int16_t* A,
   return split_b ? end_workspace_use(d, s) : GEMMI_OK;
 }
 
+// The direct convolution (conv_rows.cu): the lowered weights (K x Cout) split once into limb planes
+// in the workspace, then one launch over tiles of output rows.
+int run_conv_rows(DeviceState& d, int64_t N, int64_t H, int64_t W, int64_t Cout, int64_t R, int64_t S,
+                  const int16_t* X, const int16_t* Wt, int64_t* Y, cudaStream_t s) {
+  const int64_t k = R * S * 64;
+  const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
+  const Layout L = plane_layout(0, Cout, pitch, 2);
+  int rc = ensure_buffer(&d.ws, &d.ws_bytes, L.total);
+  if (rc != GEMMI_OK) return rc;
+  if ((rc = begin_workspace_use(d, s)) != GEMMI_OK) return rc;
+  char* ws = static_cast<char*>(d.ws);
+  const LimbPlanes pb{{ws + L.b0, ws + L.b1}, Cout, pitch};
+  const LimbPlanes none{{nullptr, nullptr}, 0, pitch};
+  cudaEvent_t t0 = timer_begin(GEMMI_KERNEL_SPLIT, s);
+  cudaError_t e = gemmi::split_i16(nullptr, k, Wt, Cout, 0, Cout, k, none, pb, s, d.status, timeout_ns());
+  timer_end(GEMMI_KERNEL_SPLIT, t0, s);
+  if (e != cudaSuccess) return cuda_error(e, "limb split launch");
+  gemmi::ConvRowsArgs ca;
+  ca.X = X;
+  ca.N = N;
+  ca.H = H;
+  ca.W = W;
+  ca.R = R;
+  ca.S = S;
+  ca.cout = Cout;
+  ca.b = pb;
+  ca.Y = Y;
+  ca.status = d.status;
+  ca.timeout_ns = timeout_ns();
+  ca.num_sms = d.sm_count;
+  ca.chunk_scale = static_cast<int>(g_tc_chunk_scale);
+  const char* why = "direct convolution launch";
+  cudaEvent_t t1 = timer_begin(GEMMI_KERNEL_CONV_ROWS, s);
+  e = gemmi::conv_rows_i16(ca, s, &why);
+  timer_end(GEMMI_KERNEL_CONV_ROWS, t1, s);
+  if (e != cudaSuccess) return cuda_error(e, why);
+  return end_workspace_use(d, s);
+}
+
 int run_tc(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k, const void* A, int64_t lda, const void* B,
            int64_t ldb, void* C, int64_t ldc, cudaStream_t s, const LimbPlanes* packed_b = nullptr) {
   if (fused_applies(nl, n, A, lda, C))
@@ -593,6 +633,12 @@ int conv2d_locked(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout, in
   DeviceState* d = nullptr;
   int rc = device_state(&d);
   if (rc != GEMMI_OK) return rc;
+  int geo[4];
+  if (g_conv_rows != 0 && Ho == H && Wo == W && Cin == 64 && M > g_skinny_max_m && Cout % 2 == 0 &&
+      N * H * W < (int64_t(1) << 31) && reinterpret_cast<uintptr_t>(X) % 16 == 0 &&
+      reinterpret_cast<uintptr_t>(Y) % 16 == 0 &&
+      gemmi::conv_rows_geometry(W, R, S, static_cast<int>(g_tc_chunk_scale), &geo[0], &geo[1], &geo[2], &geo[3]))
+    return run_conv_rows(*d, N, H, W, Cout, R, S, X, Wt, Y, s);
   const bool implicit = Ho == H && Wo == W && Cin % 64 == 0 && M > g_skinny_max_m && Cout <= 256 &&
                         N * H * W < (int64_t(1) << 31) && reinterpret_cast<uintptr_t>(X) % 16 == 0 &&
                         reinterpret_cast<uintptr_t>(Y) % 8 == 0;
@@ -1379,6 +1425,10 @@ int gemmi_set_option(int option, int64_t value) {
       if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "overlapped-split option must be 0 or 1");
       g_split_ahead = value;
       return GEMMI_OK;
+    case GEMMI_OPT_CONV_ROWS:
+      if (value != 0 && value != 1) return set_error(GEMMI_EINVAL, "direct-convolution option must be 0 or 1");
+      g_conv_rows = value;
+      return GEMMI_OK;
     default:
       return set_error(GEMMI_EINVAL, "unknown option");
   }
@@ -1398,6 +1448,7 @@ int64_t gemmi_get_option(int option) {
     case GEMMI_OPT_SMALL_MAX_MACS: return g_small_max_macs;
     case GEMMI_OPT_KARATSUBA: return g_karatsuba;
     case GEMMI_OPT_SPLIT_AHEAD: return g_split_ahead;
+    case GEMMI_OPT_CONV_ROWS: return g_conv_rows;
     default: return -1;
   }
 }

@@ -184,6 +184,16 @@ def test_split_ahead_option(L):
             gm.set_option(gm.OPT_SPLIT_AHEAD, bad)
 
 
+def test_conv_rows_option(L):
+    assert gm.get_option(gm.OPT_CONV_ROWS) == 1
+    gm.set_option(gm.OPT_CONV_ROWS, 0)
+    assert gm.get_option(gm.OPT_CONV_ROWS) == 0
+    gm.set_option(gm.OPT_CONV_ROWS, 1)
+    for bad in (-1, 2):
+        with pytest.raises(gm.GemmiError):
+            gm.set_option(gm.OPT_CONV_ROWS, bad)
+
+
 def test_small_problem_option(L):
     assert gm.get_option(gm.OPT_SMALL_MAX_MACS) == 1 << 28
     gm.set_option(gm.OPT_SMALL_MAX_MACS, 0)

@@ -1,9 +1,12 @@
 """GPU parity of gemmi_conv2d_i16: a convolution through the lowered GEMM (IM2COL).
 
-"Same" stride-1 convolutions with Cin % 64 == 0 run the fused kernel directly on
-the NHWC tensor (the lowered matrix is never formed); other shapes lower X with
-im2col.cu first.  Expected values come from the oracle's direct convolution
-(oracle.conv2d) on the same seeded inputs, bit for bit.
+"Same" stride-1 convolutions with 64 input channels (odd R and S, one exact chunk,
+an even Cout, padded rows of at most 128 pixels) run the direct kernel
+(conv_rows.cu), which splits every input pixel once; other "same" convolutions
+with Cin % 64 == 0 run the fused kernel directly on the NHWC tensor (the lowered
+matrix is never formed); other shapes lower X with im2col.cu first.  Expected
+values come from the oracle's direct convolution (oracle.conv2d) on the same
+seeded inputs, bit for bit.
 """
 import numpy as np
 import pytest
@@ -49,6 +52,22 @@ def run(gm, X, Wt, Y, R, S, ph, pw):
     return dY.cpu().numpy(), counts
 
 
+def direct_applies(gm, shape):
+    """Whether gemmi_conv2d_i16 takes the direct kernel for this shape (aligned tensors, default
+    options otherwise): the rule of the library's dispatch, restated."""
+    N, H, W, Ci, Co, R, S, ph, pw = shape
+    if gm.get_option(gm.OPT_CONV_ROWS) == 0 or Ci != 64 or R % 2 == 0 or S % 2 == 0:
+        return False
+    if 2 * ph != R - 1 or 2 * pw != S - 1 or Co % 2 or N * H * W <= gm.get_option(gm.OPT_SKINNY_MAX_M):
+        return False
+    if R * S * 64 > 512 * gm.get_option(gm.OPT_TC_CHUNK_SCALE):
+        return False
+    wp, wpad = W + S - 1, (W + 7) // 8 * 8
+    if wp > 128 or min(128 // wp, 136 // wpad) < 1:
+        return False
+    return (128 + (R - 1) * wp + (S - 1) + 7) // 8 * 8 <= 256
+
+
 def expected(X, Wt, Y, R, S, ph, pw):
     Z = Y.copy()
     oracle.conv2d(X, Wt, Z, R, S, ph, pw, nthreads=8)
@@ -75,13 +94,84 @@ IMPLICIT = [
 ]
 
 
+@pytest.fixture
+def conv_rows_option(gm, request):
+    gm.set_option(gm.OPT_CONV_ROWS, request.param)
+    yield request.param
+    gm.set_option(gm.OPT_CONV_ROWS, 1)
+
+
+@pytest.mark.parametrize("conv_rows_option", [1, 0], indirect=True, ids=["direct_on", "direct_off"])
 @pytest.mark.parametrize("shape", IMPLICIT)
-def test_conv_implicit(gm, shape):
+def test_conv_implicit(gm, shape, conv_rows_option):
     N, H, W, Ci, Co, R, S, ph, pw = shape
     X, Wt, Y = make(900 + sum(shape), *shape)
     got, counts = run(gm, X, Wt, Y, R, S, ph, pw)
-    assert counts["fused_i16"] == 1 and counts["tc_i16"] + counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 0, counts
+    kernel = "conv_rows" if direct_applies(gm, shape) else "fused_i16"
+    assert counts[kernel] == 1, (kernel, counts)
+    assert counts["tc_i16"] + counts["tc_pair_i16"] + counts["tc_pair_i16_ahead"] == 0, counts
+    assert counts["conv_rows"] + counts["fused_i16"] == 1, counts
     assert_same(got, expected(X, Wt, Y, R, S, ph, pw), f"implicit {shape}")
+
+
+# shapes at the edges of the direct kernel's rule, and a few just beyond it (the fused kernel)
+DIRECT_EDGES = [
+    (1, 5, 61, 64, 64, 3, 3, 1, 1),     # padded row of 63: the largest 3x3 window buffer (256 positions)
+    (1, 5, 62, 64, 64, 3, 3, 1, 1),     # padded row of 64: beyond the buffer -> fused kernel
+    (2, 6, 7, 64, 2, 3, 3, 1, 1),       # two output channels
+    (2, 5, 9, 64, 130, 3, 3, 1, 1),     # three channel blocks, the last one partial
+    (1, 4, 12, 64, 256, 3, 3, 1, 1),    # four channel blocks
+    (3, 5, 8, 64, 48, 5, 3, 2, 1),      # 5x3: 960 reduction indices
+    (2, 7, 20, 64, 64, 1, 3, 0, 1),     # 1x3
+    (1, 3, 126, 64, 64, 1, 3, 0, 1),    # padded row of 128: one output row per tile
+    (2, 6, 8, 64, 63, 3, 3, 1, 1),      # odd Cout -> fused kernel
+    (5, 20, 3, 64, 64, 3, 3, 1, 1),     # narrow images, 17 rows per tile, ragged last tile
+]
+
+
+@pytest.mark.parametrize("shape", DIRECT_EDGES)
+def test_conv_direct_edges(gm, shape):
+    N, H, W, Ci, Co, R, S, ph, pw = shape
+    X, Wt, Y = make(1100 + sum(shape), *shape)
+    got, counts = run(gm, X, Wt, Y, R, S, ph, pw)
+    kernel = "conv_rows" if direct_applies(gm, shape) else "fused_i16"
+    assert counts[kernel] == 1, (kernel, counts)
+    assert_same(got, expected(X, Wt, Y, R, S, ph, pw), f"direct edge {shape}")
+
+
+def test_conv_direct_chunk_scale_one(gm):
+    """At chunk scale 1 a 3x3 filter (576 reduction indices) exceeds one exact chunk, so the fused
+    kernel takes it; a 1x1 filter still runs direct.  Both exact."""
+    gm.set_option(gm.OPT_TC_CHUNK_SCALE, 1)
+    try:
+        for shape, kernel in (((2, 6, 9, 64, 64, 3, 3, 1, 1), "fused_i16"), ((2, 6, 9, 64, 64, 1, 1, 0, 0), "conv_rows")):
+            N, H, W, Ci, Co, R, S, ph, pw = shape
+            X, Wt, Y = make(1200 + sum(shape), *shape)
+            got, counts = run(gm, X, Wt, Y, R, S, ph, pw)
+            assert counts[kernel] == 1, (shape, counts)
+            assert_same(got, expected(X, Wt, Y, R, S, ph, pw), f"chunk scale 1 {shape}")
+    finally:
+        gm.set_option(gm.OPT_TC_CHUNK_SCALE, 2)
+
+
+def test_conv_direct_every_int16_value(gm):
+    """Every int16 value passes through the direct kernel's on-chip split: X holds all 65536
+    values (64 channels x 1024 pixels), against weights with extreme and ragged values."""
+    X = np.arange(-32768, 32768, dtype=np.int64).astype(np.int16).reshape(1, 16, 64, 64)
+    Wt = gi.uniform_int(1301, (9 * 64, 64), -32768, 32767, np.int16)
+    Wt[0, :] = -32768
+    Wt[1, :] = 32767
+    Y = np.zeros((1, 16, 64, 64), np.int64)
+    # W = 64 needs a padded row of 66 > 63: run it as 1x3 (padded row 66, window 128 + 2)
+    Wt13 = Wt[:3 * 64].copy()
+    got, counts = run(gm, X, Wt13, Y, 1, 3, 0, 1)
+    assert counts["conv_rows"] == 1, counts
+    assert_same(got, expected(X, Wt13, Y, 1, 3, 0, 1), "every int16 value, 1x3")
+    X2 = X.reshape(1, 32, 32, 64)
+    Y2 = np.zeros((1, 32, 32, 64), np.int64)
+    got, counts = run(gm, X2, Wt, Y2, 3, 3, 1, 1)
+    assert counts["conv_rows"] == 1, counts
+    assert_same(got, expected(X2, Wt, Y2, 3, 3, 1, 1), "every int16 value, 3x3")
 
 
 FALLBACK = [
@@ -109,17 +199,18 @@ def test_conv_extremes(gm):
         assert_same(got, expected(X, Wt, Y, 3, 3, 1, 1), f"constant {(a, b)}")
 
 
-def test_conv_workload_images(gm):
+@pytest.mark.parametrize("conv_rows_option", [1, 0], indirect=True, ids=["direct", "fused"])
+def test_conv_workload_every_element(gm, conv_rows_option):
     """The convolution of the im2col workload (batch 32, 56x56, 64 -> 64 channels, 3x3, pad 1),
-    run whole; the oracle checks images 0, 13 and 31 (images are independent)."""
+    run whole on the direct kernel and on the fused one; every element against the oracle."""
     N, H, W, Ci, Co = 32, 56, 56, 64, 64
     X, Wt, _ = make(1003, N, H, W, Ci, Co, 3, 3, 1, 1, dist="conv")
-    Y = np.zeros((N, H, W, Co), np.int64)
+    Y = gi.uniform_int(1004, (N, H, W, Co), -(1 << 40), 1 << 40, np.int64)
     got, counts = run(gm, X, Wt, Y, 3, 3, 1, 1)
-    assert counts["fused_i16"] == 1, counts
-    for n in (0, 13, 31):
-        exp = expected(X[n:n + 1].copy(), Wt, Y[n:n + 1].copy(), 3, 3, 1, 1)
-        assert_same(got[n:n + 1], exp, f"image {n}")
+    assert counts["conv_rows" if conv_rows_option else "fused_i16"] == 1, counts
+    Z = Y.copy()
+    oracle.conv2d(X, Wt, Z, 3, 3, 1, 1, nthreads=oracle.host_cores())
+    assert_same(got, Z, "conv workload")
 
 
 def test_conv_argument_errors(gm):
