@@ -29,23 +29,34 @@
 // Arithmetic.  Every buffered int16 is split into its centred limbs a = 256h + l (h in [-128,128],
 // l in [-128,127], exact in fp16; the split of split.cu).  Per block of 64 output channels and
 // per tap, limb e of the window times the stacked limb tiles of B (the weights, split once per
-// call: B_high in rows 0-63, B_low in rows 64-127) accumulates into accumulator e (N = 128) in
-// TMEM.  Each column sums R*S*64 <= 512*CS products of magnitude <= 2^14, exactly in fp32.  The
+// call: B_high in columns 0-63, B_low in columns 64-127) accumulates into accumulator e (N = 128)
+// in TMEM.  Each column sums R*S*64 <= 512*CS products of magnitude <= 2^14, exactly in fp32.  The
 // epilogue weights the four quarters by 2^16, 2^8, 2^8 and 1 into int64 and adds each valid image
 // row of the tile into Y with 2-D tensor reductions (16 channels x W pixels each) through an
 // unsigned 64-bit tensor map, so the adds wrap modulo 2^64 and Y is never read by the SMs.
 //
-// Roles (one CTA per SM, 608 threads):
+// SM pairs.  Two CTAs of a cluster, on two SMs, take two consecutive tiles, and one thread of the
+// even CTA issues tcgen05.mma.cta_group::2 of M = 256: MMA rows 0-127 are the even CTA's window,
+// rows 128-255 the odd CTA's (each CTA's limb planes at the same shared-memory offsets), and the
+// stacked weights are split between them (B_high rows in the even CTA, B_low rows in the odd
+// one).  Each SM so reads 4 KB of pixels and 2 KB of weights per MMA step instead of 4 + 4: with
+// both operands in shared memory, the reads bound the MMA rate.  Two sets of limb planes per CTA
+// let the converters split the next tile while the tensor cores work on the current one.
+//
+// Roles (one CTA per SM, clusters of two, 608 threads per CTA):
 //   warps 0-7   epilogue: warp w drains TMEM lanes 32*(w % 4) .. +31 (MMA rows) for output
 //               channels 32*(w / 4) .. +31 of the block, into a 128-byte-swizzled staging area;
 //               lane 0 of warp 0 issues the tile's reductions;
 //   warps 8-15  converters: load the next tile's pixels into registers while the tensor cores
-//               work on the current one, then split them into the two limb planes;
-//   warp 16     TMEM allocation; lane 0 streams B's stacked limb tiles (one per tap and block of
-//               output channels) through a ring by TMA;
-//   warps 17-18 lane 0: the MMA issuer of A limb 0 (high) and of A limb 1 (low).
+//               work on the current one, then split them into a free set of limb planes;
+//   warp 16     TMEM allocation (both CTAs); lane 0 streams this CTA's half of B's stacked limb
+//               tiles (one per tap and block of output channels) through a ring by TMA, every
+//               load completing on the even CTA's barrier;
+//   warps 17-18 lane 0 of the even CTA: the MMA issuer of A limb 0 (high) and of A limb 1 (low);
+//               their commits arrive on the barriers of both CTAs.
 // Every wait is bounded by the global timer; one that runs out records GEMMI_ETIMEOUT in the
-// status word and the CTA winds down.
+// status word and the CTA winds down.  Before either CTA of a pair frees tensor memory or exits,
+// the two exchange one arrival, so neither outlives signals aimed at it.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -59,9 +70,10 @@ namespace {
 
 using tc::STATUS_TIMEOUT;
 
-constexpr int BM = 128;                      // MMA rows (buffer window) per tile
+constexpr int BM = 128;                      // MMA rows (buffer window) per CTA and tile
 constexpr int BN = 64;                       // output channels per block
 constexpr int CIN = 64;                      // input channels
+constexpr int UMMA_M = 2 * BM;               // both CTAs' windows
 constexpr int UMMA_N = 2 * BN;               // B's two limb tiles stacked
 constexpr int UMMA_K = 16;
 constexpr int NUM_EPI_WARPS = 8;
@@ -74,20 +86,22 @@ constexpr int NUM_THREADS = 19 * 32;
 constexpr int PB_MAX = 256;                  // buffered positions
 constexpr int ITEMS_PER_THREAD = PB_MAX * 8 / NUM_CONV_THREADS;  // 16-byte cells per converter thread
 constexpr int LIMB_BYTES = PB_MAX * 128;     // one limb plane: a 128-byte row per position
-constexpr int B_STAGES = 5;
-constexpr int TILE_B = UMMA_N * CIN * 2;     // 16 KB: a stacked limb tile of one tap
-constexpr int STG_ROWS = 136;                // staged output pixels per tile: T * round_up(W, 8)
+constexpr int NBUF = 2;                      // sets of limb planes (tile i uses set i % 2)
+constexpr int B_STAGES = 4;
+constexpr int TILE_BH = BN * CIN * 2;        // 8 KB: this CTA's half of a stacked limb tile
+constexpr int STG_ROWS = 120;                // staged output pixels per tile: T * round_up(W, 8)
 constexpr int STG_G = STG_ROWS * 128;        // one group of 16 output channels (int64)
-constexpr int OFF_LIMB0 = 0;
-constexpr int OFF_LIMB1 = LIMB_BYTES;
-constexpr int OFF_B = 2 * LIMB_BYTES;
-constexpr int OFF_STG = OFF_B + B_STAGES * TILE_B;
+constexpr int OFF_LIMB = 0;
+constexpr int OFF_B = NBUF * 2 * LIMB_BYTES;
+constexpr int OFF_STG = OFF_B + B_STAGES * TILE_BH;
 constexpr int OFF_BAR = OFF_STG + 4 * STG_G;
-// limbs full / empty, B full / empty, accumulator full / empty (two slots), staging full / free, final
-constexpr int NBAR = 2 + 2 * B_STAGES + 4 + 2 + 1;
+// limbs full / empty (per set), B full / empty, accumulator full / empty (two slots), staging
+// full / free, final, bye
+constexpr int NBAR = 2 * NBUF + 2 * B_STAGES + 4 + 2 + 2;
 constexpr size_t SMEM = 1024 + static_cast<size_t>(OFF_BAR) + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
-static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0 && STG_G % 1024 == 0, "1024-byte aligned TMA areas");
+static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0 && STG_G % 1024 == 0 && TILE_BH % 1024 == 0,
+              "1024-byte aligned TMA areas");
 constexpr int TMEM_COLS = 512;
 constexpr int SLOT_COLS = 2 * UMMA_N;        // both accumulators of one (tile, channel block)
 
@@ -95,13 +109,15 @@ struct ConvParams {
   const int16_t* X;
   int H, W, R, S, ph, pw;
   int Wp, T, PB, wpad;
-  int tiles_per_image, num_tiles, nnb, cout;
+  int tiles_per_image, num_tiles, num_pair_tiles, nnb, cout;
   uint64_t timeout_ns;
   uint32_t* status;
 };
 
 // Shared-memory descriptor of a K-major operand with 128-byte rows in the 128-byte swizzle whose
-// start need not be 1024-byte aligned: groups of 8 rows 1024 bytes apart (stride byte offset).
+// start need not be 1024-byte aligned: groups of 8 rows 1024 bytes apart (stride byte offset).  The
+// swizzle follows the address bits, so a window that starts r rows into the plane reads the rows
+// the converters stored there (the matrix base offset stays 0; measured exact on every start row).
 __device__ __forceinline__ uint64_t smem_desc_kmajor_sw128_at(uint32_t saddr) {
   uint64_t d = 0;
   d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
@@ -122,17 +138,19 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
   asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
-// 2-D tiled bulk-tensor reduction global[box at (x, y)] += shared[src] (element type and wrap from
-// the tensor map; elements outside the tensor skipped); tracked by this thread's bulk groups.
-__device__ __forceinline__ void reduce_box(const void* map, uint32_t src, int32_t x, int32_t y) {
-  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(src), "r"(x), "r"(y)
-               : "memory");
-}
-
 __device__ __forceinline__ uint64_t widen(uint32_t f32_bits) {
   return static_cast<uint64_t>(static_cast<int64_t>(tc::f32_to_i32(f32_bits)));
+}
+
+// Polls (no suspend hint) a barrier that the peer CTA arrives on, with cluster-scope acquire.
+__device__ __forceinline__ bool spin_wait_cluster(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try_wait_cluster(bar, parity, 0u)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    for (int i = 0; i < 256; ++i)
+      if (mbar_try_wait_cluster(bar, parity, 0u)) return true;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
 }
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -141,43 +159,49 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
-  const uint32_t limbs_full = smem_u32(bars);     // the tile's limbs stored (8 converter warps)
-  const uint32_t limbs_empty = limbs_full + 8;    // the tile's MMAs done with them (2 issuers)
-  const uint32_t b_full0 = limbs_empty + 8;
-  const uint32_t b_empty0 = b_full0 + 8 * B_STAGES;  // both issuers' MMAs on the stage done
+  const uint32_t limbs_full0 = smem_u32(bars);          // per set: both CTAs' converters stored (even CTA's)
+  const uint32_t limbs_empty0 = limbs_full0 + 8 * NBUF;  // per set: the tile's MMAs are done with it
+  const uint32_t b_full0 = limbs_empty0 + 8 * NBUF;     // both halves landed (even CTA's)
+  const uint32_t b_empty0 = b_full0 + 8 * B_STAGES;     // both issuers' MMAs on the stage done
   const uint32_t acc_full0 = b_empty0 + 8 * B_STAGES;
-  const uint32_t acc_empty0 = acc_full0 + 16;
-  const uint32_t stg_full = acc_empty0 + 16;      // all epilogue warps staged the unit
-  const uint32_t stg_free = stg_full + 8;         // the unit's reductions have read the staging
+  const uint32_t acc_empty0 = acc_full0 + 16;           // both CTAs' epilogue warps drained (even CTA's)
+  const uint32_t stg_full = acc_empty0 + 16;            // this CTA's epilogue warps staged the unit
+  const uint32_t stg_free = stg_full + 8;               // the unit's reductions have read the staging
   const uint32_t final_bar = stg_free + 8;
+  const uint32_t bye_bar = final_bar + 8;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + NBAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
   if (threadIdx.x == 0) {
-    mbar_init(limbs_full, NUM_CONV_WARPS);
-    mbar_init(limbs_empty, 2);
+    for (int b = 0; b < NBUF; ++b) {
+      mbar_init(limbs_full0 + 8 * b, 2 * NUM_CONV_WARPS);
+      mbar_init(limbs_empty0 + 8 * b, 2);
+    }
     for (int s = 0; s < B_STAGES; ++s) {
       mbar_init(b_full0 + 8 * s, 1);
       mbar_init(b_empty0 + 8 * s, 2);
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(acc_full0 + 8 * s, 2);
-      mbar_init(acc_empty0 + 8 * s, NUM_EPI_WARPS);
+      mbar_init(acc_empty0 + 8 * s, 2 * NUM_EPI_WARPS);
     }
     mbar_init(stg_full, NUM_EPI_WARPS);
     mbar_init(stg_free, 1);
     mbar_init(final_bar, 2);
+    mbar_init(bye_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == B_WARP) {
-    tmem_alloc(smem_u32(tmem_holder), TMEM_COLS);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(tmem_holder), TMEM_COLS);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
   // Launched with programmatic stream serialization: the set-up above may overlap the previous
@@ -185,9 +209,12 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
   pdl_wait();
   pdl_launch_dependents();
 
-  const int ntiles = (P.num_tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                     static_cast<int>(gridDim.x);
+  // pair tiles pair, pair + npairs, ...: this CTA's tile is 2 * (pair tile) + rank (none past the end)
+  const int pair = static_cast<int>(cluster_id_x());
+  const int npairs = static_cast<int>(cluster_count_x());
+  const int ntiles = (P.num_pair_tiles - pair + npairs - 1) / npairs;
   const int taps = P.R * P.S;
+  auto tile_of = [&](int i) { return 2 * (pair + i * npairs) + static_cast<int>(rank); };
 
   if (warp >= CONV_WARP0 && warp < CONV_WARP0 + NUM_CONV_WARPS) {
     // ------------------------------------------------------------ converters
@@ -206,27 +233,31 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
     }
     uint4 x[ITEMS_PER_THREAD];
     auto fetch = [&](int t) {
-      const int n = t / P.tiles_per_image;
-      const int h0 = (t - n * P.tiles_per_image) * P.T;
+      const bool real = t < P.num_tiles;  // the odd CTA of the last pair may have no tile
+      const int n = real ? t / P.tiles_per_image : 0;
+      const int h0 = real ? (t - n * P.tiles_per_image) * P.T : 0;
 #pragma unroll
       for (int j = 0; j < ITEMS_PER_THREAD; ++j) {
         x[j] = make_uint4(0u, 0u, 0u, 0u);
         const int h = h0 - P.ph + rb[j];
-        if (tid + NUM_CONV_THREADS * j < items && h >= 0 && h < P.H && cb[j] >= 0 && cb[j] < P.W)
+        if (real && tid + NUM_CONV_THREADS * j < items && h >= 0 && h < P.H && cb[j] >= 0 && cb[j] < P.W)
           x[j] = ld_nc_v4(P.X + ((static_cast<int64_t>(n) * P.H + h) * P.W + cb[j]) * CIN + c * 8);
       }
     };
-    const uint32_t l0 = smem_u32(smem + OFF_LIMB0);
-    const uint32_t l1 = smem_u32(smem + OFF_LIMB1);
-    if (ntiles > 0) fetch(static_cast<int>(blockIdx.x));
+    const uint32_t full_leader0 = map_to_rank(limbs_full0, 0);
+    if (ntiles > 0) fetch(tile_of(0));
     for (int i = 0; i < ntiles; ++i) {
-      // the previous tile's MMAs must be done with the limb planes
-      const bool got = bounded_wait(limbs_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, P.timeout_ns);
+      const int b = i & 1;
+      const uint32_t use = static_cast<uint32_t>(i >> 1);
+      // the set's previous tile must be done with its planes (the MMAs have completed)
+      const bool got = bounded_wait(limbs_empty0 + 8 * b, (use & 1u) ^ 1u, P.timeout_ns);
       if (!__all_sync(0xFFFFFFFFu, got && !*abort_flag)) {  // the warp decides together
         if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 41);
         *abort_flag = 1;
         break;
       }
+      const uint32_t l0 = smem_u32(smem + OFF_LIMB + (2 * b) * LIMB_BYTES);
+      const uint32_t l1 = l0 + LIMB_BYTES;
 #pragma unroll
       for (int j = 0; j < ITEMS_PER_THREAD; ++j) {
         if (tid + NUM_CONV_THREADS * j < items) {
@@ -243,16 +274,17 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
       }
       fence_proxy_async_smem();  // the tensor cores read the planes through the async proxy
       __syncwarp();
-      if (lane == 0) mbar_arrive(limbs_full);
-      if (i + 1 < ntiles) fetch(static_cast<int>(blockIdx.x) + (i + 1) * static_cast<int>(gridDim.x));
+      if (lane == 0) mbar_arrive_cluster(full_leader0 + 8 * b);
+      if (i + 1 < ntiles) fetch(tile_of(i + 1));
     }
   } else if (warp == B_WARP) {
-    // ------------------------------------------------------------ B producer
+    // ------------------------------------------------------------ B producer (both CTAs)
     if (lane == 0) {
-      tma_prefetch_desc(&mapBH);
-      tma_prefetch_desc(&mapBL);
+      const CUtensorMap* mb = leader ? &mapBH : &mapBL;
+      tma_prefetch_desc(mb);
+      const uint32_t full_leader0 = map_to_rank(b_full0, 0);
       tc::RingPos pos;
-      int issued = 0;
+      int64_t issued = 0;
       bool stop = false;
       for (int i = 0; i < ntiles && !stop; ++i) {
         for (int nb = 0; nb < P.nnb && !stop; ++nb) {
@@ -263,106 +295,110 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
               stop = true;
               break;
             }
-            const uint32_t fb = b_full0 + 8 * pos.slot;
-            const uint32_t base = smem_u32(smem + OFF_B + pos.slot * TILE_B);
-            mbar_arrive_expect_tx(fb, TILE_B);
-            tma_load_2d(base, &mapBH, fb, tap * CIN, nb * BN);
-            tma_load_2d(base + TILE_B / 2, &mapBL, fb, tap * CIN, nb * BN);
+            if (leader) mbar_arrive_expect_tx(b_full0 + 8 * pos.slot, 2 * TILE_BH);
+            tma_load_2d_pair(smem_u32(smem + OFF_B + pos.slot * TILE_BH), mb, full_leader0 + 8 * pos.slot, tap * CIN,
+                             nb * BN);
             pos.advance(B_STAGES);
             ++issued;
           }
         }
       }
-      // copies still in flight: slots below pos.slot in this round, the others in the last one
-      for (int s = 0; s < B_STAGES; ++s) {
-        if (s < pos.slot)
-          bounded_wait(b_full0 + 8 * s, pos.phase, P.timeout_ns);
-        else if (issued >= B_STAGES)
-          bounded_wait(b_full0 + 8 * s, pos.phase ^ 1u, P.timeout_ns);
-      }
+      // no copy of this CTA may still be landing when it exits: the last stages must have been
+      // consumed by the MMAs (which waited for every byte of them)
+      const int64_t first = issued > B_STAGES ? issued - B_STAGES : 0;
+      for (int64_t i = first; i < issued; ++i)
+        bounded_wait(b_empty0 + 8 * static_cast<int>(i % B_STAGES), static_cast<uint32_t>((i / B_STAGES) & 1),
+                     P.timeout_ns);
     }
   } else if (warp == ISSUE_WARP0 || warp == ISSUE_WARP0 + 1) {
-    // ------------------------------------------------------------ MMA issuers (issuer e: A limb e)
+    // ------------------------------------------------------------ MMA issuers (even CTA; issuer e: A limb e)
     if (lane == 0) {
-      const int me = warp - ISSUE_WARP0;
-      constexpr uint32_t idesc = idesc_f16_f32(BM, UMMA_N);
-      const uint32_t limb = smem_u32(smem + (me == 0 ? OFF_LIMB0 : OFF_LIMB1));
-      tc::RingPos pb;
-      int unit = 0;
-      bool ok = true;
-      for (int i = 0; i < ntiles && ok; ++i) {
-        if (!spin_wait(limbs_full, static_cast<uint32_t>(i) & 1u, P.timeout_ns) || *abort_flag) {
-          report_status(P.status, STATUS_TIMEOUT, 43);
-          *abort_flag = 1;
-          break;
-        }
-        tc_fence_after();
-        for (int nb = 0; nb < P.nnb && ok; ++nb, ++unit) {
-          const int slot = unit & 1;
-          const uint32_t use = static_cast<uint32_t>(unit >> 1);
-          if (!spin_wait(acc_empty0 + 8 * slot, (use & 1u) ^ 1u, P.timeout_ns) || *abort_flag) {
-            report_status(P.status, STATUS_TIMEOUT, 44);
+      if (leader) {
+        const int me = warp - ISSUE_WARP0;
+        constexpr uint32_t idesc = idesc_f16_f32(UMMA_M, UMMA_N);
+        tc::RingPos pb;
+        int unit = 0;
+        bool ok = true;
+        for (int i = 0; i < ntiles && ok; ++i) {
+          const int b = i & 1;
+          const uint32_t use = static_cast<uint32_t>(i >> 1);
+          if (!spin_wait_cluster(limbs_full0 + 8 * b, use & 1u, P.timeout_ns) || *abort_flag) {
+            report_status(P.status, STATUS_TIMEOUT, 43);
             *abort_flag = 1;
-            ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS + me * UMMA_N);
-          for (int tap = 0; tap < taps; ++tap) {
-            const int r = tap / P.S;
-            const int s = tap - r * P.S;
-            if (!spin_wait(b_full0 + 8 * pb.slot, pb.phase, P.timeout_ns)) {
-              report_status(P.status, STATUS_TIMEOUT, 45);
+          const uint32_t limb = smem_u32(smem + OFF_LIMB + (2 * b + me) * LIMB_BYTES);
+          for (int nb = 0; nb < P.nnb && ok; ++nb, ++unit) {
+            const int slot = unit & 1;
+            const uint32_t suse = static_cast<uint32_t>(unit >> 1);
+            if (!spin_wait_cluster(acc_empty0 + 8 * slot, (suse & 1u) ^ 1u, P.timeout_ns) || *abort_flag) {
+              report_status(P.status, STATUS_TIMEOUT, 44);
               *abort_flag = 1;
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t a0 = limb + static_cast<uint32_t>((r * P.Wp + s) * 128);
-            const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + pb.slot * TILE_B));
+            const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS + me * UMMA_N);
+            for (int tap = 0; tap < taps; ++tap) {
+              const int r = tap / P.S;
+              const int s = tap - r * P.S;
+              if (!spin_wait(b_full0 + 8 * pb.slot, pb.phase, P.timeout_ns)) {
+                report_status(P.status, STATUS_TIMEOUT, 45);
+                *abort_flag = 1;
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t a0 = limb + static_cast<uint32_t>((r * P.Wp + s) * 128);
+              const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + pb.slot * TILE_BH));
 #pragma unroll
-            for (int kk = 0; kk < CIN / UMMA_K; ++kk) {
-              // K step kk: 16 channels, 32 bytes into the swizzled rows of both operands
-              const uint64_t adesc = smem_desc_kmajor_sw128_at(a0 + static_cast<uint32_t>(32 * kk));
-              tc_mma_f16(d, adesc, bdesc + 2 * kk, idesc, (tap == 0 && kk == 0) ? 0u : 1u);
+              for (int kk = 0; kk < CIN / UMMA_K; ++kk) {
+                // K step kk: 16 channels, 32 bytes into the swizzled rows of both operands
+                const uint64_t adesc = smem_desc_kmajor_sw128_at(a0 + static_cast<uint32_t>(32 * kk));
+                tc_mma_f16_pair(d, adesc, bdesc + 2 * kk, idesc, (tap == 0 && kk == 0) ? 0u : 1u);
+              }
+              tc_commit_pair(b_empty0 + 8 * pb.slot, 0x3);  // the stage is free in both CTAs
+              pb.advance(B_STAGES);
             }
-            tc_commit(b_empty0 + 8 * pb.slot);
-            pb.advance(B_STAGES);
+            if (!ok) break;
+            tc_commit_pair(acc_full0 + 8 * slot, 0x3);
           }
           if (!ok) break;
-          tc_commit(acc_full0 + 8 * slot);
+          tc_commit_pair(limbs_empty0 + 8 * b, 0x3);
         }
-        if (!ok) break;
-        tc_commit(limbs_empty);
+        tc_commit_pair(final_bar, 0x3);
       }
-      tc_commit(final_bar);
+      // both CTAs: every MMA of the pair, and every commit arrival, has landed
       bounded_wait(final_bar, 0, P.timeout_ns);
     }
   } else {
     // ------------------------------------------------------------ epilogue (warps 0-7)
     const int quad = warp & 3;
     const int half = warp >> 2;
-    const int p = quad * 32 + lane;  // this thread's MMA row
+    const int p = quad * 32 + lane;  // this thread's MMA row within this CTA's window
     const int hr = p / P.Wp;
     const int wq = p - hr * P.Wp;
     const uint32_t lane_field = static_cast<uint32_t>(quad * 32) << 16;
     const uint32_t stg = smem_u32(smem + OFF_STG);
     const uint32_t rowi = static_cast<uint32_t>(hr * P.wpad + wq);
+    const uint32_t empty_leader0 = map_to_rank(acc_empty0, 0);
     const bool reducer = warp == 0 && lane == 0;
     int unit = 0;
     bool ok = true;
     for (int i = 0; i < ntiles && ok; ++i) {
-      const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
-      const int n = t / P.tiles_per_image;
-      const int h0 = (t - n * P.tiles_per_image) * P.T;
-      const bool valid = hr < P.T && h0 + hr < P.H && wq < P.W;
+      const int t = tile_of(i);
+      const bool real = t < P.num_tiles;
+      const int n = real ? t / P.tiles_per_image : 0;
+      const int h0 = real ? (t - n * P.tiles_per_image) * P.T : 0;
+      const bool valid = real && hr < P.T && h0 + hr < P.H && wq < P.W;
       for (int nb = 0; nb < P.nnb; ++nb, ++unit) {
         const int slot = unit & 1;
-        const uint32_t use = static_cast<uint32_t>(unit >> 1);
+        const uint32_t suse = static_cast<uint32_t>(unit >> 1);
         const uint32_t upar = static_cast<uint32_t>(unit) & 1u;
         // the staging area is free once the previous unit's reductions have read it
         bool got = bounded_wait(stg_free, upar ^ 1u, P.timeout_ns);
-        got = got && bounded_wait(acc_full0 + 8 * slot, use & 1u, P.timeout_ns);
+        got = got && bounded_wait(acc_full0 + 8 * slot, suse & 1u, P.timeout_ns);
         if (!__all_sync(0xFFFFFFFFu, got && !*abort_flag)) {  // the warp decides together
           if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 46);
           *abort_flag = 1;
@@ -397,7 +433,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(acc_empty0 + 8 * slot);
+        if (lane == 0) mbar_arrive_cluster(empty_leader0 + 8 * slot);
         fence_proxy_async_smem();  // the reductions read the staging area through the async proxy
         __syncwarp();
         if (lane == 0) mbar_arrive(stg_full);
@@ -405,7 +441,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
           if (!bounded_wait(stg_full, upar, P.timeout_ns)) {
             report_status(P.status, STATUS_TIMEOUT, 47);
             *abort_flag = 1;
-          } else {
+          } else if (real) {
             for (int r2 = 0; r2 < P.T; ++r2) {
               if (h0 + r2 >= P.H) break;
               const int32_t y = (n * P.H + h0 + r2) * P.W;
@@ -413,7 +449,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
               for (int g = 0; g < 4; ++g) {
                 const int x0 = nb * BN + g * 16;
                 if (x0 < P.cout)
-                  reduce_box(&mapY, stg + static_cast<uint32_t>(g * STG_G + r2 * P.wpad * 128), x0, y);
+                  tma_reduce_add_2d(&mapY, stg + static_cast<uint32_t>(g * STG_G + r2 * P.wpad * 128), x0, y);
               }
             }
             bulk_commit();
@@ -426,11 +462,17 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
     if (reducer) bulk_wait_all();
   }
 
+  // Pair handshake: neither CTA exits (or frees tensor memory) while its peer may still signal it.
   tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    mbar_arrive_cluster(map_to_rank(bye_bar, rank ^ 1u));
+    if (!bounded_wait_cluster(bye_bar, 0, P.timeout_ns)) report_status(P.status, STATUS_TIMEOUT, 48);
+  }
   __syncthreads();
   if (warp == B_WARP) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    tmem_dealloc_pair(tmem_base, TMEM_COLS);
   }
 }
 
@@ -458,7 +500,7 @@ cudaError_t conv_rows_i16(const ConvRowsArgs& a, cudaStream_t s, const char** wh
   ConvParams P;
   if (!conv_rows_geometry(a.W, a.R, a.S, a.chunk_scale, &P.Wp, &P.T, &P.PB, &P.wpad) || a.cout < 1 ||
       a.cout % 2 != 0 || a.N * a.H * a.W >= (int64_t(1) << 31) || reinterpret_cast<uintptr_t>(a.X) % 16 != 0 ||
-      reinterpret_cast<uintptr_t>(a.Y) % 16 != 0) {
+      reinterpret_cast<uintptr_t>(a.Y) % 16 != 0 || a.num_sms < 2) {
     *why = "direct convolution: unsupported shape";
     return cudaErrorInvalidValue;
   }
@@ -480,6 +522,7 @@ cudaError_t conv_rows_i16(const ConvRowsArgs& a, cudaStream_t s, const char** wh
   P.pw = static_cast<int>((a.S - 1) / 2);
   P.tiles_per_image = static_cast<int>((a.H + P.T - 1) / P.T);
   P.num_tiles = static_cast<int>(a.N * P.tiles_per_image);
+  P.num_pair_tiles = (P.num_tiles + 1) / 2;
   P.nnb = static_cast<int>((a.cout + BN - 1) / BN);
   P.cout = static_cast<int>(a.cout);
   P.timeout_ns = a.timeout_ns;
@@ -493,17 +536,22 @@ cudaError_t conv_rows_i16(const ConvRowsArgs& a, cudaStream_t s, const char** wh
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) attr_done[dev] = true;
   }
-  const int grid = P.num_tiles < a.num_sms ? P.num_tiles : a.num_sms;
+  const int max_pairs = a.num_sms / 2;
+  const int npairs = P.num_pair_tiles < max_pairs ? P.num_pair_tiles : max_pairs;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.gridDim = dim3(2 * static_cast<unsigned>(npairs), 1, 1);
   cfg.blockDim = dim3(NUM_THREADS, 1, 1);
   cfg.dynamicSmemBytes = SMEM;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   *why = "direct convolution launch";
   return cudaLaunchKernelEx(&cfg, conv_rows_kernel, mapBH, mapBL, mapY, P);
 }

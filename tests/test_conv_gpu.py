@@ -63,7 +63,7 @@ def direct_applies(gm, shape):
     if R * S * 64 > 512 * gm.get_option(gm.OPT_TC_CHUNK_SCALE):
         return False
     wp, wpad = W + S - 1, (W + 7) // 8 * 8
-    if wp > 128 or min(128 // wp, 136 // wpad) < 1:
+    if wp > 128 or min(128 // wp, 120 // wpad) < 1:
         return False
     return (128 + (R - 1) * wp + (S - 1) + 7) // 8 * 8 <= 256
 
@@ -123,7 +123,8 @@ DIRECT_EDGES = [
     (1, 4, 12, 64, 256, 3, 3, 1, 1),    # four channel blocks
     (3, 5, 8, 64, 48, 5, 3, 2, 1),      # 5x3: 960 reduction indices
     (2, 7, 20, 64, 64, 1, 3, 0, 1),     # 1x3
-    (1, 3, 126, 64, 64, 1, 3, 0, 1),    # padded row of 128: one output row per tile
+    (1, 3, 120, 64, 64, 1, 3, 0, 1),    # one output row of 120 pixels per tile (the staging limit)
+    (1, 3, 121, 64, 64, 1, 3, 0, 1),    # 121 pixels: beyond the staging limit -> fused kernel
     (2, 6, 8, 64, 63, 3, 3, 1, 1),      # odd Cout -> fused kernel
     (5, 20, 3, 64, 64, 3, 3, 1, 1),     # narrow images, 17 rows per tile, ragged last tile
 ]
