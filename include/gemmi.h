@@ -286,8 +286,9 @@ size_t gemmi_workspace_bytes(void);
  *                            panels while the tensor cores work, and a tile's loads wait until
  *                            its panel is complete; 0: the whole split runs before the GEMM.
  *   GEMMI_OPT_CONV_ROWS    : 1 (default): gemmi_conv2d_i16 runs "same" convolutions with 64 input
- *                            channels, odd R and S, R*S*64 within one exact chunk (512 * chunk
- *                            scale), an even Cout, W <= 120, W + S - 1 <= 128 and 16-byte aligned X and Y
+ *                            channels, odd R and S with R*S <= 12 and R*S*64 within one exact chunk
+ *                            (512 * chunk scale), an even Cout <= 64, W <= 120, W + S - 1 <= 128
+ *                            and 16-byte aligned X and Y
  *                            on the direct kernel, which splits every input pixel once per tile of
  *                            output rows (the taps are shifted windows of the split rows); 0:
  *                            such convolutions take the lowered GEMM read tap by tap.

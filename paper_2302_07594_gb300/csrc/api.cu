@@ -634,7 +634,7 @@ int conv2d_locked(int64_t N, int64_t H, int64_t W, int64_t Cin, int64_t Cout, in
   int rc = device_state(&d);
   if (rc != GEMMI_OK) return rc;
   int geo[4];
-  if (g_conv_rows != 0 && Ho == H && Wo == W && Cin == 64 && M > g_skinny_max_m && Cout % 2 == 0 &&
+  if (g_conv_rows != 0 && Ho == H && Wo == W && Cin == 64 && M > g_skinny_max_m && Cout % 2 == 0 && Cout <= 64 &&
       N * H * W < (int64_t(1) << 31) && reinterpret_cast<uintptr_t>(X) % 16 == 0 &&
       reinterpret_cast<uintptr_t>(Y) % 16 == 0 &&
       gemmi::conv_rows_geometry(W, R, S, static_cast<int>(g_tc_chunk_scale), &geo[0], &geo[1], &geo[2], &geo[3]))

@@ -3,8 +3,9 @@
 // What it computes: the convolution of gemmi_conv2d_i16,
 //   Y[n][h][w][co] += sum over r < R, s < S, c < 64 of
 //                     X[n][h + r - ph][w + s - pw][c] * Wt[(r*S + s)*64 + c][co],
-// X read as 0 outside the image, bit-exactly modulo 2^64, for 64 input channels and odd R, S with
-// ph = (R - 1) / 2, pw = (S - 1) / 2 (the output has the input's size).  Sections 2 and 3 of the
+// X read as 0 outside the image, bit-exactly modulo 2^64, for 64 input channels, at most 64 output
+// channels and odd R, S (R*S <= 12) with ph = (R - 1) / 2, pw = (S - 1) / 2 (the output has the
+// input's size).  Sections 2 and 3 of the
 // paper lower a convolution to one GEMM (IM2COL) and note that the lowering can be done on the fly
 // while the activations are packed; this kernel packs each activation once for all filter taps.
 //
@@ -39,19 +40,20 @@
 // even CTA issues tcgen05.mma.cta_group::2 of M = 256: MMA rows 0-127 are the even CTA's window,
 // rows 128-255 the odd CTA's (each CTA's limb planes at the same shared-memory offsets), and the
 // stacked weights are split between them (B_high rows in the even CTA, B_low rows in the odd
-// one).  Each SM so reads 4 KB of pixels and 2 KB of weights per MMA step instead of 4 + 4: with
-// both operands in shared memory, the reads bound the MMA rate.  Two sets of limb planes per CTA
-// let the converters split the next tile while the tensor cores work on the current one.
+// one).  Each SM so reads 4 KB of pixels and 2 KB of weights per MMA step instead of 4 + 4.  Each
+// CTA loads its half of the weights' limb tiles for every tap once, when it starts, and keeps them:
+// the MMA threads then wait and commit once per tile, not once per tap (the per-tap stage
+// handshakes drained the tensor pipe at every tap boundary).
 //
 // Roles (one CTA per SM, clusters of two, 608 threads per CTA):
 //   warps 0-7   epilogue: warp w drains TMEM lanes 32*(w % 4) .. +31 (MMA rows) for output
 //               channels 32*(w / 4) .. +31 of the block, into a 128-byte-swizzled staging area;
 //               lane 0 of warp 0 issues the tile's reductions;
 //   warps 8-15  converters: load the next tile's pixels into registers while the tensor cores
-//               work on the current one, then split them into a free set of limb planes;
-//   warp 16     TMEM allocation (both CTAs); lane 0 streams this CTA's half of B's stacked limb
-//               tiles (one per tap and block of output channels) through a ring by TMA, every
-//               load completing on the even CTA's barrier;
+//               work on the current one, then split them into the limb planes once those MMAs
+//               are done;
+//   warp 16     TMEM allocation (both CTAs); lane 0 loads this CTA's half of B's stacked limb
+//               tiles (one per tap) by TMA, every load completing on the even CTA's barrier;
 //   warps 17-18 lane 0 of the even CTA: the MMA issuer of A limb 0 (high) and of A limb 1 (low);
 //               their commits arrive on the barriers of both CTAs.
 // Every wait is bounded by the global timer; one that runs out records GEMMI_ETIMEOUT in the
@@ -86,18 +88,16 @@ constexpr int NUM_THREADS = 19 * 32;
 constexpr int PB_MAX = 256;                  // buffered positions
 constexpr int ITEMS_PER_THREAD = PB_MAX * 8 / NUM_CONV_THREADS;  // 16-byte cells per converter thread
 constexpr int LIMB_BYTES = PB_MAX * 128;     // one limb plane: a 128-byte row per position
-constexpr int NBUF = 2;                      // sets of limb planes (tile i uses set i % 2)
-constexpr int B_STAGES = 4;
+constexpr int MAX_TAPS = 12;                 // R * S: this CTA's weight halves stay resident
 constexpr int TILE_BH = BN * CIN * 2;        // 8 KB: this CTA's half of a stacked limb tile
 constexpr int STG_ROWS = 120;                // staged output pixels per tile: T * round_up(W, 8)
 constexpr int STG_G = STG_ROWS * 128;        // one group of 16 output channels (int64)
 constexpr int OFF_LIMB = 0;
-constexpr int OFF_B = NBUF * 2 * LIMB_BYTES;
-constexpr int OFF_STG = OFF_B + B_STAGES * TILE_BH;
+constexpr int OFF_B = 2 * LIMB_BYTES;
+constexpr int OFF_STG = OFF_B + MAX_TAPS * TILE_BH;
 constexpr int OFF_BAR = OFF_STG + 4 * STG_G;
-// limbs full / empty (per set), B full / empty, accumulator full / empty (two slots), staging
-// full / free, final, bye
-constexpr int NBAR = 2 * NBUF + 2 * B_STAGES + 4 + 2 + 2;
+// limbs full / empty, B full, accumulator full / empty (two slots), staging full / free, final, bye
+constexpr int NBAR = 2 + 1 + 4 + 2 + 2;
 constexpr size_t SMEM = 1024 + static_cast<size_t>(OFF_BAR) + 8 * NBAR + 16;
 static_assert(SMEM <= 227 * 1024, "shared memory budget");
 static_assert(OFF_B % 1024 == 0 && OFF_STG % 1024 == 0 && STG_G % 1024 == 0 && TILE_BH % 1024 == 0,
@@ -109,7 +109,7 @@ struct ConvParams {
   const int16_t* X;
   int H, W, R, S, ph, pw;
   int Wp, T, PB, wpad;
-  int tiles_per_image, num_tiles, num_pair_tiles, nnb, cout;
+  int tiles_per_image, num_tiles, num_pair_tiles, cout;
   uint64_t timeout_ns;
   uint32_t* status;
 };
@@ -159,11 +159,10 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
-  const uint32_t limbs_full0 = smem_u32(bars);          // per set: both CTAs' converters stored (even CTA's)
-  const uint32_t limbs_empty0 = limbs_full0 + 8 * NBUF;  // per set: the tile's MMAs are done with it
-  const uint32_t b_full0 = limbs_empty0 + 8 * NBUF;     // both halves landed (even CTA's)
-  const uint32_t b_empty0 = b_full0 + 8 * B_STAGES;     // both issuers' MMAs on the stage done
-  const uint32_t acc_full0 = b_empty0 + 8 * B_STAGES;
+  const uint32_t limbs_full = smem_u32(bars);           // both CTAs' converters stored (even CTA's)
+  const uint32_t limbs_empty = limbs_full + 8;          // the tile's MMAs are done with the planes
+  const uint32_t b_full = limbs_empty + 8;              // every tap's halves landed (even CTA's)
+  const uint32_t acc_full0 = b_full + 8;
   const uint32_t acc_empty0 = acc_full0 + 16;           // both CTAs' epilogue warps drained (even CTA's)
   const uint32_t stg_full = acc_empty0 + 16;            // this CTA's epilogue warps staged the unit
   const uint32_t stg_free = stg_full + 8;               // the unit's reductions have read the staging
@@ -177,14 +176,9 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
   const uint32_t rank = cluster_ctarank();
   const bool leader = rank == 0;
   if (threadIdx.x == 0) {
-    for (int b = 0; b < NBUF; ++b) {
-      mbar_init(limbs_full0 + 8 * b, 2 * NUM_CONV_WARPS);
-      mbar_init(limbs_empty0 + 8 * b, 2);
-    }
-    for (int s = 0; s < B_STAGES; ++s) {
-      mbar_init(b_full0 + 8 * s, 1);
-      mbar_init(b_empty0 + 8 * s, 2);
-    }
+    mbar_init(limbs_full, 2 * NUM_CONV_WARPS);
+    mbar_init(limbs_empty, 2);
+    mbar_init(b_full, 1);
     for (int s = 0; s < 2; ++s) {
       mbar_init(acc_full0 + 8 * s, 2);
       mbar_init(acc_empty0 + 8 * s, 2 * NUM_EPI_WARPS);
@@ -244,20 +238,18 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
           x[j] = ld_nc_v4(P.X + ((static_cast<int64_t>(n) * P.H + h) * P.W + cb[j]) * CIN + c * 8);
       }
     };
-    const uint32_t full_leader0 = map_to_rank(limbs_full0, 0);
+    const uint32_t full_leader = map_to_rank(limbs_full, 0);
+    const uint32_t l0 = smem_u32(smem + OFF_LIMB);
+    const uint32_t l1 = l0 + LIMB_BYTES;
     if (ntiles > 0) fetch(tile_of(0));
     for (int i = 0; i < ntiles; ++i) {
-      const int b = i & 1;
-      const uint32_t use = static_cast<uint32_t>(i >> 1);
-      // the set's previous tile must be done with its planes (the MMAs have completed)
-      const bool got = bounded_wait(limbs_empty0 + 8 * b, (use & 1u) ^ 1u, P.timeout_ns);
+      // the previous tile's MMAs must be done with the planes
+      const bool got = bounded_wait(limbs_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, P.timeout_ns);
       if (!__all_sync(0xFFFFFFFFu, got && !*abort_flag)) {  // the warp decides together
         if (lane == 0) report_status(P.status, STATUS_TIMEOUT, 41);
         *abort_flag = 1;
         break;
       }
-      const uint32_t l0 = smem_u32(smem + OFF_LIMB + (2 * b) * LIMB_BYTES);
-      const uint32_t l1 = l0 + LIMB_BYTES;
 #pragma unroll
       for (int j = 0; j < ITEMS_PER_THREAD; ++j) {
         if (tid + NUM_CONV_THREADS * j < items) {
@@ -274,41 +266,21 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
       }
       fence_proxy_async_smem();  // the tensor cores read the planes through the async proxy
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(full_leader0 + 8 * b);
+      if (lane == 0) mbar_arrive_cluster(full_leader);
       if (i + 1 < ntiles) fetch(tile_of(i + 1));
     }
   } else if (warp == B_WARP) {
-    // ------------------------------------------------------------ B producer (both CTAs)
-    if (lane == 0) {
+    // ------------------------------------------------------------ weights (both CTAs), once
+    if (lane == 0 && ntiles > 0) {
       const CUtensorMap* mb = leader ? &mapBH : &mapBL;
       tma_prefetch_desc(mb);
-      const uint32_t full_leader0 = map_to_rank(b_full0, 0);
-      tc::RingPos pos;
-      int64_t issued = 0;
-      bool stop = false;
-      for (int i = 0; i < ntiles && !stop; ++i) {
-        for (int nb = 0; nb < P.nnb && !stop; ++nb) {
-          for (int tap = 0; tap < taps; ++tap) {
-            if (!spin_wait(b_empty0 + 8 * pos.slot, pos.phase ^ 1u, P.timeout_ns) || *abort_flag) {
-              report_status(P.status, STATUS_TIMEOUT, 42);
-              *abort_flag = 1;
-              stop = true;
-              break;
-            }
-            if (leader) mbar_arrive_expect_tx(b_full0 + 8 * pos.slot, 2 * TILE_BH);
-            tma_load_2d_pair(smem_u32(smem + OFF_B + pos.slot * TILE_BH), mb, full_leader0 + 8 * pos.slot, tap * CIN,
-                             nb * BN);
-            pos.advance(B_STAGES);
-            ++issued;
-          }
-        }
-      }
-      // no copy of this CTA may still be landing when it exits: the last stages must have been
-      // consumed by the MMAs (which waited for every byte of them)
-      const int64_t first = issued > B_STAGES ? issued - B_STAGES : 0;
-      for (int64_t i = first; i < issued; ++i)
-        bounded_wait(b_empty0 + 8 * static_cast<int>(i % B_STAGES), static_cast<uint32_t>((i / B_STAGES) & 1),
-                     P.timeout_ns);
+      if (leader) mbar_arrive_expect_tx(b_full, static_cast<uint32_t>(2 * taps * TILE_BH));
+      const uint32_t full_leader = map_to_rank(b_full, 0);
+      for (int tap = 0; tap < taps; ++tap)
+        tma_load_2d_pair(smem_u32(smem + OFF_B + tap * TILE_BH), mb, full_leader, tap * CIN, 0);
+      // no copy of this CTA may still be landing when it exits: every MMA of the pair has waited
+      // for all of them, and this warp's lane 0 waits for the MMAs to be done (final barrier)
+      bounded_wait(final_bar, 0, P.timeout_ns);
     }
   } else if (warp == ISSUE_WARP0 || warp == ISSUE_WARP0 + 1) {
     // ------------------------------------------------------------ MMA issuers (even CTA; issuer e: A limb e)
@@ -316,56 +288,38 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
       if (leader) {
         const int me = warp - ISSUE_WARP0;
         constexpr uint32_t idesc = idesc_f16_f32(UMMA_M, UMMA_N);
-        tc::RingPos pb;
-        int unit = 0;
-        bool ok = true;
+        bool ok = ntiles == 0 || spin_wait(b_full, 0, P.timeout_ns);
+        if (!ok) {
+          report_status(P.status, STATUS_TIMEOUT, 45);
+          *abort_flag = 1;
+        }
+        const uint32_t bbase = smem_u32(smem + OFF_B);
         for (int i = 0; i < ntiles && ok; ++i) {
-          const int b = i & 1;
+          const int slot = i & 1;
           const uint32_t use = static_cast<uint32_t>(i >> 1);
-          if (!spin_wait_cluster(limbs_full0 + 8 * b, use & 1u, P.timeout_ns) || *abort_flag) {
+          if (!spin_wait_cluster(limbs_full, static_cast<uint32_t>(i) & 1u, P.timeout_ns) ||
+              !spin_wait_cluster(acc_empty0 + 8 * slot, (use & 1u) ^ 1u, P.timeout_ns) || *abort_flag) {
             report_status(P.status, STATUS_TIMEOUT, 43);
             *abort_flag = 1;
             break;
           }
           tc_fence_after();
-          const uint32_t limb = smem_u32(smem + OFF_LIMB + (2 * b + me) * LIMB_BYTES);
-          for (int nb = 0; nb < P.nnb && ok; ++nb, ++unit) {
-            const int slot = unit & 1;
-            const uint32_t suse = static_cast<uint32_t>(unit >> 1);
-            if (!spin_wait_cluster(acc_empty0 + 8 * slot, (suse & 1u) ^ 1u, P.timeout_ns) || *abort_flag) {
-              report_status(P.status, STATUS_TIMEOUT, 44);
-              *abort_flag = 1;
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS + me * UMMA_N);
-            for (int tap = 0; tap < taps; ++tap) {
-              const int r = tap / P.S;
-              const int s = tap - r * P.S;
-              if (!spin_wait(b_full0 + 8 * pb.slot, pb.phase, P.timeout_ns)) {
-                report_status(P.status, STATUS_TIMEOUT, 45);
-                *abort_flag = 1;
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              const uint32_t a0 = limb + static_cast<uint32_t>((r * P.Wp + s) * 128);
-              const uint64_t bdesc = smem_desc_kmajor<128>(smem_u32(smem + OFF_B + pb.slot * TILE_BH));
+          const uint32_t limb = smem_u32(smem + OFF_LIMB + me * LIMB_BYTES);
+          const uint32_t d = tmem_base + static_cast<uint32_t>(slot * SLOT_COLS + me * UMMA_N);
+          for (int tap = 0; tap < taps; ++tap) {
+            const int r = tap / P.S;
+            const int s = tap - r * P.S;
+            const uint32_t a0 = limb + static_cast<uint32_t>((r * P.Wp + s) * 128);
+            const uint64_t bdesc = smem_desc_kmajor<128>(bbase + static_cast<uint32_t>(tap * TILE_BH));
 #pragma unroll
-              for (int kk = 0; kk < CIN / UMMA_K; ++kk) {
-                // K step kk: 16 channels, 32 bytes into the swizzled rows of both operands
-                const uint64_t adesc = smem_desc_kmajor_sw128_at(a0 + static_cast<uint32_t>(32 * kk));
-                tc_mma_f16_pair(d, adesc, bdesc + 2 * kk, idesc, (tap == 0 && kk == 0) ? 0u : 1u);
-              }
-              tc_commit_pair(b_empty0 + 8 * pb.slot, 0x3);  // the stage is free in both CTAs
-              pb.advance(B_STAGES);
+            for (int kk = 0; kk < CIN / UMMA_K; ++kk) {
+              // K step kk: 16 channels, 32 bytes into the swizzled rows of both operands
+              const uint64_t adesc = smem_desc_kmajor_sw128_at(a0 + static_cast<uint32_t>(32 * kk));
+              tc_mma_f16_pair(d, adesc, bdesc + 2 * kk, idesc, (tap == 0 && kk == 0) ? 0u : 1u);
             }
-            if (!ok) break;
-            tc_commit_pair(acc_full0 + 8 * slot, 0x3);
           }
-          if (!ok) break;
-          tc_commit_pair(limbs_empty0 + 8 * b, 0x3);
+          tc_commit_pair(acc_full0 + 8 * slot, 0x3);
+          tc_commit_pair(limbs_empty, 0x3);
         }
         tc_commit_pair(final_bar, 0x3);
       }
@@ -392,7 +346,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
       const int n = real ? t / P.tiles_per_image : 0;
       const int h0 = real ? (t - n * P.tiles_per_image) * P.T : 0;
       const bool valid = real && hr < P.T && h0 + hr < P.H && wq < P.W;
-      for (int nb = 0; nb < P.nnb; ++nb, ++unit) {
+      {
         const int slot = unit & 1;
         const uint32_t suse = static_cast<uint32_t>(unit >> 1);
         const uint32_t upar = static_cast<uint32_t>(unit) & 1u;
@@ -447,7 +401,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
               const int32_t y = (n * P.H + h0 + r2) * P.W;
 #pragma unroll
               for (int g = 0; g < 4; ++g) {
-                const int x0 = nb * BN + g * 16;
+                const int x0 = g * 16;
                 if (x0 < P.cout)
                   tma_reduce_add_2d(&mapY, stg + static_cast<uint32_t>(g * STG_G + r2 * P.wpad * 128), x0, y);
               }
@@ -457,6 +411,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
           bulk_wait_read_all();
           mbar_arrive(stg_free);
         }
+        ++unit;
       }
     }
     if (reducer) bulk_wait_all();
@@ -480,7 +435,7 @@ conv_rows_kernel(const __grid_constant__ CUtensorMap mapBH, const __grid_constan
 
 bool conv_rows_geometry(int64_t W, int64_t R, int64_t S, int chunk_scale, int* Wp, int* T, int* PB, int* wpad) {
   if (W < 1 || R < 1 || S < 1 || (R % 2) == 0 || (S % 2) == 0) return false;
-  if (R * S * CIN > 512 * chunk_scale) return false;  // one exact chunk per tile
+  if (R * S * CIN > 512 * chunk_scale || R * S > MAX_TAPS) return false;  // one exact chunk per tile
   const int64_t wp = W + S - 1;
   if (wp > BM) return false;
   const int64_t wpd = (W + 7) / 8 * 8;
@@ -499,7 +454,7 @@ bool conv_rows_geometry(int64_t W, int64_t R, int64_t S, int chunk_scale, int* W
 cudaError_t conv_rows_i16(const ConvRowsArgs& a, cudaStream_t s, const char** why) {
   ConvParams P;
   if (!conv_rows_geometry(a.W, a.R, a.S, a.chunk_scale, &P.Wp, &P.T, &P.PB, &P.wpad) || a.cout < 1 ||
-      a.cout % 2 != 0 || a.N * a.H * a.W >= (int64_t(1) << 31) || reinterpret_cast<uintptr_t>(a.X) % 16 != 0 ||
+      a.cout % 2 != 0 || a.cout > BN || a.N * a.H * a.W >= (int64_t(1) << 31) || reinterpret_cast<uintptr_t>(a.X) % 16 != 0 ||
       reinterpret_cast<uintptr_t>(a.Y) % 16 != 0 || a.num_sms < 2) {
     *why = "direct convolution: unsupported shape";
     return cudaErrorInvalidValue;
@@ -523,7 +478,6 @@ cudaError_t conv_rows_i16(const ConvRowsArgs& a, cudaStream_t s, const char** wh
   P.tiles_per_image = static_cast<int>((a.H + P.T - 1) / P.T);
   P.num_tiles = static_cast<int>(a.N * P.tiles_per_image);
   P.num_pair_tiles = (P.num_tiles + 1) / 2;
-  P.nnb = static_cast<int>((a.cout + BN - 1) / BN);
   P.cout = static_cast<int>(a.cout);
   P.timeout_ns = a.timeout_ns;
   P.status = a.status;

@@ -109,8 +109,9 @@ struct FusedArgs {
 };
 cudaError_t tc_gemm_fused_i16(const FusedArgs& args, cudaStream_t s, const char** why);
 
-// ---- conv_rows.cu: "same" stride-1 int16 convolution with 64 input channels, odd R and S; each
-// input pixel split once per tile (the filter taps are shifted windows of the split rows).
+// ---- conv_rows.cu: "same" stride-1 int16 convolution with 64 input channels, at most 64 output
+// channels, odd R and S; each input pixel split once per tile (the filter taps are shifted windows
+// of the split rows).
 struct ConvRowsArgs {
   const int16_t* X;  // N x H x W x 64 (NHWC), 16-byte aligned
   int64_t N, H, W, R, S, cout;
@@ -122,8 +123,8 @@ struct ConvRowsArgs {
   int chunk_scale;
 };
 // The tile geometry of the direct convolution for image width W and an R x S filter, or false when
-// the kernel does not cover the shape (even R or S, R*S*64 above one exact chunk of 512*chunk_scale,
-// padded rows wider than 128 pixels or a shifted window beyond its buffer).
+// the kernel does not cover the shape (even R or S, R*S above 12, R*S*64 above one exact chunk of
+// 512*chunk_scale, padded rows wider than 128 pixels or a shifted window beyond its buffer).
 bool conv_rows_geometry(int64_t W, int64_t R, int64_t S, int chunk_scale, int* Wp, int* T, int* PB, int* wpad);
 cudaError_t conv_rows_i16(const ConvRowsArgs& args, cudaStream_t s, const char** why);
 // ---- skinny.cu: m <= 16 int16 GEMM streaming B once.

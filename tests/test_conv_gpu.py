@@ -58,9 +58,9 @@ def direct_applies(gm, shape):
     N, H, W, Ci, Co, R, S, ph, pw = shape
     if gm.get_option(gm.OPT_CONV_ROWS) == 0 or Ci != 64 or R % 2 == 0 or S % 2 == 0:
         return False
-    if 2 * ph != R - 1 or 2 * pw != S - 1 or Co % 2 or N * H * W <= gm.get_option(gm.OPT_SKINNY_MAX_M):
+    if 2 * ph != R - 1 or 2 * pw != S - 1 or Co % 2 or Co > 64 or N * H * W <= gm.get_option(gm.OPT_SKINNY_MAX_M):
         return False
-    if R * S * 64 > 512 * gm.get_option(gm.OPT_TC_CHUNK_SCALE):
+    if R * S > 12 or R * S * 64 > 512 * gm.get_option(gm.OPT_TC_CHUNK_SCALE):
         return False
     wp, wpad = W + S - 1, (W + 7) // 8 * 8
     if wp > 128 or min(128 // wp, 120 // wpad) < 1:
@@ -119,9 +119,11 @@ DIRECT_EDGES = [
     (1, 5, 61, 64, 64, 3, 3, 1, 1),     # padded row of 63: the largest 3x3 window buffer (256 positions)
     (1, 5, 62, 64, 64, 3, 3, 1, 1),     # padded row of 64: beyond the buffer -> fused kernel
     (2, 6, 7, 64, 2, 3, 3, 1, 1),       # two output channels
-    (2, 5, 9, 64, 130, 3, 3, 1, 1),     # three channel blocks, the last one partial
-    (1, 4, 12, 64, 256, 3, 3, 1, 1),    # four channel blocks
-    (3, 5, 8, 64, 48, 5, 3, 2, 1),      # 5x3: 960 reduction indices
+    (2, 5, 9, 64, 130, 3, 3, 1, 1),     # more than 64 output channels -> fused kernel
+    (1, 4, 12, 64, 256, 3, 3, 1, 1),    # four channel blocks -> fused kernel
+    (3, 5, 8, 64, 48, 5, 3, 2, 1),      # 5x3: 15 taps -> fused kernel
+    (2, 6, 20, 64, 40, 1, 5, 0, 2),     # 1x5, 40 output channels
+    (2, 7, 9, 64, 34, 3, 3, 1, 1),      # 34 output channels: a partial group of 16
     (2, 7, 20, 64, 64, 1, 3, 0, 1),     # 1x3
     (1, 3, 120, 64, 64, 1, 3, 0, 1),    # one output row of 120 pixels per tile (the staging limit)
     (1, 3, 121, 64, 64, 1, 3, 0, 1),    # 121 pixels: beyond the staging limit -> fused kernel
