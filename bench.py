@@ -52,7 +52,7 @@ KERNEL_INFO = {
     "tc_karatsuba": ("tc_gemm_kernel<3>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
     "tc_pair_i16_ahead": ("tc_pair_kernel<2,ahead>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"),
                           "tensor"),
-    "conv_rows": ("conv_rows_kernel", ("conv_rows.cu", "tc_common.cuh", "ptx.cuh"), "hbm"),
+    "conv_rows": ("conv_rows_kernel", ("conv_rows.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "hbm"),
 }
 FP8_PER_BF16 = 2.0  # nominal dense fp8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s)
 FULL16_RANGE = ("uniform", -32768, 32767)
