@@ -5,9 +5,9 @@
 //                     X[n][h + r - ph][w + s - pw][c] * Wt[(r*S + s)*64 + c][co],
 // X read as 0 outside the image, bit-exactly modulo 2^64, for 64 input channels, at most 64 output
 // channels and odd R, S (R*S <= 12) with ph = (R - 1) / 2, pw = (S - 1) / 2 (the output has the
-// input's size).  Sections 2 and 3 of the
-// paper lower a convolution to one GEMM (IM2COL) and note that the lowering can be done on the fly
-// while the activations are packed; this kernel packs each activation once for all filter taps.
+// input's size).  Sections 2 and 3 of the paper lower a convolution to one GEMM (IM2COL) and note
+// that the lowering can be done on the fly while the activations are packed; this kernel packs
+// each activation once for all filter taps.
 //
 // Why a kernel of its own.  The lowered matrix holds every input pixel R*S times.  The narrow-n
 // fused kernel (gemm_fused.cu) reads it tap by tap and splits every copy into limbs, so its
@@ -23,15 +23,14 @@
 //
 // Shared-memory layout of a limb plane: K-major with the 128-byte swizzle, one 128-byte row per
 // position (64 channels), the 16-byte chunk of channel octet c of position q at chunk c ^ (q % 8).
-// The window from position q0 on is the matrix descriptor with start address + 128*q0 and matrix
-// base offset q0 % 8 (the swizzle pattern's phase at a start that is not 1024-byte aligned); the
+// The window from position q0 on is the matrix descriptor with start address + 128*q0 (the
+// swizzle follows the address bits, so the matrix base offset stays 0 at any start row); the
 // eight threads that store one position's eight chunks hit distinct bank groups.
 //
 // Arithmetic.  Every buffered int16 is split into its centred limbs a = 256h + l (h in [-128,128],
-// l in [-128,127], exact in fp16; the split of split.cu).  Per block of 64 output channels and
-// per tap, limb e of the window times the stacked limb tiles of B (the weights, split once per
-// call: B_high in columns 0-63, B_low in columns 64-127) accumulates into accumulator e (N = 128)
-// in TMEM.  Each column sums R*S*64 <= 512*CS products of magnitude <= 2^14, exactly in fp32.  The
+// l in [-128,127], exact in fp16; the split of split.cu).  Per tap, limb e of the window times
+// the stacked limb tiles of B (the weights, split once per call: B_high in columns 0-63, B_low in
+// columns 64-127) accumulates into accumulator e (N = 128) in TMEM.  Each column sums R*S*64 <= 512*CS products of magnitude <= 2^14, exactly in fp32.  The
 // epilogue weights the four quarters by 2^16, 2^8, 2^8 and 1 into int64 and adds each valid image
 // row of the tile into Y with 2-D tensor reductions (16 channels x W pixels each) through an
 // unsigned 64-bit tensor map, so the adds wrap modulo 2^64 and Y is never read by the SMs.
@@ -47,7 +46,7 @@
 //
 // Roles (one CTA per SM, clusters of two, 608 threads per CTA):
 //   warps 0-7   epilogue: warp w drains TMEM lanes 32*(w % 4) .. +31 (MMA rows) for output
-//               channels 32*(w / 4) .. +31 of the block, into a 128-byte-swizzled staging area;
+//               channels 32*(w / 4) .. +31, into a 128-byte-swizzled staging area;
 //               lane 0 of warp 0 issues the tile's reductions;
 //   warps 8-15  converters: load the next tile's pixels into registers while the tensor cores
 //               work on the current one, then split them into the limb planes once those MMAs
