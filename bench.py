@@ -40,7 +40,7 @@ KERNEL_INFO = {
     "split": ("split_tma_kernel", ("split.cu", "ptx.cuh", "tc_common.cuh"), "hbm"),
     "tc_i16": ("tc_gemm_kernel<2>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
     "tc_i8": ("tc_gemm_kernel<1>", ("gemm_tc.cu", "tc_common.cuh", "ptx.cuh"), "tensor"),
-    "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh"), "hbm"),
+    "skinny": ("skinny_kernel", ("skinny.cu", "ptx.cuh", "tc_common.cuh"), "hbm"),
     "fused_i16": ("fused_kernel", ("gemm_fused.cu", "tc_common.cuh", "ptx.cuh"), "hbm"),
     "srs": ("srs_add_kernel", ("requant.cu",), "hbm"),
     "tc_pair_i16": ("tc_pair_kernel<2>", ("gemm_pair.cu", "tc_common.cuh", "ptx.cuh", "ptx_pair.cuh"), "tensor"),

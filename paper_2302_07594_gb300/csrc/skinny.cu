@@ -31,15 +31,21 @@
 //     share of a stage (32 reduction indices x 32 columns) into registers, transposed with
 //     ldmatrix (the "A" operand of C^T = B^T A^T), and releases the stage at once, so the
 //     producer refills it while the warp computes (holding the stage through the arithmetic
-//     stretched every refill by about half a microsecond).  It then splits every int16 into
-//     8-bit limbs
-//         b = 256*hi + lo,  hi = b >> 8 in [-128,127],  lo = b & 255 in [0,255],
-//     exactly representable in fp16, and multiplies on the tensor cores with
-//     mma.sync m16n8k16 (fp16 in, fp32 accumulate) against the limbs of A;
-//   * three fp32 accumulator sets HH, X, LL hold exact integer sums while every
-//     partial sum stays within 2^24 (a run of 256 reduction indices:
-//     256 * 255 * 255 < 2^24 and 256 * 2 * 128 * 255 = 16,711,680 < 2^24), then are drained
-//     into int64 registers as HH*2^16 + X*2^8 + LL;
+//     stretched every refill by about half a microsecond).  For m <= 8 it then takes the two bytes of
+//         u = b + 32768 = 256*H + L,  H = (b >> 8) + 128 and L = b & 255, both in [0,255],
+//     as fp16 subnormals (bit pattern 0x00XX is the value XX * 2^-24, exactly), one mask for L
+//     and a shift and a mask for H, and multiplies them on the tensor cores with mma.sync
+//     m16n8k16 (fp16 in, fp32 accumulate) against the centred limbs of A (a = 256*h + l,
+//     |h|, |l| <= 128, split once per CTA).  Since u = b + 32768, the sums over the CTA's
+//     reduction range are sum(a*b) + 32768 * sum(a); the row sums of the CTA's slice of A,
+//     formed once, take the second term back off where the partial sums go into C.  (The 16-row
+//     instantiation splits B into its signed high and unsigned low byte as fp16 values 1024 + x
+//     less 1024, two more operations per pair; it measured faster there, its A limbs being
+//     non-centred: hi = a >> 8, lo = a & 255.)
+//   * three fp32 accumulator sets HH, X, LL hold exact sums, in units of 2^-24, while every
+//     partial sum stays within 2^24 units (a run of 256 reduction indices of products of at
+//     most 255 * 128: 256 * 2 * 32640 = 16,711,680 < 2^24 for the cross terms), then are
+//     scaled by 2^24, converted and drained into int64 registers as HH*2^16 + X*2^8 + LL;
 //   * each warp adds its partial sums into C: 64-bit atomic adds (exact and order-independent
 //     modulo 2^64) when the reduction range is split, a plain read-modify-write otherwise.
 #include <cuda.h>
@@ -47,6 +53,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace gemmi {
 namespace {
@@ -93,15 +100,24 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
 }
 
 // Dynamic shared memory: alignment slack, the B ring, the interleaved A limbs (16 rows of a_stride
-// words), the raw A slice as it lands (16 rows of `pairs` words: two int16 per word), the barriers.
+// words), the raw A slice as it lands (16 rows of `pairs` words: two int16 per word), the barriers,
+// the row sums of the A slice (16 int32).
 constexpr size_t sk_smem(int stages, int a_stride, int pairs) {
   return 1024 + static_cast<size_t>(stages) * STAGE_BYTES + static_cast<size_t>(A_ROWS) * a_stride * 4 +
-         static_cast<size_t>(A_ROWS) * pairs * 4 + 8 * (2 * stages + 1) + 16;
+         static_cast<size_t>(A_ROWS) * pairs * 4 + 8 * (2 * stages + 1) + 4 * A_ROWS + 16;
 }
 static_assert(sk_smem(4, KMAX_CTA + 16, KMAX_CTA / 2) <= SMEM_MAX, "four stages fit beside the largest A slice");
 
-// int16 pair -> fp16 pairs of its high (signed) and low (unsigned) bytes, exactly.
-// 0x64xx as fp16 is 1024 + xx, so each byte is recovered by one subtraction.
+// int16 pair -> fp16 subnormal pairs of the bytes of u = b + 32768: L = b & 255 and H = (b >> 8) + 128
+// (the high byte with its sign bit flipped), each the value byte * 2^-24 exactly.
+__device__ __forceinline__ void split_pair_u(uint32_t x, uint32_t& hi, uint32_t& lo) {
+  lo = x & 0x00FF00FFu;
+  hi = ((x >> 8) & 0x00FF00FFu) ^ 0x00800080u;
+}
+
+// int16 pair -> fp16 pairs of its high (signed) and low (unsigned) bytes, exactly (the 16-row
+// instantiation's B split, and its A split).  0x64xx as fp16 is 1024 + xx, so each byte is
+// recovered by one subtraction.
 __device__ __forceinline__ void split_pair(uint32_t x, uint32_t& hi, uint32_t& lo) {
   const uint32_t lo_bits = (x & 0x00FF00FFu) | 0x64006400u;         // 1024 + lo
   const uint32_t hi_bits = ((x >> 8) & 0x00FF00FFu) ^ 0x64806480u;  // 1024 + (hi + 128)
@@ -151,6 +167,7 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   uint32_t* a_limb = reinterpret_cast<uint32_t*>(smem + static_cast<size_t>(stages) * STAGE_BYTES);  // [16][a_stride]
   uint32_t* a_raw = a_limb + A_ROWS * a_stride;                                                      // [16][cta_pairs]
   uint64_t* bars = reinterpret_cast<uint64_t*>(a_raw + A_ROWS * cta_pairs);
+  int32_t* row_sum = reinterpret_cast<int32_t*>(bars + 2 * stages + 1);  // [16]: the A slice's row sums
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * stages;
   const uint32_t abar = empty0 + 8 * stages;  // the CTA's A slice has landed
@@ -239,7 +256,8 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
   // at word (kp / 4) % 2 and low limb two words further.
   auto store_limbs = [&](int row, int kp, uint32_t x) {
     uint32_t hi, lo;
-    split_pair(x, hi, lo);
+    if constexpr (NT == 1) tc::limbs16x2(x, hi, lo);  // centred limbs: |h|, |l| <= 128
+    else split_pair(x, hi, lo);
     const int w = row * a_stride + (kp >> 3) * 16 + (kp & 3) * 4 + ((kp >> 2) & 1);
     a_limb[w] = hi;
     a_limb[w + 2] = lo;
@@ -258,6 +276,18 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
       const int kp = idx - row * pairs;
       store_limbs(row, kp, (row < mrows && 2 * kp < kv) ? a_raw[row * cta_pairs + kp] : 0u);
     }
+    if constexpr (NT == 1) {
+      // warp w sums row w of the slice (two int16 per word): the correction of B's offset
+      int32_t rs = 0;
+      if (warp < mrows)
+        for (int kp = lane; kp < pairs && 2 * kp < kv; kp += 32) {
+          const uint32_t x = a_raw[warp * cta_pairs + kp];
+          rs += static_cast<int32_t>(static_cast<int16_t>(x & 0xFFFFu)) +
+                static_cast<int32_t>(static_cast<int16_t>(x >> 16));
+        }
+      for (int o = 16; o > 0; o >>= 1) rs += __shfl_xor_sync(0xFFFFFFFFu, rs, o);
+      if (lane == 0 && warp < A_ROWS) row_sum[warp] = rs;
+    }
     asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // every consumer warp arrives
     ok = landed;
   } else {
@@ -275,6 +305,16 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         x = v0 | (v1 << 16);
       }
       store_limbs(row, kp, x);
+    }
+    if constexpr (NT == 1) {
+      // warp w sums row w of the slice: the correction of B's offset
+      int32_t rs = 0;
+      if (warp < mrows) {
+        const int64_t kend = min(k0 + static_cast<int64_t>(nst) * KS, P.k);
+        for (int64_t k = k0 + lane; k < kend; k += 32) rs += Ag[warp * P.lda + k];
+      }
+      for (int o = 16; o > 0; o >>= 1) rs += __shfl_xor_sync(0xFFFFFFFFu, rs, o);
+      if (lane == 0 && warp < A_ROWS) row_sum[warp] = rs;
     }
     asm volatile("bar.sync 1, %0;" ::"n"(NCONS * 32) : "memory");  // consumer warps only
   }
@@ -333,7 +373,10 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
     for (int mt = 0; mt < MT; ++mt) {
       uint32_t bhi[4], blo[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) split_pair(bk[mt][q], bhi[q], blo[q]);
+      for (int q = 0; q < 4; ++q) {
+        if constexpr (NT == 1) split_pair_u(bk[mt][q], bhi[q], blo[q]);
+        else split_pair(bk[mt][q], bhi[q], blo[q]);
+      }
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
         mma16816(hh[mt][nt], bhi, ahi[nt][0], ahi[nt][1]);
@@ -382,9 +425,11 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
-            acc[mt][nt][c] += (static_cast<uint64_t>(static_cast<int64_t>(f2i(hh[mt][nt][c]))) << 16) +
-                              (static_cast<uint64_t>(static_cast<int64_t>(f2i(xx[mt][nt][c]))) << 8) +
-                              static_cast<uint64_t>(static_cast<int64_t>(f2i(ll[mt][nt][c])));
+            // m <= 8: the sums are in units of 2^-24 (the subnormal bytes of B); scaling is exact
+            constexpr float unit = NT == 1 ? 16777216.0f : 1.0f;
+            acc[mt][nt][c] += (static_cast<uint64_t>(static_cast<int64_t>(f2i(hh[mt][nt][c] * unit))) << 16) +
+                              (static_cast<uint64_t>(static_cast<int64_t>(f2i(xx[mt][nt][c] * unit))) << 8) +
+                              static_cast<uint64_t>(static_cast<int64_t>(f2i(ll[mt][nt][c] * unit)));
             hh[mt][nt][c] = xx[mt][nt][c] = ll[mt][nt][c] = 0.f;
           }
     }
@@ -402,7 +447,9 @@ skinny_kernel(const __grid_constant__ CUtensorMap mapB, SkParams P) {
         const int64_t j = j_base + warp * (16 * MT) + mt * 16 + g + 8 * (c >> 1);
         if (i < mrows && j < P.n) {
           unsigned long long* dst = reinterpret_cast<unsigned long long*>(Cg + i * P.ldc + j);
-          const unsigned long long v = static_cast<unsigned long long>(acc[mt][nt][c]);
+          // m <= 8: B entered as u = b + 32768, so 32768 times the row's sum of A comes back off
+          unsigned long long v = static_cast<unsigned long long>(acc[mt][nt][c]);
+          if constexpr (NT == 1) v -= static_cast<unsigned long long>(static_cast<int64_t>(row_sum[i])) << 15;
           if (P.atomic_out) atomicAdd(dst, v);
           else *dst = *dst + v;
         }
