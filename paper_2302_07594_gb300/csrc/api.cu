@@ -822,6 +822,30 @@ int ensure_pipeline(DeviceState& d) {
 constexpr int kPipeSlots = 3;
 constexpr int64_t kPanelMin = 512;
 
+// First rows of the pipelined host path's row panels, then m: panels of at most mb rows, with a
+// quarter and a half panel at each end when m has room for them.  The small first panel starts
+// the copies out sooner; the small last panels shorten the end of the call, where the last GEMM
+// and its copy out run with nothing left to overlap them.
+std::vector<int64_t> panel_starts(int64_t m, int64_t mb) {
+  std::vector<int64_t> starts{0};
+  const int64_t q = mb / 4, h = mb / 2;
+  if (q < 1 || m < 2 * (q + h) + mb) {
+    for (int64_t r = mb; r < m; r += mb) starts.push_back(r);
+  } else {
+    starts.push_back(q);
+    starts.push_back(q + h);
+    // whole panels in the middle, the remainder of the rows as one panel in front of them
+    const int64_t mid = m - 2 * (q + h);
+    int64_t r = q + h + mid % mb;
+    if (r > q + h) starts.push_back(r);
+    for (r += mb; r < m - q - h; r += mb) starts.push_back(r);
+    starts.push_back(m - q - h);
+    starts.push_back(m - q);
+  }
+  starts.push_back(m);
+  return starts;
+}
+
 // Host-buffer GEMM of m >= 2 * kPanelMin rows as a pipeline over row panels of A and C.  B is
 // copied and split into limb planes once; then each panel's copy in (A and C rows), GEMM and
 // copy out run on three streams (copy in, the caller's stream, copy out) through a ring of
@@ -835,7 +859,8 @@ int host_gemm_pipelined(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k,
   cudaStream_t s = g_stream;
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 8));
   const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 15) / 16), 128)));
-  const int64_t panels = (m + mb - 1) / mb;
+  const std::vector<int64_t> starts = panel_starts(m, mb);
+  const int64_t panels = static_cast<int64_t>(starts.size()) - 1;
   const size_t b_raw = round_up(static_cast<size_t>(k) * n * sizeof(OP), kAlign);
   const size_t b_plane = round_up(static_cast<size_t>(n) * pitch * 2, kAlign);
   const size_t a_slot = round_up(static_cast<size_t>(mb) * k * sizeof(OP), kAlign);
@@ -880,7 +905,7 @@ int host_gemm_pipelined(DeviceState& d, int nl, int64_t m, int64_t n, int64_t k,
   }
   for (int64_t p = 0; p < panels; ++p) {
     const int r = static_cast<int>(p % kPipeSlots);
-    const int64_t r0 = p * mb, mi = std::min(mb, m - r0);
+    const int64_t r0 = starts[p], mi = starts[p + 1] - r0;
     OP* dA = reinterpret_cast<OP*>(slots + r * (a_slot + c_slot));
     CT* dC = reinterpret_cast<CT*>(slots + r * (a_slot + c_slot) + a_slot);
     e = p >= kPipeSlots ? cudaStreamWaitEvent(d.h2d, ev[8 + r], 0) : cudaSuccess;  // slot's last copy out
@@ -977,7 +1002,8 @@ int host_gemm_i4_pipelined(DeviceState& d, int64_t m, int64_t n, int64_t k, cons
   const int64_t dldc = static_cast<int64_t>(round_up(static_cast<size_t>(n), 4));
   const int64_t pitch = static_cast<int64_t>(round_up(static_cast<size_t>(k), 16));
   const int64_t mb = std::max<int64_t>(kPanelMin, static_cast<int64_t>(round_up(static_cast<size_t>((m + 15) / 16), 128)));
-  const int64_t panels = (m + mb - 1) / mb;
+  const std::vector<int64_t> starts = panel_starts(m, mb);
+  const int64_t panels = static_cast<int64_t>(starts.size()) - 1;
   const size_t b_raw = round_up(static_cast<size_t>(k) * dldb, kAlign);
   const size_t b_plane = round_up(static_cast<size_t>(n) * pitch, kAlign);
   const size_t a_slot = round_up(static_cast<size_t>(mb) * dlda, kAlign);
@@ -1018,7 +1044,7 @@ int host_gemm_i4_pipelined(DeviceState& d, int64_t m, int64_t n, int64_t k, cons
   }
   for (int64_t p = 0; p < panels; ++p) {
     const int r = static_cast<int>(p % kPipeSlots);
-    const int64_t r0 = p * mb, mi = std::min(mb, m - r0);
+    const int64_t r0 = starts[p], mi = starts[p + 1] - r0;
     uint8_t* dA = reinterpret_cast<uint8_t*>(slots + r * (a_slot + c_slot));
     int32_t* dC = reinterpret_cast<int32_t*>(slots + r * (a_slot + c_slot) + a_slot);
     e = p >= kPipeSlots ? cudaStreamWaitEvent(d.h2d, ev[8 + r], 0) : cudaSuccess;  // slot's last copy out
