@@ -227,3 +227,51 @@ def test_conv_argument_errors(gm):
     assert L.gemmi_conv2d_i16(1, 2, 2, 64, 8, 5, 5, 0, 0, dX.data_ptr(), dW.data_ptr(), dY.data_ptr(), None) == gm.EINVAL
     # an empty output is a no-op
     assert L.gemmi_conv2d_i16(0, 4, 4, 64, 8, 3, 3, 1, 1, None, None, None, None) == gm.OK
+
+
+def _random_conv_shapes(count, seed):
+    """Seeded random convolution shapes over the three paths: "same" 64-channel convolutions with
+    odd filters (the direct kernel when its rule holds), other "same" ones with Cin % 64 == 0 (the
+    fused kernel on the NHWC tensor) and everything else (lowered first).  The oracle's work per
+    case stays below about 4e7 multiply-adds."""
+    rng = np.random.Generator(np.random.Philox(seed))
+    shapes = []
+    while len(shapes) < count:
+        kind = len(shapes) % 3
+        R = int(rng.choice([1, 3, 5])) if kind < 2 else int(rng.integers(1, 5))
+        S = int(rng.choice([1, 3, 5])) if kind < 2 else int(rng.integers(1, 5))
+        if kind == 0:
+            Ci, ph, pw = 64, (R - 1) // 2, (S - 1) // 2
+            Co = int(rng.integers(1, 33)) * 2
+        elif kind == 1:
+            Ci, ph, pw = int(rng.choice([64, 128])), (R - 1) // 2, (S - 1) // 2
+            Co = int(rng.integers(1, 80))
+        else:
+            Ci = int(rng.choice([3, 8, 16, 40, 64]))
+            ph, pw = int(rng.integers(0, R)), int(rng.integers(0, S))
+            Co = int(rng.integers(1, 70))
+        N = int(rng.integers(1, 4))
+        H = int(rng.integers(1, 30))
+        W = int(rng.choice([int(rng.integers(1, 40)), int(rng.integers(100, 121))]))
+        Ho, Wo = H + 2 * ph - R + 1, W + 2 * pw - S + 1
+        if Ho < 1 or Wo < 1 or N * Ho * Wo * Co * R * S * Ci > 4e7:
+            continue
+        shapes.append((N, H, W, Ci, Co, R, S, ph, pw))
+    return shapes
+
+
+RANDOM_CONV = _random_conv_shapes(45, 2302)
+
+
+@pytest.mark.parametrize("shape", RANDOM_CONV, ids=lambda s: "x".join(map(str, s)))
+def test_conv_random_sweep(gm, shape):
+    """Every element of a seeded random convolution against the oracle; where the direct kernel's
+    rule holds, that kernel is the one that ran."""
+    N, H, W, Ci, Co, R, S, ph, pw = shape
+    X, Wt, Y = make(9300 + sum(shape) * 7, *shape)
+    got, counts = run(gm, X, Wt, Y, R, S, ph, pw)
+    if direct_applies(gm, shape):
+        assert counts["conv_rows"] == 1, counts
+    else:
+        assert counts["conv_rows"] == 0, counts
+    assert_same(got, expected(X, Wt, Y, R, S, ph, pw), f"random {shape}")
