@@ -435,9 +435,11 @@ def test_host_api_padded(gm):
 # m >= 1024: the host path pipelines row panels of A and C (a ring of three device slots, so
 # panels reuse slots) with B copied and split once.  From m = 1280 on, the first two and the last
 # two panels are a quarter and a half panel (m = 2000: 128, 256, 208, 512, 512, 256, 128 rows;
-# m = 8192: 128, 256, 256, fourteen of 512, 256, 128); m = 1024 keeps two whole panels.
+# m = 8192: 128, 256, 256, fourteen of 512, 256, 128); m = 1024 and m = 1279 (512, 512, 255) keep
+# whole panels.
 @pytest.mark.parametrize("kind,m,n,k", [("i16", 2000, 300, 500), ("i8", 2000, 300, 500), ("i16", 1024, 64, 200),
-                                        ("i16", 5000, 130, 96), ("i16", 8192, 72, 64), ("i8", 1280, 40, 80)])
+                                        ("i16", 5000, 130, 96), ("i16", 8192, 72, 64), ("i8", 1280, 40, 80),
+                                        ("i16", 1279, 24, 40)])
 def test_host_api_pipelined_panels(gm, kind, m, n, k):
     A, B, C = gi.random_problem(905 + m + n, m, n, k, kind)
     # host operands with padded rows: the panel copies must honour the leading dimensions
